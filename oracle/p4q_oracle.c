@@ -1,0 +1,331 @@
+/*
+ * P4Q oracle: a plain, slow CPU restatement of the pruned W4A4 hot path.
+ *
+ * TEST INFRASTRUCTURE ONLY. Nothing in the product path may link, load or call
+ * this file; only the tests, the smoke check and the CPU-baseline leg of the
+ * benchmark do. It shares no code, header or table with the CUDA library.
+ *
+ * What it computes (P4Q, Sec. 3.2 "Quantization-Aware Pre-LLM Selection",
+ * Eq. 4, and App. A / App. B.3 for the W4A4 quantizer settings):
+ *   - q4_quantize_rows: symmetric round-to-nearest 4-bit quantizer, one scale
+ *     per row (per token for activations and selector copies, per output
+ *     channel for weights), clip ratio 1.0, no groups.
+ *   - q4_cosine: CosSim of two fake-quantized vectors s_a*c_a and s_b*c_b,
+ *     evaluated on their integer codes (the positive scales cancel).
+ *   - p4q_select_one: the three sequential selection stages of Eq. 4 (query
+ *     relevance per concept, CLS saliency on the rest, greedy max-min
+ *     diversity), then the retained indices in ascending order.
+ *   - w4a4_gemm_s32 / w4a4_linear: the integer matmul of INT4 codes and the
+ *     dequantization (acc * s_a) * s_w.
+ *
+ * Readings where the paper is silent (each is also listed in the design
+ * notes):
+ *   R1 quantizer arithmetic is IEEE fp32: a = max|x|, s = a / 7 (one rounded
+ *      division), code = clamp(round_half_even(x / s), -8, 7) where x / s is
+ *      one rounded fp32 division; a == 0 gives s = 0 and all codes 0.
+ *   R2 the selector's fake quantizer is the deployment activation quantizer
+ *      (4-bit, per token).
+ *   R3 cosine := (float)dot / sqrtf((float)n_a * (float)n_b), every operation
+ *      rounded to fp32 in that order, with n = sum of squared codes; 0 when
+ *      n_a * n_b == 0.
+ *   R4 budget split in integers: K_q = floor(alpha*K/1000),
+ *      K_s = floor(beta*K/1000), K_d = K - K_q - K_s (alpha, beta in
+ *      per mille); without concepts K_q moves to diversity, without CLS
+ *      attention K_s moves to diversity.
+ *   R5 query stage: concept j = 0..J-1 in order, quota
+ *      floor(K_q/J) + (j < K_q mod J); each concept takes its best-scoring
+ *      tokens not kept yet; ties go to the lower token index.
+ *   R6 saliency stage: best A_cls among tokens not kept; ties to lower index.
+ *   R7 diversity stage: m_i = max over kept r of cos(i, r), -inf when nothing
+ *      is kept; pick argmin m_i (ties to lower index), keep it, repeat K_d
+ *      times. Updating m_i with the newest pick equals recomputing the max
+ *      over the whole kept set, because max is associative.
+ *   R8 output indices are sorted ascending.
+ *
+ * Build: plain C11, -O2 -ffp-contract=off (no fused multiply-add, no
+ * fast-math), optional OpenMP over independent rows / images.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORACLE_OK 0
+#define ORACLE_BAD_ARG 1
+#define ORACLE_OVERFLOW 2
+
+int oracle_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+  return omp_get_max_threads();
+#else
+  (void)n;
+  return 1;
+#endif
+}
+
+/* ------------------------------------------------------------------ */
+/* Symmetric per-row 4-bit quantizer (App. A: symmetric round-to-nearest,  */
+/* per-token activations / per-output-channel weights, group size -1,      */
+/* clip ratio 1.0; App. B.3 repeats the settings). Reading R1.            */
+/* ------------------------------------------------------------------ */
+static void quantize_row(const float* x, int64_t cols, int8_t* code, float* scale) {
+  float a = 0.0f;
+  for (int64_t k = 0; k < cols; ++k) {
+    float m = fabsf(x[k]);
+    if (m > a) a = m;
+  }
+  if (a == 0.0f) {
+    *scale = 0.0f;
+    for (int64_t k = 0; k < cols; ++k) code[k] = 0;
+    return;
+  }
+  float s = a / 7.0f;           /* one rounded fp32 division */
+  for (int64_t k = 0; k < cols; ++k) {
+    float q = x[k] / s;          /* one rounded fp32 division */
+    float r = nearbyintf(q);     /* round half to even (default mode) */
+    if (r < -8.0f) r = -8.0f;
+    if (r > 7.0f) r = 7.0f;
+    code[k] = (int8_t)r;
+  }
+  *scale = s;
+}
+
+int q4_quantize_rows(const float* x, int64_t rows, int64_t cols, int8_t* code, float* scale) {
+  if (!x || !code || !scale || rows < 0 || cols <= 0) return ORACLE_BAD_ARG;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r)
+    quantize_row(x + r * cols, cols, code + r * cols, scale + r);
+  return ORACLE_OK;
+}
+
+/* Squared code norm n = sum c^2 (exact integer). */
+static int64_t code_norm2(const int8_t* c, int64_t d) {
+  int64_t n = 0;
+  for (int64_t k = 0; k < d; ++k) n += (int64_t)c[k] * c[k];
+  return n;
+}
+
+static int64_t code_dot(const int8_t* a, const int8_t* b, int64_t d) {
+  int64_t g = 0;
+  for (int64_t k = 0; k < d; ++k) g += (int64_t)a[k] * b[k];
+  return g;
+}
+
+/* CosSim of fake-quantized vectors, Eq. 4; reading R3. */
+static float cosine_from(int64_t dot, int64_t na, int64_t nb) {
+  if (na == 0 || nb == 0) return 0.0f;
+  float prod = (float)na * (float)nb;
+  float den = sqrtf(prod);
+  return (float)dot / den;
+}
+
+float q4_cosine(const int8_t* ca, const int8_t* cb, int64_t d) {
+  return cosine_from(code_dot(ca, cb, d), code_norm2(ca, d), code_norm2(cb, d));
+}
+
+/* ------------------------------------------------------------------ */
+/* Budget split (Sec. 3.2: alpha = 0.3, beta = 0.2, gamma = 0.5); R4.     */
+/* ------------------------------------------------------------------ */
+void p4q_budget(int K, int alpha_pm, int beta_pm, int have_q, int have_a, int* Kq, int* Ks, int* Kd) {
+  int q = (int)(((int64_t)alpha_pm * K) / 1000);
+  int s = (int)(((int64_t)beta_pm * K) / 1000);
+  if (!have_q) q = 0;
+  if (!have_a) s = 0;
+  *Kq = q;
+  *Ks = s;
+  *Kd = K - q - s;
+}
+
+/* Pick the best not-kept token under score (higher better), lower index on ties. */
+static int argbest_free(const float* score, const unsigned char* kept, int N) {
+  int best = -1;
+  for (int i = 0; i < N; ++i) {
+    if (kept[i]) continue;
+    if (best < 0 || score[i] > score[best]) best = i;
+  }
+  return best;
+}
+
+static int cmp_i32(const void* a, const void* b) {
+  int32_t x = *(const int32_t*)a, y = *(const int32_t*)b;
+  return (x > y) - (x < y);
+}
+
+/*
+ * One image of the selector (Eq. 4 and the three stage paragraphs of
+ * Sec. 3.2). V: [N, d] fp32 copies of fp16 features. Q: [J, d] or NULL.
+ * A: [N] CLS saliency or NULL. Outputs:
+ *   idx[K]          retained token indices, ascending (R8)
+ *   order[K]        (optional) indices in the order they were kept
+ *   stage[K]        (optional) 1 + concept j for query picks, -1 saliency,
+ *                   -2 diversity, aligned with order[]
+ */
+int p4q_select_one(const float* V, int N, int d, const float* Q, int J, const float* A,
+                   int K, int alpha_pm, int beta_pm, int32_t* idx, int32_t* order, int32_t* stage) {
+  if (!V || N <= 0 || d <= 0 || K < 1 || K > N || !idx) return ORACLE_BAD_ARG;
+  if (J < 0 || (J > 0 && !Q)) return ORACLE_BAD_ARG;
+  int have_q = (Q != NULL && J > 0);
+  int have_a = (A != NULL);
+  int Kq, Ks, Kd;
+  p4q_budget(K, alpha_pm, beta_pm, have_q, have_a, &Kq, &Ks, &Kd);
+  if (Kq < 0 || Ks < 0 || Kd < 0) return ORACLE_BAD_ARG;
+
+  /* Fake-quantized copies of the projector features and concept embeddings (R2). */
+  int8_t* cv = (int8_t*)malloc((size_t)N * d);
+  float* sv = (float*)malloc(sizeof(float) * N);
+  int64_t* nv = (int64_t*)malloc(sizeof(int64_t) * N);
+  unsigned char* kept = (unsigned char*)calloc(N, 1);
+  float* score = (float*)malloc(sizeof(float) * N);
+  int32_t* picks = (int32_t*)malloc(sizeof(int32_t) * K);
+  int32_t* stg = (int32_t*)malloc(sizeof(int32_t) * K);
+  if (!cv || !sv || !nv || !kept || !score || !picks || !stg) {
+    free(cv); free(sv); free(nv); free(kept); free(score); free(picks); free(stg);
+    return ORACLE_BAD_ARG;
+  }
+  for (int i = 0; i < N; ++i) {
+    quantize_row(V + (int64_t)i * d, d, cv + (int64_t)i * d, sv + i);
+    nv[i] = code_norm2(cv + (int64_t)i * d, d);
+  }
+  int nk = 0;
+
+  /* Stage 1: query relevance, one ranking per concept (R5). */
+  if (Kq > 0) {
+    int8_t* cq = (int8_t*)malloc((size_t)d);
+    float sq;
+    for (int j = 0; j < J; ++j) {
+      int quota = Kq / J + (j < Kq % J ? 1 : 0);
+      quantize_row(Q + (int64_t)j * d, d, cq, &sq);
+      int64_t nq = code_norm2(cq, d);
+      for (int i = 0; i < N; ++i)
+        score[i] = cosine_from(code_dot(cq, cv + (int64_t)i * d, d), nq, nv[i]);
+      for (int t = 0; t < quota; ++t) {
+        int b = argbest_free(score, kept, N);
+        kept[b] = 1;
+        picks[nk] = b;
+        stg[nk] = 1 + j;
+        ++nk;
+      }
+    }
+    free(cq);
+  }
+
+  /* Stage 2: visual saliency on the tokens left by stage 1 (R6). */
+  for (int t = 0; t < Ks; ++t) {
+    int b = argbest_free(A, kept, N);
+    kept[b] = 1;
+    picks[nk] = b;
+    stg[nk] = -1;
+    ++nk;
+  }
+
+  /* Stage 3: greedy max-min diversity (R7). */
+  if (Kd > 0) {
+    float* m = score; /* reuse: m_i = max cosine to the kept set */
+    for (int i = 0; i < N; ++i) {
+      m[i] = -INFINITY;
+      if (kept[i]) continue;
+      for (int r = 0; r < nk; ++r) {
+        int p = picks[r];
+        float c = cosine_from(code_dot(cv + (int64_t)i * d, cv + (int64_t)p * d, d), nv[i], nv[p]);
+        if (c > m[i]) m[i] = c;
+      }
+    }
+    for (int t = 0; t < Kd; ++t) {
+      int b = -1;
+      for (int i = 0; i < N; ++i) {
+        if (kept[i]) continue;
+        if (b < 0 || m[i] < m[b]) b = i;
+      }
+      kept[b] = 1;
+      picks[nk] = b;
+      stg[nk] = -2;
+      ++nk;
+      for (int i = 0; i < N; ++i) {
+        if (kept[i]) continue;
+        float c = cosine_from(code_dot(cv + (int64_t)i * d, cv + (int64_t)b * d, d), nv[i], nv[b]);
+        if (c > m[i]) m[i] = c;
+      }
+    }
+  }
+
+  for (int t = 0; t < K; ++t) {
+    idx[t] = picks[t];
+    if (order) order[t] = picks[t];
+    if (stage) stage[t] = stg[t];
+  }
+  qsort(idx, (size_t)K, sizeof(int32_t), cmp_i32);
+  free(cv); free(sv); free(nv); free(kept); free(score); free(picks); free(stg);
+  return ORACLE_OK;
+}
+
+/* Batched selector: images are independent. */
+int p4q_select_batch(const float* V, int B, int N, int d, const float* Q, int J, const float* A,
+                     int K, int alpha_pm, int beta_pm, int32_t* idx) {
+  if (B < 0) return ORACLE_BAD_ARG;
+  int bad = 0;
+#pragma omp parallel for schedule(dynamic, 1) reduction(| : bad)
+  for (int b = 0; b < B; ++b) {
+    const float* Qb = Q ? Q + (int64_t)b * J * d : NULL;
+    const float* Ab = A ? A + (int64_t)b * N : NULL;
+    bad |= p4q_select_one(V + (int64_t)b * N * d, N, d, Qb, J, Ab, K, alpha_pm, beta_pm,
+                          idx + (int64_t)b * K, NULL, NULL);
+  }
+  return bad ? ORACLE_BAD_ARG : ORACLE_OK;
+}
+
+/* ------------------------------------------------------------------ */
+/* W4A4 linear (App. B.3): integer matmul of the codes, then dequant.      */
+/* ------------------------------------------------------------------ */
+int w4a4_gemm_s32(const int8_t* a, const int8_t* w, int64_t M, int64_t N, int64_t K, int32_t* acc) {
+  if (!a || !w || !acc || M < 0 || N < 0 || K <= 0) return ORACLE_BAD_ARG;
+  int overflow = 0;
+#pragma omp parallel for schedule(static) reduction(| : overflow)
+  for (int64_t m = 0; m < M; ++m) {
+    for (int64_t n = 0; n < N; ++n) {
+      int64_t g = code_dot(a + m * K, w + n * K, K);
+      if (g > INT32_MAX || g < INT32_MIN) overflow = 1;
+      acc[m * N + n] = (int32_t)g;
+    }
+  }
+  return overflow ? ORACLE_OVERFLOW : ORACLE_OK;
+}
+
+/* y[m, n] = ((float)acc * s_a[m]) * s_w[n], each product rounded to fp32. */
+int w4a4_linear(const int8_t* a, const float* sa, const int8_t* w, const float* sw,
+                int64_t M, int64_t N, int64_t K, float* y) {
+  if (!sa || !sw || !y) return ORACLE_BAD_ARG;
+  int32_t* acc = (int32_t*)malloc(sizeof(int32_t) * (size_t)(M * N > 0 ? M * N : 1));
+  if (!acc) return ORACLE_BAD_ARG;
+  int rc = w4a4_gemm_s32(a, w, M, N, K, acc);
+  if (rc == ORACLE_OK) {
+    for (int64_t m = 0; m < M; ++m)
+      for (int64_t n = 0; n < N; ++n) {
+        float t = (float)acc[m * N + n] * sa[m];
+        y[m * N + n] = t * sw[n];
+      }
+  }
+  free(acc);
+  return rc;
+}
+
+/* Gather of the FP16 originals (Sec. 3.2: the originals, not the fake-quantized
+ * copies, go to the language model): X = [V[idx]; text] per image. */
+int p4q_gather(const float* V, int B, int N, int d, const int32_t* idx, int K, const float* text, int T,
+               float* X) {
+  if (!V || !idx || !X || B < 0 || K < 0 || T < 0 || (T > 0 && !text)) return ORACLE_BAD_ARG;
+  for (int b = 0; b < B; ++b) {
+    float* xb = X + (int64_t)b * (K + T) * d;
+    for (int t = 0; t < K; ++t) {
+      int i = idx[(int64_t)b * K + t];
+      if (i < 0 || i >= N) return ORACLE_BAD_ARG;
+      memcpy(xb + (int64_t)t * d, V + ((int64_t)b * N + i) * d, sizeof(float) * d);
+    }
+    for (int t = 0; t < T; ++t)
+      memcpy(xb + (int64_t)(K + t) * d, text + ((int64_t)b * T + t) * d, sizeof(float) * d);
+  }
+  return ORACLE_OK;
+}
