@@ -1,0 +1,183 @@
+/*
+ * p4q.h - C ABI of the P4Q pruned W4A4 hot path on NVIDIA GB300 (sm_103a).
+ *
+ * P4Q (co-designed visual-token pruning and W4A4 quantization) runs two things
+ * between the vision projector and the low-bit language model:
+ *   1. a quantization-aware visual-token selector (Sec. 3.2, Eq. 4): the
+ *      projector features and the question's concept embeddings are copied,
+ *      fake-quantized to 4 bits, and scored in three sequential stages (query
+ *      relevance per concept, CLS saliency, greedy max-min diversity) until the
+ *      token budget K is filled; the original FP16 features of the kept tokens
+ *      are forwarded;
+ *   2. W4A4 linear layers on the shortened sequence (App. A and App. B.3):
+ *      symmetric round-to-nearest INT4 weights with one scale per output
+ *      channel, INT4 activations with one scale per token, integer matmul and
+ *      dequantization.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers are DEVICE pointers unless a parameter says otherwise. The
+ *     caller owns every buffer; the library allocates nothing per call.
+ *   - fp16 tensors are passed as uint16_t bit patterns (IEEE binary16).
+ *   - Packed INT4: two codes per byte, the even index in the low nibble, each
+ *     nibble a two's complement integer. Codes produced here lie in [-7, 7].
+ *   - All work is enqueued asynchronously on `stream` (NULL = legacy default
+ *     stream); p4q_stream_t has the same type as cudaStream_t.
+ *   - Arguments are validated on the host before anything is launched; a
+ *     failed check returns an error status and launches nothing.
+ *     P4Q_ERR_CUDA reports a launch error (query cudaGetLastError for detail).
+ *     Device-side waits are bounded: a wait that runs out sets a device error
+ *     word, the kernel returns, and the next p4q_device_status() call reports
+ *     P4Q_ERR_TIMEOUT. No call aborts the process or traps the GPU.
+ *   - Behaviour on non-finite inputs is unspecified (no fault, values undefined).
+ *   - Alignment: every device pointer must be 16-byte aligned.
+ */
+#ifndef P4Q_H_
+#define P4Q_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* p4q_stream_t;
+
+typedef enum {
+  P4Q_OK = 0,
+  P4Q_ERR_INVALID_ARG = 1,          /* null pointer, negative size, K > N, ... */
+  P4Q_ERR_UNSUPPORTED_SHAPE = 2,    /* size outside the documented limits */
+  P4Q_ERR_MISALIGNED = 3,           /* a device pointer not 16-byte aligned */
+  P4Q_ERR_WORKSPACE_TOO_SMALL = 4,  /* ws_bytes below the queried size */
+  P4Q_ERR_CUDA = 5,                 /* a CUDA runtime / launch error */
+  P4Q_ERR_TIMEOUT = 6,              /* a bounded device wait ran out */
+  P4Q_ERR_NO_DEVICE = 7             /* no sm_103 device current */
+} p4q_status;
+
+/* Budget split of the selector (Sec. 3.2: alpha = 0.3, beta = 0.2, gamma =
+ * 0.5). K_q = floor(alpha_permille * K / 1000) tokens go to query relevance,
+ * K_s = floor(beta_permille * K / 1000) to CLS saliency, the rest
+ * K_d = K - K_q - K_s to diversity. When no concept embeddings are given
+ * (Q == NULL or J == 0) K_q moves to diversity; when A_cls == NULL K_s does. */
+typedef struct {
+  int32_t K;               /* retained visual tokens per image, 1 <= K <= N */
+  int32_t alpha_permille;  /* query-relevance share, 0..1000 (default 300) */
+  int32_t beta_permille;   /* saliency share, 0..1000-alpha (default 200) */
+} p4q_select_params;
+
+/* Limits checked by the calls below. */
+#define P4Q_MAX_TOKENS 4096   /* N, visual tokens per image */
+#define P4Q_MAX_CONCEPTS 16   /* J, concept embeddings per image */
+#define P4Q_MAX_ROW 16384     /* d and Kin (elements per row) */
+
+/* Human-readable name of a status code (static storage, never NULL). */
+const char* p4q_status_string(p4q_status s);
+
+/* Reads and clears the device error word of the current device after
+ * synchronizing `stream`. Returns P4Q_ERR_TIMEOUT if a bounded device wait ran
+ * out since the last call, P4Q_ERR_CUDA on a CUDA error, else P4Q_OK. */
+p4q_status p4q_device_status(p4q_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* Per-row 4-bit quantizers (App. A, App. B.3)                             */
+/* ---------------------------------------------------------------------- */
+
+/* Per-token activation quantization (App. A: symmetric round-to-nearest,
+ * per-token 4-bit activations, group size -1, clip ratio 1.0).
+ * For each row m of X:
+ *   a = max_k |X[m,k]|, s_a[m] = a / 7 (fp32, rounded once),
+ *   code[m,k] = clamp(round_half_even(X[m,k] / s_a[m]), -8, 7) with the
+ *   quotient rounded to fp32; a == 0 gives s_a[m] = 0 and zero codes.
+ *   X   [M, Kin] fp16 row-major (device, read)
+ *   Xq  [M, Kin/2] packed INT4 (device, written)
+ *   s_a [M] fp32 (device, written)
+ * Requires M >= 0, 2 <= Kin <= P4Q_MAX_ROW, Kin % 16 == 0. M == 0 is a no-op. */
+p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* s_a,
+                         p4q_stream_t stream);
+
+/* Per-output-channel weight quantization (App. B.3: symmetric, per output
+ * channel, then round-to-nearest): the same per-row quantizer applied to each
+ * output row of W.
+ *   W   [N, Kin] fp16 row-major, one row per output channel (device, read)
+ *   Wq  [N, Kin/2] packed INT4 (device, written)
+ *   s_w [N] fp32 (device, written)
+ * Same size limits as p4q_quant_act. Not on the timed path (offline). */
+p4q_status p4q_quant_weight(const uint16_t* W, int N, int Kin, uint8_t* Wq, float* s_w,
+                            p4q_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* W4A4 linear (App. B.3: INT4 weights per output channel, INT4 activations */
+/* per token)                                                              */
+/* ---------------------------------------------------------------------- */
+
+/* Y[m,n] = fp16_rne( ((float)acc[m,n] * s_a[m]) * s_w[n] ),
+ * acc[m,n] = sum_k code_x[m,k] * code_w[n,k] computed exactly (int32).
+ *   Xq  [M, Kin/2] packed INT4, s_a [M] fp32   (device, read)
+ *   Wq  [N, Kin/2] packed INT4, s_w [N] fp32   (device, read)
+ *   Y   [M, N] fp16 row-major                  (device, written)
+ * Requires M >= 0, N >= 1, Kin % 128 == 0, 128 <= Kin <= P4Q_MAX_ROW,
+ * N % 8 == 0. Runs on the tcgen05 tensor cores. */
+p4q_status p4q_w4a4_linear(const uint8_t* Xq, const float* s_a, int M, int Kin,
+                           const uint8_t* Wq, const float* s_w, int N, uint16_t* Y,
+                           p4q_stream_t stream);
+
+/* Test entry: the exact int32 accumulators of the same integer matmul,
+ * acc [M, N] int32 row-major (device, written). Same limits as above. */
+p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N,
+                             int32_t* acc, p4q_stream_t stream);
+
+/* ---------------------------------------------------------------------- */
+/* Quantization-aware visual-token selector (Sec. 3.2, Eq. 4)               */
+/* ---------------------------------------------------------------------- */
+
+/* Device workspace needed by p4q_select / p4q_select_gather_quant for these
+ * sizes (bytes, a multiple of 256). Returns 0 if the sizes are invalid. */
+size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_params* params);
+
+/* Selects K of the N visual tokens of each image (Sec. 3.2, Eq. 4):
+ *   - V and Q are fake-quantized per row with the 4-bit quantizer above
+ *     (the selector sees only the fake-quantized copies);
+ *   - CosSim(a, b) of fake-quantized rows is evaluated on their codes as
+ *     (float)dot / sqrtf((float)|c_a|^2 * (float)|c_b|^2), fp32, 0 if a norm
+ *     is 0 (the positive scales cancel);
+ *   - stage 1 (query relevance): concept j = 0..J-1 in turn keeps its
+ *     floor(K_q/J) + (j < K_q % J) best-cosine tokens not kept yet;
+ *   - stage 2 (visual saliency): the K_s largest A_cls among tokens not kept;
+ *   - stage 3 (visual diversity): K_d times, keep the token whose largest
+ *     cosine to the kept set is smallest (the first token when nothing is kept);
+ *   - every tie goes to the lower token index.
+ *   V     [B, N, d] fp16 projector features (device, read)
+ *   Q     [B, J, d] fp16 concept embeddings, or NULL (then J is ignored)
+ *   A_cls [B, N] fp32 CLS-to-patch attention (head-averaged), or NULL
+ *   idx   [B, K] int32, kept token indices in ascending order (device, written)
+ *   ws    device workspace of at least p4q_select_workspace_bytes() bytes,
+ *         256-byte aligned; its contents are scratch.
+ * Requires 1 <= B, 1 <= K <= N <= P4Q_MAX_TOKENS, 0 <= J <= P4Q_MAX_CONCEPTS,
+ * d % 128 == 0, 128 <= d <= P4Q_MAX_ROW, 0 <= alpha, beta and
+ * alpha + beta <= 1000. */
+p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
+                      const float* A_cls, const p4q_select_params* params, int32_t* idx,
+                      void* ws, size_t ws_bytes, p4q_stream_t stream);
+
+/* The selector followed by the gather of the original FP16 features of the
+ * kept tokens (Sec. 3.2: the fake-quantized copies only decide the indices)
+ * and the per-token INT4 quantization of the pruned sequence for the first
+ * W4A4 linear. Per image b the pruned sequence is
+ *   X[b] = [ V[b, idx[b,0]], ..., V[b, idx[b,K-1]], text[b,0], ..., text[b,T-1] ]
+ *   text [B, T, d] fp16 (device, read), or NULL when T == 0
+ *   idx  [B, K] int32 ascending (device, written)
+ *   X    [B, K+T, d] fp16 (device, written)
+ *   Xq   [B*(K+T), d/2] packed INT4, s_a [B*(K+T)] fp32 (device, written):
+ *        the activation quantizer of p4q_quant_act applied to every row of X.
+ * Other arguments and limits as p4q_select; T >= 0. */
+p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
+                                   int J, const float* A_cls, const uint16_t* text, int T,
+                                   const p4q_select_params* params, int32_t* idx, uint16_t* X,
+                                   uint8_t* Xq, float* s_a, void* ws, size_t ws_bytes,
+                                   p4q_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* P4Q_H_ */

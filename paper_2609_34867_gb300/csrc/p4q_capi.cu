@@ -1,0 +1,246 @@
+// The extern "C" boundary of libp4q.so (declared in include/p4q.h): argument
+// validation on the host, then the kernel launches of each entry point on the
+// caller's stream. Nothing here allocates memory.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "p4q.h"
+#include "p4q_internal.h"
+
+using namespace p4q;
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// The kernels are built for sm_103a only; refuse to launch on anything else.
+p4q_status check_device() {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess) return P4Q_ERR_NO_DEVICE;
+  int major = 0, minor = 0;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return P4Q_ERR_NO_DEVICE;
+  return (major == 10 && minor == 3) ? P4Q_OK : P4Q_ERR_NO_DEVICE;
+}
+
+p4q_status from_cuda(cudaError_t e) { return e == cudaSuccess ? P4Q_OK : P4Q_ERR_CUDA; }
+
+struct Budget {
+  int Kq, Ks, Kd;
+};
+
+// Budget split of Sec. 3.2 in integers; absent signals hand their share to diversity.
+Budget split(const p4q_select_params& p, bool have_q, bool have_a) {
+  Budget b;
+  b.Kq = have_q ? static_cast<int>((static_cast<long long>(p.alpha_permille) * p.K) / 1000) : 0;
+  b.Ks = have_a ? static_cast<int>((static_cast<long long>(p.beta_permille) * p.K) / 1000) : 0;
+  b.Kd = p.K - b.Kq - b.Ks;
+  return b;
+}
+
+p4q_status check_select_args(const uint16_t* V, int B, int N, int d, int J, const p4q_select_params* params,
+                             const int32_t* idx) {
+  if (!V || !params || !idx || B < 1 || N < 1 || d < 1 || J < 0) return P4Q_ERR_INVALID_ARG;
+  if (params->K < 1 || params->K > N || params->alpha_permille < 0 || params->beta_permille < 0 ||
+      params->alpha_permille + params->beta_permille > 1000)
+    return P4Q_ERR_INVALID_ARG;
+  if (N > P4Q_MAX_TOKENS || J > P4Q_MAX_CONCEPTS || d % 128 != 0 || d > P4Q_MAX_ROW || B > 65535)
+    return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned16(V) || !aligned16(idx)) return P4Q_ERR_MISALIGNED;
+  return P4Q_OK;
+}
+
+p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
+                      const p4q_select_params* params, int32_t* idx, void* ws, size_t ws_bytes,
+                      cudaStream_t stream) {
+  const bool have_q = (Q != nullptr && J > 0);
+  const int Jeff = have_q ? J : 0;
+  if (have_q && !aligned16(Q)) return P4Q_ERR_MISALIGNED;
+  if (A_cls && !aligned16(A_cls)) return P4Q_ERR_MISALIGNED;
+  const size_t need = select_workspace_layout(B, N, d, Jeff, nullptr, nullptr);
+  if (!ws || ws_bytes < need) return P4Q_ERR_WORKSPACE_TOO_SMALL;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return P4Q_ERR_MISALIGNED;
+  SelectWorkspace w;
+  select_workspace_layout(B, N, d, Jeff, &w, ws);
+  const Budget bud = split(*params, have_q, A_cls != nullptr);
+  SelectPlan plan{B, N, d, Jeff, params->K, bud.Kq, bud.Ks, bud.Kd};
+
+  // Fake-quantized copies of the projector features (and the concepts).
+  RowSource src;
+  src.X = V;
+  RowSinks sv;
+  sv.codes = w.vcodes;
+  sv.scale = w.vscale;
+  sv.norm2 = w.vnorm;
+  cudaError_t e = launch_quant_rows(src, B * N, d, sv, stream);
+  if (e != cudaSuccess) return from_cuda(e);
+  if (bud.Kq > 0) {
+    RowSource sq;
+    sq.X = Q;
+    RowSinks oq;
+    oq.codes = w.qcodes;
+    oq.scale = w.qscale;
+    oq.norm2 = w.qnorm;
+    e = launch_quant_rows(sq, B * Jeff, d, oq, stream);
+    if (e == cudaSuccess) e = launch_query_scores(plan, w, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+  }
+  if (bud.Kd > 0) {
+    GemmArgs g;
+    g.A = w.vcodes;
+    g.B = w.vcodes;
+    g.M = N;
+    g.N = N;
+    g.K = d;
+    g.batch = B;
+    g.a_batch_stride = N;
+    g.b_batch_stride = N;
+    g.out = GemmOut::kCos;
+    g.D = w.gram;
+    g.norm_a = w.vnorm;
+    g.norm_b = w.vnorm;
+    e = launch_w4a4_gemm(g, stream);
+    if (e != cudaSuccess) return from_cuda(e);
+  }
+  return from_cuda(launch_select_stages(plan, w, A_cls, idx, stream));
+}
+
+p4q_status check_rows(const void* X, int M, int Kin, const void* Xq, const void* s) {
+  if (M < 0 || Kin < 1) return P4Q_ERR_INVALID_ARG;
+  if (M > 0 && (!X || !Xq || !s)) return P4Q_ERR_INVALID_ARG;
+  if (Kin % 16 != 0 || Kin > P4Q_MAX_ROW) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (M > 0 && (!aligned16(X) || !aligned16(Xq) || !aligned16(s))) return P4Q_ERR_MISALIGNED;
+  return P4Q_OK;
+}
+
+p4q_status check_gemm(const void* Xq, int M, int Kin, const void* Wq, int N, const void* out) {
+  if (M < 0 || N < 1 || Kin < 1 || !Wq || (M > 0 && (!Xq || !out))) return P4Q_ERR_INVALID_ARG;
+  if (Kin % 128 != 0 || Kin > P4Q_MAX_ROW || N % 8 != 0 || M > 65535 * 128) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned16(Wq) || (M > 0 && (!aligned16(Xq) || !aligned16(out)))) return P4Q_ERR_MISALIGNED;
+  return P4Q_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* p4q_status_string(p4q_status s) {
+  switch (s) {
+    case P4Q_OK: return "ok";
+    case P4Q_ERR_INVALID_ARG: return "invalid argument";
+    case P4Q_ERR_UNSUPPORTED_SHAPE: return "unsupported shape";
+    case P4Q_ERR_MISALIGNED: return "device pointer not 16-byte aligned";
+    case P4Q_ERR_WORKSPACE_TOO_SMALL: return "workspace too small";
+    case P4Q_ERR_CUDA: return "CUDA error";
+    case P4Q_ERR_TIMEOUT: return "a bounded device wait timed out";
+    case P4Q_ERR_NO_DEVICE: return "no sm_103 device is current";
+  }
+  return "unknown status";
+}
+
+p4q_status p4q_device_status(p4q_stream_t stream) {
+  if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
+  const unsigned int g = gemm_read_and_clear_error();
+  if (cudaGetLastError() != cudaSuccess) return P4Q_ERR_CUDA;
+  return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
+}
+
+p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* s_a, p4q_stream_t stream) {
+  p4q_status st = check_rows(X, M, Kin, Xq, s_a);
+  if (st != P4Q_OK || M == 0) return st;
+  if ((st = check_device()) != P4Q_OK) return st;
+  RowSource src;
+  src.X = X;
+  RowSinks o;
+  o.codes = Xq;
+  o.scale = s_a;
+  return from_cuda(launch_quant_rows(src, M, Kin, o, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+p4q_status p4q_quant_weight(const uint16_t* W, int N, int Kin, uint8_t* Wq, float* s_w, p4q_stream_t stream) {
+  return p4q_quant_act(W, N, Kin, Wq, s_w, stream);
+}
+
+p4q_status p4q_w4a4_linear(const uint8_t* Xq, const float* s_a, int M, int Kin, const uint8_t* Wq,
+                           const float* s_w, int N, uint16_t* Y, p4q_stream_t stream) {
+  p4q_status st = check_gemm(Xq, M, Kin, Wq, N, Y);
+  if (st != P4Q_OK) return st;
+  if (!s_w || (M > 0 && !s_a)) return P4Q_ERR_INVALID_ARG;
+  if (M == 0) return P4Q_OK;
+  if ((st = check_device()) != P4Q_OK) return st;
+  GemmArgs g;
+  g.A = Xq;
+  g.B = Wq;
+  g.M = M;
+  g.N = N;
+  g.K = Kin;
+  g.out = GemmOut::kHalf;
+  g.D = Y;
+  g.s_a = s_a;
+  g.s_b = s_w;
+  return from_cuda(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,
+                             p4q_stream_t stream) {
+  p4q_status st = check_gemm(Xq, M, Kin, Wq, N, acc);
+  if (st != P4Q_OK || M == 0) return st;
+  if ((st = check_device()) != P4Q_OK) return st;
+  GemmArgs g;
+  g.A = Xq;
+  g.B = Wq;
+  g.M = M;
+  g.N = N;
+  g.K = Kin;
+  g.out = GemmOut::kS32;
+  g.D = acc;
+  return from_cuda(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_params* params) {
+  if (!params || B < 1 || N < 1 || d < 1 || J < 0 || N > P4Q_MAX_TOKENS || J > P4Q_MAX_CONCEPTS ||
+      d % 128 != 0 || d > P4Q_MAX_ROW || params->K < 1 || params->K > N)
+    return 0;
+  return select_workspace_layout(B, N, d, J, nullptr, nullptr);
+}
+
+p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
+                      const p4q_select_params* params, int32_t* idx, void* ws, size_t ws_bytes,
+                      p4q_stream_t stream) {
+  p4q_status st = check_select_args(V, B, N, d, J, params, idx);
+  if (st != P4Q_OK) return st;
+  if ((st = check_device()) != P4Q_OK) return st;
+  return run_select(V, B, N, d, Q, J, A_cls, params, idx, ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
+                                   const float* A_cls, const uint16_t* text, int T,
+                                   const p4q_select_params* params, int32_t* idx, uint16_t* X, uint8_t* Xq,
+                                   float* s_a, void* ws, size_t ws_bytes, p4q_stream_t stream) {
+  p4q_status st = check_select_args(V, B, N, d, J, params, idx);
+  if (st != P4Q_OK) return st;
+  if (T < 0 || (T > 0 && !text) || !X || !Xq || !s_a) return P4Q_ERR_INVALID_ARG;
+  if ((T > 0 && !aligned16(text)) || !aligned16(X) || !aligned16(Xq) || !aligned16(s_a)) return P4Q_ERR_MISALIGNED;
+  if ((st = check_device()) != P4Q_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  st = run_select(V, B, N, d, Q, J, A_cls, params, idx, ws, ws_bytes, s);
+  if (st != P4Q_OK) return st;
+  // Gather the FP16 originals of the kept tokens, then the text rows, and
+  // quantize every row of the pruned sequence.
+  RowSource src;
+  src.X = V;
+  src.idx = idx;
+  src.text = text;
+  src.N = N;
+  src.K = params->K;
+  src.T = T;
+  RowSinks o;
+  o.codes = Xq;
+  o.scale = s_a;
+  o.copy = X;
+  return from_cuda(launch_quant_rows(src, B * (params->K + T), d, o, s));
+}
+
+}  // extern "C"

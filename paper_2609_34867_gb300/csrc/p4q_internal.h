@@ -1,0 +1,77 @@
+// Host-side declarations shared by the translation units of libp4q.so.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace p4q {
+
+// ------------------------------------------------------------ quantizer
+// Row source for the per-row quantizer: either a dense [rows, L] fp16 matrix,
+// or the pruned sequence of the selector (kept visual rows, then text rows).
+struct RowSource {
+  const uint16_t* X = nullptr;     // dense source, or V [B, N, L] when idx != nullptr
+  const int32_t* idx = nullptr;    // [B, K] kept indices (gather mode)
+  const uint16_t* text = nullptr;  // [B, T, L] (gather mode)
+  int N = 0, K = 0, T = 0;         // gather mode sizes
+};
+
+// Outputs of the per-row quantizer. Optional pointers may be null.
+struct RowSinks {
+  uint8_t* codes = nullptr;   // [rows, L/2] packed INT4 (required)
+  float* scale = nullptr;     // [rows] (required)
+  int32_t* norm2 = nullptr;   // [rows] sum of squared codes
+  uint16_t* copy = nullptr;   // [rows, L] fp16 copy of the source row (gather mode)
+};
+
+cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
+                              cudaStream_t stream);
+
+// ------------------------------------------------------------ GEMM
+enum class GemmOut { kHalf = 0, kS32 = 1, kCos = 2 };
+
+struct GemmArgs {
+  const uint8_t* A = nullptr;  // [batch, M, K/2] packed INT4
+  const uint8_t* B = nullptr;  // [batch, N, K/2] packed INT4
+  int M = 0, N = 0, K = 0, batch = 1;
+  long long a_batch_stride = 0;  // rows between batches of A (0 for batch 1)
+  long long b_batch_stride = 0;
+  GemmOut out = GemmOut::kHalf;
+  void* D = nullptr;              // [batch, M, N] fp16 / int32 / fp32
+  const float* s_a = nullptr;     // kHalf: [M]
+  const float* s_b = nullptr;     // kHalf: [N]
+  const int32_t* norm_a = nullptr;  // kCos: [batch, M] squared code norms
+  const int32_t* norm_b = nullptr;  // kCos: [batch, N]
+};
+
+// Returns cudaSuccess or the launch error; sets *unsupported when the shape
+// cannot run on this kernel.
+cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream);
+
+// ------------------------------------------------------------ selector
+struct SelectPlan {
+  int B, N, d, J, K, Kq, Ks, Kd;
+};
+
+struct SelectWorkspace {
+  uint8_t* vcodes;   // [B*N, d/2]
+  float* vscale;     // [B*N]
+  int32_t* vnorm;    // [B*N]
+  uint8_t* qcodes;   // [B*J, d/2]
+  float* qscale;     // [B*J]
+  int32_t* qnorm;    // [B*J]
+  float* scores;     // [B, J, N] query cosines
+  float* gram;       // [B, N, N] cosine of every token pair
+};
+
+size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, void* base);
+
+cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls,
+                                 int32_t* idx, cudaStream_t stream);
+
+// Device error word of the GEMM (the only kernel with bounded waits).
+unsigned int gemm_read_and_clear_error();
+
+}  // namespace p4q

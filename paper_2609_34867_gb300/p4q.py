@@ -1,0 +1,216 @@
+"""Thin Python binding of libp4q.so (include/p4q.h), argument marshalling only.
+
+Each function has the name of the C entry point it calls and passes torch
+tensors as raw device pointers plus the current CUDA stream; every step of the
+work runs in the library's sm_103a kernels. A missing library raises: there is
+no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+P4Q_OK = 0
+STATUS_NAMES = {0: "P4Q_OK", 1: "P4Q_ERR_INVALID_ARG", 2: "P4Q_ERR_UNSUPPORTED_SHAPE", 3: "P4Q_ERR_MISALIGNED",
+                4: "P4Q_ERR_WORKSPACE_TOO_SMALL", 5: "P4Q_ERR_CUDA", 6: "P4Q_ERR_TIMEOUT", 7: "P4Q_ERR_NO_DEVICE"}
+
+
+class P4QError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {STATUS_NAMES.get(status, status)} ({p4q_status_string(status)})")
+
+
+class SelectParams(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libp4q.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(_build.LIB):
+            raise RuntimeError(f"{_build.LIB} is missing: run __graft_entry__.build() first")
+        L = ctypes.CDLL(_build.LIB)
+        P, I, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        st = ctypes.c_int
+        L.p4q_status_string.argtypes = [st]
+        L.p4q_status_string.restype = ctypes.c_char_p
+        L.p4q_device_status.argtypes = [P]
+        L.p4q_device_status.restype = st
+        L.p4q_quant_act.argtypes = [P, I, I, P, P, P]
+        L.p4q_quant_act.restype = st
+        L.p4q_quant_weight.argtypes = [P, I, I, P, P, P]
+        L.p4q_quant_weight.restype = st
+        L.p4q_w4a4_linear.argtypes = [P, P, I, I, P, P, I, P, P]
+        L.p4q_w4a4_linear.restype = st
+        L.p4q_w4a4_gemm_s32.argtypes = [P, I, I, P, I, P, P]
+        L.p4q_w4a4_gemm_s32.restype = st
+        L.p4q_select_workspace_bytes.argtypes = [I, I, I, I, ctypes.POINTER(SelectParams)]
+        L.p4q_select_workspace_bytes.restype = S
+        L.p4q_select.argtypes = [P, I, I, I, P, I, P, ctypes.POINTER(SelectParams), P, P, S, P]
+        L.p4q_select.restype = st
+        L.p4q_select_gather_quant.argtypes = [P, I, I, I, P, I, P, P, I, ctypes.POINTER(SelectParams), P, P, P,
+                                              P, P, S, P]
+        L.p4q_select_gather_quant.restype = st
+        _lib = L
+    return _lib
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(status: int, what: str):
+    if status != P4Q_OK:
+        raise P4QError(status, what)
+
+
+def _need(t, dtype, ndim, name):
+    if not isinstance(t, torch.Tensor) or t.dtype != dtype or t.dim() != ndim or not t.is_contiguous():
+        raise TypeError(f"{name}: expected a contiguous {dtype} tensor with {ndim} dims")
+    if not t.is_cuda:
+        raise TypeError(f"{name}: expected a CUDA tensor")
+
+
+def p4q_status_string(status: int) -> str:
+    return lib().p4q_status_string(int(status)).decode()
+
+
+def p4q_device_status(stream=None) -> int:
+    return int(lib().p4q_device_status(_stream(stream)))
+
+
+def p4q_quant_act(X, Xq, s_a, stream=None):
+    """X [M, Kin] fp16 -> Xq [M, Kin/2] uint8 (packed INT4), s_a [M] fp32."""
+    _need(X, torch.float16, 2, "X"); _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    M, K = X.shape
+    _check(lib().p4q_quant_act(_ptr(X), M, K, _ptr(Xq), _ptr(s_a), _stream(stream)), "p4q_quant_act")
+
+
+def p4q_quant_weight(W, Wq, s_w, stream=None):
+    """W [N, Kin] fp16 -> Wq [N, Kin/2] uint8, s_w [N] fp32 (one scale per output channel)."""
+    _need(W, torch.float16, 2, "W"); _need(Wq, torch.uint8, 2, "Wq"); _need(s_w, torch.float32, 1, "s_w")
+    N, K = W.shape
+    _check(lib().p4q_quant_weight(_ptr(W), N, K, _ptr(Wq), _ptr(s_w), _stream(stream)), "p4q_quant_weight")
+
+
+def p4q_w4a4_linear(Xq, s_a, Wq, s_w, Y, stream=None):
+    """Y [M, N] fp16 = dequant(Xq Wq^T) with per-token s_a and per-channel s_w."""
+    _need(Xq, torch.uint8, 2, "Xq"); _need(Wq, torch.uint8, 2, "Wq"); _need(Y, torch.float16, 2, "Y")
+    M, K = Xq.shape[0], Xq.shape[1] * 2
+    N = Wq.shape[0]
+    _check(lib().p4q_w4a4_linear(_ptr(Xq), _ptr(s_a), M, K, _ptr(Wq), _ptr(s_w), N, _ptr(Y), _stream(stream)),
+           "p4q_w4a4_linear")
+
+
+def p4q_w4a4_gemm_s32(Xq, Wq, acc, stream=None):
+    """acc [M, N] int32 = exact integer product of the packed INT4 codes."""
+    _need(Xq, torch.uint8, 2, "Xq"); _need(Wq, torch.uint8, 2, "Wq"); _need(acc, torch.int32, 2, "acc")
+    M, K = Xq.shape[0], Xq.shape[1] * 2
+    N = Wq.shape[0]
+    _check(lib().p4q_w4a4_gemm_s32(_ptr(Xq), M, K, _ptr(Wq), N, _ptr(acc), _stream(stream)), "p4q_w4a4_gemm_s32")
+
+
+def p4q_select_workspace_bytes(B: int, N: int, d: int, J: int, K: int, alpha_permille: int = 300,
+                               beta_permille: int = 200) -> int:
+    p = SelectParams(K, alpha_permille, beta_permille)
+    return int(lib().p4q_select_workspace_bytes(B, N, d, J, ctypes.byref(p)))
+
+
+def p4q_select(V, Q, A_cls, K, idx, ws, alpha_permille=300, beta_permille=200, stream=None):
+    """V [B, N, d] fp16, Q [B, J, d] fp16 or None, A_cls [B, N] fp32 or None -> idx [B, K] int32."""
+    _need(V, torch.float16, 3, "V"); _need(idx, torch.int32, 2, "idx"); _need(ws, torch.uint8, 1, "ws")
+    B, N, d = V.shape
+    J = 0 if Q is None else Q.shape[1]
+    p = SelectParams(K, alpha_permille, beta_permille)
+    _check(lib().p4q_select(_ptr(V), B, N, d, _ptr(Q), J, _ptr(A_cls), ctypes.byref(p), _ptr(idx), _ptr(ws),
+                            ws.numel(), _stream(stream)), "p4q_select")
+
+
+def p4q_select_gather_quant(V, Q, A_cls, text, K, idx, X, Xq, s_a, ws, alpha_permille=300, beta_permille=200,
+                            stream=None):
+    """Selector, gather of [kept V rows; text rows] into X [B, K+T, d] fp16, and its INT4 quantization."""
+    _need(V, torch.float16, 3, "V"); _need(idx, torch.int32, 2, "idx"); _need(ws, torch.uint8, 1, "ws")
+    _need(X, torch.float16, 3, "X"); _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    B, N, d = V.shape
+    J = 0 if Q is None else Q.shape[1]
+    T = 0 if text is None else text.shape[1]
+    p = SelectParams(K, alpha_permille, beta_permille)
+    _check(lib().p4q_select_gather_quant(_ptr(V), B, N, d, _ptr(Q), J, _ptr(A_cls), _ptr(text), T,
+                                         ctypes.byref(p), _ptr(idx), _ptr(X), _ptr(Xq), _ptr(s_a), _ptr(ws),
+                                         ws.numel(), _stream(stream)), "p4q_select_gather_quant")
+
+
+# ---------------------------------------------------------------- helpers
+def quant_act(X, stream=None):
+    """Allocating wrapper of p4q_quant_act: returns (Xq, s_a)."""
+    M, K = X.shape
+    Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=X.device)
+    s = torch.empty((M,), dtype=torch.float32, device=X.device)
+    p4q_quant_act(X, Xq, s, stream)
+    return Xq, s
+
+
+def quant_weight(W, stream=None):
+    N, K = W.shape
+    Wq = torch.empty((N, K // 2), dtype=torch.uint8, device=W.device)
+    s = torch.empty((N,), dtype=torch.float32, device=W.device)
+    p4q_quant_weight(W, Wq, s, stream)
+    return Wq, s
+
+
+def w4a4_linear(Xq, s_a, Wq, s_w, stream=None):
+    Y = torch.empty((Xq.shape[0], Wq.shape[0]), dtype=torch.float16, device=Xq.device)
+    p4q_w4a4_linear(Xq, s_a, Wq, s_w, Y, stream)
+    return Y
+
+
+def w4a4_gemm_s32(Xq, Wq, stream=None):
+    acc = torch.empty((Xq.shape[0], Wq.shape[0]), dtype=torch.int32, device=Xq.device)
+    p4q_w4a4_gemm_s32(Xq, Wq, acc, stream)
+    return acc
+
+
+def select_workspace(B, N, d, J, K, device, alpha_permille=300, beta_permille=200):
+    n = p4q_select_workspace_bytes(B, N, d, J, K, alpha_permille, beta_permille)
+    if n == 0:
+        raise P4QError(1, "p4q_select_workspace_bytes")
+    return torch.empty((n,), dtype=torch.uint8, device=device)
+
+
+def select(V, Q, A_cls, K, ws=None, alpha_permille=300, beta_permille=200, stream=None):
+    B, N, d = V.shape
+    J = 0 if Q is None else Q.shape[1]
+    if ws is None:
+        ws = select_workspace(B, N, d, J, K, V.device, alpha_permille, beta_permille)
+    idx = torch.empty((B, K), dtype=torch.int32, device=V.device)
+    p4q_select(V, Q, A_cls, K, idx, ws, alpha_permille, beta_permille, stream)
+    return idx
+
+
+def select_gather_quant(V, Q, A_cls, text, K, ws=None, alpha_permille=300, beta_permille=200, stream=None):
+    B, N, d = V.shape
+    J = 0 if Q is None else Q.shape[1]
+    T = 0 if text is None else text.shape[1]
+    if ws is None:
+        ws = select_workspace(B, N, d, J, K, V.device, alpha_permille, beta_permille)
+    idx = torch.empty((B, K), dtype=torch.int32, device=V.device)
+    X = torch.empty((B, K + T, d), dtype=torch.float16, device=V.device)
+    Xq = torch.empty((B * (K + T), d // 2), dtype=torch.uint8, device=V.device)
+    s_a = torch.empty((B * (K + T),), dtype=torch.float32, device=V.device)
+    p4q_select_gather_quant(V, Q, A_cls, text, K, idx, X, Xq, s_a, ws, alpha_permille, beta_permille, stream)
+    return idx, X, Xq, s_a

@@ -1,0 +1,88 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds, exports
+every entry point include/p4q.h declares, and validates arguments before it
+touches a device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_34867_gb300 import build as B
+
+HEADER = os.path.join(B.ROOT, "include", "p4q.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(p4q_[a-z0-9_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return ctypes.CDLL(B.LIB)
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ["p4q_select", "p4q_quant_act", "p4q_w4a4_linear", "p4q_select_gather_quant",
+                     "p4q_quant_weight", "p4q_w4a4_gemm_s32", "p4q_select_workspace_bytes",
+                     "p4q_status_string", "p4q_device_status"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    lib.p4q_status_string.restype = ctypes.c_char_p
+    lib.p4q_status_string.argtypes = [ctypes.c_int]
+    for s in range(8):
+        assert lib.p4q_status_string(s)
+    assert lib.p4q_status_string(0) == b"ok"
+
+
+def test_invalid_arguments_are_rejected_before_any_launch(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_quant_act.argtypes = [P, I, I, P, P, P]
+    assert lib.p4q_quant_act(None, -1, 128, None, None, None) == 1         # negative M
+    assert lib.p4q_quant_act(P(16), 4, 100, P(16), P(16), None) == 2      # Kin % 16
+    assert lib.p4q_quant_act(P(8), 4, 128, P(16), P(16), None) == 3       # misaligned X
+    assert lib.p4q_quant_act(None, 0, 128, None, None, None) == 0         # empty is a no-op
+    lib.p4q_w4a4_linear.argtypes = [P, P, I, I, P, P, I, P, P]
+    assert lib.p4q_w4a4_linear(P(16), P(16), 4, 100, P(16), P(16), 8, P(16), None) == 2   # Kin % 128
+    assert lib.p4q_w4a4_linear(P(16), P(16), 4, 128, P(16), P(16), 12, P(16), None) == 2  # N % 8
+    assert lib.p4q_w4a4_linear(P(16), P(16), 4, 128, None, P(16), 8, P(16), None) == 1
+
+
+class Params(ctypes.Structure):
+    _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
+
+
+def test_workspace_query_and_select_validation(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_select_workspace_bytes.argtypes = [I, I, I, I, ctypes.POINTER(Params)]
+    lib.p4q_select_workspace_bytes.restype = ctypes.c_size_t
+    p = Params(64, 300, 200)
+    n = lib.p4q_select_workspace_bytes(1, 576, 4096, 3, ctypes.byref(p))
+    assert n > 576 * 576 * 4 and n % 256 == 0
+    assert lib.p4q_select_workspace_bytes(1, 576, 4000, 3, ctypes.byref(p)) == 0   # d % 128
+    bad = Params(700, 300, 200)
+    assert lib.p4q_select_workspace_bytes(1, 576, 4096, 3, ctypes.byref(bad)) == 0  # K > N
+    lib.p4q_select.argtypes = [P, I, I, I, P, I, P, ctypes.POINTER(Params), P, P, ctypes.c_size_t, P]
+    assert lib.p4q_select(P(16), 1, 576, 4096, None, 0, None, ctypes.byref(bad), P(16), P(256), 0, None) == 1
+    over = Params(64, 800, 300)
+    assert lib.p4q_select(P(16), 1, 576, 4096, None, 0, None, ctypes.byref(over), P(16), P(256), 0, None) == 1
+
+
+def test_no_device_is_reported_not_faked(lib):
+    """Without an sm_103 device a valid call returns P4Q_ERR_NO_DEVICE instead of computing on the CPU."""
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_quant_act.argtypes = [P, I, I, P, P, P]
+    assert lib.p4q_quant_act(P(16), 4, 128, P(16), P(16), None) == 7

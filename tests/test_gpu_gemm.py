@@ -1,0 +1,68 @@
+"""GPU parity of the W4A4 integer GEMM (tcgen05, FP8 path) against the oracle:
+int32 accumulators bit-exact; fp16 dequantized outputs within 1e-3 relative
+(2e-3 absolute floor) of the oracle's fp32 dequant."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+
+def _packed(rng, rows, K):
+    return rng.integers(0, 256, size=(rows, K // 2), dtype=np.uint8)  # any byte is a valid pair of codes
+
+
+def _gemm(p4q, dev, a, w):
+    acc = p4q.w4a4_gemm_s32(torch.from_numpy(a).to(dev), torch.from_numpy(w).to(dev))
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    return acc.cpu().numpy()
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 8, 128), (128, 128, 128), (96, 4096, 4096), (200, 136, 256),
+                                   (300, 1032, 384), (129, 1024, 1024), (64, 2048, 11008)])
+def test_gemm_s32_bit_exact(p4q, dev, M, N, K):
+    rng = np.random.default_rng(M * 7 + N)
+    a, w = _packed(rng, M, K), _packed(rng, N, K)
+    got = _gemm(p4q, dev, a, w)
+    ref = oracle.gemm_s32(oracle.unpack_codes(a), oracle.unpack_codes(w))
+    bad = np.argwhere(got != ref)
+    assert bad.size == 0, f"{len(bad)} of {ref.size} differ, first {bad[:4].tolist()}"
+
+
+@pytest.mark.parametrize("K", [13824, 16384])
+def test_gemm_extreme_codes_exact(p4q, dev, K):
+    """Largest magnitudes: +7 x +7 (offset codes 15 x 15), -8 x -8, -8 x +7, and alternating signs."""
+    pat = {"p7": 0x77, "m7": 0x99, "m8": 0x88, "alt": 0x97, "zero": 0x00}
+    names = list(pat)
+    a = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 26)[:128]
+    w = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 2)[:8]
+    got = _gemm(p4q, dev, a, w)
+    ref = oracle.gemm_s32(oracle.unpack_codes(a), oracle.unpack_codes(w))
+    assert np.array_equal(got, ref)
+    assert ref.max() == 64 * K
+
+
+def test_gemm_zero_rows_is_noop(p4q, dev):
+    a = torch.empty((0, 64), dtype=torch.uint8, device=dev)
+    w = torch.zeros((8, 64), dtype=torch.uint8, device=dev)
+    acc = torch.empty((0, 8), dtype=torch.int32, device=dev)
+    p4q.p4q_w4a4_gemm_s32(a, w, acc)
+
+
+@pytest.mark.parametrize("M,N,K", [(96, 4096, 4096), (257, 1032, 512), (33, 128, 13824)])
+def test_linear_fp16_within_tolerance(p4q, dev, M, N, K):
+    rng = np.random.default_rng(K + M)
+    a, w = _packed(rng, M, K), _packed(rng, N, K)
+    sa = (rng.random(M) * 0.5 + 0.01).astype(np.float32)
+    sw = (rng.random(N) * 0.002 + 1e-4).astype(np.float32)
+    Y = p4q.w4a4_linear(torch.from_numpy(a).to(dev), torch.from_numpy(sa).to(dev),
+                        torch.from_numpy(w).to(dev), torch.from_numpy(sw).to(dev))
+    torch.cuda.synchronize()
+    y = Y.float().cpu().numpy()
+    ref = oracle.linear(oracle.unpack_codes(a), sa, oracle.unpack_codes(w), sw)
+    err = np.abs(y - ref)
+    lim = np.maximum(1e-3 * np.abs(ref), 2e-3)
+    assert np.all(err <= lim), f"max err {err.max()} at {np.unravel_index(np.argmax(err - lim), err.shape)}"

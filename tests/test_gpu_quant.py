@@ -1,0 +1,68 @@
+"""GPU parity of the per-row INT4 quantizer (App. A / App. B.3) against the
+oracle: packed codes and fp32 scale bits must be bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_34867_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(p4q, dev, x):
+    X = torch.from_numpy(x).to(dev)
+    Xq, s = p4q.quant_act(X)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    return Xq.cpu().numpy(), s.cpu().numpy()
+
+
+def _check(p4q, dev, x):
+    q, s = _run(p4q, dev, x)
+    c, sr = oracle.quantize_rows(x)
+    assert np.array_equal(s.view(np.uint32), sr.view(np.uint32)), "scale bits differ"
+    got = oracle.unpack_codes(q)
+    bad = np.argwhere(got != c)
+    assert bad.size == 0, f"{len(bad)} codes differ, first at {bad[:3].tolist()}"
+
+
+@pytest.mark.parametrize("M,K", [(1, 16), (7, 128), (33, 4096), (96, 4096), (300, 11008), (17, 13824),
+                                 (5, 16384), (257, 5120)])
+def test_quant_act_matches_oracle(p4q, dev, M, K):
+    _check(p4q, dev, wl.activations(M, K, seed=M + K))
+
+
+def test_quant_heavy_tail_and_zero_rows(p4q, dev):
+    x = wl.activations(64, 5120, seed=3, heavy_tail=True)
+    x[5] = 0
+    x[17, :] = 0
+    x[17, 4000] = -0.0
+    _check(p4q, dev, x)
+
+
+def test_quant_worked_example_ties(p4q, dev, golden_dir):
+    import os
+    rows = []
+    for line in open(os.path.join(golden_dir, "quant_worked_examples.txt")):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            xs = [float(v) for v in line.split("|")[0].split()]
+            rows.append(xs + [0.0] * (16 - len(xs)))
+    _check(p4q, dev, np.array(rows, np.float16))
+
+
+def test_quant_weight_matches_oracle(p4q, dev):
+    W = wl.weight(4096, 136, seed=5)
+    Wt = torch.from_numpy(W).to(dev)
+    Wq, s = p4q.quant_weight(Wt)
+    c, sr = oracle.quantize_rows(W)
+    assert np.array_equal(s.cpu().numpy().view(np.uint32), sr.view(np.uint32))
+    assert np.array_equal(oracle.unpack_codes(Wq.cpu().numpy()), c)
+
+
+def test_quant_empty_is_noop(p4q, dev):
+    X = torch.empty((0, 128), dtype=torch.float16, device=dev)
+    Xq = torch.empty((0, 64), dtype=torch.uint8, device=dev)
+    s = torch.empty((0,), dtype=torch.float32, device=dev)
+    p4q.p4q_quant_act(X, Xq, s)

@@ -1,0 +1,90 @@
+"""GPU parity of the quantization-aware selector (Sec. 3.2, Eq. 4) and of the
+fused gather + quantize against the oracle: kept index sets identical,
+gathered rows and their INT4 codes / scales bit-exact."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_34867_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+def _t(x, dev):
+    return None if x is None else torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+
+def _select(p4q, dev, x, K, use_q=True, use_a=True, alpha=300, beta=200):
+    Q = x.Q if use_q else None
+    A = x.A if use_a else None
+    idx = p4q.select(_t(x.V, dev), _t(Q, dev), _t(A, dev), K, alpha_permille=alpha, beta_permille=beta)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    ref = oracle.select_batch(x.V, K, Q, A, alpha, beta)
+    return idx.cpu().numpy(), ref
+
+
+@pytest.mark.parametrize("B,N,d,K,J,seed", [(2, 100, 128, 20, 3, 0), (3, 576, 256, 64, 3, 1),
+                                            (1, 30, 128, 10, 2, 2), (2, 301, 384, 77, 5, 3),
+                                            (1, 1152, 128, 200, 3, 4)])
+def test_select_matches_oracle(p4q, dev, B, N, d, K, J, seed):
+    w = wl.Workload("t", B=B, N=N, d=d, K=K, T=0, J=J, seed=seed, heavy_tail=False, linears=())
+    got, ref = _select(p4q, dev, wl.selector_inputs(w), K)
+    assert np.array_equal(got, ref)
+
+
+@pytest.mark.parametrize("use_q,use_a,alpha,beta", [(False, True, 300, 200), (True, False, 300, 200),
+                                                    (False, False, 300, 200), (True, True, 0, 0),
+                                                    (True, True, 1000, 0), (True, True, 0, 1000)])
+def test_select_signal_variants(p4q, dev, use_q, use_a, alpha, beta):
+    w = wl.Workload("t", B=2, N=200, d=256, K=40, T=0, J=3, seed=9, heavy_tail=True, linears=())
+    got, ref = _select(p4q, dev, wl.selector_inputs(w), 40, use_q, use_a, alpha, beta)
+    assert np.array_equal(got, ref)
+
+
+@pytest.mark.parametrize("K", [1, 576])
+def test_select_budget_extremes(p4q, dev, K):
+    w = wl.Workload("t", B=1, N=576, d=128, K=K, T=0, J=3, seed=5, heavy_tail=False, linears=())
+    got, ref = _select(p4q, dev, wl.selector_inputs(w), K)
+    assert np.array_equal(got, ref)
+
+
+def test_select_orthogonal_ties(p4q, dev):
+    """All cosines 0: every diversity pick is a tie won by the lowest index."""
+    N, d = 130, 256
+    V = np.zeros((1, N, d), np.float16)
+    V[0, np.arange(N), np.arange(N)] = 1.0
+    idx = p4q.select(_t(V, dev), None, None, 17)
+    assert np.array_equal(idx.cpu().numpy()[0], np.arange(17))
+
+
+def test_select_one_image_576_tokens_4096d(p4q, dev):
+    """The single-image LLaVA-1.5 shape: 576 tokens x 4096, budget 64."""
+    w = wl.LLAVA15_7B_ONE
+    got, ref = _select(p4q, dev, wl.selector_inputs(w), w.K)
+    assert np.array_equal(got, ref)
+
+
+def test_select_gather_quant_matches_oracle(p4q, dev):
+    w = wl.Workload("t", B=3, N=320, d=512, K=48, T=16, J=3, seed=7, heavy_tail=False, linears=())
+    x = wl.selector_inputs(w)
+    idx, X, Xq, s_a = p4q.select_gather_quant(_t(x.V, dev), _t(x.Q, dev), _t(x.A, dev), _t(x.text, dev), w.K)
+    torch.cuda.synchronize()
+    ref_idx = oracle.select_batch(x.V, w.K, x.Q, x.A)
+    assert np.array_equal(idx.cpu().numpy(), ref_idx)
+    Xr = oracle.gather(x.V, ref_idx, x.text)
+    assert np.array_equal(X.cpu().numpy().astype(np.float32), Xr)
+    c, s = oracle.quantize_rows(Xr.reshape(-1, w.d))
+    assert np.array_equal(oracle.unpack_codes(Xq.cpu().numpy()), c)
+    assert np.array_equal(s_a.cpu().numpy().view(np.uint32), s.view(np.uint32))
+
+
+def test_select_gather_quant_without_text(p4q, dev):
+    w = wl.Workload("t", B=2, N=200, d=256, K=30, T=0, J=3, seed=8, heavy_tail=False, linears=())
+    x = wl.selector_inputs(w)
+    idx, X, Xq, s_a = p4q.select_gather_quant(_t(x.V, dev), _t(x.Q, dev), _t(x.A, dev), None, w.K)
+    torch.cuda.synchronize()
+    ref_idx = oracle.select_batch(x.V, w.K, x.Q, x.A)
+    assert np.array_equal(idx.cpu().numpy(), ref_idx)
+    assert np.array_equal(X.cpu().numpy().astype(np.float32), oracle.gather(x.V, ref_idx))
