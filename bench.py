@@ -1,0 +1,455 @@
+"""Benchmark of the P4Q pruned W4A4 hot path on GB300.
+
+One step = the whole path over one batch of the LLaVA-1.5-7B-shaped workload
+(8 images x 576 visual tokens of 4096 fp16 features + 64 text tokens each,
+budget 192 kept tokens per image):
+  p4q_select_gather_quant  fake-quant -> query / saliency / diversity stages
+                           -> gather of the kept FP16 rows + text -> INT4
+  p4q_w4a4_linear x 7      q, k, v, gate, up on the pruned sequence (M = 2048),
+                           o on the re-quantized q output, down on the
+                           re-quantized up output (2 x p4q_quant_act).
+The metric is W4A4 linear TOPS: 2 * M * N * K integer ops of the seven linears
+per step divided by the step time (the selector's time included); the
+selector's share is also reported as microseconds per image.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {p4q,reference}]
+
+--impl reference times the CPU oracle (test infrastructure) on a bounded
+sample of the same workload. Under torchrun each rank runs its own batch
+(weak scaling, no collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2609_34867_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "W4A4 prefill linear TOPS (% INT8 tensor peak); select+prune µs/image"
+WORKLOAD = wl.LLAVA15_7B
+FLUSH_BYTES = 512 << 20  # > 129 MB L2, written between timed steps
+
+# Latest ncu capture of the dominant kernel (see profiles/): DRAM bytes per
+# launch, valid while the GEMM source is unchanged since the capture.
+PROFILED_GEMM = {"source_sha1": None, "dram_bytes_per_launch": None}
+
+
+def gemm_source_sha1() -> str:
+    p = os.path.join(ROOT, "paper_2609_34867_gb300", "csrc", "p4q_gemm.cu")
+    return hashlib.sha1(open(p, "rb").read()).hexdigest()
+
+
+def linear_ops(w: wl.Workload) -> int:
+    return sum(2 * w.M * l.n_out * l.k_in for l in w.linears)
+
+
+def measured_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except (OSError, ValueError):
+        return None
+
+
+def fp8_peak_tops(sustained: bool):
+    """Dense FP8 tensor peak: the measured bf16 peak x the nominal fp8 / bf16 ratio (4.5 / 2.25)."""
+    pk = measured_peaks()
+    if pk:
+        bf = pk.get("bf16_tflops_sustained" if sustained else "bf16_tflops")
+        return 2.0 * bf, ("measured bf16 %s x 2 (nominal fp8/bf16 ratio), MEASURED_PEAKS.json"
+                          % ("sustained" if sustained else "burst"))
+    return 2.0 * (1700.0 if sustained else 1900.0), "fallback bf16 x 2"
+
+
+# --------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"p4q_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        os.remove(self.path)
+        if not rows:
+            return None
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, v in enumerate(r) if v.lower() == "active"})
+        return {"sm_mhz": float(np.median([r[0] for r in rows])), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------------- GPU arm
+class Step:
+    """Device buffers and weights of one rank, and the step itself."""
+
+    def __init__(self, w: wl.Workload, dev, seed: int):
+        import torch
+        from paper_2609_34867_gb300 import p4q
+        self.torch, self.p4q, self.w, self.dev = torch, p4q, w, dev
+        x = wl.selector_inputs(w, seed=seed)
+        self.host = {"V": x.V, "Q": x.Q, "A": x.A, "text": x.text}
+        self.V = torch.from_numpy(x.V).to(dev)
+        self.Q = torch.from_numpy(x.Q).to(dev)
+        self.A = torch.from_numpy(x.A).to(dev)
+        self.text = torch.from_numpy(x.text).to(dev)
+        B, N, d, K, T = w.B, w.N, w.d, w.K, w.T
+        self.ws = p4q.select_workspace(B, N, d, w.J, K, dev)
+        self.idx = torch.empty((B, K), dtype=torch.int32, device=dev)
+        self.X = torch.empty((B, K + T, d), dtype=torch.float16, device=dev)
+        M = w.M
+        self.Xq = torch.empty((M, d // 2), dtype=torch.uint8, device=dev)
+        self.s_a = torch.empty((M,), dtype=torch.float32, device=dev)
+        self.Wq, self.s_w, self.Y = {}, {}, {}
+        for lid, lin in enumerate(w.linears):
+            W = torch.from_numpy(wl.weight(lin.k_in, lin.n_out, wl.weight_seed(seed, lid))).to(dev)
+            self.Wq[lin.name], self.s_w[lin.name] = p4q.quant_weight(W)
+            del W
+            self.Y[lin.name] = torch.empty((M, lin.n_out), dtype=torch.float16, device=dev)
+        dims = {l.name: l for l in w.linears}
+        self.Xq_o = torch.empty((M, dims["o"].k_in // 2), dtype=torch.uint8, device=dev)
+        self.s_o = torch.empty((M,), dtype=torch.float32, device=dev)
+        self.Xq_d = torch.empty((M, dims["down"].k_in // 2), dtype=torch.uint8, device=dev)
+        self.s_d = torch.empty((M,), dtype=torch.float32, device=dev)
+        self.gemm_events = []  # (start, end, ops) of every linear launched while recording
+        self.select_events = []
+        self.record = False
+
+    def _lin(self, name, Xq, s):
+        p4q, torch = self.p4q, self.torch
+        if self.record:
+            e0 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+        p4q.p4q_w4a4_linear(Xq, s, self.Wq[name], self.s_w[name], self.Y[name])
+        if self.record:
+            e1 = torch.cuda.Event(enable_timing=True)
+            e1.record()
+            lin = next(l for l in self.w.linears if l.name == name)
+            self.gemm_events.append((e0, e1, 2 * Xq.shape[0] * lin.n_out * lin.k_in))
+
+    def __call__(self):
+        p4q, torch = self.p4q, self.torch
+        if self.record:
+            s0 = torch.cuda.Event(enable_timing=True)
+            s0.record()
+        p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
+                                    self.s_a, self.ws)
+        if self.record:
+            s1 = torch.cuda.Event(enable_timing=True)
+            s1.record()
+            self.select_events.append((s0, s1))
+        for name in ("q", "k", "v", "gate", "up"):
+            self._lin(name, self.Xq, self.s_a)
+        p4q.p4q_quant_act(self.Y["q"], self.Xq_o, self.s_o)
+        self._lin("o", self.Xq_o, self.s_o)
+        p4q.p4q_quant_act(self.Y["up"], self.Xq_d, self.s_d)
+        self._lin("down", self.Xq_d, self.s_d)
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    from paper_2609_34867_gb300 import build as _build
+    from paper_2609_34867_gb300 import p4q
+    if rank == 0 or not os.path.exists(_build.LIB):
+        _build.build()
+    if world > 1:
+        dist.barrier()
+    p4q.lib()
+    w = WORKLOAD
+    step = Step(w, dev, seed=w.seed + rank)
+    flush = torch.empty((FLUSH_BYTES,), dtype=torch.uint8, device=dev)
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    if p4q.p4q_device_status() != 0:
+        raise RuntimeError("device status not ok after warm-up")
+
+    # ---- device-timed region: K steps, L2 flushed before each, events per step
+    clocks = ClockSampler(int(os.environ.get("P4Q_NVSMI_INDEX", local_rank)))
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    step.record = True
+    launches0 = p4q.p4q_launch_count()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    t_wall = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()
+        ev[i][0].record()
+        step()
+        ev[i][1].record()
+    torch.cuda.synchronize()
+    t_wall = time.perf_counter() - t_wall
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    launches = p4q.p4q_launch_count() - launches0
+    step.record = False
+    if p4q.p4q_device_status() != 0:
+        raise RuntimeError("device status not ok after the timed region")
+    step_ms = [a.elapsed_time(b) for a, b in ev]
+    total_ms = float(np.sum(step_ms))
+    gemm_ms = np.array([a.elapsed_time(b) for a, b, _ in step.gemm_events])
+    gemm_ops = np.array([o for _, _, o in step.gemm_events], dtype=np.float64)
+    sel_ms = np.array([a.elapsed_time(b) for a, b in step.select_events])
+
+    # ---- end to end through the C ABI with host buffers (pinned), copies timed
+    e2e_ms = None
+    h2d = d2h = 0
+    if args.e2e_steps > 0:
+        hostV = torch.from_numpy(step.host["V"]).pin_memory()
+        hostQ = torch.from_numpy(step.host["Q"]).pin_memory()
+        hostA = torch.from_numpy(step.host["A"]).pin_memory()
+        hostT = torch.from_numpy(step.host["text"]).pin_memory()
+        outY = torch.empty(step.Y["down"].shape, dtype=torch.float16).pin_memory()
+        outI = torch.empty(step.idx.shape, dtype=torch.int32).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in (hostV, hostQ, hostA, hostT))
+        d2h = outY.numel() * 2 + outI.numel() * 4
+        times = []
+        for i in range(args.e2e_steps + 2):
+            flush.zero_()
+            torch.cuda.synchronize()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record()
+            step.V.copy_(hostV, non_blocking=True)
+            step.Q.copy_(hostQ, non_blocking=True)
+            step.A.copy_(hostA, non_blocking=True)
+            step.text.copy_(hostT, non_blocking=True)
+            step()
+            outY.copy_(step.Y["down"], non_blocking=True)
+            outI.copy_(step.idx, non_blocking=True)
+            b.record()
+            torch.cuda.synchronize()
+            if i >= 2:
+                times.append(a.elapsed_time(b))
+        e2e_ms = float(np.mean(times))
+
+    # ---- reduce over ranks (max time)
+    stats = torch.tensor([total_ms, e2e_ms or 0.0], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(stats, op=dist.ReduceOp.MAX)
+    total_ms, e2e_max = float(stats[0]), float(stats[1])
+    if rank != 0:
+        return None
+
+    ops = linear_ops(w)
+    ms_per_step = total_ms / args.steps
+    value = ops * world / (ms_per_step * 1e-3) / 1e12
+    sustained = t_wall > 1.0
+    peak, peak_src = fp8_peak_tops(sustained)
+    ach = float(gemm_ops.sum() / (gemm_ms.sum() * 1e-3) / 1e12)
+    n_gemm = len(gemm_ms)
+    traffic = None
+    if PROFILED_GEMM["source_sha1"] == gemm_source_sha1():
+        traffic = PROFILED_GEMM["dram_bytes_per_launch"]
+    rec = {
+        "metric": METRIC,
+        "value": round(value, 3),
+        "unit": "TOPS",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int4",
+        "data": "synthetic",
+        "config": {
+            "workload": w.name, "B": w.B, "N": w.N, "d": w.d, "K": w.K, "T": w.T, "J": w.J, "M": w.M,
+            "linears": "q,k,v,o 4096x4096; gate,up 4096->11008; down 11008->4096",
+            "alpha_beta_gamma": "0.3/0.2/0.5", "l2": "flushed (512 MiB write) before every timed step",
+            "parallelism": f"dp{world} (independent batches)"},
+        "select_prune_us_per_image": round(float(sel_ms.mean()) * 1e3 / w.B, 3),
+        "gemm_tops": round(ach, 3),
+        "pct_int8_tensor_peak": None,
+        "pct_fp8_tensor_peak": round(100.0 * ach / peak, 2),
+        "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_kernel (tcgen05 kind::f8f6f4)",
+                     "achieved": round(ach, 3), "peak": round(peak, 1), "unit": "TFLOP/s",
+                     "frac": round(ach / peak, 4), "traffic": traffic, "peak_source": peak_src,
+                     "launches_timed": n_gemm,
+                     "note": "integer ops on the FP8 tensor pipe; sm_103a has no integer tcgen05 MMA kind"},
+        "gpu_launches": int(launches),
+        "clocks": clk,
+    }
+    if e2e_ms is not None:
+        rec["e2e"] = {"value": round(ops * world / (e2e_max * 1e-3) / 1e12, 3), "unit": "TOPS",
+                      "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+                      "ms_per_step": round(e2e_max, 4), "steps": args.e2e_steps}
+    if not args.no_cpu_baseline and world == 1:
+        rec["cpu_baseline"] = cpu_baseline(w, args.cpu_threads)
+    return rec
+
+
+# --------------------------------------------------------------------- CPU oracle
+class OracleSampler:
+    """Times the CPU oracle on bounded pieces of one step and scales them up.
+
+    Pieces: the selector + gather + quantize of one image (x B images), and each
+    of the seven linears on `rows` rows of the pruned sequence (x M / rows),
+    with the o and down inputs re-quantized from the q and up outputs as in the
+    step. Weight quantization is offline and not timed."""
+
+    def __init__(self, w: wl.Workload, threads: int, rows: int = 4):
+        import oracle
+        self.o, self.w, self.rows = oracle, w, rows
+        self.cores = oracle.set_threads(threads)
+        self.x = wl.selector_inputs(w)
+        idx = oracle.select_batch(self.x.V[:1], w.K, self.x.Q[:1], self.x.A[:1])
+        X = oracle.gather(self.x.V[:1], idx, self.x.text[:1]).reshape(-1, w.d)[:rows]
+        self.ca, self.sa = oracle.quantize_rows(X)
+        self.cw = {}
+        for lid, lin in enumerate(w.linears):
+            self.cw[lin.name] = oracle.quantize_rows(wl.weight(lin.k_in, lin.n_out, wl.weight_seed(w.seed, lid)))
+        self.y = {n: oracle.linear(self.ca, self.sa, *self.cw[n]) for n in ("q", "up")}
+        self.pieces = [("select", None)] + [("linear", l.name) for l in w.linears]
+        self.times = {i: [] for i in range(len(self.pieces))}
+        self.image = 0
+
+    def run_piece(self, i: int) -> float:
+        o, w = self.o, self.w
+        kind, name = self.pieces[i % len(self.pieces)]
+        t0 = time.perf_counter()
+        if kind == "select":
+            b = self.image % w.B
+            self.image += 1
+            idx = o.select_batch(self.x.V[b:b + 1], w.K, self.x.Q[b:b + 1], self.x.A[b:b + 1])
+            o.quantize_rows(o.gather(self.x.V[b:b + 1], idx, self.x.text[b:b + 1]).reshape(-1, w.d))
+        elif name in ("o", "down"):
+            a, s = o.quantize_rows(self.y["q" if name == "o" else "up"])
+            o.linear(a, s, *self.cw[name])
+        else:
+            o.linear(self.ca, self.sa, *self.cw[name])
+        dt = time.perf_counter() - t0
+        self.times[i % len(self.pieces)].append(dt)
+        return dt
+
+    def estimate(self) -> float:
+        """Estimated seconds of one full step from the mean time of each piece."""
+        w = self.w
+        est = 0.0
+        for i, (kind, _) in enumerate(self.pieces):
+            if not self.times[i]:
+                raise RuntimeError("piece not sampled")
+            est += float(np.mean(self.times[i])) * (w.B if kind == "select" else w.M / self.rows)
+        return est
+
+    def describe(self) -> str:
+        w = self.w
+        return (f"selector+gather+quantize on 1 of {w.B} images (x{w.B}) and each of the 7 linears on "
+                f"{self.rows} of {w.M} rows (x{w.M // self.rows}), o/down inputs re-quantized; "
+                f"weight quantization untimed")
+
+
+def cpu_baseline(w: wl.Workload, threads: int, reps: int = 2):
+    s = OracleSampler(w, threads)
+    for _ in range(reps):
+        for i in range(len(s.pieces)):
+            s.run_piece(i)
+    est = s.estimate()
+    return {"value": round(linear_ops(w) / est / 1e12, 6), "unit": "TOPS", "cores": s.cores, "kind": "oracle",
+            "sample": s.describe(), "est_step_s": round(est, 3)}
+
+
+def run_reference(args, rank):
+    """The oracle as it stands: each step runs one piece of the workload (round
+    robin over the selector and the seven linears); the reported step time is
+    the sum of the pieces' mean times scaled to the full workload."""
+    if rank != 0:
+        return None
+    w = WORKLOAD
+    s = OracleSampler(w, args.cpu_threads)
+    n = len(s.pieces)
+    for i in range(args.warmup):
+        s.run_piece(i)
+    s.times = {i: [] for i in range(n)}
+    for i in range(max(args.steps, n)):
+        s.run_piece(i)
+    est = s.estimate()
+    value = linear_ops(w) / est / 1e12
+    return {
+        "metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(est * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int4", "data": "synthetic", "impl": "reference",
+        "config": {"workload": w.name, "B": w.B, "N": w.N, "d": w.d, "K": w.K, "T": w.T, "J": w.J, "M": w.M},
+        "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": s.cores, "kind": "oracle",
+                         "sample": "each step one piece: " + s.describe()},
+        "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["p4q", "reference"], default="p4q")
+    ap.add_argument("--e2e-steps", type=int, default=50)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-threads", type=int, default=0, help="oracle threads (0 = all cores)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        rec = run_reference(args, rank)
+    else:
+        if world > 1:
+            import torch.distributed as dist
+            os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+            dist.init_process_group("nccl")
+        rec = run_gpu(args, rank, world, local_rank)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+    if rec is not None:
+        print(json.dumps(rec), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -78,6 +78,11 @@ const char* p4q_status_string(p4q_status s);
  * out since the last call, P4Q_ERR_CUDA on a CUDA error, else P4Q_OK. */
 p4q_status p4q_device_status(p4q_stream_t stream);
 
+/* Number of kernels this library has launched in the process so far (all
+ * devices, all streams). Host-side counter for launch accounting; no device
+ * work. */
+uint64_t p4q_launch_count(void);
+
 /* ---------------------------------------------------------------------- */
 /* Per-row 4-bit quantizers (App. A, App. B.3)                             */
 /* ---------------------------------------------------------------------- */

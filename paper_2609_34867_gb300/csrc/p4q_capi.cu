@@ -3,6 +3,7 @@
 // caller's stream. Nothing here allocates memory.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
 
 #include "p4q.h"
@@ -13,6 +14,14 @@ using namespace p4q;
 namespace {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+std::atomic<uint64_t> g_launches{0};
+
+// Counts one kernel launch when `e` reports success.
+cudaError_t counted(cudaError_t e) {
+  if (e == cudaSuccess) g_launches.fetch_add(1, std::memory_order_relaxed);
+  return e;
+}
 
 // The kernels are built for sm_103a only; refuse to launch on anything else.
 p4q_status check_device() {
@@ -74,7 +83,7 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   sv.codes = w.vcodes;
   sv.scale = w.vscale;
   sv.norm2 = w.vnorm;
-  cudaError_t e = launch_quant_rows(src, B * N, d, sv, stream);
+  cudaError_t e = counted(launch_quant_rows(src, B * N, d, sv, stream));
   if (e != cudaSuccess) return from_cuda(e);
   if (bud.Kq > 0) {
     RowSource sq;
@@ -83,8 +92,8 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     oq.codes = w.qcodes;
     oq.scale = w.qscale;
     oq.norm2 = w.qnorm;
-    e = launch_quant_rows(sq, B * Jeff, d, oq, stream);
-    if (e == cudaSuccess) e = launch_query_scores(plan, w, stream);
+    e = counted(launch_quant_rows(sq, B * Jeff, d, oq, stream));
+    if (e == cudaSuccess) e = counted(launch_query_scores(plan, w, stream));
     if (e != cudaSuccess) return from_cuda(e);
   }
   if (bud.Kd > 0) {
@@ -99,12 +108,13 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     g.b_batch_stride = N;
     g.out = GemmOut::kCos;
     g.D = w.gram;
+    g.d_pitch = w.gram_pitch;
     g.norm_a = w.vnorm;
     g.norm_b = w.vnorm;
-    e = launch_w4a4_gemm(g, stream);
+    e = counted(launch_w4a4_gemm(g, stream));
     if (e != cudaSuccess) return from_cuda(e);
   }
-  return from_cuda(launch_select_stages(plan, w, A_cls, idx, stream));
+  return from_cuda(counted(launch_select_stages(plan, w, A_cls, idx, stream)));
 }
 
 p4q_status check_rows(const void* X, int M, int Kin, const void* Xq, const void* s) {
@@ -140,6 +150,8 @@ const char* p4q_status_string(p4q_status s) {
   return "unknown status";
 }
 
+uint64_t p4q_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
   const unsigned int g = gemm_read_and_clear_error();
@@ -156,7 +168,7 @@ p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* 
   RowSinks o;
   o.codes = Xq;
   o.scale = s_a;
-  return from_cuda(launch_quant_rows(src, M, Kin, o, reinterpret_cast<cudaStream_t>(stream)));
+  return from_cuda(counted(launch_quant_rows(src, M, Kin, o, reinterpret_cast<cudaStream_t>(stream))));
 }
 
 p4q_status p4q_quant_weight(const uint16_t* W, int N, int Kin, uint8_t* Wq, float* s_w, p4q_stream_t stream) {
@@ -180,7 +192,7 @@ p4q_status p4q_w4a4_linear(const uint8_t* Xq, const float* s_a, int M, int Kin, 
   g.D = Y;
   g.s_a = s_a;
   g.s_b = s_w;
-  return from_cuda(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream)));
+  return from_cuda(counted(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream))));
 }
 
 p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,
@@ -196,7 +208,7 @@ p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* W
   g.K = Kin;
   g.out = GemmOut::kS32;
   g.D = acc;
-  return from_cuda(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream)));
+  return from_cuda(counted(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream))));
 }
 
 size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_params* params) {
@@ -240,7 +252,7 @@ p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const
   o.codes = Xq;
   o.scale = s_a;
   o.copy = X;
-  return from_cuda(launch_quant_rows(src, B * (params->K + T), d, o, s));
+  return from_cuda(counted(launch_quant_rows(src, B * (params->K + T), d, o, s)));
 }
 
 }  // extern "C"

@@ -14,20 +14,23 @@
 // byte u = v + 8 in [0, 15]; the E4M3 bytes 0..15 encode exactly u * 2^-9
 // (subnormals 0..7, then the first binade), so one nibble becomes one byte with
 // a mask and an xor. The tensor core sums P = sum_k u_a u_b * 2^-18 in fp32;
-// P * 2^18 < 225 * 16384 < 2^22 is an integer that fp32 holds exactly, and
+// P * 2^18 <= 225 * 16384 < 2^22 is an integer that fp32 holds exactly, and
 //   acc = P - 8 * (sum_k u_a) - 8 * (sum_k u_b) + 64 K
 // restores the signed product. The row sums of u are accumulated by the same
 // threads that unpack the nibbles.
 //
-// Pipeline of one CTA (one 128 x BN output tile):
-//   warp 0      TMA: packed tiles of A [128 x 64 B] and B [BN x 64 B] per
-//               128-deep k-block into a ring of packed stages;
-//   warps 2-9   unpack: packed stage -> E4M3 stage in the 128-byte swizzled
-//               K-major layout the tensor core reads; also the row sums;
-//   warp 1      MMA: 4 x tcgen05.mma (K = 32 each) per stage, accumulator in
-//               TMEM (128 lanes x BN fp32 columns), commit frees the stage;
-//   warps 2-5   epilogue: tcgen05.ld of the accumulator, correction, scaling,
-//               store.
+// Persistent kernel, one CTA per SM, static round-robin over output tiles
+// (m fastest, so CTAs running together share the same B tile in L2):
+//   warp 0       TMA: packed tiles of A [128 x 64 B] and B [BN x 64 B] per
+//                128-deep k-block into a ring of SP packed stages;
+//   warps 2-9    unpack: packed stage -> E4M3 stage in the 128-byte swizzled
+//                K-major layout the tensor core reads (ring of SC stages),
+//                plus the per-row sums of u for the correction;
+//   warp 1       MMA: 4 x tcgen05.mma (K = 32 each) per k-block into one of
+//                two TMEM accumulators (128 lanes x BN fp32 columns each);
+//   warps 10-13  epilogue of the previous tile, overlapped with the next
+//                tile's main loop: tcgen05.ld, correction, scaling, a 32 x 32
+//                box staged in swizzled shared memory, TMA store.
 // The nibble order inside a 16-byte packed chunk is permuted identically for
 // A and B (even k, then odd k), which leaves every dot product unchanged.
 #include <cuda.h>
@@ -48,32 +51,40 @@ constexpr int BM = 128;                      // tile rows (TMEM lanes)
 constexpr int BK = 128;                      // k-elements per stage
 constexpr int BKP = BK / 2;                  // packed bytes per row per stage
 constexpr int kConvWarps = 8;
-constexpr int kThreads = (2 + kConvWarps) * 32;
+constexpr int kEpiWarps = 4;
 constexpr int kConvThreads = kConvWarps * 32;
+constexpr int kFirstConvWarp = 2;
+constexpr int kFirstEpiWarp = kFirstConvWarp + kConvWarps;
+constexpr int kThreads = (kFirstEpiWarp + kEpiWarps) * 32;
 
-template <int BN>
+template <int BN, int MODE>
 struct Cfg {
-  static constexpr int SC = (BN == 256) ? 3 : 4;  // E4M3 stages
-  static constexpr int SP = (BN == 256) ? 3 : 4;  // packed stages
+  static constexpr int SC = (BN == 256) ? 2 : 3;  // E4M3 stages
+  static constexpr int SP = (BN == 256) ? 4 : 5;  // packed stages
   static constexpr int A_CONV = BM * BK;
   static constexpr int B_CONV = BN * BK;
   static constexpr int A_PACK = BM * BKP;
   static constexpr int B_PACK = BN * BKP;
   static constexpr int CONV_STAGE = A_CONV + B_CONV;
   static constexpr int PACK_STAGE = A_PACK + B_PACK;
+  static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
+  static constexpr int BOX_BYTES = 32 * 32 * ELEM;  // one 32 x 32 output box
   static constexpr int OFF_PACK = SC * CONV_STAGE;
-  static constexpr int OFF_BAR = OFF_PACK + SP * PACK_STAGE;
-  static constexpr int NBAR = 2 * SP + 2 * SC + 2;
-  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;      // tmem slot, abort flag
-  static constexpr int OFF_SUM = OFF_MISC + 16;
-  static constexpr int SMEM = 1024 + OFF_SUM + (BM + BN) * 4;
-  static constexpr uint32_t TMEM_COLS = BN;
+  static constexpr int OFF_STAGE = OFF_PACK + SP * PACK_STAGE;  // epilogue boxes, 2 per warp
+  static constexpr int OFF_SUMA = OFF_STAGE + kEpiWarps * 2 * BOX_BYTES;
+  static constexpr int OFF_SUMB = OFF_SUMA + 2 * BM * 4;
+  static constexpr int OFF_SCOL = OFF_SUMB + 2 * BN * 4;           // per-warp column scale / norm cache
+  static constexpr int OFF_BAR = OFF_SCOL + kEpiWarps * BN * 4;
+  static constexpr int NBAR = 2 * SP + 2 * SC + 8;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int SMEM = 1024 + OFF_MISC + 16;
+  static constexpr uint32_t TMEM_COLS = 2 * BN;
+  static_assert(SMEM <= 232448, "shared memory budget");
 };
 
 struct Params {
-  int M, N, K;
-  int out;  // GemmOut
-  void* D;
+  int M, N, K, batch;
+  int num_m, num_n, tiles;
   const float* s_a;
   const float* s_b;
   const int32_t* norm_a;
@@ -83,11 +94,10 @@ struct Params {
 __device__ __forceinline__ uint32_t nib_lo(uint32_t w) { return (w & 0x0F0F0F0Fu) ^ 0x08080808u; }
 __device__ __forceinline__ uint32_t nib_hi(uint32_t w) { return ((w >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u; }
 
-// Unpacks one 16-byte packed chunk (32 codes of one row) into 32 E4M3 bytes at
-// logical byte offset 32*c of row r of a 128-byte-swizzled K-major tile, and
+// Writes the 32 E4M3 bytes of one 16-byte packed chunk (32 codes of one row)
+// at logical byte offset 32*c of row r of a 128-byte-swizzled K-major tile and
 // returns the sum of the 32 offset codes u.
-__device__ __forceinline__ int unpack_chunk(const uint8_t* pack_row, uint8_t* conv_tile, int r, int c) {
-  const uint4 p = *reinterpret_cast<const uint4*>(pack_row + c * 16);
+__device__ __forceinline__ int convert_chunk(const uint4 p, uint8_t* conv_tile, int r, int c) {
   const uint32_t l0 = nib_lo(p.x), h0 = nib_hi(p.x), l1 = nib_lo(p.y), h1 = nib_hi(p.y);
   const uint32_t l2 = nib_lo(p.z), h2 = nib_hi(p.z), l3 = nib_lo(p.w), h3 = nib_hi(p.w);
   uint8_t* row = conv_tile + r * 128;
@@ -98,26 +108,28 @@ __device__ __forceinline__ int unpack_chunk(const uint8_t* pack_row, uint8_t* co
   return __dp4a(bytesum, 0x01010101u, 0u);
 }
 
-template <int BN>
+template <int BN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const Params p) {
-  using C = Cfg<BN>;
+                     const __grid_constant__ CUtensorMap tmD, const Params p) {
+  using C = Cfg<BN, MODE>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-  uint64_t* full_p = bars;
-  uint64_t* empty_p = bars + C::SP;
-  uint64_t* full_c = bars + 2 * C::SP;
-  uint64_t* empty_c = bars + 2 * C::SP + C::SC;
-  uint64_t* acc_full = bars + 2 * C::SP + 2 * C::SC;
+  uint64_t* full_p = bars;                        // TMA -> unpack
+  uint64_t* empty_p = full_p + C::SP;             // unpack -> TMA
+  uint64_t* full_c = empty_p + C::SP;             // unpack -> MMA
+  uint64_t* empty_c = full_c + C::SC;             // MMA -> unpack
+  uint64_t* acc_full = empty_c + C::SC;           // [2] MMA -> epilogue
+  uint64_t* acc_empty = acc_full + 2;             // [2] epilogue -> MMA
+  uint64_t* sums_full = acc_empty + 2;            // [2] unpack -> epilogue
+  uint64_t* sums_empty = sums_full + 2;           // [2] epilogue -> unpack
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
-  int* sumA = reinterpret_cast<int*>(smem + C::OFF_SUM);
-  int* sumB = sumA + BM;
+  int* sumA = reinterpret_cast<int*>(smem + C::OFF_SUMA);   // [2][BM]
+  int* sumB = reinterpret_cast<int*>(smem + C::OFF_SUMB);   // [2][BN]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN, m0 = blockIdx.y * BM, bz = blockIdx.z;
   const int KB = p.K / BK;
 
   if (threadIdx.x == 0) {
@@ -129,7 +141,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&full_c[i], kConvWarps);
       mbar_init(&empty_c[i], 1);
     }
-    mbar_init(acc_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], kEpiWarps);
+      mbar_init(&sums_full[i], kConvWarps);
+      mbar_init(&sums_empty[i], kEpiWarps);
+    }
     *abort_flag = 0;
     fence_barrier_init();
   }
@@ -141,188 +158,258 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  const int per = p.num_m * p.num_n;
 
   if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
     if (lane == 0) {
       tma_prefetch_desc(&tmA);
       tma_prefetch_desc(&tmB);
-      int issued = 0;
-      for (int kb = 0; kb < KB; ++kb) {
-        const int s = kb % C::SP;
-        const uint32_t ph = (kb / C::SP) & 1;
-        if (!mbar_wait(&empty_p[s], ph ^ 1, abort_flag, &g_gemm_err)) break;
-        uint8_t* pa = smem + C::OFF_PACK + s * C::PACK_STAGE;
-        mbar_arrive_expect_tx(&full_p[s], C::PACK_STAGE);
-        tma_load_3d(&tmA, &full_p[s], pa, kb * BKP, m0, bz);
-        tma_load_3d(&tmB, &full_p[s], pa + C::A_PACK, kb * BKP, n0, bz);
-        issued = kb + 1;
+      int g = 0, issued = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x) {
+        const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
+        const int m0 = (r - nb * p.num_m) * BM, n0 = nb * BN;
+        for (int kb = 0; kb < KB; ++kb, ++g) {
+          const int s = g % C::SP;
+          if (!mbar_wait(&empty_p[s], ((g / C::SP) & 1) ^ 1, abort_flag, &g_gemm_err)) {
+            ok = false;
+            break;
+          }
+          uint8_t* pa = smem + C::OFF_PACK + s * C::PACK_STAGE;
+          mbar_arrive_expect_tx(&full_p[s], C::PACK_STAGE);
+          tma_load_3d(&tmA, &full_p[s], pa, kb * BKP, m0, bz);
+          tma_load_3d(&tmB, &full_p[s], pa + C::A_PACK, kb * BKP, n0, bz);
+          issued = g + 1;
+        }
       }
       if (*abort_flag) {
         // Let the copies already in flight land before the CTA exits.
-        for (int kb = max(0, issued - C::SP); kb < issued; ++kb) {
-          const uint32_t a = smem_u32(&full_p[kb % C::SP]);
+        for (int q = max(0, issued - C::SP); q < issued; ++q) {
+          const uint32_t a = smem_u32(&full_p[q % C::SP]);
           const unsigned long long t0 = globaltimer();
-          while (!mbar_try_wait(a, (kb / C::SP) & 1) && globaltimer() - t0 < 100000000ull) {
+          while (!mbar_try_wait(a, (q / C::SP) & 1) && globaltimer() - t0 < 100000000ull) {
           }
         }
       }
     }
   } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
-      for (int kb = 0; kb < KB; ++kb) {
-        const int t = kb % C::SC;
-        const uint32_t ph = (kb / C::SC) & 1;
-        if (!mbar_wait(&full_c[t], ph, abort_flag, &g_gemm_err)) break;
+      int g = 0, it = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++it) {
+        const int ab = it & 1;
+        if (!mbar_wait(&acc_empty[ab], ((it >> 1) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
         tc_fence_after();
-        const uint32_t a0 = smem_u32(smem + t * C::CONV_STAGE);
-        const uint32_t b0 = a0 + C::A_CONV;
+        const uint32_t d = tmem_base + static_cast<uint32_t>(ab * BN);
+        for (int kb = 0; kb < KB; ++kb, ++g) {
+          const int s = g % C::SC;
+          if (!mbar_wait(&full_c[s], (g / C::SC) & 1, abort_flag, &g_gemm_err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(smem + s * C::CONV_STAGE);
+          const uint32_t b0 = a0 + C::A_CONV;
 #pragma unroll
-        for (int k = 0; k < BK / 32; ++k)
-          mma_f8f6f4(tmem_base, sw128_kmajor_desc(a0 + k * 32), sw128_kmajor_desc(b0 + k * 32), idesc,
-                     (kb | k) != 0 ? 1u : 0u);
-        mma_commit(&empty_c[t]);
+          for (int k = 0; k < BK / 32; ++k)
+            mma_f8f6f4(d, sw128_kmajor_desc(a0 + k * 32), sw128_kmajor_desc(b0 + k * 32), idesc,
+                       (kb | k) != 0 ? 1u : 0u);
+          mma_commit(&empty_c[s]);
+        }
+        mma_commit(&acc_full[ab]);
       }
-      mma_commit(acc_full);
+    }
+  } else if (warp < kFirstEpiWarp) {
+    // ------------------------------------------------------------ unpack warps
+    const int tc = threadIdx.x - kFirstConvWarp * 32;
+    constexpr int NA = BM * 4 / kConvThreads, NB = BN * 4 / kConvThreads;
+    int g = 0, it = 0;
+    bool ok = true;
+    for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++it) {
+      int accA[NA], accB[NB];
+#pragma unroll
+      for (int j = 0; j < NA; ++j) accA[j] = 0;
+#pragma unroll
+      for (int j = 0; j < NB; ++j) accB[j] = 0;
+      for (int kb = 0; kb < KB; ++kb, ++g) {
+        const int s = g % C::SP, c = g % C::SC;
+        if (!mbar_wait(&full_p[s], (g / C::SP) & 1, abort_flag, &g_gemm_err) ||
+            !mbar_wait(&empty_c[c], ((g / C::SC) & 1) ^ 1, abort_flag, &g_gemm_err)) {
+          ok = false;
+          break;
+        }
+        const uint8_t* pa = smem + C::OFF_PACK + s * C::PACK_STAGE;
+        const uint8_t* pb = pa + C::A_PACK;
+        uint8_t* ca = smem + c * C::CONV_STAGE;
+        uint8_t* cb = ca + C::A_CONV;
+        uint4 va[NA], vb[NB];
+#pragma unroll
+        for (int j = 0; j < NA; ++j) {
+          const int task = tc + j * kConvThreads;
+          va[j] = *reinterpret_cast<const uint4*>(pa + (task >> 2) * BKP + (task & 3) * 16);
+        }
+#pragma unroll
+        for (int j = 0; j < NB; ++j) {
+          const int task = tc + j * kConvThreads;
+          vb[j] = *reinterpret_cast<const uint4*>(pb + (task >> 2) * BKP + (task & 3) * 16);
+        }
+#pragma unroll
+        for (int j = 0; j < NA; ++j) {
+          const int task = tc + j * kConvThreads;
+          accA[j] += convert_chunk(va[j], ca, task >> 2, task & 3);
+        }
+#pragma unroll
+        for (int j = 0; j < NB; ++j) {
+          const int task = tc + j * kConvThreads;
+          accB[j] += convert_chunk(vb[j], cb, task >> 2, task & 3);
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&empty_p[s]);  // packed stage consumed
+          mbar_arrive(&full_c[c]);   // E4M3 stage ready for the tensor core
+        }
+      }
+      if (!ok) break;
+      // Row sums of u over the whole K for this tile: reduce the 4 threads sharing a row.
+      const int ab = it & 1;
+      if (!mbar_wait(&sums_empty[ab], ((it >> 1) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
+#pragma unroll
+      for (int j = 0; j < NA; ++j) {
+        int v = accA[j];
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
+        if ((tc & 3) == 0) sumA[ab * BM + ((tc + j * kConvThreads) >> 2)] = v;
+      }
+#pragma unroll
+      for (int j = 0; j < NB; ++j) {
+        int v = accB[j];
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
+        if ((tc & 3) == 0) sumB[ab * BN + ((tc + j * kConvThreads) >> 2)] = v;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sums_full[ab]);
     }
   } else {
-    // ---------------- unpack warps
-    const int tc = threadIdx.x - 64;
-    int accA[BM * 4 / kConvThreads];
-    int accB[BN * 4 / kConvThreads];
-#pragma unroll
-    for (int j = 0; j < BM * 4 / kConvThreads; ++j) accA[j] = 0;
-#pragma unroll
-    for (int j = 0; j < BN * 4 / kConvThreads; ++j) accB[j] = 0;
-    for (int kb = 0; kb < KB; ++kb) {
-      const int s = kb % C::SP, t = kb % C::SC;
-      if (!mbar_wait(&full_p[s], (kb / C::SP) & 1, abort_flag, &g_gemm_err)) break;
-      if (!mbar_wait(&empty_c[t], ((kb / C::SC) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
-      const uint8_t* pa = smem + C::OFF_PACK + s * C::PACK_STAGE;
-      const uint8_t* pb = pa + C::A_PACK;
-      uint8_t* ca = smem + t * C::CONV_STAGE;
-      uint8_t* cb = ca + C::A_CONV;
-#pragma unroll
-      for (int j = 0; j < BM * 4 / kConvThreads; ++j) {
-        const int task = tc + j * kConvThreads;
-        const int r = task >> 2, c = task & 3;
-        accA[j] += unpack_chunk(pa + r * BKP, ca, r, c);
-      }
-#pragma unroll
-      for (int j = 0; j < BN * 4 / kConvThreads; ++j) {
-        const int task = tc + j * kConvThreads;
-        const int r = task >> 2, c = task & 3;
-        accB[j] += unpack_chunk(pb + r * BKP, cb, r, c);
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&empty_p[s]);
-        mbar_arrive(&full_c[t]);
-      }
-    }
-    // row sums of u over the whole K: reduce the 4 threads sharing a row
-#pragma unroll
-    for (int j = 0; j < BM * 4 / kConvThreads; ++j) {
-      int v = accA[j];
-      v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
-      v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
-      if ((tc & 3) == 0) sumA[(tc + j * kConvThreads) >> 2] = v;
-    }
-#pragma unroll
-    for (int j = 0; j < BN * 4 / kConvThreads; ++j) {
-      int v = accB[j];
-      v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
-      v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
-      if ((tc & 3) == 0) sumB[(tc + j * kConvThreads) >> 2] = v;
-    }
-    asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");
-
-    if (warp < 6) {
-      // ---------------- epilogue: warps 2..5 cover TMEM lane quarters 2,3,0,1
-      const bool ok = mbar_wait(acc_full, 0, abort_flag, &g_gemm_err);
+    // ------------------------------------------------------------ epilogue warps
+    const int ew = warp - kFirstEpiWarp;
+    const int q = warp & 3;  // TMEM lane quarter this warp may read
+    uint8_t* boxes = smem + C::OFF_STAGE + ew * 2 * C::BOX_BYTES;
+    float* colv = reinterpret_cast<float*>(smem + C::OFF_SCOL) + ew * BN;  // s_b or norms of this tile
+    int it = 0, nbox = 0;
+    for (int t = blockIdx.x; t < p.tiles; t += gridDim.x, ++it) {
+      const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
+      const int m0 = (r - nb * p.num_m) * BM, n0 = nb * BN;
+      const int ab = it & 1;
+      const uint32_t ph = (it >> 1) & 1;
+      if (!mbar_wait(&acc_full[ab], ph, abort_flag, &g_gemm_err)) break;
+      if (!mbar_wait(&sums_full[ab], ph, abort_flag, &g_gemm_err)) break;
       tc_fence_after();
-      const int q = warp & 3;
       const int row = q * 32 + lane;
       const int m = m0 + row;
-      const int corrA = 64 * p.K - 8 * sumA[row];
+      const int corrA = 64 * p.K - 8 * sumA[ab * BM + row];
       float sa = 0.0f;
       int na = 0;
-      if (ok && m < p.M) {
-        if (p.out == static_cast<int>(GemmOut::kHalf)) sa = p.s_a[m];
-        if (p.out == static_cast<int>(GemmOut::kCos)) na = p.norm_a[static_cast<size_t>(bz) * p.M + m];
+      if (m < p.M) {
+        if (MODE == static_cast<int>(GemmOut::kHalf)) sa = p.s_a[m];
+        if (MODE == static_cast<int>(GemmOut::kCos)) na = p.norm_a[static_cast<size_t>(bz) * p.M + m];
+      }
+      if (MODE != static_cast<int>(GemmOut::kS32)) {
+        for (int i = lane; i < BN; i += 32) {
+          const int n = n0 + i;
+          float v = 0.0f;
+          if (n < p.N) {
+            if (MODE == static_cast<int>(GemmOut::kHalf)) v = p.s_b[n];
+            else v = static_cast<float>(p.norm_b[static_cast<size_t>(bz) * p.N + n]);
+          }
+          colv[i] = v;
+        }
+        __syncwarp();
       }
 #pragma unroll 1
       for (int cc = 0; cc < BN / 32; ++cc) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + cc * 32, r);
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ab * BN + cc * 32, v);
         tmem_ld_wait();
-        const int nb = n0 + cc * 32;
-        if (!ok || m >= p.M || nb >= p.N) continue;
-        int acc[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const int P = __float2int_rn(__uint_as_float(r[i]) * 262144.0f);
-          acc[i] = P + corrA - 8 * sumB[cc * 32 + i];
+        if (cc == BN / 32 - 1) {
+          // Accumulator and sums fully read: hand them back.
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) {
+            mbar_arrive(&acc_empty[ab]);
+          }
         }
-        const size_t base = (static_cast<size_t>(bz) * p.M + m) * p.N + nb;
-        if (p.out == static_cast<int>(GemmOut::kHalf)) {
-          __half* y = reinterpret_cast<__half*>(p.D) + base;
+        const int* sb = sumB + ab * BN + cc * 32;
+        uint8_t* box = boxes + (nbox & 1) * C::BOX_BYTES;
+        if (lane == 0) bulk_wait_group_read<1>();  // the box about to be written is free again
+        __syncwarp();
+        uint8_t* rowp = box + lane * (32 * C::ELEM);
+        if (MODE == static_cast<int>(GemmOut::kHalf)) {
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            if (nb + g * 8 >= p.N) break;
+          for (int g4 = 0; g4 < 4; ++g4) {
             uint32_t w[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-              const int i0 = g * 8 + 2 * e;
-              const float y0 = __fmul_rn(__fmul_rn(static_cast<float>(acc[i0]), sa), p.s_b[nb + i0]);
-              const float y1 = __fmul_rn(__fmul_rn(static_cast<float>(acc[i0 + 1]), sa), p.s_b[nb + i0 + 1]);
+              const int i0 = g4 * 8 + 2 * e;
+              const int a0 = __float2int_rn(__uint_as_float(v[i0]) * 262144.0f) + corrA - 8 * sb[i0];
+              const int a1 = __float2int_rn(__uint_as_float(v[i0 + 1]) * 262144.0f) + corrA - 8 * sb[i0 + 1];
+              const float y0 = __fmul_rn(__fmul_rn(static_cast<float>(a0), sa), colv[cc * 32 + i0]);
+              const float y1 = __fmul_rn(__fmul_rn(static_cast<float>(a1), sa), colv[cc * 32 + i0 + 1]);
               const __half2 h = __floats2half2_rn(y0, y1);
               w[e] = *reinterpret_cast<const uint32_t*>(&h);
             }
-            *reinterpret_cast<uint4*>(y + g * 8) = make_uint4(w[0], w[1], w[2], w[3]);
-          }
-        } else if (p.out == static_cast<int>(GemmOut::kS32)) {
-          int32_t* y = reinterpret_cast<int32_t*>(p.D) + base;
-#pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            if (nb + g * 4 >= p.N) break;
-            *reinterpret_cast<int4*>(y + g * 4) = make_int4(acc[g * 4], acc[g * 4 + 1], acc[g * 4 + 2], acc[g * 4 + 3]);
+            // 64-byte rows, 64-byte swizzle: chunk g4 of row lane
+            *reinterpret_cast<uint4*>(rowp + ((g4 ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
           }
         } else {
-          // Token counts need not be multiples of 4: vector stores only when
-          // every row of the output starts on a 16-byte boundary.
-          float* y = reinterpret_cast<float*>(p.D) + base;
-          const int32_t* nbv = p.norm_b + static_cast<size_t>(bz) * p.N;
-          const int ncol = min(32, p.N - nb);
-          float o[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int nn = (i < ncol) ? nbv[nb + i] : 0;
-            o[i] = (na == 0 || nn == 0)
-                       ? 0.0f
-                       : __fdiv_rn(static_cast<float>(acc[i]),
-                                   __fsqrt_rn(__fmul_rn(static_cast<float>(na), static_cast<float>(nn))));
-          }
-          if ((p.N & 3) == 0) {
+          for (int g4 = 0; g4 < 8; ++g4) {
+            uint32_t w[4];
 #pragma unroll
-            for (int g = 0; g < 8; ++g)
-              if (g * 4 < ncol) *reinterpret_cast<float4*>(y + g * 4) = make_float4(o[g * 4], o[g * 4 + 1], o[g * 4 + 2], o[g * 4 + 3]);
-          } else {
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (i < ncol) y[i] = o[i];
+            for (int e = 0; e < 4; ++e) {
+              const int i = g4 * 4 + e;
+              const int a = __float2int_rn(__uint_as_float(v[i]) * 262144.0f) + corrA - 8 * sb[i];
+              if (MODE == static_cast<int>(GemmOut::kS32)) {
+                w[e] = static_cast<uint32_t>(a);
+              } else {
+                const float nn = colv[cc * 32 + i];
+                const float cs = (na == 0 || nn == 0.0f)
+                                     ? 0.0f
+                                     : __fdiv_rn(static_cast<float>(a),
+                                                 __fsqrt_rn(__fmul_rn(static_cast<float>(na), nn)));
+                w[e] = __float_as_uint(cs);
+              }
+            }
+            // 128-byte rows, 128-byte swizzle: chunk g4 of row lane
+            *reinterpret_cast<uint4*>(rowp + ((g4 ^ (lane & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
           }
         }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(&tmD, box, n0 + cc * 32, m0 + q * 32, bz);
+          bulk_commit_group();
+        }
+        ++nbox;
       }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sums_empty[ab]);
     }
+    if (lane == 0) bulk_wait_group_all();
+    __syncwarp();
   }
 
   // Teardown: every MMA must have completed before TMEM is released.
   if (warp == 1 && lane == 0 && *abort_flag) {
-    const uint32_t a = smem_u32(acc_full);
-    const unsigned long long t0 = globaltimer();
-    while (!mbar_try_wait(a, 0) && globaltimer() - t0 < 100000000ull) {
+    for (int i = 0; i < 2; ++i) {
+      const unsigned long long t0 = globaltimer();
+      const uint32_t a = smem_u32(&acc_full[i]);
+      while (!mbar_try_wait(a, 0) && !mbar_try_wait(a, 1) && globaltimer() - t0 < 100000000ull) {
+      }
     }
   }
   tc_fence_before();
@@ -348,8 +435,8 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
 }
 
 // 3-D map over packed rows: dims (K/2 bytes, rows, batch), box (64, box_rows, 1).
-bool make_map(CUtensorMap* map, const uint8_t* base, int K, int rows, int batch, long long batch_stride_rows,
-              int box_rows) {
+bool make_operand_map(CUtensorMap* map, const uint8_t* base, int K, int rows, int batch,
+                      long long batch_stride_rows, int box_rows) {
   auto enc = get_encode_fn();
   if (!enc) return false;
   const cuuint64_t kb = static_cast<cuuint64_t>(K / 2);
@@ -358,27 +445,69 @@ bool make_map(CUtensorMap* map, const uint8_t* base, int K, int rows, int batch,
   cuuint64_t strides[2] = {kb, static_cast<cuuint64_t>(bs) * kb};
   cuuint32_t box[3] = {static_cast<cuuint32_t>(BKP), static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
-  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t*>(base), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS;
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN>
-cudaError_t launch_bn(const GemmArgs& g, cudaStream_t stream) {
-  using C = Cfg<BN>;
+// 3-D map over the output [batch][rows][cols] with row pitch `pitch` elements;
+// 32 x 32 boxes in the swizzle the epilogue writes.
+bool make_output_map(CUtensorMap* map, void* base, GemmOut out, int rows, int cols, int pitch, int batch) {
+  auto enc = get_encode_fn();
+  if (!enc) return false;
+  const int es = (out == GemmOut::kHalf) ? 2 : 4;
+  const CUtensorMapDataType dt = (out == GemmOut::kHalf)  ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                 : (out == GemmOut::kS32) ? CU_TENSOR_MAP_DATA_TYPE_INT32
+                                                          : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows), static_cast<cuuint64_t>(batch)};
+  cuuint64_t strides[2] = {static_cast<cuuint64_t>(pitch) * es, static_cast<cuuint64_t>(pitch) * es * rows};
+  cuuint32_t box[3] = {32, 32, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, dt, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             es == 2 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+template <int BN, int MODE>
+cudaError_t launch_cfg(const GemmArgs& g, cudaStream_t stream) {
+  using C = Cfg<BN, MODE>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(w4a4_gemm_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+    cudaError_t e =
+        cudaFuncSetAttribute(w4a4_gemm_kernel<BN, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, g.A, g.K, g.M, g.batch, g.a_batch_stride, BM)) return cudaErrorInvalidValue;
-  if (!make_map(&mb, g.B, g.K, g.N, g.batch, g.b_batch_stride, BN)) return cudaErrorInvalidValue;
-  Params p{g.M, g.N, g.K, static_cast<int>(g.out), g.D, g.s_a, g.s_b, g.norm_a, g.norm_b};
-  dim3 grid((g.N + BN - 1) / BN, (g.M + BM - 1) / BM, g.batch);
-  w4a4_gemm_kernel<BN><<<grid, kThreads, C::SMEM, stream>>>(ma, mb, p);
+  CUtensorMap ma, mb, md;
+  if (!make_operand_map(&ma, g.A, g.K, g.M, g.batch, g.a_batch_stride, BM)) return cudaErrorInvalidValue;
+  if (!make_operand_map(&mb, g.B, g.K, g.N, g.batch, g.b_batch_stride, BN)) return cudaErrorInvalidValue;
+  const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
+  if (!make_output_map(&md, g.D, g.out, g.M, g.N, pitch, g.batch)) return cudaErrorInvalidValue;
+  Params p;
+  p.M = g.M;
+  p.N = g.N;
+  p.K = g.K;
+  p.batch = g.batch;
+  p.num_m = (g.M + BM - 1) / BM;
+  p.num_n = (g.N + BN - 1) / BN;
+  p.tiles = p.num_m * p.num_n * g.batch;
+  p.s_a = g.s_a;
+  p.s_b = g.s_b;
+  p.norm_a = g.norm_a;
+  p.norm_b = g.norm_b;
+  const int grid = p.tiles < num_sms() ? p.tiles : num_sms();
+  w4a4_gemm_kernel<BN, MODE><<<grid, kThreads, C::SMEM, stream>>>(ma, mb, md, p);
   return cudaGetLastError();
 }
 
@@ -386,8 +515,15 @@ cudaError_t launch_bn(const GemmArgs& g, cudaStream_t stream) {
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream) {
   if (g.M <= 0 || g.N <= 0 || g.batch <= 0) return cudaSuccess;
-  if (g.N >= 1024 && g.out != GemmOut::kCos) return launch_bn<256>(g, stream);
-  return launch_bn<128>(g, stream);
+  switch (g.out) {
+    case GemmOut::kHalf:
+      return (g.N >= 1024) ? launch_cfg<256, 0>(g, stream) : launch_cfg<128, 0>(g, stream);
+    case GemmOut::kS32:
+      return launch_cfg<128, 1>(g, stream);
+    case GemmOut::kCos:
+      return launch_cfg<128, 2>(g, stream);
+  }
+  return cudaErrorInvalidValue;
 }
 
 unsigned int gemm_read_and_clear_error() {

@@ -38,7 +38,8 @@ struct GemmArgs {
   long long a_batch_stride = 0;  // rows between batches of A (0 for batch 1)
   long long b_batch_stride = 0;
   GemmOut out = GemmOut::kHalf;
-  void* D = nullptr;              // [batch, M, N] fp16 / int32 / fp32
+  void* D = nullptr;              // [batch, M, d_pitch] fp16 / int32 / fp32
+  int d_pitch = 0;                // output row pitch in elements (0 = N); pitch * size % 16 == 0
   const float* s_a = nullptr;     // kHalf: [M]
   const float* s_b = nullptr;     // kHalf: [N]
   const int32_t* norm_a = nullptr;  // kCos: [batch, M] squared code norms
@@ -62,7 +63,8 @@ struct SelectWorkspace {
   float* qscale;     // [B*J]
   int32_t* qnorm;    // [B*J]
   float* scores;     // [B, J, N] query cosines
-  float* gram;       // [B, N, N] cosine of every token pair
+  float* gram;       // [B, N, gram_pitch] cosine of every token pair
+  int gram_pitch;    // N rounded up to a multiple of 4
 };
 
 size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, void* base);

@@ -206,8 +206,8 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
 
 __global__ void __launch_bounds__(kSelThreads, 1)
     select_stages_kernel(const float* __restrict__ scores, const float* __restrict__ A_cls,
-                         const float* __restrict__ gram, int N, int J, int K, int Kq, int Ks, int Kd,
-                         int32_t* __restrict__ idx) {
+                         const float* __restrict__ gram, int gp, int N, int J, int K, int Kq, int Ks,
+                         int Kd, int32_t* __restrict__ idx) {
   extern __shared__ uint8_t smem_raw[];
   BlockScratch& s = *reinterpret_cast<BlockScratch*>(smem_raw);
   const int b = blockIdx.x;
@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   }
   // Stage 3: greedy max-min diversity.
   if (Kd > 0) {
-    const float* G = gram + static_cast<size_t>(b) * N * N;
+    const float* G = gram + static_cast<size_t>(b) * N * gp;
     // list of the kept set R0
     int cnt = 0;
 #pragma unroll
@@ -248,9 +248,9 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     float m[kPer];
 #pragma unroll
     for (int e = 0; e < kPer; ++e) m[e] = -INFINITY;
-    const bool full4 = (N % 4 == 0) && (base + kPer <= N);  // 16-byte aligned row slices
+    const bool full4 = (base + kPer <= N);  // rows start 16-byte aligned (pitch % 4 == 0)
     for (int r = 0; r < total; ++r) {
-      const float* row = G + static_cast<size_t>(s.list[r]) * N;
+      const float* row = G + static_cast<size_t>(s.list[r]) * gp;
       if (full4) {
         const float4 g = *reinterpret_cast<const float4*>(row + base);
         m[0] = fmaxf(m[0], g.x); m[1] = fmaxf(m[1], g.y); m[2] = fmaxf(m[2], g.z); m[3] = fmaxf(m[3], g.w);
@@ -287,7 +287,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       }
       const int pick = static_cast<int>(best & 0xFFFFFFFFull);
       if (pick >= base && pick < base + kPer) kept[pick - base] = true;
-      const float* row = G + static_cast<size_t>(pick) * N;
+      const float* row = G + static_cast<size_t>(pick) * gp;
       if (full4) {
         const float4 g = *reinterpret_cast<const float4*>(row + base);
         m[0] = fmaxf(m[0], g.x); m[1] = fmaxf(m[1], g.y); m[2] = fmaxf(m[2], g.z); m[3] = fmaxf(m[3], g.w);
@@ -323,7 +323,8 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
   };
   const size_t o_vc = take(BN * (d / 2)), o_vs = take(BN * 4), o_vn = take(BN * 4);
   const size_t o_qc = take(BJ * (d / 2)), o_qs = take(BJ * 4), o_qn = take(BJ * 4);
-  const size_t o_sc = take(BJ * N * 4), o_g = take(BN * N * 4);
+  const int gp = (N + 3) & ~3;
+  const size_t o_sc = take(BJ * N * 4), o_g = take(BN * gp * 4);
   if (ws && base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     ws->vcodes = p + o_vc;
@@ -334,6 +335,7 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
     ws->qnorm = reinterpret_cast<int32_t*>(p + o_qn);
     ws->scores = reinterpret_cast<float*>(p + o_sc);
     ws->gram = reinterpret_cast<float*>(p + o_g);
+    ws->gram_pitch = gp;
   }
   return off;
 }
@@ -354,8 +356,8 @@ cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws,
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  select_stages_kernel<<<p.B, kSelThreads, smem, stream>>>(ws.scores, A_cls, ws.gram, p.N, p.J, p.K, p.Kq, p.Ks,
-                                                           p.Kd, idx);
+  select_stages_kernel<<<p.B, kSelThreads, smem, stream>>>(ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J,
+                                                           p.K, p.Kq, p.Ks, p.Kd, idx);
   return cudaGetLastError();
 }
 

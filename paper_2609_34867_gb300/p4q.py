@@ -43,6 +43,8 @@ def lib() -> ctypes.CDLL:
         st = ctypes.c_int
         L.p4q_status_string.argtypes = [st]
         L.p4q_status_string.restype = ctypes.c_char_p
+        L.p4q_launch_count.argtypes = []
+        L.p4q_launch_count.restype = ctypes.c_uint64
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_quant_act.argtypes = [P, I, I, P, P, P]
@@ -88,6 +90,11 @@ def _need(t, dtype, ndim, name):
 
 def p4q_status_string(status: int) -> str:
     return lib().p4q_status_string(int(status)).decode()
+
+
+def p4q_launch_count() -> int:
+    """Kernels launched by libp4q.so in this process so far."""
+    return int(lib().p4q_launch_count())
 
 
 def p4q_device_status(stream=None) -> int:

@@ -22,7 +22,8 @@ def _gemm(p4q, dev, a, w):
 
 
 @pytest.mark.parametrize("M,N,K", [(1, 8, 128), (128, 128, 128), (96, 4096, 4096), (200, 136, 256),
-                                   (300, 1032, 384), (129, 1024, 1024), (64, 2048, 11008)])
+                                   (300, 1032, 384), (129, 1024, 1024), (64, 2048, 11008),
+                                   (1100, 2056, 256), (2048, 4096, 512)])
 def test_gemm_s32_bit_exact(p4q, dev, M, N, K):
     rng = np.random.default_rng(M * 7 + N)
     a, w = _packed(rng, M, K), _packed(rng, N, K)
@@ -52,7 +53,8 @@ def test_gemm_zero_rows_is_noop(p4q, dev):
     p4q.p4q_w4a4_gemm_s32(a, w, acc)
 
 
-@pytest.mark.parametrize("M,N,K", [(96, 4096, 4096), (257, 1032, 512), (33, 128, 13824)])
+@pytest.mark.parametrize("M,N,K", [(96, 4096, 4096), (257, 1032, 512), (33, 128, 13824), (2048, 4096, 1024),
+                                   (300, 11008, 256)])
 def test_linear_fp16_within_tolerance(p4q, dev, M, N, K):
     rng = np.random.default_rng(K + M)
     a, w = _packed(rng, M, K), _packed(rng, N, K)
