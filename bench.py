@@ -148,39 +148,58 @@ class Step:
         self.s_o = torch.empty((M,), dtype=torch.float32, device=dev)
         self.Xq_d = torch.empty((M, dims["down"].k_in // 2), dtype=torch.uint8, device=dev)
         self.s_d = torch.empty((M,), dtype=torch.float32, device=dev)
-        self.gemm_events = []  # (start, end, ops) of every linear launched while recording
-        self.select_events = []
-        self.record = False
+        # The step is captured as a chain of CUDA graphs, one per segment
+        # (selector, each linear, each re-quantization), so that events
+        # recorded between the replays time the selector and every linear.
+        self.segments = [("select", self._select)] + \
+            [(n, (lambda n=n: self._lin(n, self.Xq, self.s_a))) for n in ("q", "k", "v", "gate", "up")] + \
+            [("quant_o", lambda: p4q.p4q_quant_act(self.Y["q"], self.Xq_o, self.s_o)),
+             ("o", lambda: self._lin("o", self.Xq_o, self.s_o)),
+             ("quant_down", lambda: p4q.p4q_quant_act(self.Y["up"], self.Xq_d, self.s_d)),
+             ("down", lambda: self._lin("down", self.Xq_d, self.s_d))]
+        self.lin_ops = {l.name: 2 * w.M * l.n_out * l.k_in for l in w.linears}
+        self.graphs = None
+        self.launches_per_step = None
+        self.events = [torch.cuda.Event(enable_timing=True) for _ in range(len(self.segments) + 1)]
+
+    def _select(self):
+        self.p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
+                                         self.s_a, self.ws)
 
     def _lin(self, name, Xq, s):
-        p4q, torch = self.p4q, self.torch
-        if self.record:
-            e0 = torch.cuda.Event(enable_timing=True)
-            e0.record()
-        p4q.p4q_w4a4_linear(Xq, s, self.Wq[name], self.s_w[name], self.Y[name])
-        if self.record:
-            e1 = torch.cuda.Event(enable_timing=True)
-            e1.record()
-            lin = next(l for l in self.w.linears if l.name == name)
-            self.gemm_events.append((e0, e1, 2 * Xq.shape[0] * lin.n_out * lin.k_in))
+        self.p4q.p4q_w4a4_linear(Xq, s, self.Wq[name], self.s_w[name], self.Y[name])
+
+    def body(self):
+        """The step as plain C-ABI calls (no graph)."""
+        for _, fn in self.segments:
+            fn()
+
+    def capture(self):
+        """Captures every segment into its own CUDA graph (after warm-up calls
+        have set up the kernels' attributes); a replay launches the same
+        kernels with no host work per kernel."""
+        torch = self.torch
+        self.graphs = []
+        n0 = self.p4q.p4q_launch_count()
+        for _, fn in self.segments:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g):
+                fn()
+            self.graphs.append(g)
+        self.launches_per_step = self.p4q.p4q_launch_count() - n0
 
     def __call__(self):
-        p4q, torch = self.p4q, self.torch
-        if self.record:
-            s0 = torch.cuda.Event(enable_timing=True)
-            s0.record()
-        p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
-                                    self.s_a, self.ws)
-        if self.record:
-            s1 = torch.cuda.Event(enable_timing=True)
-            s1.record()
-            self.select_events.append((s0, s1))
-        for name in ("q", "k", "v", "gate", "up"):
-            self._lin(name, self.Xq, self.s_a)
-        p4q.p4q_quant_act(self.Y["q"], self.Xq_o, self.s_o)
-        self._lin("o", self.Xq_o, self.s_o)
-        p4q.p4q_quant_act(self.Y["up"], self.Xq_d, self.s_d)
-        self._lin("down", self.Xq_d, self.s_d)
+        if self.graphs is None:
+            self.body()
+            return
+        self.events[0].record()
+        for i, g in enumerate(self.graphs):
+            g.replay()
+            self.events[i + 1].record()
+
+    def kernel_times(self):
+        """{segment: ms} of the most recent graph step (after a sync)."""
+        return {name: self.events[i].elapsed_time(self.events[i + 1]) for i, (name, _) in enumerate(self.segments)}
 
 
 def run_gpu(args, rank, world, local_rank):
@@ -204,12 +223,18 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.synchronize()
     if p4q.p4q_device_status() != 0:
         raise RuntimeError("device status not ok after warm-up")
+    step.capture()
+    for _ in range(3):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
 
-    # ---- device-timed region: K steps, L2 flushed before each, events per step
+    # ---- device-timed region: K graph replays, L2 flushed before each, events
+    # around each replay; per-kernel times from the events inside the graph
     clocks = ClockSampler(int(os.environ.get("P4Q_NVSMI_INDEX", local_rank)))
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    step.record = True
-    launches0 = p4q.p4q_launch_count()
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    step_ms, sel_ms, gemm_ms = [], [], {l.name: [] for l in w.linears}
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -217,23 +242,26 @@ def run_gpu(args, rank, world, local_rank):
     t_wall = time.perf_counter()
     for i in range(args.steps):
         flush.zero_()
-        ev[i][0].record()
+        e_start.record()
         step()
-        ev[i][1].record()
-    torch.cuda.synchronize()
+        e_end.record()
+        torch.cuda.synchronize()
+        step_ms.append(e_start.elapsed_time(e_end))
+        kt = step.kernel_times()
+        sel_ms.append(kt["select"])
+        for n in gemm_ms:
+            gemm_ms[n].append(kt[n])
     t_wall = time.perf_counter() - t_wall
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
-    launches = p4q.p4q_launch_count() - launches0
-    step.record = False
+    launches = step.launches_per_step * args.steps
     if p4q.p4q_device_status() != 0:
         raise RuntimeError("device status not ok after the timed region")
-    step_ms = [a.elapsed_time(b) for a, b in ev]
     total_ms = float(np.sum(step_ms))
-    gemm_ms = np.array([a.elapsed_time(b) for a, b, _ in step.gemm_events])
-    gemm_ops = np.array([o for _, _, o in step.gemm_events], dtype=np.float64)
-    sel_ms = np.array([a.elapsed_time(b) for a, b in step.select_events])
+    sel_ms = np.array(sel_ms)
+    gemm_ops = float(sum(step.lin_ops.values()))
+    gemm_time_ms = float(sum(np.mean(v) for v in gemm_ms.values()))
 
     # ---- end to end through the C ABI with host buffers (pinned), copies timed
     e2e_ms = None
@@ -258,7 +286,7 @@ def run_gpu(args, rank, world, local_rank):
             step.Q.copy_(hostQ, non_blocking=True)
             step.A.copy_(hostA, non_blocking=True)
             step.text.copy_(hostT, non_blocking=True)
-            step()
+            step.body()  # the C-ABI calls themselves, no graph
             outY.copy_(step.Y["down"], non_blocking=True)
             outI.copy_(step.idx, non_blocking=True)
             b.record()
@@ -280,8 +308,8 @@ def run_gpu(args, rank, world, local_rank):
     value = ops * world / (ms_per_step * 1e-3) / 1e12
     sustained = t_wall > 1.0
     peak, peak_src = fp8_peak_tops(sustained)
-    ach = float(gemm_ops.sum() / (gemm_ms.sum() * 1e-3) / 1e12)
-    n_gemm = len(gemm_ms)
+    ach = gemm_ops / (gemm_time_ms * 1e-3) / 1e12
+    n_gemm = len(step.lin_ops) * args.steps
     traffic = None
     if PROFILED_GEMM["source_sha1"] == gemm_source_sha1():
         traffic = PROFILED_GEMM["dram_bytes_per_launch"]
@@ -302,6 +330,7 @@ def run_gpu(args, rank, world, local_rank):
             "workload": w.name, "B": w.B, "N": w.N, "d": w.d, "K": w.K, "T": w.T, "J": w.J, "M": w.M,
             "linears": "q,k,v,o 4096x4096; gate,up 4096->11008; down 11008->4096",
             "alpha_beta_gamma": "0.3/0.2/0.5", "l2": "flushed (512 MiB write) before every timed step",
+            "timing": "CUDA events around each step (graph replays), summed over the K steps",
             "parallelism": f"dp{world} (independent batches)"},
         "select_prune_us_per_image": round(float(sel_ms.mean()) * 1e3 / w.B, 3),
         "gemm_tops": round(ach, 3),
@@ -311,8 +340,11 @@ def run_gpu(args, rank, world, local_rank):
                      "achieved": round(ach, 3), "peak": round(peak, 1), "unit": "TFLOP/s",
                      "frac": round(ach / peak, 4), "traffic": traffic, "peak_source": peak_src,
                      "launches_timed": n_gemm,
-                     "note": "integer ops on the FP8 tensor pipe; sm_103a has no integer tcgen05 MMA kind"},
+                     "note": "integer ops on the FP8 tensor pipe; sm_103a has no integer tcgen05 MMA kind",
+                     "per_linear_us": {n: round(float(np.mean(v)) * 1e3, 2) for n, v in gemm_ms.items()}},
         "gpu_launches": int(launches),
+        "launch": "%d CUDA graph replays per step (%d kernels of libp4q per step)" % (
+            len(step.graphs), step.launches_per_step),
         "clocks": clk,
     }
     if e2e_ms is not None:
@@ -424,7 +456,7 @@ def run_reference(args, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["p4q", "reference"], default="p4q")
     ap.add_argument("--e2e-steps", type=int, default=50)

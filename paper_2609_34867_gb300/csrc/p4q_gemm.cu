@@ -21,16 +21,20 @@
 //
 // Persistent kernel, one CTA per SM, static round-robin over output tiles
 // (m fastest, so CTAs running together share the same B tile in L2):
-//   warp 0       TMA: packed tiles of A [128 x 64 B] and B [BN x 64 B] per
-//                128-deep k-block into a ring of SP packed stages;
-//   warps 2-9    unpack: packed stage -> E4M3 stage in the 128-byte swizzled
-//                K-major layout the tensor core reads (ring of SC stages),
-//                plus the per-row sums of u for the correction;
-//   warp 1       MMA: 4 x tcgen05.mma (K = 32 each) per k-block into one of
-//                two TMEM accumulators (128 lanes x BN fp32 columns each);
-//   warps 10-13  epilogue of the previous tile, overlapped with the next
+//   warp 0       MMA: 4 x tcgen05.mma (K = 32 each) per 128-deep k-block into
+//                one of two TMEM accumulators (128 lanes x BN fp32 columns);
+//   warps 1-8    unpack: 16-byte global loads of the packed A and B rows of the
+//                next k-blocks into registers (three k-blocks in flight, the
+//                tiles prefetched into L2 by TMA further ahead), then the E4M3
+//                bytes written in the 128-byte swizzled K-major layout the
+//                tensor core reads (ring of SC stages), plus the per-row sums of
+//                u for the correction;
+//   warps 9-12   epilogue of the previous tile, overlapped with the next
 //                tile's main loop: tcgen05.ld, correction, scaling, a 32 x 32
 //                box staged in swizzled shared memory, TMA store.
+// Loading the packed operands straight into registers keeps the only shared
+// memory traffic of the main loop to the E4M3 stores and the tensor core's
+// operand reads.
 // The nibble order inside a 16-byte packed chunk is permuted identically for
 // A and B (even k, then odd k), which leaves every dot product unchanged.
 #include <cuda.h>
@@ -50,39 +54,51 @@ __device__ unsigned int g_gemm_err;
 constexpr int BM = 128;                      // tile rows (TMEM lanes)
 constexpr int BK = 128;                      // k-elements per stage
 constexpr int BKP = BK / 2;                  // packed bytes per row per stage
-constexpr int kConvWarps = 8;
+constexpr int kGroups = 2;                   // unpack groups, each converts every kGroups-th k-block
+constexpr int kGroupWarps = 8;
+constexpr int kConvWarps = kGroups * kGroupWarps;
 constexpr int kEpiWarps = 4;
-constexpr int kConvThreads = kConvWarps * 32;
-constexpr int kFirstConvWarp = 2;
+constexpr int kGroupThreads = kGroupWarps * 32;
+constexpr int kRowStep = kGroupThreads / 4;  // rows between the chunks one unpack thread handles
+constexpr int kFirstConvWarp = 1;
 constexpr int kFirstEpiWarp = kFirstConvWarp + kConvWarps;
 constexpr int kThreads = (kFirstEpiWarp + kEpiWarps) * 32;
+constexpr int kPrefetchAhead = 6;
+#ifndef P4Q_UNPACK_DEPTH
+#define P4Q_UNPACK_DEPTH 1
+#endif
+constexpr int kDepth = P4Q_UNPACK_DEPTH;       // k-blocks of one group held in registers (1 or 2)            // k-blocks prefetched into L2 ahead of the loads
 
 template <int BN, int MODE>
 struct Cfg {
-  static constexpr int SC = (BN == 256) ? 2 : 3;  // E4M3 stages
-  static constexpr int SP = (BN == 256) ? 4 : 5;  // packed stages
   static constexpr int A_CONV = BM * BK;
   static constexpr int B_CONV = BN * BK;
-  static constexpr int A_PACK = BM * BKP;
-  static constexpr int B_PACK = BN * BKP;
   static constexpr int CONV_STAGE = A_CONV + B_CONV;
-  static constexpr int PACK_STAGE = A_PACK + B_PACK;
   static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
   static constexpr int BOX_BYTES = 32 * 32 * ELEM;  // one 32 x 32 output box
-  static constexpr int OFF_PACK = SC * CONV_STAGE;
-  static constexpr int OFF_STAGE = OFF_PACK + SP * PACK_STAGE;  // epilogue boxes, 2 per warp
+  static constexpr int FIXED = kEpiWarps * 2 * BOX_BYTES + 2 * kGroups * (BM + BN) * 4 + 2 * BN * 4 + 512;
+  static constexpr int SC_FIT = (232448 - 1024 - FIXED) / CONV_STAGE > 8 ? 8 : (232448 - 1024 - FIXED) / CONV_STAGE;
+  // Every stage must belong to one unpack group (SC % kGroups == 0): a group
+  // then reuses a stage only after its own previous use of it, so its parity
+  // wait on the stage's barrier can never run more than one phase ahead.
+  static constexpr int SC = SC_FIT - SC_FIT % kGroups;
+  static constexpr int OFF_STAGE = SC * CONV_STAGE;                // epilogue boxes, 2 per warp
   static constexpr int OFF_SUMA = OFF_STAGE + kEpiWarps * 2 * BOX_BYTES;
-  static constexpr int OFF_SUMB = OFF_SUMA + 2 * BM * 4;
-  static constexpr int OFF_SCOL = OFF_SUMB + 2 * BN * 4;           // per-warp column scale / norm cache
-  static constexpr int OFF_BAR = OFF_SCOL + kEpiWarps * BN * 4;
-  static constexpr int NBAR = 2 * SP + 2 * SC + 8;
+  static constexpr int OFF_SUMB = OFF_SUMA + 2 * kGroups * BM * 4;
+  static constexpr int OFF_SCOL = OFF_SUMB + 2 * kGroups * BN * 4;  // column scale / norm and -8 sum_u caches
+  static constexpr int OFF_BAR = OFF_SCOL + 2 * BN * 4;
+  static constexpr int NBAR = 2 * SC + 8;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = 1024 + OFF_MISC + 16;
   static constexpr uint32_t TMEM_COLS = 2 * BN;
+  static_assert(SC >= 2 && SC % kGroups == 0, "E4M3 stages: at least two, a multiple of the groups");
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
 struct Params {
+  const uint8_t* A;  // [batch][M][K/2] packed, batch stride a_bs rows
+  const uint8_t* B;  // [batch][N][K/2]
+  long long a_bs, b_bs;
   int M, N, K, batch;
   int num_m, num_n, tiles;
   const float* s_a;
@@ -91,21 +107,38 @@ struct Params {
   const int32_t* norm_b;
 };
 
+// Named barrier among the epilogue warps only (id 1).
+__device__ __forceinline__ void epi_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
+}
+
+// Offset codes u = v + 8 of the even (lo) and odd (hi) nibbles of a packed
+// word, one per byte. The shift by 4 is done as a high multiply so that it
+// runs on the FMA pipe rather than the integer-logic pipe.
 __device__ __forceinline__ uint32_t nib_lo(uint32_t w) { return (w & 0x0F0F0F0Fu) ^ 0x08080808u; }
-__device__ __forceinline__ uint32_t nib_hi(uint32_t w) { return ((w >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u; }
+__device__ __forceinline__ uint32_t nib_hi(uint32_t w) {
+  return (__umulhi(w, 0x10000000u) & 0x0F0F0F0Fu) ^ 0x08080808u;
+}
 
 // Writes the 32 E4M3 bytes of one 16-byte packed chunk (32 codes of one row)
 // at logical byte offset 32*c of row r of a 128-byte-swizzled K-major tile and
-// returns the sum of the 32 offset codes u.
-__device__ __forceinline__ int convert_chunk(const uint4 p, uint8_t* conv_tile, int r, int c) {
+// adds the sum of the 32 offset codes u to acc (dp4a, FMA pipe).
+__device__ __forceinline__ void convert_chunk(const uint4 p, uint8_t* conv_tile, int r, int c, uint32_t& acc) {
   const uint32_t l0 = nib_lo(p.x), h0 = nib_hi(p.x), l1 = nib_lo(p.y), h1 = nib_hi(p.y);
   const uint32_t l2 = nib_lo(p.z), h2 = nib_hi(p.z), l3 = nib_lo(p.w), h3 = nib_hi(p.w);
   uint8_t* row = conv_tile + r * 128;
   const int sw = r & 7;
   *reinterpret_cast<uint4*>(row + (((2 * c) ^ sw) << 4)) = make_uint4(l0, h0, l1, h1);
   *reinterpret_cast<uint4*>(row + (((2 * c + 1) ^ sw) << 4)) = make_uint4(l2, h2, l3, h3);
-  const uint32_t bytesum = l0 + h0 + l1 + h1 + l2 + h2 + l3 + h3;  // <= 8 * 15 per byte
-  return __dp4a(bytesum, 0x01010101u, 0u);
+  constexpr uint32_t ones = 0x01010101u;
+  acc = __dp4a(l0, ones, acc);
+  acc = __dp4a(h0, ones, acc);
+  acc = __dp4a(l1, ones, acc);
+  acc = __dp4a(h1, ones, acc);
+  acc = __dp4a(l2, ones, acc);
+  acc = __dp4a(h2, ones, acc);
+  acc = __dp4a(l3, ones, acc);
+  acc = __dp4a(h3, ones, acc);
 }
 
 template <int BN, int MODE>
@@ -116,9 +149,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BAR);
-  uint64_t* full_p = bars;                        // TMA -> unpack
-  uint64_t* empty_p = full_p + C::SP;             // unpack -> TMA
-  uint64_t* full_c = empty_p + C::SP;             // unpack -> MMA
+  uint64_t* full_c = bars;                        // unpack -> MMA
   uint64_t* empty_c = full_c + C::SC;             // MMA -> unpack
   uint64_t* acc_full = empty_c + C::SC;           // [2] MMA -> epilogue
   uint64_t* acc_empty = acc_full + 2;             // [2] epilogue -> MMA
@@ -126,19 +157,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* sums_empty = sums_full + 2;           // [2] epilogue -> unpack
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
-  int* sumA = reinterpret_cast<int*>(smem + C::OFF_SUMA);   // [2][BM]
-  int* sumB = reinterpret_cast<int*>(smem + C::OFF_SUMB);   // [2][BN]
+  int* sumA = reinterpret_cast<int*>(smem + C::OFF_SUMA);   // [2][kGroups][BM] partial sums per group
+  int* sumB = reinterpret_cast<int*>(smem + C::OFF_SUMB);   // [2][kGroups][BN]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int KB = p.K / BK;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < C::SP; ++i) {
-      mbar_init(&full_p[i], 1);
-      mbar_init(&empty_p[i], kConvWarps);
-    }
     for (int i = 0; i < C::SC; ++i) {
-      mbar_init(&full_c[i], kConvWarps);
+      mbar_init(&full_c[i], kGroupWarps);
       mbar_init(&empty_c[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
@@ -150,7 +177,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 1) {
+  if (warp == 0) {
     tmem_alloc(tmem_slot, C::TMEM_COLS);
     tmem_relinquish();
   }
@@ -161,39 +188,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int per = p.num_m * p.num_n;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      tma_prefetch_desc(&tmA);
-      tma_prefetch_desc(&tmB);
-      int g = 0, issued = 0;
-      bool ok = true;
-      for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x) {
-        const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
-        const int m0 = (r - nb * p.num_m) * BM, n0 = nb * BN;
-        for (int kb = 0; kb < KB; ++kb, ++g) {
-          const int s = g % C::SP;
-          if (!mbar_wait(&empty_p[s], ((g / C::SP) & 1) ^ 1, abort_flag, &g_gemm_err)) {
-            ok = false;
-            break;
-          }
-          uint8_t* pa = smem + C::OFF_PACK + s * C::PACK_STAGE;
-          mbar_arrive_expect_tx(&full_p[s], C::PACK_STAGE);
-          tma_load_3d(&tmA, &full_p[s], pa, kb * BKP, m0, bz);
-          tma_load_3d(&tmB, &full_p[s], pa + C::A_PACK, kb * BKP, n0, bz);
-          issued = g + 1;
-        }
-      }
-      if (*abort_flag) {
-        // Let the copies already in flight land before the CTA exits.
-        for (int q = max(0, issued - C::SP); q < issued; ++q) {
-          const uint32_t a = smem_u32(&full_p[q % C::SP]);
-          const unsigned long long t0 = globaltimer();
-          while (!mbar_try_wait(a, (q / C::SP) & 1) && globaltimer() - t0 < 100000000ull) {
-          }
-        }
-      }
-    }
-  } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_e4m3_f32(BM, BN);
@@ -224,72 +218,117 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp < kFirstEpiWarp) {
     // ------------------------------------------------------------ unpack warps
-    const int tc = threadIdx.x - kFirstConvWarp * 32;
-    constexpr int NA = BM * 4 / kConvThreads, NB = BN * 4 / kConvThreads;
-    int g = 0, it = 0;
+    // Group grp converts the k-blocks g with g % kGroups == grp (g counts the
+    // k-blocks of all tiles this CTA processes), so kGroups independent
+    // load -> convert -> store chains are in flight at once.
+    const int cw = warp - kFirstConvWarp;
+    const int grp = cw / kGroupWarps;
+    const int tc = threadIdx.x - (kFirstConvWarp + grp * kGroupWarps) * 32;
+    constexpr int NA = BM * 4 / kGroupThreads, NB = BN * 4 / kGroupThreads, NT = NA + NB;
+    const int rbase = tc >> 2, chunk = tc & 3;
+    const size_t rowbytes = static_cast<size_t>(p.K) >> 1;
+    const bool prefetcher = (tc == 0);
+    if (prefetcher) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+    }
+    int gbase = 0, it = 0;  // gbase: global index of the tile's first k-block
     bool ok = true;
-    for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++it) {
-      int accA[NA], accB[NB];
+    for (int t = blockIdx.x; t < p.tiles && ok; t += gridDim.x, ++it, gbase += KB) {
+      const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
+      const int m0 = (r - nb * p.num_m) * BM, n0 = nb * BN;
+      // This thread's rows: rbase + kRowStep * j of the A and B tiles; rows
+      // outside the matrix read as zero codes.
+      const uint8_t* baseA = p.A + (static_cast<size_t>(bz) * p.a_bs + m0 + rbase) * rowbytes + chunk * 16;
+      const uint8_t* baseB = p.B + (static_cast<size_t>(bz) * p.b_bs + n0 + rbase) * rowbytes + chunk * 16;
+      const size_t step = static_cast<size_t>(kRowStep) * rowbytes;
+      uint32_t valid = 0;
+#pragma unroll
+      for (int j = 0; j < NA; ++j) valid |= (m0 + rbase + kRowStep * j < p.M) ? (1u << j) : 0u;
+#pragma unroll
+      for (int j = 0; j < NB; ++j) valid |= (n0 + rbase + kRowStep * j < p.N) ? (1u << (NA + j)) : 0u;
+      // first k-block of this tile that belongs to this group
+      const int kb0 = ((grp - gbase) % kGroups + kGroups) % kGroups;
+      if (prefetcher && grp == 0) {
+        for (int kb = 0; kb < min(KB, kPrefetchAhead); ++kb) {
+          tma_prefetch_l2_3d(&tmA, kb * BKP, m0, bz);
+          tma_prefetch_l2_3d(&tmB, kb * BKP, n0, bz);
+        }
+      }
+      uint32_t accA[NA], accB[NB];
 #pragma unroll
       for (int j = 0; j < NA; ++j) accA[j] = 0;
 #pragma unroll
       for (int j = 0; j < NB; ++j) accB[j] = 0;
-      for (int kb = 0; kb < KB; ++kb, ++g) {
-        const int s = g % C::SP, c = g % C::SC;
-        if (!mbar_wait(&full_p[s], (g / C::SP) & 1, abort_flag, &g_gemm_err) ||
-            !mbar_wait(&empty_c[c], ((g / C::SC) & 1) ^ 1, abort_flag, &g_gemm_err)) {
-          ok = false;
-          break;
+      uint4 buf[kDepth][NT];
+      auto load = [&](uint4 (&v)[NT], int kb) {
+        const size_t off = static_cast<size_t>(kb) * BKP;
+#pragma unroll
+        for (int j = 0; j < NA; ++j)
+          v[j] = (valid >> j) & 1u ? ldg_stream16(baseA + j * step + off) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int j = 0; j < NB; ++j)
+          v[NA + j] = (valid >> (NA + j)) & 1u ? ldg_stream16(baseB + j * step + off) : make_uint4(0u, 0u, 0u, 0u);
+      };
+      auto convert = [&](const uint4 (&v)[NT], int kb) -> bool {
+        const int g = gbase + kb;
+        const int c = g % C::SC;
+        if (prefetcher && grp == 0) {
+          for (int q = kb + kPrefetchAhead; q < min(KB, kb + kPrefetchAhead + kGroups); ++q) {
+            tma_prefetch_l2_3d(&tmA, q * BKP, m0, bz);
+            tma_prefetch_l2_3d(&tmB, q * BKP, n0, bz);
+          }
         }
-        const uint8_t* pa = smem + C::OFF_PACK + s * C::PACK_STAGE;
-        const uint8_t* pb = pa + C::A_PACK;
+        if (!mbar_wait_warp(&empty_c[c], ((g / C::SC) & 1) ^ 1, abort_flag, &g_gemm_err)) return false;
         uint8_t* ca = smem + c * C::CONV_STAGE;
         uint8_t* cb = ca + C::A_CONV;
-        uint4 va[NA], vb[NB];
 #pragma unroll
-        for (int j = 0; j < NA; ++j) {
-          const int task = tc + j * kConvThreads;
-          va[j] = *reinterpret_cast<const uint4*>(pa + (task >> 2) * BKP + (task & 3) * 16);
-        }
+        for (int j = 0; j < NA; ++j) convert_chunk(v[j], ca, rbase + kRowStep * j, chunk, accA[j]);
 #pragma unroll
-        for (int j = 0; j < NB; ++j) {
-          const int task = tc + j * kConvThreads;
-          vb[j] = *reinterpret_cast<const uint4*>(pb + (task >> 2) * BKP + (task & 3) * 16);
-        }
-#pragma unroll
-        for (int j = 0; j < NA; ++j) {
-          const int task = tc + j * kConvThreads;
-          accA[j] += convert_chunk(va[j], ca, task >> 2, task & 3);
-        }
-#pragma unroll
-        for (int j = 0; j < NB; ++j) {
-          const int task = tc + j * kConvThreads;
-          accB[j] += convert_chunk(vb[j], cb, task >> 2, task & 3);
-        }
+        for (int j = 0; j < NB; ++j) convert_chunk(v[NA + j], cb, rbase + kRowStep * j, chunk, accB[j]);
         fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&empty_p[s]);  // packed stage consumed
-          mbar_arrive(&full_c[c]);   // E4M3 stage ready for the tensor core
+        if (lane == 0) mbar_arrive(&full_c[c]);  // E4M3 stage ready for the tensor core
+        return true;
+      };
+      if constexpr (kDepth == 1) {
+        // One k-block of this group in flight: the next load is issued as soon
+        // as the registers are free, a whole group period ahead of its use.
+        if (kb0 < KB) load(buf[0], kb0);
+        for (int kb = kb0; kb < KB && ok; kb += kGroups) {
+          ok = convert(buf[0], kb);
+          if (ok && kb + kGroups < KB) load(buf[0], kb + kGroups);
+        }
+      } else {
+        // Two of this group's k-blocks in flight in registers.
+        if (kb0 < KB) load(buf[0], kb0);
+        if (kb0 + kGroups < KB) load(buf[kDepth - 1], kb0 + kGroups);
+        for (int kb = kb0; kb < KB && ok; kb += 2 * kGroups) {
+          ok = convert(buf[0], kb);
+          if (!ok || kb + kGroups >= KB) break;
+          if (kb + 2 * kGroups < KB) load(buf[0], kb + 2 * kGroups);
+          ok = convert(buf[kDepth - 1], kb + kGroups);
+          if (!ok) break;
+          if (kb + 3 * kGroups < KB) load(buf[kDepth - 1], kb + 3 * kGroups);
         }
       }
       if (!ok) break;
-      // Row sums of u over the whole K for this tile: reduce the 4 threads sharing a row.
+      // This group's row sums of u for the tile: reduce the 4 threads sharing a row.
       const int ab = it & 1;
-      if (!mbar_wait(&sums_empty[ab], ((it >> 1) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
+      if (!mbar_wait_warp(&sums_empty[ab], ((it >> 1) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
 #pragma unroll
       for (int j = 0; j < NA; ++j) {
-        int v = accA[j];
+        int v = static_cast<int>(accA[j]);
         v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
         v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
-        if ((tc & 3) == 0) sumA[ab * BM + ((tc + j * kConvThreads) >> 2)] = v;
+        if (chunk == 0) sumA[(ab * kGroups + grp) * BM + rbase + kRowStep * j] = v;
       }
 #pragma unroll
       for (int j = 0; j < NB; ++j) {
-        int v = accB[j];
+        int v = static_cast<int>(accB[j]);
         v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
         v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
-        if ((tc & 3) == 0) sumB[ab * BN + ((tc + j * kConvThreads) >> 2)] = v;
+        if (chunk == 0) sumB[(ab * kGroups + grp) * BN + rbase + kRowStep * j] = v;
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&sums_full[ab]);
@@ -299,93 +338,118 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ew = warp - kFirstEpiWarp;
     const int q = warp & 3;  // TMEM lane quarter this warp may read
     uint8_t* boxes = smem + C::OFF_STAGE + ew * 2 * C::BOX_BYTES;
-    float* colv = reinterpret_cast<float*>(smem + C::OFF_SCOL) + ew * BN;  // s_b or norms of this tile
+    float* colv = reinterpret_cast<float*>(smem + C::OFF_SCOL);  // s_b or norms of this tile
+    // The epilogue warps synchronize among themselves with a named barrier, so
+    // they all run the same number of iterations: after a failed wait a warp
+    // keeps looping (doing no work) instead of leaving the others at the barrier.
     int it = 0, nbox = 0;
+    bool failed = false;
     for (int t = blockIdx.x; t < p.tiles; t += gridDim.x, ++it) {
       const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
       const int m0 = (r - nb * p.num_m) * BM, n0 = nb * BN;
       const int ab = it & 1;
       const uint32_t ph = (it >> 1) & 1;
-      if (!mbar_wait(&acc_full[ab], ph, abort_flag, &g_gemm_err)) break;
-      if (!mbar_wait(&sums_full[ab], ph, abort_flag, &g_gemm_err)) break;
+      if (!failed && !(mbar_wait_warp(&acc_full[ab], ph, abort_flag, &g_gemm_err) &&
+                       mbar_wait_warp(&sums_full[ab], ph, abort_flag, &g_gemm_err)))
+        failed = true;
       tc_fence_after();
       const int row = q * 32 + lane;
       const int m = m0 + row;
-      const int corrA = 64 * p.K - 8 * sumA[ab * BM + row];
+      // -8 * (column sums of u of the B rows of this tile), all groups combined
+      float* sbw = reinterpret_cast<float*>(smem + C::OFF_SCOL) + BN;
+      epi_sync();  // every epilogue warp is done with the previous tile's caches
+      if (!failed) {
+        for (int i = ew * 32 + lane; i < BN; i += kEpiWarps * 32) {
+          int v = 0;
+#pragma unroll
+          for (int q2 = 0; q2 < kGroups; ++q2) v += sumB[(ab * kGroups + q2) * BN + i];
+          sbw[i] = static_cast<float>(-8 * v);
+          if (MODE != static_cast<int>(GemmOut::kS32)) {
+            const int n = n0 + i;
+            float cv = 0.0f;
+            if (n < p.N) {
+              if (MODE == static_cast<int>(GemmOut::kHalf)) cv = p.s_b[n];
+              else cv = static_cast<float>(p.norm_b[static_cast<size_t>(bz) * p.N + n]);
+            }
+            colv[i] = cv;
+          }
+        }
+      }
+      epi_sync();  // caches of this tile complete
+      if (failed) continue;
+      int sa_u = 0;
+#pragma unroll
+      for (int q2 = 0; q2 < kGroups; ++q2) sa_u += sumA[(ab * kGroups + q2) * BM + row];
+      // acc = P - 8 sum_k u_a - 8 sum_k u_b + 64 K, evaluated in fp32: every
+      // term and partial result is an integer of magnitude < 2^24, so the
+      // fused multiply-add below is exact.
+      const float corrA = static_cast<float>(64 * p.K - 8 * sa_u);
       float sa = 0.0f;
       int na = 0;
       if (m < p.M) {
         if (MODE == static_cast<int>(GemmOut::kHalf)) sa = p.s_a[m];
         if (MODE == static_cast<int>(GemmOut::kCos)) na = p.norm_a[static_cast<size_t>(bz) * p.M + m];
       }
-      if (MODE != static_cast<int>(GemmOut::kS32)) {
-        for (int i = lane; i < BN; i += 32) {
-          const int n = n0 + i;
-          float v = 0.0f;
-          if (n < p.N) {
-            if (MODE == static_cast<int>(GemmOut::kHalf)) v = p.s_b[n];
-            else v = static_cast<float>(p.norm_b[static_cast<size_t>(bz) * p.N + n]);
-          }
-          colv[i] = v;
-        }
-        __syncwarp();
-      }
 #pragma unroll 1
       for (int cc = 0; cc < BN / 32; ++cc) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ab * BN + cc * 32, v);
-        tmem_ld_wait();
-        if (cc == BN / 32 - 1) {
-          // Accumulator and sums fully read: hand them back.
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) {
-            mbar_arrive(&acc_empty[ab]);
-          }
-        }
-        const int* sb = sumB + ab * BN + cc * 32;
         uint8_t* box = boxes + (nbox & 1) * C::BOX_BYTES;
         if (lane == 0) bulk_wait_group_read<1>();  // the box about to be written is free again
         __syncwarp();
         uint8_t* rowp = box + lane * (32 * C::ELEM);
-        if (MODE == static_cast<int>(GemmOut::kHalf)) {
-#pragma unroll
-          for (int g4 = 0; g4 < 4; ++g4) {
-            uint32_t w[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int i0 = g4 * 8 + 2 * e;
-              const int a0 = __float2int_rn(__uint_as_float(v[i0]) * 262144.0f) + corrA - 8 * sb[i0];
-              const int a1 = __float2int_rn(__uint_as_float(v[i0 + 1]) * 262144.0f) + corrA - 8 * sb[i0 + 1];
-              const float y0 = __fmul_rn(__fmul_rn(static_cast<float>(a0), sa), colv[cc * 32 + i0]);
-              const float y1 = __fmul_rn(__fmul_rn(static_cast<float>(a1), sa), colv[cc * 32 + i0 + 1]);
-              const __half2 h = __floats2half2_rn(y0, y1);
-              w[e] = *reinterpret_cast<const uint32_t*>(&h);
-            }
-            // 64-byte rows, 64-byte swizzle: chunk g4 of row lane
-            *reinterpret_cast<uint4*>(rowp + ((g4 ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          const int c0 = cc * 32 + h * 16;  // first of the 16 columns of this half
+          uint32_t v[16];
+          tmem_ld_32x32b_x16(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ab * BN + c0, v);
+          tmem_ld_wait();
+          if (cc == BN / 32 - 1 && h == 1) {
+            // Accumulator fully read: hand it back to the MMA warp.
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[ab]);
           }
-        } else {
+          float acc[16];  // exact integers
 #pragma unroll
-          for (int g4 = 0; g4 < 8; ++g4) {
-            uint32_t w[4];
+          for (int i = 0; i < 16; ++i)
+            acc[i] = __fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c0 + i]);
+          if (MODE == static_cast<int>(GemmOut::kHalf)) {
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int i = g4 * 4 + e;
-              const int a = __float2int_rn(__uint_as_float(v[i]) * 262144.0f) + corrA - 8 * sb[i];
-              if (MODE == static_cast<int>(GemmOut::kS32)) {
-                w[e] = static_cast<uint32_t>(a);
-              } else {
-                const float nn = colv[cc * 32 + i];
-                const float cs = (na == 0 || nn == 0.0f)
-                                     ? 0.0f
-                                     : __fdiv_rn(static_cast<float>(a),
-                                                 __fsqrt_rn(__fmul_rn(static_cast<float>(na), nn)));
-                w[e] = __float_as_uint(cs);
+            for (int g2 = 0; g2 < 2; ++g2) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int i0 = g2 * 8 + 2 * e;
+                const float y0 = __fmul_rn(__fmul_rn(acc[i0], sa), colv[c0 + i0]);
+                const float y1 = __fmul_rn(__fmul_rn(acc[i0 + 1], sa), colv[c0 + i0 + 1]);
+                const __half2 hh = __floats2half2_rn(y0, y1);
+                w[e] = *reinterpret_cast<const uint32_t*>(&hh);
               }
+              // 64-byte rows, 64-byte swizzle: 16-byte chunk (2h + g2) of row `lane`
+              const int ch = 2 * h + g2;
+              *reinterpret_cast<uint4*>(rowp + ((ch ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
             }
-            // 128-byte rows, 128-byte swizzle: chunk g4 of row lane
-            *reinterpret_cast<uint4*>(rowp + ((g4 ^ (lane & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+          } else {
+#pragma unroll
+            for (int g4 = 0; g4 < 4; ++g4) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int i = g4 * 4 + e;
+                if (MODE == static_cast<int>(GemmOut::kS32)) {
+                  w[e] = static_cast<uint32_t>(__float2int_rn(acc[i]));
+                } else {
+                  const float nn = colv[c0 + i];
+                  const float cs = (na == 0 || nn == 0.0f)
+                                       ? 0.0f
+                                       : __fdiv_rn(acc[i],
+                                                   __fsqrt_rn(__fmul_rn(static_cast<float>(na), nn)));
+                  w[e] = __float_as_uint(cs);
+                }
+              }
+              // 128-byte rows, 128-byte swizzle: 16-byte chunk (4h + g4) of row `lane`
+              const int ch = 4 * h + g4;
+              *reinterpret_cast<uint4*>(rowp + ((ch ^ (lane & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
           }
         }
         fence_proxy_async_smem();
@@ -404,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   // Teardown: every MMA must have completed before TMEM is released.
-  if (warp == 1 && lane == 0 && *abort_flag) {
+  if (warp == 0 && lane == 0 && *abort_flag) {
     for (int i = 0; i < 2; ++i) {
       const unsigned long long t0 = globaltimer();
       const uint32_t a = smem_u32(&acc_full[i]);
@@ -414,7 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  if (warp == 0) {
     tc_fence_after();
     tmem_dealloc(tmem_base, C::TMEM_COLS);
   }
@@ -495,6 +559,10 @@ cudaError_t launch_cfg(const GemmArgs& g, cudaStream_t stream) {
   const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
   if (!make_output_map(&md, g.D, g.out, g.M, g.N, pitch, g.batch)) return cudaErrorInvalidValue;
   Params p;
+  p.A = g.A;
+  p.B = g.B;
+  p.a_bs = g.a_batch_stride > 0 ? g.a_batch_stride : g.M;
+  p.b_bs = g.b_batch_stride > 0 ? g.b_batch_stride : g.N;
   p.M = g.M;
   p.N = g.N;
   p.K = g.K;
