@@ -22,16 +22,38 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kMaxChunks = 8;  // 8 halves per chunk: rows of up to 256 * 8 * 8 = 16384
 
-__device__ __forceinline__ uint32_t quant_pair(uint32_t h2, float s, int& n2) {
-  // h2 holds two fp16 values; returns their two 4-bit codes in bits [0,8).
-  const __half2 hv = *reinterpret_cast<const __half2*>(&h2);
-  const float x0 = __low2float(hv), x1 = __high2float(hv);
-  int c0 = __float2int_rn(__fdiv_rn(x0, s));
-  int c1 = __float2int_rn(__fdiv_rn(x1, s));
-  c0 = min(max(c0, -8), 7);
-  c1 = min(max(c1, -8), 7);
-  n2 += c0 * c0 + c1 * c1;
-  return (static_cast<uint32_t>(c0) & 0xFu) | ((static_cast<uint32_t>(c1) & 0xFu) << 4);
+// Rounded quotient code = round_half_even(fl(x / s)), computed as
+// round(x * inv) with inv = fl(1 / s): the two quotients differ by less than
+// 2^-19 for |x / s| <= 7 (three roundings of relative size 2^-24), so they
+// round to the same integer unless x * inv lies within 2^-17 of a .5
+// boundary; there the exact quotient fl(x / s) is computed and rounded.
+// |x| <= max|x| bounds the code to [-7, 7], so the clamp to [-8, 7] cannot
+// bind. Returns the code as a float and adds its square to n2.
+__device__ __forceinline__ float quant_code(float x, float s, float inv, float& n2) {
+  const float q = __fmul_rn(x, inv);
+  float c = rintf(q);
+  if (fabsf(q - c) > 0.5f - 0x1p-17f) c = rintf(__fdiv_rn(x, s));
+  n2 = __fmaf_rn(c, c, n2);
+  return c;
+}
+
+// The low 4 bits of a small integer-valued float's two's complement, via the
+// bits of c + 1.5 * 2^23 (exact for |c| < 2^22).
+__device__ __forceinline__ uint32_t nibble(float c) { return __float_as_uint(c + 12582912.0f) & 0xFu; }
+
+// Eight fp16 values (one 16-byte chunk) -> eight packed 4-bit codes.
+__device__ __forceinline__ uint32_t quant_chunk(const uint4 v, float s, float inv, float& n2) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  uint32_t packed = 0;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const __half2 hv = *reinterpret_cast<const __half2*>(&w[k]);
+    const float2 f = __half22float2(hv);
+    const uint32_t n0 = nibble(quant_code(f.x, s, inv, n2));
+    const uint32_t n1 = nibble(quant_code(f.y, s, inv, n2));
+    packed |= (n0 | (n1 << 4)) << (8 * k);
+  }
+  return packed;
 }
 
 __global__ void __launch_bounds__(kThreads) quant_rows_kernel(RowSource src, int L, RowSinks out) {
@@ -76,26 +98,21 @@ __global__ void __launch_bounds__(kThreads) quant_rows_kernel(RowSource src, int
   for (int w = 1; w < kThreads / 32; ++w) mm = max(mm, red[w]);
   const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
   const float s = __fdiv_rn(a, 7.0f);
+  const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
 
-  int n2 = 0;
+  float n2 = 0.0f;  // exact: sum of squared codes <= 49 * 16384 < 2^24
   uint32_t* q4 = reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(row) * (L >> 1));
 #pragma unroll
   for (int i = 0; i < kMaxChunks; ++i) {
     const int c = threadIdx.x + i * kThreads;
     if (c < nch) {
-      uint32_t packed = 0;
-      if (a != 0.0f) {
-        packed = quant_pair(v[i].x, s, n2) | (quant_pair(v[i].y, s, n2) << 8) |
-                 (quant_pair(v[i].z, s, n2) << 16) | (quant_pair(v[i].w, s, n2) << 24);
-      }
-      q4[c] = packed;
+      q4[c] = (a != 0.0f) ? quant_chunk(v[i], s, inv, n2) : 0u;
       if (out.copy) reinterpret_cast<uint4*>(out.copy + static_cast<size_t>(row) * L)[c] = v[i];
     }
   }
   if (out.norm2) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) n2 += __shfl_xor_sync(0xFFFFFFFFu, n2, o);
-    if (lane == 0) red_n[warp] = n2;
+    const int wn = __reduce_add_sync(0xFFFFFFFFu, static_cast<int>(n2));
+    if (lane == 0) red_n[warp] = wn;
     __syncthreads();
     if (threadIdx.x == 0) {
       int t = 0;

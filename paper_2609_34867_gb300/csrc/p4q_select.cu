@@ -8,10 +8,9 @@
 // with every operation rounded to fp32 in that order, and 0 when a norm is 0.
 //
 // Kernels:
-//   query_scores_kernel   one warp per visual token: integer dot products with
-//                         the J concept codes (dp4a on the offset codes
-//                         u = c + 8, corrected by the code sums), then the
-//                         cosine per concept.
+//   query_scores_kernel   one warp per visual token: signed integer dot
+//                         products (dp4a on sign-extended nibbles) with the J
+//                         concept codes, then the cosine per concept.
 //   select_stages_kernel  one 1024-thread CTA per image: stage 1 (per-concept
 //                         top quota), stage 2 (CLS-saliency top K_s), stage 3
 //                         (greedy max-min diversity on the cosine matrix of
@@ -27,8 +26,6 @@
 namespace p4q {
 namespace {
 
-__device__ __forceinline__ uint32_t lo_u(uint32_t w) { return (w & 0x0F0F0F0Fu) ^ 0x08080808u; }
-__device__ __forceinline__ uint32_t hi_u(uint32_t w) { return ((w >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u; }
 
 __device__ __forceinline__ float code_cosine(int dot, int na, int nb) {
   if (na == 0 || nb == 0) return 0.0f;
@@ -37,7 +34,27 @@ __device__ __forceinline__ float code_cosine(int dot, int na, int nb) {
 
 constexpr int kScoreWarps = 8;
 
-// scores[b, j, i] = cos(concept j of image b, token i of image b)
+// Four two's complement nibbles (the even or odd codes of a packed word,
+// already moved to the low nibble of each byte) sign-extended to bytes.
+__device__ __forceinline__ int sext_nibbles(uint32_t n) {
+  return static_cast<int>((n & 0x0F0F0F0Fu) | ((n & 0x08080808u) * 0x1Eu));
+}
+
+// Signed dot product of 32 packed codes (one 16-byte chunk) of two rows.
+__device__ __forceinline__ int dot32(const uint4& x, const uint4& y, int acc) {
+  acc = __dp4a(sext_nibbles(x.x), sext_nibbles(y.x), acc);
+  acc = __dp4a(sext_nibbles(x.x >> 4), sext_nibbles(y.x >> 4), acc);
+  acc = __dp4a(sext_nibbles(x.y), sext_nibbles(y.y), acc);
+  acc = __dp4a(sext_nibbles(x.y >> 4), sext_nibbles(y.y >> 4), acc);
+  acc = __dp4a(sext_nibbles(x.z), sext_nibbles(y.z), acc);
+  acc = __dp4a(sext_nibbles(x.z >> 4), sext_nibbles(y.z >> 4), acc);
+  acc = __dp4a(sext_nibbles(x.w), sext_nibbles(y.w), acc);
+  acc = __dp4a(sext_nibbles(x.w >> 4), sext_nibbles(y.w >> 4), acc);
+  return acc;
+}
+
+// scores[b, j, i] = cos(concept j of image b, token i of image b); one warp
+// per token, the token's packed codes loaded with 16-byte loads by all lanes.
 __global__ void __launch_bounds__(kScoreWarps * 32)
     query_scores_kernel(const uint8_t* __restrict__ vcodes, const int32_t* __restrict__ vnorm,
                         const uint8_t* __restrict__ qcodes, const int32_t* __restrict__ qnorm, int B, int N, int d,
@@ -46,58 +63,50 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
   const int tok = blockIdx.x * kScoreWarps + warp;
   if (tok >= B * N) return;
   const int b = tok / N, i = tok - b * N;
-  const int words = d >> 3;  // 8 codes per 32-bit word
-  const uint32_t* tv = reinterpret_cast<const uint32_t*>(vcodes + static_cast<size_t>(tok) * (d >> 1));
-  const uint32_t* tq = reinterpret_cast<const uint32_t*>(qcodes + static_cast<size_t>(b) * J * (d >> 1));
-  unsigned int P[P4Q_MAX_CONCEPTS];
-  unsigned int SQ[P4Q_MAX_CONCEPTS];
+  const int nvec = d >> 5;  // 16-byte chunks (32 codes) per row
+  const uint4* tv = reinterpret_cast<const uint4*>(vcodes + static_cast<size_t>(tok) * (d >> 1));
+  const uint4* tq = reinterpret_cast<const uint4*>(qcodes + static_cast<size_t>(b) * J * (d >> 1));
+  int acc[P4Q_MAX_CONCEPTS];
 #pragma unroll
-  for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) P[j] = SQ[j] = 0;
-  unsigned int SV = 0;
-  for (int w = lane; w < words; w += 32) {
-    const uint32_t x = __ldg(tv + w);
-    const uint32_t xl = lo_u(x), xh = hi_u(x);
-    SV = __dp4a(xl + xh, 0x01010101u, SV);
+  for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) acc[j] = 0;
+  for (int c0 = 0; c0 < nvec; c0 += 4 * 32) {
+    uint4 x[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int c = c0 + u * 32 + lane;
+      x[u] = c < nvec ? __ldg(tv + c) : make_uint4(0u, 0u, 0u, 0u);
+    }
 #pragma unroll
     for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) {
       if (j < J) {
-        const uint32_t y = __ldg(tq + static_cast<size_t>(j) * words + w);
-        const uint32_t yl = lo_u(y), yh = hi_u(y);
-        P[j] = __dp4a(xl, yl, P[j]);
-        P[j] = __dp4a(xh, yh, P[j]);
-        SQ[j] = __dp4a(yl + yh, 0x01010101u, SQ[j]);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int c = c0 + u * 32 + lane;
+          if (c < nvec) acc[j] = dot32(x[u], __ldg(tq + static_cast<size_t>(j) * nvec + c), acc[j]);
+        }
       }
     }
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) SV += __shfl_xor_sync(0xFFFFFFFFu, SV, o);
   const int nv = vnorm[tok];
 #pragma unroll
   for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) {
     if (j < J) {
-      unsigned int pj = P[j], sj = SQ[j];
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        pj += __shfl_xor_sync(0xFFFFFFFFu, pj, o);
-        sj += __shfl_xor_sync(0xFFFFFFFFu, sj, o);
-      }
-      if (lane == 0) {
-        const int dot = static_cast<int>(pj) - 8 * static_cast<int>(SV) - 8 * static_cast<int>(sj) + 64 * d;
-        scores[(static_cast<size_t>(b) * J + j) * N + i] = code_cosine(dot, qnorm[b * J + j], nv);
-      }
+      const int dot = __reduce_add_sync(0xFFFFFFFFu, acc[j]);
+      if (lane == 0) scores[(static_cast<size_t>(b) * J + j) * N + i] = code_cosine(dot, qnorm[b * J + j], nv);
     }
   }
 }
 
 constexpr int kSelThreads = 1024;
+constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kPer = 4;  // tokens per thread: token i = kPer * threadIdx.x + e
 
 struct BlockScratch {
   unsigned int hist[256];
   unsigned int wsum[32];
-  unsigned long long wmin[2][32];
+  unsigned int wkey[2][32];  // per-warp minimum keys of a greedy round (double buffered)
+  unsigned int widx[2][32];  // and the lowest token index holding that key
   int digit, above;
-  int list_len;
   int list[P4Q_MAX_TOKENS];
 };
 
@@ -130,9 +139,13 @@ __device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
 
 // Marks as kept the q free tokens with the largest keys (keys are the
 // order-preserving images of fp32 scores; ties go to the lower token index).
-__device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], int n_valid_base, int N, int q,
+// Radix select, 8 bits per pass, from the most significant byte; the
+// histogram updates are aggregated per warp over equal digits, since scores
+// of similar magnitude share their leading bytes.
+__device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], int base, int N, int q,
                                BlockScratch& s) {
   if (q <= 0) return;
+  const int lane = threadIdx.x & 31;
   uint32_t prefix = 0, mask = 0;
   int need = q;
   for (int pass = 0; pass < 4; ++pass) {
@@ -141,27 +154,27 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
     __syncthreads();
 #pragma unroll
     for (int e = 0; e < kPer; ++e) {
-      const int i = n_valid_base + e;
-      if (i < N && !kept[e] && (key[e] & mask) == prefix) atomicAdd(&s.hist[(key[e] >> shift) & 255u], 1u);
+      const bool live = (base + e < N) && !kept[e] && (key[e] & mask) == prefix;
+      const uint32_t dig = live ? ((key[e] >> shift) & 255u) : 256u;  // 256: not counted
+      const unsigned peers = __match_any_sync(0xFFFFFFFFu, dig);
+      if (live && (__ffs(peers) - 1) == lane) atomicAdd(&s.hist[dig], static_cast<unsigned>(__popc(peers)));
     }
     __syncthreads();
     if (threadIdx.x < 32) {
       // lane l owns digits [8l, 8l+8); find the digit where the count from the top reaches need
-      const int lane = threadIdx.x;
       unsigned int c[8], own = 0;
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         c[k] = s.hist[8 * lane + k];
         own += c[k];
       }
-      unsigned int above = 0;  // counts of lanes with higher digits
       unsigned int x = own;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const unsigned int y = __shfl_down_sync(0xFFFFFFFFu, x, o);
         if (lane + o < 32) x += y;
       }
-      above = x - own;  // sum over lanes > lane
+      const unsigned int above = x - own;  // sum over lanes > lane
       if (above < static_cast<unsigned>(need) && above + own >= static_cast<unsigned>(need)) {
         unsigned int acc = above;
         for (int k = 7; k >= 0; --k) {
@@ -183,16 +196,13 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
   // keys > prefix are taken; among keys == prefix the first `need` in index order
   int eq = 0;
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) {
-    const int i = n_valid_base + e;
-    if (i < N && !kept[e] && key[e] == prefix) ++eq;
-  }
+  for (int e = 0; e < kPer; ++e)
+    if (base + e < N && !kept[e] && key[e] == prefix) ++eq;
   int total;
   int rank = block_exclusive_scan(eq, &total, s);
 #pragma unroll
   for (int e = 0; e < kPer; ++e) {
-    const int i = n_valid_base + e;
-    if (i < N && !kept[e]) {
+    if (base + e < N && !kept[e]) {
       if (key[e] > prefix) {
         kept[e] = true;
       } else if (key[e] == prefix) {
@@ -212,6 +222,7 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   BlockScratch& s = *reinterpret_cast<BlockScratch*>(smem_raw);
   const int b = blockIdx.x;
   const int base = kPer * threadIdx.x;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   bool kept[kPer];
 #pragma unroll
   for (int e = 0; e < kPer; ++e) kept[e] = false;
@@ -232,10 +243,9 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(a[base + e]) : 0u;
     block_take_top(key, kept, base, N, Ks, s);
   }
-  // Stage 3: greedy max-min diversity.
+  // Stage 3: greedy max-min diversity on the cosine matrix G of the image.
   if (Kd > 0) {
     const float* G = gram + static_cast<size_t>(b) * N * gp;
-    // list of the kept set R0
     int cnt = 0;
 #pragma unroll
     for (int e = 0; e < kPer; ++e) cnt += (base + e < N && kept[e]) ? 1 : 0;
@@ -245,12 +255,13 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     for (int e = 0; e < kPer; ++e)
       if (base + e < N && kept[e]) s.list[pos++] = base + e;
     __syncthreads();
+    // m_i = max over the kept set R0 of cos(i, r); -inf when R0 is empty.
     float m[kPer];
 #pragma unroll
     for (int e = 0; e < kPer; ++e) m[e] = -INFINITY;
     const bool full4 = (base + kPer <= N);  // rows start 16-byte aligned (pitch % 4 == 0)
-    for (int r = 0; r < total; ++r) {
-      const float* row = G + static_cast<size_t>(s.list[r]) * gp;
+    auto take_row = [&](int r) {
+      const float* row = G + static_cast<size_t>(r) * gp;
       if (full4) {
         const float4 g = *reinterpret_cast<const float4*>(row + base);
         m[0] = fmaxf(m[0], g.x); m[1] = fmaxf(m[1], g.y); m[2] = fmaxf(m[2], g.z); m[3] = fmaxf(m[3], g.w);
@@ -259,43 +270,38 @@ __global__ void __launch_bounds__(kSelThreads, 1)
         for (int e = 0; e < kPer; ++e)
           if (base + e < N) m[e] = fmaxf(m[e], row[base + e]);
       }
-    }
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    };
+    for (int r = 0; r < total; ++r) take_row(s.list[r]);
+    // Greedy rounds: argmin of m over the free tokens (lower index on ties),
+    // one block barrier per round.
     for (int t = 0; t < Kd; ++t) {
-      unsigned long long best = ~0ull;
+      uint32_t bk = 0xFFFFFFFFu, bi = 0xFFFFFFFFu;
 #pragma unroll
       for (int e = 0; e < kPer; ++e) {
         if (base + e < N && !kept[e]) {
-          const unsigned long long k =
-              (static_cast<unsigned long long>(float_order_key(m[e])) << 32) | static_cast<unsigned>(base + e);
-          best = k < best ? k : best;
+          const uint32_t k = float_order_key(m[e]);
+          if (k < bk) {  // strictly smaller: the lower index of this thread wins ties
+            bk = k;
+            bi = static_cast<uint32_t>(base + e);
+          }
         }
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, best, o);
-        best = y < best ? y : best;
-      }
+      uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, bk);
+      uint32_t wi = __reduce_min_sync(0xFFFFFFFFu, bk == wk ? bi : 0xFFFFFFFFu);
       const int slot = t & 1;
-      if (lane == 0) s.wmin[slot][warp] = best;
+      if (lane == 0) {
+        s.wkey[slot][warp] = wk;
+        s.widx[slot][warp] = wi;
+      }
       __syncthreads();
-      best = s.wmin[slot][lane];
+      const uint32_t ck = s.wkey[slot][lane], ci = s.widx[slot][lane];
+      wk = __reduce_min_sync(0xFFFFFFFFu, ck);
+      wi = __reduce_min_sync(0xFFFFFFFFu, ck == wk ? ci : 0xFFFFFFFFu);
+      const int pick = static_cast<int>(wi);
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long y = __shfl_xor_sync(0xFFFFFFFFu, best, o);
-        best = y < best ? y : best;
-      }
-      const int pick = static_cast<int>(best & 0xFFFFFFFFull);
-      if (pick >= base && pick < base + kPer) kept[pick - base] = true;
-      const float* row = G + static_cast<size_t>(pick) * gp;
-      if (full4) {
-        const float4 g = *reinterpret_cast<const float4*>(row + base);
-        m[0] = fmaxf(m[0], g.x); m[1] = fmaxf(m[1], g.y); m[2] = fmaxf(m[2], g.z); m[3] = fmaxf(m[3], g.w);
-      } else {
-#pragma unroll
-        for (int e = 0; e < kPer; ++e)
-          if (base + e < N) m[e] = fmaxf(m[e], row[base + e]);
-      }
+      for (int e = 0; e < kPer; ++e)
+        if (base + e == pick) kept[e] = true;
+      take_row(pick);
     }
   }
   // Output: the kept set in ascending index order.

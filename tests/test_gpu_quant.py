@@ -66,3 +66,14 @@ def test_quant_empty_is_noop(p4q, dev):
     Xq = torch.empty((0, 64), dtype=torch.uint8, device=dev)
     s = torch.empty((0,), dtype=torch.float32, device=dev)
     p4q.p4q_quant_act(X, Xq, s)
+
+
+def test_quant_rows_full_of_exact_ties(p4q, dev):
+    """Rows whose quotients x / s land on exact .5 boundaries (s = 1 or 2^k),
+    plus rows near them: the rounding decisions must match the oracle's."""
+    rng = np.random.default_rng(21)
+    x = (rng.integers(-28, 29, size=(64, 512)) * 0.25).astype(np.float32)
+    x[:, 0] = 7.0                      # absmax 7 -> s = 1 exactly
+    x[32:] *= np.float32(2.0 ** -3)    # s = 2^-3
+    x[48:, 1:] = np.nextafter(x[48:, 1:], np.float32(np.inf))  # just off the boundaries
+    _check(p4q, dev, x.astype(np.float16))
