@@ -271,7 +271,23 @@ __global__ void __launch_bounds__(kSelThreads, 1)
           if (base + e < N) m[e] = fmaxf(m[e], row[base + e]);
       }
     };
-    for (int r = 0; r < total; ++r) take_row(s.list[r]);
+    // The kept rows are independent: fetch them eight at a time so their
+    // L2 latencies overlap.
+    int r = 0;
+    if (full4) {
+      for (; r + 8 <= total; r += 8) {
+        float4 g[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          g[u] = *reinterpret_cast<const float4*>(G + static_cast<size_t>(s.list[r + u]) * gp + base);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          m[0] = fmaxf(m[0], g[u].x); m[1] = fmaxf(m[1], g[u].y);
+          m[2] = fmaxf(m[2], g[u].z); m[3] = fmaxf(m[3], g[u].w);
+        }
+      }
+    }
+    for (; r < total; ++r) take_row(s.list[r]);
     // Greedy rounds: argmin of m over the free tokens (lower index on ties),
     // one block barrier per round.
     for (int t = 0; t < Kd; ++t) {
