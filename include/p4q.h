@@ -83,6 +83,16 @@ p4q_status p4q_device_status(p4q_stream_t stream);
  * work. */
 uint64_t p4q_launch_count(void);
 
+/* GEMM kernel variant used by p4q_w4a4_linear and p4q_w4a4_gemm_s32, for all
+ * later calls in the process (for tests and tuning; results are identical):
+ *   0 automatic (default): CTA-pair kernel for fp16 outputs with M >= 256 and
+ *     N >= 256, single-CTA kernel otherwise;
+ *   1 single-CTA kernel only;
+ *   2 CTA-pair kernel whenever N >= 256 (also for int32 outputs).
+ * Returns P4Q_ERR_INVALID_ARG for other values. Not thread-safe against
+ * concurrent launches. */
+p4q_status p4q_set_gemm_variant(int variant);
+
 /* ---------------------------------------------------------------------- */
 /* Per-row 4-bit quantizers (App. A, App. B.3)                             */
 /* ---------------------------------------------------------------------- */

@@ -152,6 +152,12 @@ const char* p4q_status_string(p4q_status s) {
 
 uint64_t p4q_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+p4q_status p4q_set_gemm_variant(int variant) {
+  if (variant < 0 || variant > 2) return P4Q_ERR_INVALID_ARG;
+  set_gemm_pair_mode(variant == 0 ? -1 : variant == 1 ? 0 : 1);
+  return P4Q_OK;
+}
+
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
   const unsigned int g = gemm_read_and_clear_error();

@@ -484,6 +484,360 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ============================================================================
+// CTA-pair variant (tcgen05 cta_group::2): a cluster of two CTAs computes a
+// 256 x 256 output tile. CTA r of the pair unpacks rows 128r..128r+127 of the
+// A tile and of the B tile into its own shared memory; the leader (r = 0)
+// issues M = 256 MMAs that read both CTAs' operands, and each CTA's TMEM
+// receives its 128 rows of the accumulator. Per SM this halves the B rows
+// unpacked per multiply-accumulate compared with a 128 x 256 tile of one CTA.
+// The per-row sums of u of the B tile are exchanged between the two CTAs
+// through distributed shared memory.
+// ============================================================================
+namespace pair {
+
+constexpr int BN = 256;      // output columns per pair
+constexpr int HB = BN / 2;   // B rows unpacked per CTA
+constexpr int A_CONV = BM * BK;
+constexpr int B_CONV = HB * BK;
+constexpr int CONV_STAGE = A_CONV + B_CONV;
+constexpr uint32_t TMEM_COLS = 2 * BN;
+
+template <int MODE>  // GemmOut::kHalf or kS32
+struct Lay {
+  static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
+  static constexpr int BOX_BYTES = 32 * 32 * ELEM;  // one 32 x 32 output box
+  static constexpr int FIXED = kEpiWarps * 2 * BOX_BYTES + 2 * kGroups * (BM + BN) * 4 + 2 * BN * 4 + 512;
+  static constexpr int SC_FIT = (232448 - 1024 - FIXED) / CONV_STAGE > 8 ? 8 : (232448 - 1024 - FIXED) / CONV_STAGE;
+  static constexpr int SC = SC_FIT - SC_FIT % kGroups;
+  static constexpr int OFF_STAGE = SC * CONV_STAGE;
+  static constexpr int OFF_SUMA = OFF_STAGE + kEpiWarps * 2 * BOX_BYTES;
+  static constexpr int OFF_SUMB = OFF_SUMA + 2 * kGroups * BM * 4;
+  static constexpr int OFF_SCOL = OFF_SUMB + 2 * kGroups * BN * 4;
+  static constexpr int OFF_BAR = OFF_SCOL + 2 * BN * 4;
+  static constexpr int NBAR = 2 * SC + 8;
+  static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
+  static constexpr int SMEM = 1024 + OFF_MISC + 16;
+  static_assert(SC >= 2 && SC % kGroups == 0, "E4M3 stages");
+  static_assert(SMEM <= 232448, "shared memory budget");
+};
+
+template <int MODE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    w4a4_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                          const __grid_constant__ CUtensorMap tmD, const Params p) {
+  using L = Lay<MODE>;
+  constexpr int SC = L::SC, BOX_BYTES = L::BOX_BYTES, OFF_STAGE = L::OFF_STAGE, OFF_SUMA = L::OFF_SUMA,
+                OFF_SUMB = L::OFF_SUMB, OFF_SCOL = L::OFF_SCOL, OFF_BAR = L::OFF_BAR, OFF_MISC = L::OFF_MISC;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  uint64_t* full_c = bars;              // [SC] leader: both CTAs' unpack -> MMA
+  uint64_t* empty_c = full_c + SC;      // [SC] MMA commit (both CTAs) -> unpack
+  uint64_t* acc_full = empty_c + SC;    // [2] MMA commit (both CTAs) -> epilogue
+  uint64_t* acc_empty = acc_full + 2;   // [2] leader: both CTAs' epilogues -> MMA
+  uint64_t* sums_full = acc_empty + 2;  // [2] both CTAs' unpack -> epilogue
+  uint64_t* sums_empty = sums_full + 2; // [2] both CTAs' epilogues -> unpack
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + OFF_MISC + 4);
+  int* sumA = reinterpret_cast<int*>(smem + OFF_SUMA);  // [2][kGroups][BM]
+  int* sumB = reinterpret_cast<int*>(smem + OFF_SUMB);  // [2][kGroups][BN], both halves
+  float* colv = reinterpret_cast<float*>(smem + OFF_SCOL);
+  float* sbw = colv + BN;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank(), peer = rank ^ 1u;
+  const int KB = p.K / BK;
+  const int per = p.num_m * p.num_n;  // pair tiles per batch (num_m counts 256-row tiles)
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < SC; ++i) {
+      mbar_init(&full_c[i], 2 * kGroupWarps);  // the unpack warps of both CTAs
+      mbar_init(&empty_c[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 2 * kEpiWarps);
+      mbar_init(&sums_full[i], 2 * kConvWarps);
+      mbar_init(&sums_empty[i], 2 * kEpiWarps);
+    }
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc_pair(tmem_slot, TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();  // barriers of both CTAs initialized, TMEM allocated in both
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ MMA issuer (leader)
+    if (lane == 0 && rank == 0) {
+      constexpr uint32_t idesc = idesc_e4m3_f32(2 * BM, BN);
+      int g = 0, it = 0;
+      bool ok = true;
+      for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x(), ++it) {
+        const int ab = it & 1;
+        if (!mbar_wait(&acc_empty[ab], ((it >> 1) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
+        tc_fence_after();
+        const uint32_t d = tmem_base + static_cast<uint32_t>(ab * BN);
+        for (int kb = 0; kb < KB; ++kb, ++g) {
+          const int s = g % SC;
+          if (!mbar_wait(&full_c[s], (g / SC) & 1, abort_flag, &g_gemm_err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(smem + s * CONV_STAGE);
+          const uint32_t b0 = a0 + A_CONV;
+#pragma unroll
+          for (int k = 0; k < BK / 32; ++k)
+            mma_f8f6f4_pair(d, sw128_kmajor_desc(a0 + k * 32), sw128_kmajor_desc(b0 + k * 32), idesc,
+                            (kb | k) != 0 ? 1u : 0u);
+          mma_commit_pair(&empty_c[s], 3);
+        }
+        mma_commit_pair(&acc_full[ab], 3);
+      }
+    }
+  } else if (warp < kFirstEpiWarp) {
+    // ------------------------------------------------------------ unpack warps
+    const int cw = warp - kFirstConvWarp;
+    const int grp = cw / kGroupWarps;
+    const int tc = threadIdx.x - (kFirstConvWarp + grp * kGroupWarps) * 32;
+    constexpr int NA = BM * 4 / kGroupThreads, NB = HB * 4 / kGroupThreads, NT = NA + NB;
+    const int rbase = tc >> 2, chunk = tc & 3;
+    const size_t rowbytes = static_cast<size_t>(p.K) >> 1;
+    const bool prefetcher = (tc == 0);
+    const uint32_t full_c_leader = mapa_shared(smem_u32(full_c), 0);
+    if (prefetcher) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+    }
+    int gbase = 0, it = 0;
+    bool ok = true;
+    for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x(), ++it, gbase += KB) {
+      const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
+      const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
+      const int n0 = nb * BN + static_cast<int>(rank) * HB;                       // this CTA's B rows
+      const uint8_t* baseA = p.A + (static_cast<size_t>(bz) * p.a_bs + m0 + rbase) * rowbytes + chunk * 16;
+      const uint8_t* baseB = p.B + (static_cast<size_t>(bz) * p.b_bs + n0 + rbase) * rowbytes + chunk * 16;
+      const size_t step = static_cast<size_t>(kRowStep) * rowbytes;
+      uint32_t valid = 0;
+#pragma unroll
+      for (int j = 0; j < NA; ++j) valid |= (m0 + rbase + kRowStep * j < p.M) ? (1u << j) : 0u;
+#pragma unroll
+      for (int j = 0; j < NB; ++j) valid |= (n0 + rbase + kRowStep * j < p.N) ? (1u << (NA + j)) : 0u;
+      const int kb0 = ((grp - gbase) % kGroups + kGroups) % kGroups;
+      if (prefetcher && grp == 0) {
+        for (int kb = 0; kb < min(KB, kPrefetchAhead); ++kb) {
+          tma_prefetch_l2_3d(&tmA, kb * BKP, m0, bz);
+          tma_prefetch_l2_3d(&tmB, kb * BKP, n0, bz);
+        }
+      }
+      uint32_t accA[NA], accB[NB];
+#pragma unroll
+      for (int j = 0; j < NA; ++j) accA[j] = 0;
+#pragma unroll
+      for (int j = 0; j < NB; ++j) accB[j] = 0;
+      uint4 buf[2][NT];
+      auto load = [&](uint4 (&v)[NT], int kb) {
+        const size_t off = static_cast<size_t>(kb) * BKP;
+#pragma unroll
+        for (int j = 0; j < NA; ++j)
+          v[j] = (valid >> j) & 1u ? ldg_stream16(baseA + j * step + off) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int j = 0; j < NB; ++j)
+          v[NA + j] = (valid >> (NA + j)) & 1u ? ldg_stream16(baseB + j * step + off) : make_uint4(0u, 0u, 0u, 0u);
+      };
+      auto convert = [&](const uint4 (&v)[NT], int kb) -> bool {
+        const int g = gbase + kb;
+        const int c = g % SC;
+        if (prefetcher && grp == 0) {
+          for (int q = kb + kPrefetchAhead; q < min(KB, kb + kPrefetchAhead + kGroups); ++q) {
+            tma_prefetch_l2_3d(&tmA, q * BKP, m0, bz);
+            tma_prefetch_l2_3d(&tmB, q * BKP, n0, bz);
+          }
+        }
+        if (!mbar_wait_warp(&empty_c[c], ((g / SC) & 1) ^ 1, abort_flag, &g_gemm_err)) return false;
+        uint8_t* ca = smem + c * CONV_STAGE;
+        uint8_t* cb = ca + A_CONV;
+#pragma unroll
+        for (int j = 0; j < NA; ++j) convert_chunk(v[j], ca, rbase + kRowStep * j, chunk, accA[j]);
+#pragma unroll
+        for (int j = 0; j < NB; ++j) convert_chunk(v[NA + j], cb, rbase + kRowStep * j, chunk, accB[j]);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote(full_c_leader + 8u * c);  // the leader's full_c[c]
+        return true;
+      };
+      // Two of this group's k-blocks in flight in registers.
+      if (kb0 < KB) load(buf[0], kb0);
+      if (kb0 + kGroups < KB) load(buf[1], kb0 + kGroups);
+      for (int kb = kb0; kb < KB && ok; kb += 2 * kGroups) {
+        ok = convert(buf[0], kb);
+        if (!ok || kb + kGroups >= KB) break;
+        if (kb + 2 * kGroups < KB) load(buf[0], kb + 2 * kGroups);
+        ok = convert(buf[1], kb + kGroups);
+        if (!ok) break;
+        if (kb + 3 * kGroups < KB) load(buf[1], kb + 3 * kGroups);
+      }
+      if (!ok) break;
+      // Row sums of u: A rows locally, B rows into this CTA's half of sumB in both CTAs.
+      const int ab = it & 1;
+      if (!mbar_wait_warp(&sums_empty[ab], ((it >> 1) & 1) ^ 1, abort_flag, &g_gemm_err)) break;
+#pragma unroll
+      for (int j = 0; j < NA; ++j) {
+        int v = static_cast<int>(accA[j]);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
+        if (chunk == 0) sumA[(ab * kGroups + grp) * BM + rbase + kRowStep * j] = v;
+      }
+#pragma unroll
+      for (int j = 0; j < NB; ++j) {
+        int v = static_cast<int>(accB[j]);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 1);
+        v += __shfl_xor_sync(0xFFFFFFFFu, v, 2);
+        if (chunk == 0) {
+          int* dst = &sumB[(ab * kGroups + grp) * BN + static_cast<int>(rank) * HB + rbase + kRowStep * j];
+          *dst = v;
+          st_shared_cluster_u32(mapa_shared(smem_u32(dst), peer), static_cast<uint32_t>(v));
+        }
+      }
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive_remote(mapa_shared(smem_u32(&sums_full[ab]), rank));
+        mbar_arrive_remote(mapa_shared(smem_u32(&sums_full[ab]), peer));
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue warps
+    const int ew = warp - kFirstEpiWarp;
+    const int q = warp & 3;
+    uint8_t* boxes = smem + OFF_STAGE + ew * 2 * BOX_BYTES;
+    const uint32_t acc_empty_leader = mapa_shared(smem_u32(acc_empty), 0);
+    int it = 0, nbox = 0;
+    bool failed = false;
+    for (int t = cluster_id_x(); t < p.tiles; t += nclusters_x(), ++it) {
+      const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
+      const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;
+      const int n0 = nb * BN;
+      const int ab = it & 1;
+      const uint32_t ph = (it >> 1) & 1;
+      if (!failed && !(mbar_wait_warp(&acc_full[ab], ph, abort_flag, &g_gemm_err) &&
+                       mbar_wait_warp(&sums_full[ab], ph, abort_flag, &g_gemm_err)))
+        failed = true;
+      tc_fence_after();
+      const int row = q * 32 + lane;
+      const int m = m0 + row;
+      epi_sync();
+      if (!failed) {
+        for (int i = ew * 32 + lane; i < BN; i += kEpiWarps * 32) {
+          int v = 0;
+#pragma unroll
+          for (int q2 = 0; q2 < kGroups; ++q2) v += sumB[(ab * kGroups + q2) * BN + i];
+          sbw[i] = static_cast<float>(-8 * v);
+          if (MODE == static_cast<int>(GemmOut::kHalf)) colv[i] = (n0 + i < p.N) ? p.s_b[n0 + i] : 0.0f;
+        }
+      }
+      epi_sync();
+      if (failed) continue;
+      int sa_u = 0;
+#pragma unroll
+      for (int q2 = 0; q2 < kGroups; ++q2) sa_u += sumA[(ab * kGroups + q2) * BM + row];
+      const float corrA = static_cast<float>(64 * p.K - 8 * sa_u);
+      const float sa = (MODE == static_cast<int>(GemmOut::kHalf) && m < p.M) ? p.s_a[m] : 0.0f;
+#pragma unroll 1
+      for (int cc = 0; cc < BN / 32; ++cc) {
+        uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
+        if (lane == 0) bulk_wait_group_read<1>();
+        __syncwarp();
+        uint8_t* rowp = box + lane * (32 * L::ELEM);
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          const int c0 = cc * 32 + h * 16;
+          uint32_t v[16];
+          tmem_ld_32x32b_x16(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ab * BN + c0, v);
+          tmem_ld_wait();
+          if (cc == BN / 32 - 1 && h == 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote(acc_empty_leader + 8u * ab);
+          }
+          if (MODE == static_cast<int>(GemmOut::kHalf)) {
+#pragma unroll
+            for (int g2 = 0; g2 < 2; ++g2) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int i0 = g2 * 8 + 2 * e;
+                const float a0 = __fmaf_rn(__uint_as_float(v[i0]), 262144.0f, corrA + sbw[c0 + i0]);
+                const float a1 = __fmaf_rn(__uint_as_float(v[i0 + 1]), 262144.0f, corrA + sbw[c0 + i0 + 1]);
+                const float y0 = __fmul_rn(__fmul_rn(a0, sa), colv[c0 + i0]);
+                const float y1 = __fmul_rn(__fmul_rn(a1, sa), colv[c0 + i0 + 1]);
+                const __half2 hh = __floats2half2_rn(y0, y1);
+                w[e] = *reinterpret_cast<const uint32_t*>(&hh);
+              }
+              // 64-byte rows, 64-byte swizzle: 16-byte chunk (2h + g2) of row `lane`
+              const int ch = 2 * h + g2;
+              *reinterpret_cast<uint4*>(rowp + ((ch ^ ((lane >> 1) & 3)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+          } else {
+#pragma unroll
+            for (int g4 = 0; g4 < 4; ++g4) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int i = g4 * 4 + e;
+                w[e] = static_cast<uint32_t>(
+                    __float2int_rn(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c0 + i])));
+              }
+              // 128-byte rows, 128-byte swizzle: 16-byte chunk (4h + g4) of row `lane`
+              const int ch = 4 * h + g4;
+              *reinterpret_cast<uint4*>(rowp + ((ch ^ (lane & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+            }
+          }
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          tma_store_3d(&tmD, box, n0 + cc * 32, m0 + q * 32, bz);
+          bulk_commit_group();
+        }
+        ++nbox;
+      }
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive_remote(mapa_shared(smem_u32(&sums_empty[ab]), rank));
+        mbar_arrive_remote(mapa_shared(smem_u32(&sums_empty[ab]), peer));
+      }
+    }
+    if (lane == 0) bulk_wait_group_all();
+    __syncwarp();
+  }
+
+  // Teardown: the pair's MMAs (which write both CTAs' TMEM) must be complete
+  // before either CTA releases its TMEM.
+  if (warp == 0 && lane == 0 && rank == 0 && *abort_flag) {
+    for (int i = 0; i < 2; ++i) {
+      const unsigned long long t0 = globaltimer();
+      const uint32_t a = smem_u32(&acc_full[i]);
+      while (!mbar_try_wait(a, 0) && !mbar_try_wait(a, 1) && globaltimer() - t0 < 100000000ull) {
+      }
+    }
+  }
+  tc_fence_before();
+  cluster_sync();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, TMEM_COLS);
+  }
+}
+
+}  // namespace pair
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   static std::once_flag once;
@@ -579,9 +933,53 @@ cudaError_t launch_cfg(const GemmArgs& g, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+template <int MODE>
+cudaError_t launch_pair(const GemmArgs& g, cudaStream_t stream) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(pair::w4a4_gemm_pair_kernel<MODE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, pair::Lay<MODE>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  CUtensorMap ma, mb, md;
+  if (!make_operand_map(&ma, g.A, g.K, g.M, g.batch, g.a_batch_stride, BM)) return cudaErrorInvalidValue;
+  if (!make_operand_map(&mb, g.B, g.K, g.N, g.batch, g.b_batch_stride, pair::HB)) return cudaErrorInvalidValue;
+  const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
+  if (!make_output_map(&md, g.D, g.out, g.M, g.N, pitch, g.batch)) return cudaErrorInvalidValue;
+  Params p;
+  p.A = g.A;
+  p.B = g.B;
+  p.a_bs = g.a_batch_stride > 0 ? g.a_batch_stride : g.M;
+  p.b_bs = g.b_batch_stride > 0 ? g.b_batch_stride : g.N;
+  p.M = g.M;
+  p.N = g.N;
+  p.K = g.K;
+  p.batch = g.batch;
+  p.num_m = (g.M + 2 * BM - 1) / (2 * BM);
+  p.num_n = (g.N + pair::BN - 1) / pair::BN;
+  p.tiles = p.num_m * p.num_n * g.batch;
+  p.s_a = g.s_a;
+  p.s_b = g.s_b;
+  p.norm_a = g.norm_a;
+  p.norm_b = g.norm_b;
+  const int pairs = p.tiles < num_sms() / 2 ? p.tiles : num_sms() / 2;
+  pair::w4a4_gemm_pair_kernel<MODE><<<2 * pairs, kThreads, pair::Lay<MODE>::SMEM, stream>>>(ma, mb, md, p);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
+// CTA-pair kernel selection (a test hook; the default uses it for large fp16 linears).
+static int g_pair_mode = -1;  // -1: automatic, 0: never, 1: whenever the shape allows
+
+void set_gemm_pair_mode(int mode) { g_pair_mode = mode; }
+
 cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream) {
+  const bool pair_ok = g.M > 0 && g.N >= 256 && g.batch > 0 && g_pair_mode != 0 &&
+                       (g_pair_mode == 1 || (g.M >= 256 && g.out == GemmOut::kHalf));
+  if (pair_ok && g.out == GemmOut::kHalf) return launch_pair<0>(g, stream);
+  if (pair_ok && g.out == GemmOut::kS32) return launch_pair<1>(g, stream);
   if (g.M <= 0 || g.N <= 0 || g.batch <= 0) return cudaSuccess;
   switch (g.out) {
     case GemmOut::kHalf:

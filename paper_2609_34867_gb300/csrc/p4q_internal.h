@@ -50,6 +50,11 @@ struct GemmArgs {
 // cannot run on this kernel.
 cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream);
 
+// Which GEMM kernel serves fp16 / int32 outputs: -1 automatic (the CTA-pair
+// kernel for large fp16 linears), 0 single-CTA only, 1 CTA-pair whenever the
+// shape allows (N >= 256).
+void set_gemm_pair_mode(int mode);
+
 // ------------------------------------------------------------ selector
 struct SelectPlan {
   int B, N, d, J, K, Kq, Ks, Kd;

@@ -45,6 +45,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_status_string.restype = ctypes.c_char_p
         L.p4q_launch_count.argtypes = []
         L.p4q_launch_count.restype = ctypes.c_uint64
+        L.p4q_set_gemm_variant.argtypes = [I]
+        L.p4q_set_gemm_variant.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_quant_act.argtypes = [P, I, I, P, P, P]
@@ -95,6 +97,11 @@ def p4q_status_string(status: int) -> str:
 def p4q_launch_count() -> int:
     """Kernels launched by libp4q.so in this process so far."""
     return int(lib().p4q_launch_count())
+
+
+def p4q_set_gemm_variant(variant: int):
+    """0 automatic, 1 single-CTA GEMM only, 2 CTA-pair GEMM whenever N >= 256."""
+    _check(lib().p4q_set_gemm_variant(int(variant)), "p4q_set_gemm_variant")
 
 
 def p4q_device_status(stream=None) -> int:

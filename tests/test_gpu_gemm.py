@@ -21,10 +21,17 @@ def _gemm(p4q, dev, a, w):
     return acc.cpu().numpy()
 
 
+@pytest.fixture(params=[1, 2], ids=["single_cta", "cta_pair"])
+def variant(request, p4q):
+    p4q.p4q_set_gemm_variant(request.param)
+    yield request.param
+    p4q.p4q_set_gemm_variant(0)
+
+
 @pytest.mark.parametrize("M,N,K", [(1, 8, 128), (128, 128, 128), (96, 4096, 4096), (200, 136, 256),
                                    (300, 1032, 384), (129, 1024, 1024), (64, 2048, 11008),
-                                   (1100, 2056, 256), (2048, 4096, 512)])
-def test_gemm_s32_bit_exact(p4q, dev, M, N, K):
+                                   (1100, 2056, 256), (2048, 4096, 512), (256, 256, 128), (257, 264, 256)])
+def test_gemm_s32_bit_exact(p4q, dev, variant, M, N, K):
     rng = np.random.default_rng(M * 7 + N)
     a, w = _packed(rng, M, K), _packed(rng, N, K)
     got = _gemm(p4q, dev, a, w)
@@ -34,12 +41,12 @@ def test_gemm_s32_bit_exact(p4q, dev, M, N, K):
 
 
 @pytest.mark.parametrize("K", [13824, 16384])
-def test_gemm_extreme_codes_exact(p4q, dev, K):
+def test_gemm_extreme_codes_exact(p4q, dev, variant, K):
     """Largest magnitudes: +7 x +7 (offset codes 15 x 15), -8 x -8, -8 x +7, and alternating signs."""
     pat = {"p7": 0x77, "m7": 0x99, "m8": 0x88, "alt": 0x97, "zero": 0x00}
     names = list(pat)
     a = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 26)[:128]
-    w = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 2)[:8]
+    w = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 52)[:256]
     got = _gemm(p4q, dev, a, w)
     ref = oracle.gemm_s32(oracle.unpack_codes(a), oracle.unpack_codes(w))
     assert np.array_equal(got, ref)
@@ -54,8 +61,8 @@ def test_gemm_zero_rows_is_noop(p4q, dev):
 
 
 @pytest.mark.parametrize("M,N,K", [(96, 4096, 4096), (257, 1032, 512), (33, 128, 13824), (2048, 4096, 1024),
-                                   (300, 11008, 256)])
-def test_linear_fp16_within_tolerance(p4q, dev, M, N, K):
+                                   (300, 11008, 256), (512, 264, 128)])
+def test_linear_fp16_within_tolerance(p4q, dev, variant, M, N, K):
     rng = np.random.default_rng(K + M)
     a, w = _packed(rng, M, K), _packed(rng, N, K)
     sa = (rng.random(M) * 0.5 + 0.01).astype(np.float32)
