@@ -40,9 +40,11 @@ METRIC = "W4A4 prefill linear TOPS (% INT8 tensor peak); select+prune µs/image"
 WORKLOAD = wl.LLAVA15_7B
 FLUSH_BYTES = 512 << 20  # > 129 MB L2, written between timed steps
 
-# Latest ncu capture of the dominant kernel (see profiles/): DRAM bytes per
-# launch, valid while the GEMM source is unchanged since the capture.
-PROFILED_GEMM = {"source_sha1": None, "dram_bytes_per_launch": None}
+# Latest ncu capture of the dominant kernel: mean DRAM bytes (read + write)
+# per launch over the seven linears of one step (profiles/
+# w4a4_gemm_pair_llava15_7b_b8_step.md), valid only while the GEMM source is
+# unchanged since the capture.
+PROFILED_GEMM = {"source_sha1": "192947517df2e4813855a1cc8715f43bfde5cb45", "dram_bytes_per_launch": 19820470}
 
 
 def gemm_source_sha1() -> str:
