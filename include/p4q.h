@@ -174,6 +174,26 @@ p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
                       const float* A_cls, const p4q_select_params* params, int32_t* idx,
                       void* ws, size_t ws_bytes, p4q_stream_t stream);
 
+/* p4q_select for callers that cannot allocate device memory when they select
+ * (a fixed memory budget set at start-up, a plugin inside a runtime that owns
+ * the allocator): same inputs, outputs and results as p4q_select, without the
+ * workspace arguments. The paper has no counterpart; this is a deployment
+ * convenience of this library.
+ *
+ * Scratch: a fixed array of P4Q_NOALLOC_SCRATCH_BYTES inside the library's
+ * device image, held by every GPU that loads the library until the process
+ * exits. Sizes whose workspace (p4q_select_workspace_bytes) exceeds it return
+ * P4Q_ERR_WORKSPACE_TOO_SMALL and launch nothing. The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress) and keeps it;
+ * make that first call before any stream capture. The call allocates nothing.
+ * All calls on a device share the one array: calls whose work overlaps on the
+ * GPU (other streams, or several host threads) race and give undefined
+ * results, so serialize them. */
+#define P4Q_NOALLOC_SCRATCH_BYTES (32u << 20)
+p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
+                              const float* A_cls, const p4q_select_params* params, int32_t* idx,
+                              p4q_stream_t stream);
+
 /* The selector followed by the gather of the original FP16 features of the
  * kept tokens (Sec. 3.2: the fake-quantized copies only decide the indices)
  * and the per-token INT4 quantization of the pruned sequence for the first

@@ -5,6 +5,7 @@
 
 #include <atomic>
 #include <cstdint>
+#include <mutex>
 
 #include "p4q.h"
 #include "p4q_internal.h"
@@ -262,3 +263,59 @@ p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Selector without a caller-provided workspace.
+//
+// Some callers cannot allocate device memory at the point where they run the
+// selector: code inside a fixed memory budget set up once at start-up, plugins
+// called from a runtime that owns the allocator, or hosts that must not
+// allocate while other work is in flight. p4q_select_noalloc gives them the
+// same selection with its scratch in the fixed array below. That array is
+// part of this library's device image, so every GPU that loads the library
+// reserves its bytes until the process exits.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = P4Q_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_select_scratch[kNoAllocScratchBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of g_select_scratch on the current device (looked up once per
+// device, with that device current). Host code cannot use the symbol itself:
+// in host code it names a host-side placeholder, not device memory.
+p4q_status scratch_address(void** out) {
+  int dev = -1;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return P4Q_ERR_NO_DEVICE;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (g_scratch_ptr[dev] == nullptr) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_select_scratch) != cudaSuccess || ptr == nullptr) return P4Q_ERR_CUDA;
+    g_scratch_ptr[dev] = ptr;
+  }
+  *out = g_scratch_ptr[dev];
+  return P4Q_OK;
+}
+
+}  // namespace
+
+extern "C" p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
+                                         const float* A_cls, const p4q_select_params* params, int32_t* idx,
+                                         p4q_stream_t stream) {
+  p4q_status st = check_select_args(V, B, N, d, J, params, idx);
+  if (st != P4Q_OK) return st;
+  const int Jeff = (Q != nullptr && J > 0) ? J : 0;
+  // Every region of the scratch is written before it is read on each call, so
+  // nothing needs clearing between calls.
+  if (select_workspace_layout(B, N, d, Jeff, nullptr, nullptr) > kNoAllocScratchBytes)
+    return P4Q_ERR_WORKSPACE_TOO_SMALL;
+  if ((st = check_device()) != P4Q_OK) return st;
+  void* ws = nullptr;
+  if ((st = scratch_address(&ws)) != P4Q_OK) return st;
+  return run_select(V, B, N, d, Q, J, A_cls, params, idx, ws, kNoAllocScratchBytes,
+                    reinterpret_cast<cudaStream_t>(stream));
+}
+
