@@ -13,6 +13,12 @@ per step divided by the step time (the selector's time included); the
 selector's share is also reported as microseconds per image.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl {p4q,reference}]
+                  [--workload NAME]
+
+--workload runs the same step on another of the LLaVA-shaped workloads (the
+one-image 576-token case, the 16 x 2880-token LLaVA-NeXT-7B batch over 32
+decoder layers, the 32 x 2880-token LLaVA-NeXT-13B batch); the default is the
+8-image batch above.
 
 --impl reference times the CPU oracle (test infrastructure) on a bounded
 sample of the same workload. Under torchrun each rank runs its own batch
@@ -53,7 +59,31 @@ def gemm_source_sha1() -> str:
 
 
 def linear_ops(w: wl.Workload) -> int:
-    return sum(2 * w.M * l.n_out * l.k_in for l in w.linears)
+    return w.layers * sum(2 * w.M * l.n_out * l.k_in for l in w.linears)
+
+
+def rank_seed(w: wl.Workload, rank: int) -> int:
+    """Input seed of a rank's batch: every rank draws its own images and text
+    (weights are replicated: they depend on the workload and layer only)."""
+    return w.seed + rank
+
+
+def max_over_ranks(values, world: int, device):
+    """Element-wise maximum of per-rank timings over all ranks (all_reduce MAX;
+    the identity for a single process). The job takes as long as its slowest
+    rank."""
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def whole_job_tops(ops_per_rank: int, world: int, ms_per_step: float) -> float:
+    """Aggregate throughput: the integer ops of every rank's batch over the
+    (max-over-ranks) step time."""
+    return ops_per_rank * world / (ms_per_step * 1e-3) / 1e12
 
 
 def measured_peaks():
@@ -120,7 +150,15 @@ class ClockSampler:
 
 # --------------------------------------------------------------------- GPU arm
 class Step:
-    """Device buffers and weights of one rank, and the step itself."""
+    """Device buffers and weights of one rank, and the step itself.
+
+    The inputs are drawn with `seed`; the weights of decoder layer l with
+    wl.weight_seed(w.seed + l, linear id), the same on every rank (replicated
+    weights, independent batches). Every layer runs on the pruned sequence:
+    q, k, v, gate, up on its INT4 codes, o on the re-quantized q output, down
+    on the re-quantized up output."""
+
+    REQUANT = {"o": "q", "down": "up"}  # linear -> the linear whose output it re-quantizes
 
     def __init__(self, w: wl.Workload, dev, seed: int):
         import torch
@@ -139,27 +177,36 @@ class Step:
         M = w.M
         self.Xq = torch.empty((M, d // 2), dtype=torch.uint8, device=dev)
         self.s_a = torch.empty((M,), dtype=torch.float32, device=dev)
-        self.Wq, self.s_w, self.Y = {}, {}, {}
-        for lid, lin in enumerate(w.linears):
-            W = torch.from_numpy(wl.weight(lin.k_in, lin.n_out, wl.weight_seed(seed, lid))).to(dev)
-            self.Wq[lin.name], self.s_w[lin.name] = p4q.quant_weight(W)
-            del W
-            self.Y[lin.name] = torch.empty((M, lin.n_out), dtype=torch.float16, device=dev)
+        self.Wq, self.s_w = {}, {}
+        for layer in range(w.layers):
+            for lid, lin in enumerate(w.linears):
+                W = torch.from_numpy(wl.weight(lin.k_in, lin.n_out, wl.weight_seed(w.seed + layer, lid))).to(dev)
+                self.Wq[layer, lin.name], self.s_w[layer, lin.name] = p4q.quant_weight(W)
+                del W
+        self.Y = {lin.name: torch.empty((M, lin.n_out), dtype=torch.float16, device=dev) for lin in w.linears}
         dims = {l.name: l for l in w.linears}
-        self.Xq_o = torch.empty((M, dims["o"].k_in // 2), dtype=torch.uint8, device=dev)
-        self.s_o = torch.empty((M,), dtype=torch.float32, device=dev)
-        self.Xq_d = torch.empty((M, dims["down"].k_in // 2), dtype=torch.uint8, device=dev)
-        self.s_d = torch.empty((M,), dtype=torch.float32, device=dev)
-        # The step is captured as a chain of CUDA graphs, one per segment
-        # (selector, each linear, each re-quantization), so that events
+        self.Xq_re, self.s_re = {}, {}
+        for name, src in self.REQUANT.items():
+            if name in dims:
+                assert src in dims, f"{name} needs the {src} linear"
+                self.Xq_re[name] = torch.empty((M, dims[name].k_in // 2), dtype=torch.uint8, device=dev)
+                self.s_re[name] = torch.empty((M,), dtype=torch.float32, device=dev)
+        self.out_name = w.linears[-1].name
+        # The step is a chain of segments (selector, each linear, each
+        # re-quantization) captured as one CUDA graph each, so that events
         # recorded between the replays time the selector and every linear.
-        self.segments = [("select", self._select)] + \
-            [(n, (lambda n=n: self._lin(n, self.Xq, self.s_a))) for n in ("q", "k", "v", "gate", "up")] + \
-            [("quant_o", lambda: p4q.p4q_quant_act(self.Y["q"], self.Xq_o, self.s_o)),
-             ("o", lambda: self._lin("o", self.Xq_o, self.s_o)),
-             ("quant_down", lambda: p4q.p4q_quant_act(self.Y["up"], self.Xq_d, self.s_d)),
-             ("down", lambda: self._lin("down", self.Xq_d, self.s_d))]
-        self.lin_ops = {l.name: 2 * w.M * l.n_out * l.k_in for l in w.linears}
+        self.segments = [("select", "select", self._select)]
+        for layer in range(w.layers):
+            for lin in w.linears:
+                if lin.name not in self.REQUANT:
+                    self.segments.append(("linear", lin.name, (lambda l=layer, n=lin.name: self._lin(l, n, self.Xq, self.s_a))))
+            for name, src in self.REQUANT.items():
+                if name in dims:
+                    self.segments.append(("quant", "quant_" + name, (lambda n=name, s=src: p4q.p4q_quant_act(
+                        self.Y[s], self.Xq_re[n], self.s_re[n]))))
+                    self.segments.append(("linear", name, (lambda l=layer, n=name: self._lin(
+                        l, n, self.Xq_re[n], self.s_re[n]))))
+        self.lin_ops = {l.name: 2 * w.M * l.n_out * l.k_in * w.layers for l in w.linears}
         self.graphs = None
         self.launches_per_step = None
         self.events = [torch.cuda.Event(enable_timing=True) for _ in range(len(self.segments) + 1)]
@@ -168,12 +215,12 @@ class Step:
         self.p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
                                          self.s_a, self.ws)
 
-    def _lin(self, name, Xq, s):
-        self.p4q.p4q_w4a4_linear(Xq, s, self.Wq[name], self.s_w[name], self.Y[name])
+    def _lin(self, layer, name, Xq, s):
+        self.p4q.p4q_w4a4_linear(Xq, s, self.Wq[layer, name], self.s_w[layer, name], self.Y[name])
 
     def body(self):
         """The step as plain C-ABI calls (no graph)."""
-        for _, fn in self.segments:
+        for _, _, fn in self.segments:
             fn()
 
     def capture(self):
@@ -183,7 +230,7 @@ class Step:
         torch = self.torch
         self.graphs = []
         n0 = self.p4q.p4q_launch_count()
-        for _, fn in self.segments:
+        for _, _, fn in self.segments:
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
                 fn()
@@ -200,8 +247,16 @@ class Step:
             self.events[i + 1].record()
 
     def kernel_times(self):
-        """{segment: ms} of the most recent graph step (after a sync)."""
-        return {name: self.events[i].elapsed_time(self.events[i + 1]) for i, (name, _) in enumerate(self.segments)}
+        """Milliseconds of the most recent graph step (after a sync):
+        {"select": ms, "quant": ms summed, "linear": {name: ms summed over layers}}."""
+        out = {"select": 0.0, "quant": 0.0, "linear": {l.name: 0.0 for l in self.w.linears}}
+        for i, (kind, name, _) in enumerate(self.segments):
+            ms = self.events[i].elapsed_time(self.events[i + 1])
+            if kind == "linear":
+                out["linear"][name] += ms
+            else:
+                out[kind] += ms
+        return out
 
 
 def run_gpu(args, rank, world, local_rank):
@@ -216,8 +271,8 @@ def run_gpu(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     p4q.lib()
-    w = WORKLOAD
-    step = Step(w, dev, seed=w.seed + rank)
+    w = wl.WORKLOADS[args.workload]
+    step = Step(w, dev, seed=rank_seed(w, rank))
     flush = torch.empty((FLUSH_BYTES,), dtype=torch.uint8, device=dev)
     for _ in range(args.warmup):
         flush.zero_()
@@ -252,7 +307,7 @@ def run_gpu(args, rank, world, local_rank):
         kt = step.kernel_times()
         sel_ms.append(kt["select"])
         for n in gemm_ms:
-            gemm_ms[n].append(kt[n])
+            gemm_ms[n].append(kt["linear"][n])
     t_wall = time.perf_counter() - t_wall
     if world > 1:
         dist.barrier()
@@ -273,7 +328,7 @@ def run_gpu(args, rank, world, local_rank):
         hostQ = torch.from_numpy(step.host["Q"]).pin_memory()
         hostA = torch.from_numpy(step.host["A"]).pin_memory()
         hostT = torch.from_numpy(step.host["text"]).pin_memory()
-        outY = torch.empty(step.Y["down"].shape, dtype=torch.float16).pin_memory()
+        outY = torch.empty(step.Y[step.out_name].shape, dtype=torch.float16).pin_memory()
         outI = torch.empty(step.idx.shape, dtype=torch.int32).pin_memory()
         h2d = sum(t.numel() * t.element_size() for t in (hostV, hostQ, hostA, hostT))
         d2h = outY.numel() * 2 + outI.numel() * 4
@@ -289,7 +344,7 @@ def run_gpu(args, rank, world, local_rank):
             step.A.copy_(hostA, non_blocking=True)
             step.text.copy_(hostT, non_blocking=True)
             step.body()  # the C-ABI calls themselves, no graph
-            outY.copy_(step.Y["down"], non_blocking=True)
+            outY.copy_(step.Y[step.out_name], non_blocking=True)
             outI.copy_(step.idx, non_blocking=True)
             b.record()
             torch.cuda.synchronize()
@@ -298,20 +353,18 @@ def run_gpu(args, rank, world, local_rank):
         e2e_ms = float(np.mean(times))
 
     # ---- reduce over ranks (max time)
-    stats = torch.tensor([total_ms, e2e_ms or 0.0], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(stats, op=dist.ReduceOp.MAX)
-    total_ms, e2e_max = float(stats[0]), float(stats[1])
+    total_ms, e2e_max = max_over_ranks([total_ms, e2e_ms or 0.0], world, dev)
     if rank != 0:
         return None
 
     ops = linear_ops(w)
     ms_per_step = total_ms / args.steps
-    value = ops * world / (ms_per_step * 1e-3) / 1e12
-    sustained = t_wall > 1.0
+    value = whole_job_tops(ops, world, ms_per_step)
+    # the burst peak unless the clocks show the power cap throttling the loop
+    sustained = bool(clk and "sw_power_cap" in clk["reasons"])
     peak, peak_src = fp8_peak_tops(sustained)
     ach = gemm_ops / (gemm_time_ms * 1e-3) / 1e12
-    n_gemm = len(step.lin_ops) * args.steps
+    n_gemm = len(step.lin_ops) * w.layers * args.steps
     traffic = None
     if PROFILED_GEMM["source_sha1"] == gemm_source_sha1():
         traffic = PROFILED_GEMM["dram_bytes_per_launch"]
@@ -330,7 +383,7 @@ def run_gpu(args, rank, world, local_rank):
         "data": "synthetic",
         "config": {
             "workload": w.name, "B": w.B, "N": w.N, "d": w.d, "K": w.K, "T": w.T, "J": w.J, "M": w.M,
-            "linears": "q,k,v,o 4096x4096; gate,up 4096->11008; down 11008->4096",
+            "linears": "; ".join(f"{l.name} {l.k_in}->{l.n_out}" for l in w.linears), "layers": w.layers,
             "alpha_beta_gamma": "0.3/0.2/0.5", "l2": "flushed (512 MiB write) before every timed step",
             "timing": "CUDA events around each step (graph replays), summed over the K steps",
             "parallelism": f"dp{world} (independent batches)"},
@@ -350,7 +403,7 @@ def run_gpu(args, rank, world, local_rank):
         "clocks": clk,
     }
     if e2e_ms is not None:
-        rec["e2e"] = {"value": round(ops * world / (e2e_max * 1e-3) / 1e12, 3), "unit": "TOPS",
+        rec["e2e"] = {"value": round(whole_job_tops(ops, world, e2e_max), 3), "unit": "TOPS",
                       "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                       "ms_per_step": round(e2e_max, 4), "steps": args.e2e_steps}
     if not args.no_cpu_baseline and world == 1:
@@ -378,7 +431,7 @@ class OracleSampler:
         self.cw = {}
         for lid, lin in enumerate(w.linears):
             self.cw[lin.name] = oracle.quantize_rows(wl.weight(lin.k_in, lin.n_out, wl.weight_seed(w.seed, lid)))
-        self.y = {n: oracle.linear(self.ca, self.sa, *self.cw[n]) for n in ("q", "up")}
+        self.y = {n: oracle.linear(self.ca, self.sa, *self.cw[n]) for n in ("q", "up") if n in self.cw}
         self.pieces = [("select", None)] + [("linear", l.name) for l in w.linears]
         self.times = {i: [] for i in range(len(self.pieces))}
         self.image = 0
@@ -408,13 +461,14 @@ class OracleSampler:
         for i, (kind, _) in enumerate(self.pieces):
             if not self.times[i]:
                 raise RuntimeError("piece not sampled")
-            est += float(np.mean(self.times[i])) * (w.B if kind == "select" else w.M / self.rows)
+            est += float(np.mean(self.times[i])) * (w.B if kind == "select" else w.layers * w.M / self.rows)
         return est
 
     def describe(self) -> str:
         w = self.w
-        return (f"selector+gather+quantize on 1 of {w.B} images (x{w.B}) and each of the 7 linears on "
-                f"{self.rows} of {w.M} rows (x{w.M // self.rows}), o/down inputs re-quantized; "
+        lay = f" x {w.layers} layers" if w.layers > 1 else ""
+        return (f"selector+gather+quantize on 1 of {w.B} images (x{w.B}) and each of the {len(w.linears)} linears "
+                f"on {self.rows} of {w.M} rows (x{w.M // self.rows}{lay}), o/down inputs re-quantized; "
                 f"weight quantization untimed")
 
 
@@ -434,7 +488,7 @@ def run_reference(args, rank):
     the sum of the pieces' mean times scaled to the full workload."""
     if rank != 0:
         return None
-    w = WORKLOAD
+    w = wl.WORKLOADS[args.workload]
     s = OracleSampler(w, args.cpu_threads)
     n = len(s.pieces)
     for i in range(args.warmup):
@@ -458,9 +512,11 @@ def run_reference(args, rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["p4q", "reference"], default="p4q")
+    ap.add_argument("--workload", choices=sorted(wl.WORKLOADS), default=WORKLOAD.name,
+                    help="workload of the step (default: the 8-image LLaVA-1.5-7B batch)")
     ap.add_argument("--e2e-steps", type=int, default=50)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-threads", type=int, default=0, help="oracle threads (0 = all cores)")

@@ -93,6 +93,17 @@ uint64_t p4q_launch_count(void);
  * concurrent launches. */
 p4q_status p4q_set_gemm_variant(int variant);
 
+/* Test of the bounded-wait path: launches one warp that waits on an mbarrier
+ * nothing ever completes. The wait gives up after limit_us microseconds, sets
+ * the device error word exactly as a stalled GEMM pipeline would, and the
+ * kernel returns; the next p4q_device_status() on the same stream reports
+ * P4Q_ERR_TIMEOUT (and clears it), and the context stays usable. The paper
+ * has no counterpart: this exists so that failure detection is testable
+ * without a GPU fault.
+ *   limit_us  1 .. 1000000 (else P4Q_ERR_INVALID_ARG; nothing is launched)
+ * Asynchronous on `stream`. */
+p4q_status p4q_test_wait_timeout(uint32_t limit_us, p4q_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* Per-row 4-bit quantizers (App. A, App. B.3)                             */
 /* ---------------------------------------------------------------------- */

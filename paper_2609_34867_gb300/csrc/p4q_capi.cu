@@ -166,6 +166,13 @@ p4q_status p4q_device_status(p4q_stream_t stream) {
   return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
 }
 
+p4q_status p4q_test_wait_timeout(uint32_t limit_us, p4q_stream_t stream) {
+  if (limit_us < 1u || limit_us > 1000000u) return P4Q_ERR_INVALID_ARG;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_expired_wait(1000ull * limit_us, reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* s_a, p4q_stream_t stream) {
   p4q_status st = check_rows(X, M, Kin, Xq, s_a);
   if (st != P4Q_OK || M == 0) return st;

@@ -72,17 +72,17 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parit
 
 // Waits for the phase with the given parity to complete, sleeping in the
 // barrier between checks (no busy polling). Gives up (returns false) when
-// *abort becomes non-zero or after kWaitLimitNs; on a time-out it sets *abort
+// *abort becomes non-zero or after limit_ns; on a time-out it sets *abort
 // and ORs kErrTimeout into *err so the host can report it.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          unsigned int* err) {
+                                          unsigned int* err, unsigned long long limit_ns = kWaitLimitNs) {
   const uint32_t a = smem_u32(bar);
   if (mbar_try_wait(a, parity)) return true;
   const unsigned long long t0 = globaltimer();
   while (true) {
     if (mbar_try_wait_sleep(a, parity, 200000u)) return true;
     if (*abort) return false;
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    if (globaltimer() - t0 > limit_ns) {
       *abort = 1;
       atomicOr(err, kErrTimeout);
       return false;
@@ -93,9 +93,9 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
 // Whole-warp wait: lane 0 waits on the barrier, the other lanes wait at the
 // warp barrier, so one thread per warp touches the mbarrier.
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                               unsigned int* err) {
+                                               unsigned int* err, unsigned long long limit_ns = kWaitLimitNs) {
   int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, err) ? 1 : 0;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, err, limit_ns) ? 1 : 0;
   return __shfl_sync(0xFFFFFFFFu, ok, 0) != 0;
 }
 

@@ -992,6 +992,30 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream) {
   return cudaErrorInvalidValue;
 }
 
+namespace {
+
+// One warp waits on an mbarrier that nothing ever arrives on. The bounded
+// wait gives up after limit_ns and records kErrTimeout in the same device
+// error word as the GEMM's waits, so the host sees exactly what a stalled
+// GEMM pipeline would report; the kernel then returns normally.
+__global__ void __launch_bounds__(32) expired_wait_kernel(unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+  }
+  __syncthreads();
+  mbar_wait_warp(&bar, 0, reinterpret_cast<volatile int*>(&abort_flag), &g_gemm_err, limit_ns);
+}
+
+}  // namespace
+
+cudaError_t launch_expired_wait(unsigned long long limit_ns, cudaStream_t stream) {
+  expired_wait_kernel<<<1, 32, 0, stream>>>(limit_ns);
+  return cudaGetLastError();
+}
+
 unsigned int gemm_read_and_clear_error() {
   unsigned int v = 0, z = 0;
   cudaMemcpyFromSymbol(&v, g_gemm_err, sizeof(v));

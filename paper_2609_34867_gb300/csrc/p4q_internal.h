@@ -81,4 +81,8 @@ cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws,
 // Device error word of the GEMM (the only kernel with bounded waits).
 unsigned int gemm_read_and_clear_error();
 
+// One bounded wait that nothing completes: times out after limit_ns and sets
+// the GEMM's device error word (tests the time-out path).
+cudaError_t launch_expired_wait(unsigned long long limit_ns, cudaStream_t stream);
+
 }  // namespace p4q

@@ -49,6 +49,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_set_gemm_variant.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
+        L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
+        L.p4q_test_wait_timeout.restype = st
         L.p4q_quant_act.argtypes = [P, I, I, P, P, P]
         L.p4q_quant_act.restype = st
         L.p4q_quant_weight.argtypes = [P, I, I, P, P, P]

@@ -70,6 +70,21 @@ WORKLOADS = {w.name: w for w in (LLAVA15_7B_ONE, LLAVA15_7B, LLAVANEXT_7B, LLAVA
 # GEMM + quantizer sweep: M x (K_in, N_out)
 SWEEP_M = (16, 64, 256, 1024, 4096, 16384, 65536)
 SWEEP_KN = ((4096, 4096), (4096, 11008), (11008, 4096), (5120, 13824))
+SWEEP_SEED = 4
+# selector-only sweep: tokens per image x images x budget (percent of N), d = 4096
+SWEEP_SEL_N = (576, 1152, 1728, 2304, 2880)
+SWEEP_SEL_B = (1, 4, 16, 64)
+SWEEP_SEL_PCT = (5.0, 10.0, 11.1, 25.0, 50.0)
+
+
+def sweep_budget(N: int, pct: float) -> int:
+    """Token budget of the selector sweep: pct percent of N, rounded, at least 1."""
+    return max(1, int(round(N * pct / 100.0)))
+
+
+def sweep_selector_workload(N: int, B: int, pct: float, d: int = 4096) -> Workload:
+    return Workload(f"select-sweep-b{B}-n{N}-{pct:g}pct", B=B, N=N, d=d, K=sweep_budget(N, pct), T=0, J=3,
+                    seed=SWEEP_SEED, heavy_tail=False, linears=())
 
 
 def outlier_channels(d: int) -> np.ndarray:

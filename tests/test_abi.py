@@ -86,3 +86,9 @@ def test_no_device_is_reported_not_faked(lib):
     P, I = ctypes.c_void_p, ctypes.c_int
     lib.p4q_quant_act.argtypes = [P, I, I, P, P, P]
     assert lib.p4q_quant_act(P(16), 4, 128, P(16), P(16), None) == 7
+
+
+def test_wait_timeout_test_entry_validates_its_limit(lib):
+    lib.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, ctypes.c_void_p]
+    assert lib.p4q_test_wait_timeout(0, None) == 1
+    assert lib.p4q_test_wait_timeout(1000001, None) == 1
