@@ -161,7 +161,7 @@ p4q_status p4q_set_gemm_variant(int variant) {
 
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
-  const unsigned int g = gemm_read_and_clear_error();
+  const unsigned int g = gemm_read_and_clear_error() | quant_read_and_clear_error();
   if (cudaGetLastError() != cudaSuccess) return P4Q_ERR_CUDA;
   return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
 }

@@ -78,8 +78,9 @@ cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, 
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls,
                                  int32_t* idx, cudaStream_t stream);
 
-// Device error word of the GEMM (the only kernel with bounded waits).
+// Device error words of the kernels with bounded waits (GEMM, quantizer).
 unsigned int gemm_read_and_clear_error();
+unsigned int quant_read_and_clear_error();
 
 // One bounded wait that nothing completes: times out after limit_ns and sets
 // the GEMM's device error word (tests the time-out path).

@@ -6,20 +6,37 @@
 // and zero codes. Codes are written packed, two per byte, the even index in
 // the low nibble (two's complement).
 //
-// A warp (rows up to 5120) or four warps (longer rows) quantize one row; the
-// row is read once from HBM with 16-byte loads and kept in registers between
-// the abs-max pass and the quantization pass. The same kernel serves the activation quantizer, the
-// weight quantizer, the selector's fake-quantized copies (with the squared code
-// norm as an extra output) and the fused gather of the pruned sequence.
+// Rows stream through shared memory. A group of G warps owns a ring of S row
+// buffers that its leader thread fills with bulk asynchronous copies
+// (cp.async.bulk, completion counted on one mbarrier per buffer), so that
+// while the group quantizes one row the next S - 1 rows are already on their
+// way from HBM; the group reads each row from shared memory twice, once for
+// the abs-max and once to quantize. Two persistent CTAs of 8 warps per SM. The
+// same kernel serves the activation quantizer, the weight quantizer, the
+// selector's fake-quantized copies (with the squared code norm as an extra
+// output) and the fused gather of the pruned sequence (rows addressed through
+// the kept indices, fp16 copy written beside the codes).
 #include <cuda_fp16.h>
+
+#include <algorithm>
 
 #include "p4q_device.cuh"
 #include "p4q_internal.h"
 
 namespace p4q {
+
+// Device error word of the quantizer (bounded waits on the row buffers).
+__device__ unsigned int g_quant_err;
+
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kWarps = 8;
+constexpr int kThreads = 32 * kWarps;
+constexpr int kCtasPerSm = 2;
+constexpr int kMaxStages = 16;
+constexpr uint32_t kStageBudget = 100u * 1024u;    // shared memory for row buffers per CTA
+constexpr uint32_t kInflightTarget = 48u * 1024u;  // bytes on their way per CTA (HBM latency x bandwidth share)
+constexpr int kSmemMax = 110 * 1024;
 
 // Codes of eight fp16 values (one 16-byte chunk), packed two per byte.
 //
@@ -31,7 +48,8 @@ constexpr int kThreads = 256;
 // constant 1.5 * 2^23: q + 1.5 * 2^23 rounds q to the nearest integer (ties
 // to even) and leaves its two's complement in the low mantissa bits, which
 // are the packed nibble. |x| <= max|x| bounds the codes to [-7, 7], so the
-// clamp to [-8, 7] cannot bind. Squares of the codes are added to n2.
+// clamp to [-8, 7] cannot bind. With NORM, squares of the codes are added to n2.
+template <bool NORM>
 __device__ __forceinline__ uint32_t quant_chunk(const uint4 v, float s, float inv, float2& n2) {
   const float2 inv2 = make_float2(inv, inv);
   const float2 mg = make_float2(12582912.0f, 12582912.0f);
@@ -59,100 +77,211 @@ __device__ __forceinline__ uint32_t quant_chunk(const uint4 v, float s, float in
       tb[2 * k + 1] = __float_as_uint(c[k].y + 12582912.0f);
     }
   }
+  if (NORM) {
 #pragma unroll
-  for (int k = 0; k < 4; ++k) n2 = __ffma2_rn(c[k], c[k], n2);
+    for (int k = 0; k < 4; ++k) n2 = __ffma2_rn(c[k], c[k], n2);
+  }
   // even-index codes in the low nibbles, odd-index codes in the high nibbles
   const uint32_t e = __byte_perm(__byte_perm(tb[0], tb[2], 0x0040), __byte_perm(tb[4], tb[6], 0x0040), 0x5410);
   const uint32_t o = __byte_perm(__byte_perm(tb[1], tb[3], 0x0040), __byte_perm(tb[5], tb[7], 0x0040), 0x5410);
   return (e & 0x0F0F0F0Fu) | ((o << 4) & 0xF0F0F0F0u);
 }
 
-// G warps quantize one row (8 / G rows per 256-thread CTA); each thread keeps
-// up to MAXC 16-byte chunks of its row in registers between the abs-max and
-// the quantization pass. Reductions are warp reductions, combined through
-// shared memory when G > 1.
-template <int G, int MAXC>
-__global__ void __launch_bounds__(kThreads) quant_rows_kernel(RowSource src, int rows, int L, RowSinks out) {
-  constexpr int kRowsPerCta = (kThreads / 32) / G;
-  constexpr int kRowThreads = 32 * G;
+__device__ __forceinline__ const uint16_t* row_ptr(const RowSource& src, int row, int L) {
+  if (src.idx == nullptr) return src.X + static_cast<size_t>(row) * L;
+  const int per = src.K + src.T;
+  const int b = row / per, r = row - b * per;
+  if (r < src.K) return src.X + (static_cast<size_t>(b) * src.N + src.idx[b * src.K + r]) * L;
+  return src.text + (static_cast<size_t>(b) * src.T + (r - src.K)) * L;
+}
+
+// Group g of CTA c takes rows first = c * kGroups + g, first + total, ...
+// (total = gridDim.x * kGroups). Per row j of the group: wait for its buffer,
+// abs-max pass, group reduction (named barrier when G > 1), quantize pass,
+// release of the buffer to the leader, which refills it with row j + S.
+// Waits are bounded; after a time-out the group keeps meeting its barriers
+// but skips the work, and the leader waits (bounded) for the copies it has
+// in flight before the CTA exits.
+template <int G, bool NORM>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+    quant_rows_kernel(RowSource src, int rows, int L, RowSinks out, int S, uint32_t stage_bytes) {
+  constexpr int kGroups = kWarps / G;
+  constexpr int kGroupThreads = 32 * G;
+  extern __shared__ __align__(128) unsigned char smem[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int slot = warp / G;                           // row slot inside the CTA
-  const int t = (warp % G) * 32 + lane;                // thread index inside the row
-  const int row = blockIdx.x * kRowsPerCta + slot;
-  const bool live = row < rows;
-  const uint16_t* srow = nullptr;
-  if (live) {
-    if (src.idx == nullptr) {
-      srow = src.X + static_cast<size_t>(row) * L;
-    } else {
-      const int per = src.K + src.T;
-      const int b = row / per, r = row - b * per;
-      if (r < src.K)
-        srow = src.X + (static_cast<size_t>(b) * src.N + src.idx[b * src.K + r]) * L;
-      else
-        srow = src.text + (static_cast<size_t>(b) * src.T + (r - src.K)) * L;
+  const int grp = warp / G;
+  const int gt = (warp % G) * 32 + lane;  // thread index inside the group
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(kGroups) * S * stage_bytes);
+  uint32_t* red = reinterpret_cast<uint32_t*>(bars + kGroups * kMaxStages);
+  int* red_n = reinterpret_cast<int*>(red + kWarps);
+  int* aborts = red_n + kWarps;
+  if (threadIdx.x < kGroups * S) mbar_init(&bars[threadIdx.x], 1);
+  if (threadIdx.x < kGroups) aborts[threadIdx.x] = 0;
+  fence_barrier_init();
+  __syncthreads();
+
+  unsigned char* ring = smem + static_cast<size_t>(grp) * S * stage_bytes;
+  uint64_t* full = bars + grp * S;
+  volatile int* abort = aborts + grp;
+  const int total = gridDim.x * kGroups;
+  const int first = blockIdx.x * kGroups + grp;
+  const int mine = rows > first ? (rows - first + total - 1) / total : 0;
+  const uint32_t row_bytes = 2u * static_cast<uint32_t>(L);
+  const int nch = L >> 3;  // 16-byte chunks per row
+  const bool leader = gt == 0;
+
+  int issued = 0;  // rows whose copy the leader has started
+  if (leader) {
+    for (; issued < S && issued < mine; ++issued) {
+      mbar_arrive_expect_tx(&full[issued], row_bytes);
+      bulk_load(ring + static_cast<size_t>(issued) * stage_bytes, row_ptr(src, first + issued * total, L), row_bytes,
+                &full[issued]);
     }
   }
-  const int nch = L >> 3;
-  const uint4* s4 = reinterpret_cast<const uint4*>(srow);
-
-  uint4 v[MAXC];
-  uint32_t m = 0;  // per-halfword max of |x| bit patterns (non-negative fp16 order as integers)
-#pragma unroll
-  for (int i = 0; i < MAXC; ++i) {
-    const int c = t + i * kRowThreads;
-    if (live && c < nch) {
-      v[i] = __ldg(s4 + c);
-      m = __vmaxu2(m, v[i].x & 0x7FFF7FFFu);
-      m = __vmaxu2(m, v[i].y & 0x7FFF7FFFu);
-      m = __vmaxu2(m, v[i].z & 0x7FFF7FFFu);
-      m = __vmaxu2(m, v[i].w & 0x7FFF7FFFu);
+  bool failed = false;
+  int consumed = 0;  // rows whose buffer this warp has seen complete
+  for (int j = 0; j < mine; ++j) {
+    const int st = j % S;
+    const int row = first + j * total;
+    if (!failed) {
+      failed = !mbar_wait_warp(&full[st], (j / S) & 1, abort, &g_quant_err);
+      if (!failed) consumed = j + 1;
     }
-  }
-  uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
-  __shared__ uint32_t red[kThreads / 32];
-  __shared__ int red_n[kThreads / 32];
-  if (G > 1) {
-    if (lane == 0) red[warp] = mm;
-    __syncthreads();
-#pragma unroll
-    for (int w = 0; w < G; ++w) mm = max(mm, red[slot * G + w]);
-  }
-  const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
-  const float s = __fdiv_rn(a, 7.0f);
-  const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
+    const uint4* v4 = reinterpret_cast<const uint4*>(ring + static_cast<size_t>(st) * stage_bytes);
 
-  float2 n2 = make_float2(0.0f, 0.0f);  // exact: sums of squared codes <= 49 * 16384 < 2^24
-  if (live) {
-    uint32_t* q4 = reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(row) * (L >> 1));
+    uint32_t m = 0;  // per-halfword max of |x| bit patterns (non-negative fp16 order as integers)
+    if (!failed) {
+#pragma unroll 4
+      for (int c = gt; c < nch; c += kGroupThreads) {
+        const uint4 v = v4[c];
+        m = __vmaxu2(m, v.x & 0x7FFF7FFFu);
+        m = __vmaxu2(m, v.y & 0x7FFF7FFFu);
+        m = __vmaxu2(m, v.z & 0x7FFF7FFFu);
+        m = __vmaxu2(m, v.w & 0x7FFF7FFFu);
+      }
+    }
+    uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+    if (G > 1) {
+      if (lane == 0) red[warp] = mm;
+      named_bar_sync(1 + grp, kGroupThreads);
 #pragma unroll
-    for (int i = 0; i < MAXC; ++i) {
-      const int c = t + i * kRowThreads;
-      if (c < nch) {
-        q4[c] = (a != 0.0f) ? quant_chunk(v[i], s, inv, n2) : 0u;
-        if (out.copy) reinterpret_cast<uint4*>(out.copy + static_cast<size_t>(row) * L)[c] = v[i];
+      for (int w = 0; w < G; ++w) mm = max(mm, red[grp * G + w]);
+    }
+    const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
+    const float s = __fdiv_rn(a, 7.0f);
+    const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
+
+    float2 n2 = make_float2(0.0f, 0.0f);  // exact: sums of squared codes <= 49 * 16384 < 2^24
+    if (!failed) {
+      uint32_t* q4 = reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(row) * (L >> 1));
+      uint4* cp = out.copy ? reinterpret_cast<uint4*>(out.copy + static_cast<size_t>(row) * L) : nullptr;
+#pragma unroll 4
+      for (int c = gt; c < nch; c += kGroupThreads) {
+        const uint4 v = v4[c];
+        q4[c] = (a != 0.0f) ? quant_chunk<NORM>(v, s, inv, n2) : 0u;
+        if (cp) cp[c] = v;
+      }
+    }
+    int wn = 0;
+    if (NORM) {
+      wn = __reduce_add_sync(0xFFFFFFFFu, static_cast<int>(n2.x + n2.y));
+      if (G > 1 && lane == 0) red_n[warp] = wn;
+    }
+    // every warp of the group is done with buffer st (and has published red_n)
+    if (G > 1)
+      named_bar_sync(1 + grp, kGroupThreads);
+    else
+      __syncwarp();
+    if (NORM && G > 1) {
+      wn = 0;
+#pragma unroll
+      for (int w = 0; w < G; ++w) wn += red_n[grp * G + w];
+    }
+    if (leader) {
+      if (!failed) {
+        out.scale[row] = (a != 0.0f) ? s : 0.0f;
+        if (NORM) out.norm2[row] = wn;
+        if (issued < mine) {
+          mbar_arrive_expect_tx(&full[st], row_bytes);
+          bulk_load(ring + static_cast<size_t>(st) * stage_bytes, row_ptr(src, first + issued * total, L), row_bytes,
+                    &full[st]);
+          ++issued;
+        }
       }
     }
   }
-  if (out.norm2) {
-    int wn = __reduce_add_sync(0xFFFFFFFFu, static_cast<int>(n2.x + n2.y));
-    if (G > 1) {
-      if (lane == 0) red_n[warp] = wn;
-      __syncthreads();
-      wn = 0;
-#pragma unroll
-      for (int w = 0; w < G; ++w) wn += red_n[slot * G + w];
-    }
-    if (live && t == 0) out.norm2[row] = wn;
+  if (leader && failed) {
+    // leave no copy in flight into this CTA's shared memory
+    int fresh = 0;
+    for (int j = consumed; j < issued; ++j)
+      mbar_wait(&full[j % S], (j / S) & 1, reinterpret_cast<volatile int*>(&fresh), &g_quant_err, 100000000ull);
   }
-  if (live && t == 0) out.scale[row] = (a != 0.0f) ? s : 0.0f;
 }
 
-template <int G, int MAXC>
-cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
-  constexpr int kRowsPerCta = (kThreads / 32) / G;
-  quant_rows_kernel<G, MAXC><<<(rows + kRowsPerCta - 1) / kRowsPerCta, kThreads, 0, stream>>>(src, rows, L, out);
+struct Plan {
+  int G, S;
+  uint32_t stage_bytes;
+};
+
+// Smallest group size whose ring keeps kInflightTarget bytes on their way
+// (groups x (S - 1) buffers), else the one that keeps the most.
+Plan plan_for(int L) {
+  const uint32_t sb = (2u * static_cast<uint32_t>(L) + 127u) & ~127u;
+  Plan best{kWarps, 2, sb};
+  uint64_t best_inflight = 0;
+  for (int G = 1; G <= kWarps; G *= 2) {
+    const int groups = kWarps / G;
+    const int S = std::min<int>(kMaxStages, static_cast<int>(kStageBudget / (groups * sb)));
+    if (S < 2) continue;
+    const uint64_t inflight = static_cast<uint64_t>(groups) * (S - 1) * sb;
+    if (inflight >= kInflightTarget) return Plan{G, S, sb};
+    if (inflight > best_inflight) {
+      best = Plan{G, S, sb};
+      best_inflight = inflight;
+    }
+  }
+  return best;
+}
+
+int sm_count() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
+  }
+  return n;
+}
+
+template <int G, bool NORM>
+cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out, const Plan& p,
+                     cudaStream_t stream) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(quant_rows_kernel<G, NORM>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemMax);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  constexpr int kGroups = kWarps / G;
+  const size_t smem = static_cast<size_t>(kGroups) * p.S * p.stage_bytes + kGroups * kMaxStages * 8 +
+                      2 * kWarps * 4 + kGroups * 4;
+  const int need = (rows + kGroups - 1) / kGroups;
+  const int grid = std::min(need, kCtasPerSm * sm_count());
+  quant_rows_kernel<G, NORM><<<grid, kThreads, smem, stream>>>(src, rows, L, out, p.S, p.stage_bytes);
   return cudaGetLastError();
+}
+
+template <bool NORM>
+cudaError_t launch_norm(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
+  const Plan p = plan_for(L);
+  switch (p.G) {
+    case 1: return launch_g<1, NORM>(src, rows, L, out, p, stream);
+    case 2: return launch_g<2, NORM>(src, rows, L, out, p, stream);
+    case 4: return launch_g<4, NORM>(src, rows, L, out, p, stream);
+    default: return launch_g<8, NORM>(src, rows, L, out, p, stream);
+  }
 }
 
 }  // namespace
@@ -160,11 +289,14 @@ cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out,
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
                               cudaStream_t stream) {
   if (rows <= 0) return cudaSuccess;
-  const int nch = L >> 3;  // 16-byte chunks per row
-  if (nch <= 32 * 8) return launch_g<1, 8>(src, rows, L, out, stream);    // L <= 2048
-  if (nch <= 32 * 20) return launch_g<1, 20>(src, rows, L, out, stream);  // L <= 5120
-  if (nch <= 128 * 8) return launch_g<4, 8>(src, rows, L, out, stream);   // L <= 8192
-  return launch_g<4, 16>(src, rows, L, out, stream);                      // L <= 16384
+  return out.norm2 ? launch_norm<true>(src, rows, L, out, stream) : launch_norm<false>(src, rows, L, out, stream);
+}
+
+unsigned int quant_read_and_clear_error() {
+  unsigned int v = 0, z = 0;
+  cudaMemcpyFromSymbol(&v, g_quant_err, sizeof(v));
+  cudaMemcpyToSymbol(g_quant_err, &z, sizeof(z));
+  return v;
 }
 
 }  // namespace p4q
