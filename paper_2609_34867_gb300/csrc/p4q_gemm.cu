@@ -503,31 +503,41 @@ constexpr int B_CONV = HB * BK;
 constexpr int CONV_STAGE = A_CONV + B_CONV;
 constexpr uint32_t TMEM_COLS = 2 * BN;
 
+constexpr int A_PACK = BM * BKP;            // packed A bytes per k-block (this CTA's rows)
+constexpr int PACK_STAGE = A_PACK + HB * BKP;  // packed A + B bytes per k-block
+constexpr int kProducerWarp = kFirstEpiWarp + kEpiWarps;
+constexpr int kPairThreads = (kProducerWarp + 1) * 32;
+
 template <int MODE>  // GemmOut::kHalf or kS32
 struct Lay {
   static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
   static constexpr int BOX_BYTES = 32 * 32 * ELEM;  // one 32 x 32 output box
+  // packed stages: a multiple of the unpack groups, so that each belongs to one group
+  static constexpr int P = (MODE == static_cast<int>(GemmOut::kHalf)) ? 4 : 2;
   static constexpr int FIXED = kEpiWarps * 2 * BOX_BYTES + 2 * kGroups * (BM + BN) * 4 + 2 * BN * 4 + 512;
-  static constexpr int SC_FIT = (232448 - 1024 - FIXED) / CONV_STAGE > 8 ? 8 : (232448 - 1024 - FIXED) / CONV_STAGE;
+  static constexpr int SC_ROOM = (232448 - 1024 - FIXED - P * PACK_STAGE) / CONV_STAGE;
+  static constexpr int SC_FIT = SC_ROOM > 8 ? 8 : SC_ROOM;
   static constexpr int SC = SC_FIT - SC_FIT % kGroups;
-  static constexpr int OFF_STAGE = SC * CONV_STAGE;
+  static constexpr int OFF_PACK = SC * CONV_STAGE;
+  static constexpr int OFF_STAGE = OFF_PACK + P * PACK_STAGE;
   static constexpr int OFF_SUMA = OFF_STAGE + kEpiWarps * 2 * BOX_BYTES;
   static constexpr int OFF_SUMB = OFF_SUMA + 2 * kGroups * BM * 4;
   static constexpr int OFF_SCOL = OFF_SUMB + 2 * kGroups * BN * 4;
   static constexpr int OFF_BAR = OFF_SCOL + 2 * BN * 4;
-  static constexpr int NBAR = 2 * SC + 8;
+  static constexpr int NBAR = 2 * SC + 8 + 2 * P;
   static constexpr int OFF_MISC = OFF_BAR + NBAR * 8;
   static constexpr int SMEM = 1024 + OFF_MISC + 16;
   static_assert(SC >= 2 && SC % kGroups == 0, "E4M3 stages");
+  static_assert(P >= 2 && P % kGroups == 0, "packed stages");
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
 template <int MODE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     w4a4_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                           const __grid_constant__ CUtensorMap tmD, const Params p) {
   using L = Lay<MODE>;
-  constexpr int SC = L::SC, BOX_BYTES = L::BOX_BYTES, OFF_STAGE = L::OFF_STAGE, OFF_SUMA = L::OFF_SUMA,
+  constexpr int SC = L::SC, P = L::P, BOX_BYTES = L::BOX_BYTES, OFF_STAGE = L::OFF_STAGE, OFF_SUMA = L::OFF_SUMA,
                 OFF_SUMB = L::OFF_SUMB, OFF_SCOL = L::OFF_SCOL, OFF_BAR = L::OFF_BAR, OFF_MISC = L::OFF_MISC;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -538,6 +548,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   uint64_t* acc_empty = acc_full + 2;   // [2] leader: both CTAs' epilogues -> MMA
   uint64_t* sums_full = acc_empty + 2;  // [2] both CTAs' unpack -> epilogue
   uint64_t* sums_empty = sums_full + 2; // [2] both CTAs' epilogues -> unpack
+  uint64_t* pack_full = sums_empty + 2; // [P] TMA of the packed operands -> unpack
+  uint64_t* pack_empty = pack_full + P; // [P] unpack (this CTA) -> producer
+  uint8_t* pack = smem + L::OFF_PACK;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + OFF_MISC + 4);
   int* sumA = reinterpret_cast<int*>(smem + OFF_SUMA);  // [2][kGroups][BM]
@@ -560,6 +573,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&acc_empty[i], 2 * kEpiWarps);
       mbar_init(&sums_full[i], 2 * kConvWarps);
       mbar_init(&sums_empty[i], 2 * kEpiWarps);
+    }
+    for (int i = 0; i < P; ++i) {
+      mbar_init(&pack_full[i], 1);
+      mbar_init(&pack_empty[i], kGroupWarps);  // the unpack warps of the stage's group
     }
     *abort_flag = 0;
     fence_barrier_init();
@@ -607,61 +624,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int cw = warp - kFirstConvWarp;
     const int grp = cw / kGroupWarps;
     const int tc = threadIdx.x - (kFirstConvWarp + grp * kGroupWarps) * 32;
-    constexpr int NA = BM * 4 / kGroupThreads, NB = HB * 4 / kGroupThreads, NT = NA + NB;
+    constexpr int NA = BM * 4 / kGroupThreads, NB = HB * 4 / kGroupThreads;
     const int rbase = tc >> 2, chunk = tc & 3;
-    const size_t rowbytes = static_cast<size_t>(p.K) >> 1;
-    const bool prefetcher = (tc == 0);
     const uint32_t full_c_leader = mapa_shared(smem_u32(full_c), 0);
-    if (prefetcher) {
-      tma_prefetch_desc(&tmA);
-      tma_prefetch_desc(&tmB);
-    }
     int gbase = 0, it = 0;
     bool ok = true;
     for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x(), ++it, gbase += KB) {
-      const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
-      const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
-      const int n0 = nb * BN + static_cast<int>(rank) * HB;                       // this CTA's B rows
-      const uint8_t* baseA = p.A + (static_cast<size_t>(bz) * p.a_bs + m0 + rbase) * rowbytes + chunk * 16;
-      const uint8_t* baseB = p.B + (static_cast<size_t>(bz) * p.b_bs + n0 + rbase) * rowbytes + chunk * 16;
-      const size_t step = static_cast<size_t>(kRowStep) * rowbytes;
-      uint32_t valid = 0;
-#pragma unroll
-      for (int j = 0; j < NA; ++j) valid |= (m0 + rbase + kRowStep * j < p.M) ? (1u << j) : 0u;
-#pragma unroll
-      for (int j = 0; j < NB; ++j) valid |= (n0 + rbase + kRowStep * j < p.N) ? (1u << (NA + j)) : 0u;
       const int kb0 = ((grp - gbase) % kGroups + kGroups) % kGroups;
-      if (prefetcher && grp == 0) {
-        for (int kb = 0; kb < min(KB, kPrefetchAhead); ++kb) {
-          tma_prefetch_l2_3d(&tmA, kb * BKP, m0, bz);
-          tma_prefetch_l2_3d(&tmB, kb * BKP, n0, bz);
-        }
-      }
       uint32_t accA[NA], accB[NB];
 #pragma unroll
       for (int j = 0; j < NA; ++j) accA[j] = 0;
 #pragma unroll
       for (int j = 0; j < NB; ++j) accB[j] = 0;
-      uint4 buf[2][NT];
-      auto load = [&](uint4 (&v)[NT], int kb) {
-        const size_t off = static_cast<size_t>(kb) * BKP;
-#pragma unroll
-        for (int j = 0; j < NA; ++j)
-          v[j] = (valid >> j) & 1u ? ldg_stream16(baseA + j * step + off) : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-        for (int j = 0; j < NB; ++j)
-          v[NA + j] = (valid >> (NA + j)) & 1u ? ldg_stream16(baseB + j * step + off) : make_uint4(0u, 0u, 0u, 0u);
-      };
-      auto convert = [&](const uint4 (&v)[NT], int kb) -> bool {
+      for (int kb = kb0; kb < KB; kb += kGroups) {
         const int g = gbase + kb;
-        const int c = g % SC;
-        if (prefetcher && grp == 0) {
-          for (int q = kb + kPrefetchAhead; q < min(KB, kb + kPrefetchAhead + kGroups); ++q) {
-            tma_prefetch_l2_3d(&tmA, q * BKP, m0, bz);
-            tma_prefetch_l2_3d(&tmB, q * BKP, n0, bz);
-          }
+        const int ps = g % P, c = g % SC;
+        // the packed k-block (TMA, this CTA's 128 A rows then 128 B rows of 64 bytes)
+        if (!mbar_wait_warp(&pack_full[ps], (g / P) & 1, abort_flag, &g_gemm_err)) {
+          ok = false;
+          break;
         }
-        if (!mbar_wait_warp(&empty_c[c], ((g / SC) & 1) ^ 1, abort_flag, &g_gemm_err)) return false;
+        const uint8_t* pk = pack + ps * PACK_STAGE + rbase * BKP + chunk * 16;
+        uint4 v[NA + NB];
+#pragma unroll
+        for (int j = 0; j < NA; ++j) v[j] = *reinterpret_cast<const uint4*>(pk + j * kRowStep * BKP);
+#pragma unroll
+        for (int j = 0; j < NB; ++j) v[NA + j] = *reinterpret_cast<const uint4*>(pk + A_PACK + j * kRowStep * BKP);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&pack_empty[ps]);
+        if (!mbar_wait_warp(&empty_c[c], ((g / SC) & 1) ^ 1, abort_flag, &g_gemm_err)) {
+          ok = false;
+          break;
+        }
         uint8_t* ca = smem + c * CONV_STAGE;
         uint8_t* cb = ca + A_CONV;
 #pragma unroll
@@ -671,18 +665,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive_remote(full_c_leader + 8u * c);  // the leader's full_c[c]
-        return true;
-      };
-      // Two of this group's k-blocks in flight in registers.
-      if (kb0 < KB) load(buf[0], kb0);
-      if (kb0 + kGroups < KB) load(buf[1], kb0 + kGroups);
-      for (int kb = kb0; kb < KB && ok; kb += 2 * kGroups) {
-        ok = convert(buf[0], kb);
-        if (!ok || kb + kGroups >= KB) break;
-        if (kb + 2 * kGroups < KB) load(buf[0], kb + 2 * kGroups);
-        ok = convert(buf[1], kb + kGroups);
-        if (!ok) break;
-        if (kb + 3 * kGroups < KB) load(buf[1], kb + 3 * kGroups);
       }
       if (!ok) break;
       // Row sums of u: A rows locally, B rows into this CTA's half of sumB in both CTAs.
@@ -710,6 +692,44 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (lane == 0) {
         mbar_arrive_remote(mapa_shared(smem_u32(&sums_full[ab]), rank));
         mbar_arrive_remote(mapa_shared(smem_u32(&sums_full[ab]), peer));
+      }
+    }
+  } else if (warp == kProducerWarp) {
+    // ------------------------------------------------------------ producer: packed operands by TMA
+    if (lane == 0) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+      int g = 0;
+      bool ok = true;
+      for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x()) {
+        const int bz = t / per, r = t - bz * per, nb = r / p.num_m;
+        const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
+        const int n0 = nb * BN + static_cast<int>(rank) * HB;                       // this CTA's B rows
+        for (int kb = 0; kb < min(KB, kPrefetchAhead); ++kb) {
+          tma_prefetch_l2_3d(&tmA, kb * BKP, m0, bz);
+          tma_prefetch_l2_3d(&tmB, kb * BKP, n0, bz);
+        }
+        for (int kb = 0; kb < KB; ++kb, ++g) {
+          if (kb + kPrefetchAhead < KB) {
+            tma_prefetch_l2_3d(&tmA, (kb + kPrefetchAhead) * BKP, m0, bz);
+            tma_prefetch_l2_3d(&tmB, (kb + kPrefetchAhead) * BKP, n0, bz);
+          }
+          const int ps = g % P;
+          if (!mbar_wait(&pack_empty[ps], ((g / P) & 1) ^ 1, abort_flag, &g_gemm_err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&pack_full[ps], PACK_STAGE);
+          tma_load_3d(&tmA, &pack_full[ps], pack + ps * PACK_STAGE, kb * BKP, m0, bz);
+          tma_load_3d(&tmB, &pack_full[ps], pack + ps * PACK_STAGE + A_PACK, kb * BKP, n0, bz);
+        }
+      }
+      if (!ok) {
+        // leave no TMA load in flight into this CTA's shared memory
+        int fresh = 0;
+        for (int j = (g > P ? g - P : 0); j < g; ++j)
+          mbar_wait(&pack_full[j % P], (j / P) & 1, reinterpret_cast<volatile int*>(&fresh), &g_gemm_err,
+                    100000000ull);
       }
     }
   } else {
@@ -964,7 +984,7 @@ cudaError_t launch_pair(const GemmArgs& g, cudaStream_t stream) {
   p.norm_a = g.norm_a;
   p.norm_b = g.norm_b;
   const int pairs = p.tiles < num_sms() / 2 ? p.tiles : num_sms() / 2;
-  pair::w4a4_gemm_pair_kernel<MODE><<<2 * pairs, kThreads, pair::Lay<MODE>::SMEM, stream>>>(ma, mb, md, p);
+  pair::w4a4_gemm_pair_kernel<MODE><<<2 * pairs, pair::kPairThreads, pair::Lay<MODE>::SMEM, stream>>>(ma, mb, md, p);
   return cudaGetLastError();
 }
 
