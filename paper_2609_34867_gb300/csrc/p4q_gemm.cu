@@ -496,6 +496,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ============================================================================
 namespace pair {
 
+// Pipeline shape of the pair kernel (compile-time; the defaults measured
+// best on GB300): unpack groups (each converts every kGroups-th k-block),
+// packed TMA stages, and the k-blocks prefetched into L2 ahead of them.
+#ifndef P4Q_PAIR_GROUPS
+#define P4Q_PAIR_GROUPS 2
+#endif
+#ifndef P4Q_PAIR_PACK
+#define P4Q_PAIR_PACK 4
+#endif
+#ifndef P4Q_PAIR_PREFETCH
+#define P4Q_PAIR_PREFETCH 6
+#endif
+constexpr int kPrefetchAhead = P4Q_PAIR_PREFETCH;  // k-blocks prefetched into L2 ahead of the TMA loads
+constexpr int kGroups = P4Q_PAIR_GROUPS;
+constexpr int kGroupWarps = kConvWarps / kGroups;
+constexpr int kGroupThreads = kGroupWarps * 32;
+constexpr int kRowStep = kGroupThreads / 4;
+
 constexpr int BN = 256;      // output columns per pair
 constexpr int HB = BN / 2;   // B rows unpacked per CTA
 constexpr int A_CONV = BM * BK;
@@ -513,7 +531,7 @@ struct Lay {
   static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
   static constexpr int BOX_BYTES = 32 * 32 * ELEM;  // one 32 x 32 output box
   // packed stages: a multiple of the unpack groups, so that each belongs to one group
-  static constexpr int P = (MODE == static_cast<int>(GemmOut::kHalf)) ? 4 : 2;
+  static constexpr int P = (MODE == static_cast<int>(GemmOut::kHalf)) ? P4Q_PAIR_PACK : 2;
   static constexpr int FIXED = kEpiWarps * 2 * BOX_BYTES + 2 * kGroups * (BM + BN) * 4 + 2 * BN * 4 + 512;
   static constexpr int SC_ROOM = (232448 - 1024 - FIXED - P * PACK_STAGE) / CONV_STAGE;
   static constexpr int SC_FIT = SC_ROOM > 8 ? 8 : SC_ROOM;
