@@ -5,9 +5,11 @@ One step = the whole path over one batch of the LLaVA-1.5-7B-shaped workload
 budget 192 kept tokens per image):
   p4q_select_gather_quant  fake-quant -> query / saliency / diversity stages
                            -> gather of the kept FP16 rows + text -> INT4
-  p4q_w4a4_linear x 7      q, k, v, gate, up on the pruned sequence (M = 2048),
-                           o on the re-quantized q output, down on the
-                           re-quantized up output (2 x p4q_quant_act).
+  p4q_w4a4_linear x 4      q|k|v and gate|up (each one GEMM over the
+                           concatenated output channels) on the pruned
+                           sequence (M = 2048), o on the re-quantized q
+                           output, down on the re-quantized up output
+                           (2 x p4q_quant_act_ld on column blocks).
 The metric is W4A4 linear TOPS: 2 * M * N * K integer ops of the seven linears
 per step divided by the step time (the selector's time included); the
 selector's share is also reported as microseconds per image.
@@ -172,8 +174,12 @@ class Step:
     wl.weight_seed(w.seed + l, linear id), the same on every rank (replicated
     weights, independent batches). Every layer runs on the pruned sequence:
     q, k, v, gate, up on its INT4 codes, o on the re-quantized q output, down
-    on the re-quantized up output."""
+    on the re-quantized up output. Linears that read the same input run as one
+    GEMM over their concatenated output channels (q|k|v and gate|up), which
+    computes exactly the same outputs (the weight quantizer works per output
+    channel) with fewer launches and fuller waves of tiles."""
 
+    FUSE = (("qkv", ("q", "k", "v")), ("gate_up", ("gate", "up")))
     REQUANT = {"o": "q", "down": "up"}  # linear -> the linear whose output it re-quantizes
 
     def __init__(self, w: wl.Workload, dev, seed: int):
@@ -193,14 +199,32 @@ class Step:
         M = w.M
         self.Xq = torch.empty((M, d // 2), dtype=torch.uint8, device=dev)
         self.s_a = torch.empty((M,), dtype=torch.float32, device=dev)
-        self.Wq, self.s_w = {}, {}
-        for layer in range(w.layers):
-            for lid, lin in enumerate(w.linears):
-                W = torch.from_numpy(wl.weight(lin.k_in, lin.n_out, wl.weight_seed(w.seed + layer, lid))).to(dev)
-                self.Wq[layer, lin.name], self.s_w[layer, lin.name] = p4q.quant_weight(W)
-                del W
-        self.Y = {lin.name: torch.empty((M, lin.n_out), dtype=torch.float16, device=dev) for lin in w.linears}
         dims = {l.name: l for l in w.linears}
+        lid = {l.name: i for i, l in enumerate(w.linears)}
+        # GEMMs: fused groups whose members all exist and share k_in, else single linears
+        self.gemms, taken = [], set()
+        for gname, members in self.FUSE:
+            if all(m in dims for m in members) and len({dims[m].k_in for m in members}) == 1:
+                self.gemms.append((gname, members))
+                taken.update(members)
+        for l in w.linears:
+            if l.name not in taken:
+                self.gemms.append((l.name, (l.name,)))
+        self.col = {}  # linear -> (gemm, first output column, width)
+        for gname, members in self.gemms:
+            off = 0
+            for m in members:
+                self.col[m] = (gname, off, dims[m].n_out)
+                off += dims[m].n_out
+        self.Wq, self.s_w, self.Y = {}, {}, {}
+        for gname, members in self.gemms:
+            n_out = sum(dims[m].n_out for m in members)
+            self.Y[gname] = torch.empty((M, n_out), dtype=torch.float16, device=dev)
+            for layer in range(w.layers):
+                W = torch.cat([torch.from_numpy(wl.weight(dims[m].k_in, dims[m].n_out,
+                                                          wl.weight_seed(w.seed + layer, lid[m]))) for m in members])
+                self.Wq[layer, gname], self.s_w[layer, gname] = p4q.quant_weight(W.to(dev))
+                del W
         self.Xq_re, self.s_re = {}, {}
         for name, src in self.REQUANT.items():
             if name in dims:
@@ -208,31 +232,43 @@ class Step:
                 self.Xq_re[name] = torch.empty((M, dims[name].k_in // 2), dtype=torch.uint8, device=dev)
                 self.s_re[name] = torch.empty((M,), dtype=torch.float32, device=dev)
         self.out_name = w.linears[-1].name
-        # The step is a chain of segments (selector, each linear, each
+        # The step is a chain of segments (selector, each GEMM, each
         # re-quantization) captured as one CUDA graph each, so that events
-        # recorded between the replays time the selector and every linear.
+        # recorded between the replays time the selector and every GEMM.
         self.segments = [("select", "select", self._select)]
         for layer in range(w.layers):
-            for lin in w.linears:
-                if lin.name not in self.REQUANT:
-                    self.segments.append(("linear", lin.name, (lambda l=layer, n=lin.name: self._lin(l, n, self.Xq, self.s_a))))
-            for name, src in self.REQUANT.items():
-                if name in dims:
-                    self.segments.append(("quant", "quant_" + name, (lambda n=name, s=src: p4q.p4q_quant_act(
-                        self.Y[s], self.Xq_re[n], self.s_re[n]))))
-                    self.segments.append(("linear", name, (lambda l=layer, n=name: self._lin(
-                        l, n, self.Xq_re[n], self.s_re[n]))))
-        self.lin_ops = {l.name: 2 * w.M * l.n_out * l.k_in * w.layers for l in w.linears}
+            for gname, members in self.gemms:
+                if members[0] in self.REQUANT:
+                    name = members[0]
+                    self.segments.append(("quant", "quant_" + name, (lambda n=name: p4q.p4q_quant_act_ld(
+                        self.output(self.REQUANT[n]), self.Xq_re[n], self.s_re[n]))))
+                    self.segments.append(("linear", gname, (lambda l=layer, g=gname, n=name: self._gemm(
+                        l, g, self.Xq_re[n], self.s_re[n]))))
+                else:
+                    self.segments.append(("linear", gname, (lambda l=layer, g=gname: self._gemm(
+                        l, g, self.Xq, self.s_a))))
+        self.lin_ops = {g: sum(2 * w.M * dims[m].n_out * dims[m].k_in for m in members) * w.layers
+                        for g, members in self.gemms}
         self.graphs = None
         self.launches_per_step = None
         self.events = [torch.cuda.Event(enable_timing=True) for _ in range(len(self.segments) + 1)]
+
+    def output(self, name):
+        """The [M, n_out] output of one linear (a column block of its GEMM's output)."""
+        g, off, n = self.col[name]
+        return self.Y[g][:, off:off + n]
+
+    def weight(self, layer, name):
+        """The packed INT4 rows and scales of one linear inside its GEMM's weight."""
+        g, off, n = self.col[name]
+        return self.Wq[layer, g][off:off + n], self.s_w[layer, g][off:off + n]
 
     def _select(self):
         self.p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
                                          self.s_a, self.ws)
 
-    def _lin(self, layer, name, Xq, s):
-        self.p4q.p4q_w4a4_linear(Xq, s, self.Wq[layer, name], self.s_w[layer, name], self.Y[name])
+    def _gemm(self, layer, gname, Xq, s):
+        self.p4q.p4q_w4a4_linear(Xq, s, self.Wq[layer, gname], self.s_w[layer, gname], self.Y[gname])
 
     def body(self):
         """The step as plain C-ABI calls (no graph)."""
@@ -264,8 +300,8 @@ class Step:
 
     def kernel_times(self):
         """Milliseconds of the most recent graph step (after a sync):
-        {"select": ms, "quant": ms summed, "linear": {name: ms summed over layers}}."""
-        out = {"select": 0.0, "quant": 0.0, "linear": {l.name: 0.0 for l in self.w.linears}}
+        {"select": ms, "quant": ms summed, "linear": {gemm: ms summed over layers}}."""
+        out = {"select": 0.0, "quant": 0.0, "linear": {g: 0.0 for g, _ in self.gemms}}
         for i, (kind, name, _) in enumerate(self.segments):
             ms = self.events[i].elapsed_time(self.events[i + 1])
             if kind == "linear":
@@ -307,7 +343,7 @@ def run_gpu(args, rank, world, local_rank):
     clocks = ClockSampler(int(os.environ.get("P4Q_NVSMI_INDEX", local_rank)))
     e_start = torch.cuda.Event(enable_timing=True)
     e_end = torch.cuda.Event(enable_timing=True)
-    step_ms, sel_ms, gemm_ms = [], [], {l.name: [] for l in w.linears}
+    step_ms, sel_ms, gemm_ms = [], [], {g: [] for g, _ in step.gemms}
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -344,7 +380,7 @@ def run_gpu(args, rank, world, local_rank):
         hostQ = torch.from_numpy(step.host["Q"]).pin_memory()
         hostA = torch.from_numpy(step.host["A"]).pin_memory()
         hostT = torch.from_numpy(step.host["text"]).pin_memory()
-        outY = torch.empty(step.Y[step.out_name].shape, dtype=torch.float16).pin_memory()
+        outY = torch.empty(step.output(step.out_name).shape, dtype=torch.float16).pin_memory()
         outI = torch.empty(step.idx.shape, dtype=torch.int32).pin_memory()
         h2d = sum(t.numel() * t.element_size() for t in (hostV, hostQ, hostA, hostT))
         d2h = outY.numel() * 2 + outI.numel() * 4
@@ -360,7 +396,7 @@ def run_gpu(args, rank, world, local_rank):
             step.A.copy_(hostA, non_blocking=True)
             step.text.copy_(hostT, non_blocking=True)
             step.body()  # the C-ABI calls themselves, no graph
-            outY.copy_(step.Y[step.out_name], non_blocking=True)
+            outY.copy_(step.output(step.out_name), non_blocking=True)
             outI.copy_(step.idx, non_blocking=True)
             b.record()
             torch.cuda.synchronize()
@@ -380,7 +416,7 @@ def run_gpu(args, rank, world, local_rank):
     sustained = bool(clk and "sw_power_cap" in clk["reasons"])
     peak, peak_src = fp8_peak_tops(sustained)
     ach = gemm_ops / (gemm_time_ms * 1e-3) / 1e12
-    n_gemm = len(step.lin_ops) * w.layers * args.steps
+    n_gemm = len(step.gemms) * w.layers * args.steps
     traffic = None
     if PROFILED_GEMM["source_sha1"] == gemm_source_sha1():
         traffic = PROFILED_GEMM["dram_bytes_per_launch"]
@@ -400,6 +436,7 @@ def run_gpu(args, rank, world, local_rank):
         "config": {
             "workload": w.name, "B": w.B, "N": w.N, "d": w.d, "K": w.K, "T": w.T, "J": w.J, "M": w.M,
             "linears": "; ".join(f"{l.name} {l.k_in}->{l.n_out}" for l in w.linears), "layers": w.layers,
+            "gemms": "; ".join(f"{g}={'|'.join(m)}" for g, m in step.gemms),
             "alpha_beta_gamma": "0.3/0.2/0.5", "l2": "flushed before every timed step: 512 MiB written, then another 512 MiB read (no dirty flush lines left to write back inside the timed region)",
             "timing": "CUDA events around each step (graph replays), summed over the K steps",
             "parallelism": f"dp{world} (independent batches)"},
@@ -412,7 +449,7 @@ def run_gpu(args, rank, world, local_rank):
                      "frac": round(ach / peak, 4), "traffic": traffic, "peak_source": peak_src,
                      "launches_timed": n_gemm,
                      "note": "integer ops on the FP8 tensor pipe; sm_103a has no integer tcgen05 MMA kind",
-                     "per_linear_us": {n: round(float(np.mean(v)) * 1e3, 2) for n, v in gemm_ms.items()}},
+                     "per_gemm_us": {n: round(float(np.mean(v)) * 1e3, 2) for n, v in gemm_ms.items()}},
         "gpu_launches": int(launches),
         "launch": "%d CUDA graph replays per step (%d kernels of libp4q per step)" % (
             len(step.graphs), step.launches_per_step),

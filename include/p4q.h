@@ -121,6 +121,14 @@ p4q_status p4q_test_wait_timeout(uint32_t limit_us, p4q_stream_t stream);
 p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* s_a,
                          p4q_stream_t stream);
 
+/* p4q_quant_act on rows that lie ldx elements apart: row m of X starts at
+ * X + m * ldx (a column block of a wider matrix, e.g. the q part of a fused
+ * q/k/v output). Same computation and outputs (Xq and s_a stay dense).
+ * Requires ldx >= Kin and ldx % 8 == 0 (16-byte aligned rows); otherwise as
+ * p4q_quant_act. */
+p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
+                            p4q_stream_t stream);
+
 /* Per-output-channel weight quantization (App. B.3: symmetric, per output
  * channel, then round-to-nearest): the same per-row quantizer applied to each
  * output row of W.

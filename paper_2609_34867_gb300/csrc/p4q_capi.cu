@@ -174,11 +174,20 @@ p4q_status p4q_test_wait_timeout(uint32_t limit_us, p4q_stream_t stream) {
 }
 
 p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* s_a, p4q_stream_t stream) {
+  return p4q_quant_act_ld(X, Kin, M, Kin, Xq, s_a, stream);
+}
+
+p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
+                            p4q_stream_t stream) {
   p4q_status st = check_rows(X, M, Kin, Xq, s_a);
-  if (st != P4Q_OK || M == 0) return st;
+  if (st != P4Q_OK) return st;
+  if (ldx < Kin) return P4Q_ERR_INVALID_ARG;
+  if (ldx % 8 != 0) return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
   if ((st = check_device()) != P4Q_OK) return st;
   RowSource src;
   src.X = X;
+  src.ldx = ldx;
   RowSinks o;
   o.codes = Xq;
   o.scale = s_a;

@@ -12,6 +12,7 @@ namespace p4q {
 // or the pruned sequence of the selector (kept visual rows, then text rows).
 struct RowSource {
   const uint16_t* X = nullptr;     // dense source, or V [B, N, L] when idx != nullptr
+  long long ldx = 0;               // dense mode: elements between rows (0: L)
   const int32_t* idx = nullptr;    // [B, K] kept indices (gather mode)
   const uint16_t* text = nullptr;  // [B, T, L] (gather mode)
   int N = 0, K = 0, T = 0;         // gather mode sizes

@@ -88,7 +88,7 @@ __device__ __forceinline__ uint32_t quant_chunk(const uint4 v, float s, float in
 }
 
 __device__ __forceinline__ const uint16_t* row_ptr(const RowSource& src, int row, int L) {
-  if (src.idx == nullptr) return src.X + static_cast<size_t>(row) * L;
+  if (src.idx == nullptr) return src.X + static_cast<size_t>(row) * (src.ldx > 0 ? src.ldx : L);
   const int per = src.K + src.T;
   const int b = row / per, r = row - b * per;
   if (r < src.K) return src.X + (static_cast<size_t>(b) * src.N + src.idx[b * src.K + r]) * L;

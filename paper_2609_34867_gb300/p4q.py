@@ -53,6 +53,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_test_wait_timeout.restype = st
         L.p4q_quant_act.argtypes = [P, I, I, P, P, P]
         L.p4q_quant_act.restype = st
+        L.p4q_quant_act_ld.argtypes = [P, I, I, I, P, P, P]
+        L.p4q_quant_act_ld.restype = st
         L.p4q_quant_weight.argtypes = [P, I, I, P, P, P]
         L.p4q_quant_weight.restype = st
         L.p4q_w4a4_linear.argtypes = [P, P, I, I, P, P, I, P, P]
@@ -115,6 +117,17 @@ def p4q_quant_act(X, Xq, s_a, stream=None):
     _need(X, torch.float16, 2, "X"); _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
     M, K = X.shape
     _check(lib().p4q_quant_act(_ptr(X), M, K, _ptr(Xq), _ptr(s_a), _stream(stream)), "p4q_quant_act")
+
+
+def p4q_quant_act_ld(X, Xq, s_a, stream=None):
+    """p4q_quant_act on a row-strided 2-D view X (unit column stride, rows
+    X.stride(0) elements apart), e.g. a column block of a fused output."""
+    if not isinstance(X, torch.Tensor) or X.dtype != torch.float16 or X.dim() != 2 or X.stride(1) != 1 or not X.is_cuda:
+        raise TypeError("X: expected a CUDA fp16 2-D tensor with unit column stride")
+    _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    M, K = X.shape
+    _check(lib().p4q_quant_act_ld(_ptr(X), X.stride(0), M, K, _ptr(Xq), _ptr(s_a), _stream(stream)),
+           "p4q_quant_act_ld")
 
 
 def p4q_quant_weight(W, Wq, s_w, stream=None):

@@ -92,3 +92,11 @@ def test_wait_timeout_test_entry_validates_its_limit(lib):
     lib.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, ctypes.c_void_p]
     assert lib.p4q_test_wait_timeout(0, None) == 1
     assert lib.p4q_test_wait_timeout(1000001, None) == 1
+
+
+def test_strided_quantizer_validates_its_row_pitch(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_quant_act_ld.argtypes = [P, I, I, I, P, P, P]
+    assert lib.p4q_quant_act_ld(P(16), 64, 4, 128, P(16), P(16), None) == 1   # pitch below the row length
+    assert lib.p4q_quant_act_ld(P(16), 132, 4, 128, P(16), P(16), None) == 3  # rows not 16-byte aligned
+    assert lib.p4q_quant_act_ld(None, 128, 0, 128, None, None, None) == 0     # empty is a no-op

@@ -2,8 +2,10 @@
 configuration bench.py times.
 
 Each test builds bench.Step for the workload (p4q_select_gather_quant with a
-caller workspace, the W4A4 linears on the pruned sequence, the
-re-quantizations that feed o and down), runs it once as plain calls, captures
+caller workspace, the W4A4 linears on the pruned sequence with q|k|v and
+gate|up each run as one GEMM over their concatenated output channels, the
+re-quantizations of column blocks that feed o and down), runs it once as
+plain calls, captures
 it as CUDA graphs, clears every output and replays the graphs once: the
 outputs checked are those of the replay.
 
@@ -78,9 +80,10 @@ def check_step(step, w, images, rows):
     for lid, lin in enumerate(w.linears):
         W = wl.weight(lin.k_in, lin.n_out, wl.weight_seed(w.seed + layer, lid))
         cw, sw = oracle.quantize_rows(W)
-        assert_codes_equal(step.Wq[layer, lin.name].cpu().numpy(), step.s_w[layer, lin.name].cpu().numpy(), cw, sw)
+        Wq, s_w = step.weight(layer, lin.name)
+        assert_codes_equal(Wq.cpu().numpy(), s_w.cpu().numpy(), cw, sw)
         if lin.name in step.REQUANT:
-            Yin = step.Y[step.REQUANT[lin.name]]
+            Yin = step.output(step.REQUANT[lin.name])
             every = Yin.numel() <= (64 << 20)
             r = np.arange(w.M) if every else rows
             cq, sq = oracle.quantize_rows(take(Yin, r))
@@ -88,7 +91,7 @@ def check_step(step, w, images, rows):
             a, s = (cq[rows], sq[rows]) if every else (cq, sq)
         else:
             a, s = ca[rows], sa[rows]
-        assert_close(take(step.Y[lin.name], rows), oracle.linear(a, s, cw, sw))
+        assert_close(take(step.output(lin.name), rows), oracle.linear(a, s, cw, sw))
 
 
 def test_one_image_576_to_64(run_step):

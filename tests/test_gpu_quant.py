@@ -77,3 +77,18 @@ def test_quant_rows_full_of_exact_ties(p4q, dev):
     x[32:] *= np.float32(2.0 ** -3)    # s = 2^-3
     x[48:, 1:] = np.nextafter(x[48:, 1:], np.float32(np.inf))  # just off the boundaries
     _check(p4q, dev, x.astype(np.float16))
+
+
+def test_quant_act_on_a_column_block_matches_dense(p4q, dev):
+    """p4q_quant_act_ld on the middle column block of a wider matrix equals
+    p4q_quant_act on a dense copy of that block (and the oracle)."""
+    X = torch.from_numpy(wl.activations(300, 3 * 1024, seed=21)).to(dev)
+    block = X[:, 1024:2048]
+    Xq = torch.empty((300, 512), dtype=torch.uint8, device=dev)
+    s = torch.empty((300,), dtype=torch.float32, device=dev)
+    p4q.p4q_quant_act_ld(block, Xq, s)
+    ref_q, ref_s = p4q.quant_act(block.contiguous())
+    torch.cuda.synchronize()
+    assert torch.equal(Xq, ref_q) and torch.equal(s.view(torch.int32), ref_s.view(torch.int32))
+    c, sc = oracle.quantize_rows(block.cpu().numpy())
+    assert np.array_equal(oracle.unpack_codes(Xq.cpu().numpy()), c)
