@@ -107,13 +107,19 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     g.batch = B;
     g.a_batch_stride = N;
     g.b_batch_stride = N;
-    g.out = GemmOut::kCos;
     g.D = w.gram;
     g.d_pitch = w.gram_pitch;
     g.norm_a = w.vnorm;
     g.norm_b = w.vnorm;
+    // Large token sets: exact int32 dot products on the CTA-pair GEMM, then
+    // the cosine of every entry by a full-GPU elementwise pass (the division
+    // and square root would otherwise serialize in the GEMM's four epilogue
+    // warps). Small ones: the cosine epilogue of the single-CTA GEMM.
+    const bool split = N >= 256;
+    g.out = split ? GemmOut::kS32 : GemmOut::kCos;
     e = counted(launch_w4a4_gemm(g, stream));
     if (e != cudaSuccess) return from_cuda(e);
+    if (split && (e = counted(launch_gram_cos(plan, w, stream))) != cudaSuccess) return from_cuda(e);
   }
   return from_cuda(counted(launch_select_stages(plan, w, A_cls, idx, stream)));
 }

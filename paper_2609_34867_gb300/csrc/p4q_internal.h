@@ -76,6 +76,8 @@ struct SelectWorkspace {
 size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, void* base);
 
 cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+// In place: the int32 dot products of ws.gram become the cosines of Eq. 4.
+cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls,
                                  int32_t* idx, cudaStream_t stream);
 

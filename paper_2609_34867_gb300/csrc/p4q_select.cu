@@ -11,13 +11,15 @@
 //   query_scores_kernel   one warp per visual token: signed integer dot
 //                         products (dp4a on sign-extended nibbles) with the J
 //                         concept codes, then the cosine per concept.
-//   select_stages_kernel  one 1024-thread CTA per image: stage 1 (per-concept
+//   select_stages_kernel  one CTA per image, one thread per 4 tokens: stage 1 (per-concept
 //                         top quota), stage 2 (CLS-saliency top K_s), stage 3
 //                         (greedy max-min diversity on the cosine matrix of
 //                         the image, computed beforehand on the tensor cores),
 //                         then the kept set in ascending order.
 // Every ranking orders by (score, lower token index first).
 #include <cuda_fp16.h>
+
+#include <algorithm>
 
 #include "p4q.h"
 #include "p4q_device.cuh"
@@ -97,8 +99,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
   }
 }
 
-constexpr int kSelThreads = 1024;
-constexpr int kSelWarps = kSelThreads / 32;
+constexpr int kSelThreads = 1024;  // upper bound; launches use ceil(N / kPer) threads rounded to warps
 constexpr int kPer = 4;  // tokens per thread: token i = kPer * threadIdx.x + e
 
 struct BlockScratch {
@@ -122,7 +123,7 @@ __device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
   if (lane == 31) s.wsum[warp] = x;
   __syncthreads();
   if (warp == 0) {
-    int w = s.wsum[lane];
+    int w = lane < static_cast<int>(blockDim.x >> 5) ? s.wsum[lane] : 0;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xFFFFFFFFu, w, o);
@@ -132,7 +133,7 @@ __device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
   }
   __syncthreads();
   const int before = (warp ? s.wsum[warp - 1] : 0) + x - v;
-  *total = s.wsum[31];
+  *total = s.wsum[(blockDim.x >> 5) - 1];
   __syncthreads();
   return before;
 }
@@ -310,7 +311,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
         s.widx[slot][warp] = wi;
       }
       __syncthreads();
-      const uint32_t ck = s.wkey[slot][lane], ci = s.widx[slot][lane];
+      const bool have = lane < static_cast<int>(blockDim.x >> 5);
+      const uint32_t ck = have ? s.wkey[slot][lane] : 0xFFFFFFFFu, ci = have ? s.widx[slot][lane] : 0xFFFFFFFFu;
       wk = __reduce_min_sync(0xFFFFFFFFu, ck);
       wi = __reduce_min_sync(0xFFFFFFFFu, ck == wk ? ci : 0xFFFFFFFFu);
       const int pick = static_cast<int>(wi);
@@ -369,6 +371,37 @@ cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, 
   return cudaGetLastError();
 }
 
+namespace {
+
+// Row (b, i) of the Gram buffer, four entries per thread: int32 dot products
+// in, the cosines out (same bits as the cosine epilogue of the GEMM).
+__global__ void __launch_bounds__(128) gram_cos_kernel(float* __restrict__ gram, const int32_t* __restrict__ norm,
+                                                       int N, int gp) {
+  const int row = blockIdx.x;  // b * N + i
+  const int j0 = 4 * (blockIdx.y * blockDim.x + threadIdx.x);
+  if (j0 >= N) return;
+  const int b = row / N;
+  const int na = norm[row];
+  int4* cell = reinterpret_cast<int4*>(gram + static_cast<size_t>(row) * gp + j0);
+  const int4 d = *cell;
+  const int32_t* nr = norm + static_cast<size_t>(b) * N;
+  float4 c;
+  c.x = code_cosine(d.x, na, nr[j0]);
+  c.y = (j0 + 1 < N) ? code_cosine(d.y, na, nr[j0 + 1]) : 0.0f;
+  c.z = (j0 + 2 < N) ? code_cosine(d.z, na, nr[j0 + 2]) : 0.0f;
+  c.w = (j0 + 3 < N) ? code_cosine(d.w, na, nr[j0 + 3]) : 0.0f;
+  *reinterpret_cast<float4*>(cell) = c;
+}
+
+}  // namespace
+
+cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
+  const int per_row = (p.N + 3) / 4;
+  const dim3 grid(p.B * p.N, (per_row + 127) / 128);
+  gram_cos_kernel<<<grid, 128, 0, stream>>>(ws.gram, ws.vnorm, p.N, ws.gram_pitch);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls, int32_t* idx,
                                  cudaStream_t stream) {
   static bool attr_set = false;
@@ -378,7 +411,9 @@ cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws,
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  select_stages_kernel<<<p.B, kSelThreads, smem, stream>>>(ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J,
+  // one thread per kPer tokens: idle threads would only add instructions to every round
+  const int threads = std::min(kSelThreads, ((p.N + kPer - 1) / kPer + 31) / 32 * 32);
+  select_stages_kernel<<<p.B, threads, smem, stream>>>(ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J,
                                                            p.K, p.Kq, p.Ks, p.Kd, idx);
   return cudaGetLastError();
 }
