@@ -526,7 +526,7 @@ constexpr int PACK_STAGE = A_PACK + HB * BKP;  // packed A + B bytes per k-block
 constexpr int kProducerWarp = kFirstEpiWarp + kEpiWarps;
 constexpr int kPairThreads = (kProducerWarp + 1) * 32;
 
-template <int MODE>  // GemmOut::kHalf, kS32 or kCos
+template <int MODE>  // GemmOut::kHalf or kS32
 struct Lay {
   static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
   static constexpr int BOX_BYTES = 32 * 32 * ELEM;  // one 32 x 32 output box
@@ -778,8 +778,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
           for (int q2 = 0; q2 < kGroups; ++q2) v += sumB[(ab * kGroups + q2) * BN + i];
           sbw[i] = static_cast<float>(-8 * v);
           if (MODE == static_cast<int>(GemmOut::kHalf)) colv[i] = (n0 + i < p.N) ? p.s_b[n0 + i] : 0.0f;
-          if (MODE == static_cast<int>(GemmOut::kCos))
-            colv[i] = (n0 + i < p.N) ? static_cast<float>(p.norm_b[static_cast<size_t>(bz) * p.N + n0 + i]) : 0.0f;
         }
       }
       epi_sync();
@@ -789,7 +787,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       for (int q2 = 0; q2 < kGroups; ++q2) sa_u += sumA[(ab * kGroups + q2) * BM + row];
       const float corrA = static_cast<float>(64 * p.K - 8 * sa_u);
       const float sa = (MODE == static_cast<int>(GemmOut::kHalf) && m < p.M) ? p.s_a[m] : 0.0f;
-      const int na = (MODE == static_cast<int>(GemmOut::kCos) && m < p.M) ? p.norm_a[static_cast<size_t>(bz) * p.M + m] : 0;
 #pragma unroll 1
       for (int cc = 0; cc < BN / 32; ++cc) {
         uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
@@ -832,16 +829,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
                 const int i = g4 * 4 + e;
-                const float acc = __fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c0 + i]);
-                if (MODE == static_cast<int>(GemmOut::kS32)) {
-                  w[e] = static_cast<uint32_t>(__float2int_rn(acc));
-                } else {
-                  const float nn = colv[c0 + i];
-                  const float cs = (na == 0 || nn == 0.0f)
-                                       ? 0.0f
-                                       : __fdiv_rn(acc, __fsqrt_rn(__fmul_rn(static_cast<float>(na), nn)));
-                  w[e] = __float_as_uint(cs);
-                }
+                w[e] = static_cast<uint32_t>(
+                    __float2int_rn(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c0 + i])));
               }
               // 128-byte rows, 128-byte swizzle: 16-byte chunk (4h + g4) of row `lane`
               const int ch = 4 * h + g4;
