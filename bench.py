@@ -49,10 +49,10 @@ WORKLOAD = wl.LLAVA15_7B
 FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed steps
 
 # Latest ncu capture of the dominant kernel: mean DRAM bytes (read + write)
-# per launch over the seven linears of one step (profiles/
-# w4a4_gemm_pair_llava15_7b_b8_step.md), valid only while the GEMM source is
-# unchanged since the capture.
-PROFILED_GEMM = {"source_sha1": "192947517df2e4813855a1cc8715f43bfde5cb45", "dram_bytes_per_launch": 19820470}
+# per launch over the four GEMMs of one step (profiles/
+# w4a4_gemm_pair_llava15_7b_b8_step.md, section 2), valid only while the GEMM
+# source is unchanged since the capture.
+PROFILED_GEMM = {"source_sha1": "7a7d338c9c3d6708bd71a92109b136bfdfcfb1eb", "dram_bytes_per_launch": 41999488}
 
 
 def gemm_source_sha1() -> str:
@@ -444,7 +444,7 @@ def run_gpu(args, rank, world, local_rank):
         "gemm_tops": round(ach, 3),
         "pct_int8_tensor_peak": None,
         "pct_fp8_tensor_peak": round(100.0 * ach / peak, 2),
-        "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_kernel (tcgen05 kind::f8f6f4)",
+        "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_pair_kernel (tcgen05 kind::f8f6f4, cta_group::2)",
                      "achieved": round(ach, 3), "peak": round(peak, 1), "unit": "TFLOP/s",
                      "frac": round(ach / peak, 4), "traffic": traffic, "peak_source": peak_src,
                      "launches_timed": n_gemm,

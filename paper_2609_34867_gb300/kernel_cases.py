@@ -1,0 +1,101 @@
+"""Single-call cases of the hot path, for profiling and microbenchmarks.
+
+  python -m paper_2609_34867_gb300.kernel_cases gemm M N K [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases quant M K [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [--reps R]
+
+Each case builds seeded synthetic inputs (workloads.py), makes one untimed
+warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
+graph, then times `reps` replays (default 3), each after an L2 flush (512 MiB
+written, then 512 MiB read), and prints the mean CUDA-event time per call with
+the throughput it implies. Under ncu, `-s 1 -c 1` with the kernel's name
+selects the first replayed launch.
+
+  gemm    p4q_w4a4_linear on random packed codes: M x K activations,
+          N x K weights, fp16 output (2 M N K integer ops per call);
+  quant   p4q_quant_act on M x K fp16 activations with the outlier channels
+          (bytes: 2 M K in, M K / 2 + 4 M out);
+  select  p4q_select_gather_quant on one of the LLaVA-shaped workloads.
+"""
+from __future__ import annotations
+
+import argparse
+import sys
+
+import torch
+
+from . import p4q
+from . import workloads as wl
+
+FLUSH_BYTES = 512 << 20
+
+
+def _timed(fn, reps, dev):
+    """Mean CUDA-event milliseconds of fn, replayed from a CUDA graph (so that
+    no host work sits between the events), L2 flushed before each replay."""
+    w = torch.empty((FLUSH_BYTES,), dtype=torch.uint8, device=dev)
+    r = torch.ones((FLUSH_BYTES // 4,), dtype=torch.float32, device=dev)
+    fn()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        fn()
+    total = 0.0
+    for _ in range(reps):
+        w.zero_()
+        r.amax()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        graph.replay()
+        b.record()
+        torch.cuda.synchronize()
+        total += a.elapsed_time(b)
+    status = p4q.p4q_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the timed calls")
+    return total / reps
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("case", choices=["gemm", "quant", "select"])
+    ap.add_argument("args", nargs="+")
+    ap.add_argument("--reps", type=int, default=3)
+    a = ap.parse_args(argv)
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    p4q.lib()
+    if a.case == "gemm":
+        M, N, K = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        Xq = torch.randint(0, 256, (M, K // 2), dtype=torch.uint8, device=dev, generator=g)
+        Wq = torch.randint(0, 256, (N, K // 2), dtype=torch.uint8, device=dev, generator=g)
+        s_a = torch.rand(M, device=dev, generator=g)
+        s_w = torch.rand(N, device=dev, generator=g) * 0.01
+        Y = torch.empty((M, N), dtype=torch.float16, device=dev)
+        ms = _timed(lambda: p4q.p4q_w4a4_linear(Xq, s_a, Wq, s_w, Y), a.reps, dev)
+        print(f"gemm {M}x{N}x{K}: {ms * 1e3:.1f} us/call, {2 * M * N * K / ms / 1e9:.1f} TOPS")
+    elif a.case == "quant":
+        M, K = (int(x) for x in a.args)
+        X = torch.from_numpy(wl.activations(M, K, seed=wl.SWEEP_SEED)).to(dev)
+        Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+        s = torch.empty((M,), dtype=torch.float32, device=dev)
+        ms = _timed(lambda: p4q.p4q_quant_act(X, Xq, s), a.reps, dev)
+        nbytes = 2 * M * K + M * K // 2 + 4 * M
+        print(f"quant {M}x{K}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    else:
+        w = wl.WORKLOADS[a.args[0]]
+        x = wl.selector_inputs(w)
+        V, Q, A, T = (torch.from_numpy(t).to(dev) for t in (x.V, x.Q, x.A, x.text))
+        ws = p4q.select_workspace(w.B, w.N, w.d, w.J, w.K, dev)
+        idx = torch.empty((w.B, w.K), dtype=torch.int32, device=dev)
+        X = torch.empty((w.B, w.K + w.T, w.d), dtype=torch.float16, device=dev)
+        Xq = torch.empty((w.M, w.d // 2), dtype=torch.uint8, device=dev)
+        s = torch.empty((w.M,), dtype=torch.float32, device=dev)
+        ms = _timed(lambda: p4q.p4q_select_gather_quant(V, Q, A, T, w.K, idx, X, Xq, s, ws), a.reps, dev)
+        print(f"select {w.name}: {ms * 1e3:.1f} us/call, {ms * 1e3 / w.B:.2f} us/image")
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())
