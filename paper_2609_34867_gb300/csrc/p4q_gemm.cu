@@ -141,6 +141,35 @@ __device__ __forceinline__ void convert_chunk(const uint4 p, uint8_t* conv_tile,
   acc = __dp4a(h3, ones, acc);
 }
 
+// The two halves of convert_chunk, so that the unpack can run before the
+// wait for a free stage and only the stores after it.
+struct Unpacked {
+  uint4 lo, hi;  // E4M3 bytes of the 32 codes, in the order convert_chunk stores them
+};
+
+__device__ __forceinline__ Unpacked unpack_chunk(const uint4 p, uint32_t& acc) {
+  Unpacked u;
+  u.lo = make_uint4(nib_lo(p.x), nib_hi(p.x), nib_lo(p.y), nib_hi(p.y));
+  u.hi = make_uint4(nib_lo(p.z), nib_hi(p.z), nib_lo(p.w), nib_hi(p.w));
+  constexpr uint32_t ones = 0x01010101u;
+  acc = __dp4a(u.lo.x, ones, acc);
+  acc = __dp4a(u.lo.y, ones, acc);
+  acc = __dp4a(u.lo.z, ones, acc);
+  acc = __dp4a(u.lo.w, ones, acc);
+  acc = __dp4a(u.hi.x, ones, acc);
+  acc = __dp4a(u.hi.y, ones, acc);
+  acc = __dp4a(u.hi.z, ones, acc);
+  acc = __dp4a(u.hi.w, ones, acc);
+  return u;
+}
+
+__device__ __forceinline__ void store_chunk(const Unpacked& u, uint8_t* conv_tile, int r, int c) {
+  uint8_t* row = conv_tile + r * 128;
+  const int sw = r & 7;
+  *reinterpret_cast<uint4*>(row + (((2 * c) ^ sw) << 4)) = u.lo;
+  *reinterpret_cast<uint4*>(row + (((2 * c + 1) ^ sw) << 4)) = u.hi;
+}
+
 template <int BN, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -670,6 +699,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         for (int j = 0; j < NB; ++j) v[NA + j] = *reinterpret_cast<const uint4*>(pk + A_PACK + j * kRowStep * BKP);
         __syncwarp();
         if (lane == 0) mbar_arrive(&pack_empty[ps]);
+        // unpack into registers first: after the stage frees up only the stores remain
+        Unpacked u[NA + NB];
+#pragma unroll
+        for (int j = 0; j < NA; ++j) u[j] = unpack_chunk(v[j], accA[j]);
+#pragma unroll
+        for (int j = 0; j < NB; ++j) u[NA + j] = unpack_chunk(v[NA + j], accB[j]);
         if (!mbar_wait_warp(&empty_c[c], ((g / SC) & 1) ^ 1, abort_flag, &g_gemm_err)) {
           ok = false;
           break;
@@ -677,9 +712,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         uint8_t* ca = smem + c * CONV_STAGE;
         uint8_t* cb = ca + A_CONV;
 #pragma unroll
-        for (int j = 0; j < NA; ++j) convert_chunk(v[j], ca, rbase + kRowStep * j, chunk, accA[j]);
+        for (int j = 0; j < NA; ++j) store_chunk(u[j], ca, rbase + kRowStep * j, chunk);
 #pragma unroll
-        for (int j = 0; j < NB; ++j) convert_chunk(v[NA + j], cb, rbase + kRowStep * j, chunk, accB[j]);
+        for (int j = 0; j < NB; ++j) store_chunk(u[NA + j], cb, rbase + kRowStep * j, chunk);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive_remote(full_c_leader + 8u * c);  // the leader's full_c[c]
