@@ -276,22 +276,31 @@ class Step:
             fn()
 
     def capture(self):
-        """Captures every segment into its own CUDA graph (after warm-up calls
-        have set up the kernels' attributes); a replay launches the same
-        kernels with no host work per kernel."""
+        """Captures the whole step into one CUDA graph (consecutive kernels
+        overlap their launch and set-up with the previous kernel's tail), and
+        every segment into its own graph for per-segment timing (after warm-up
+        calls have set up the kernels' attributes)."""
         torch = self.torch
         self.graphs = []
-        n0 = self.p4q.p4q_launch_count()
         for _, _, fn in self.segments:
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g):
                 fn()
             self.graphs.append(g)
+        n0 = self.p4q.p4q_launch_count()
+        self.full = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.full):
+            self.body()
         self.launches_per_step = self.p4q.p4q_launch_count() - n0
 
-    def __call__(self):
+    def __call__(self, segments: bool = False):
+        """One step: the whole-step graph, or (segments=True) the segment
+        graphs with events between them (see kernel_times)."""
         if self.graphs is None:
             self.body()
+            return
+        if not segments:
+            self.full.replay()
             return
         self.events[0].record()
         for i, g in enumerate(self.graphs):
@@ -356,11 +365,16 @@ def run_gpu(args, rank, world, local_rank):
         e_end.record()
         torch.cuda.synchronize()
         step_ms.append(e_start.elapsed_time(e_end))
+    t_wall = time.perf_counter() - t_wall
+    # per-segment times (selector, each GEMM) from the segment graphs
+    for i in range(min(args.steps, 200)):
+        flush()
+        step(segments=True)
+        torch.cuda.synchronize()
         kt = step.kernel_times()
         sel_ms.append(kt["select"])
         for n in gemm_ms:
             gemm_ms[n].append(kt["linear"][n])
-    t_wall = time.perf_counter() - t_wall
     if world > 1:
         dist.barrier()
     clk = clocks.stop()
@@ -438,7 +452,8 @@ def run_gpu(args, rank, world, local_rank):
             "linears": "; ".join(f"{l.name} {l.k_in}->{l.n_out}" for l in w.linears), "layers": w.layers,
             "gemms": "; ".join(f"{g}={'|'.join(m)}" for g, m in step.gemms),
             "alpha_beta_gamma": "0.3/0.2/0.5", "l2": "flushed before every timed step: 512 MiB written, then another 512 MiB read (no dirty flush lines left to write back inside the timed region)",
-            "timing": "CUDA events around each step (graph replays), summed over the K steps",
+            "timing": "CUDA events around each step (one CUDA graph per step), summed over the K steps; "
+                      "selector and per-GEMM times from segment graphs with events between them",
             "parallelism": f"dp{world} (independent batches)"},
         "select_prune_us_per_image": round(float(sel_ms.mean()) * 1e3 / w.B, 3),
         "gemm_tops": round(ach, 3),
@@ -451,8 +466,8 @@ def run_gpu(args, rank, world, local_rank):
                      "note": "integer ops on the FP8 tensor pipe; sm_103a has no integer tcgen05 MMA kind",
                      "per_gemm_us": {n: round(float(np.mean(v)) * 1e3, 2) for n, v in gemm_ms.items()}},
         "gpu_launches": int(launches),
-        "launch": "%d CUDA graph replays per step (%d kernels of libp4q per step)" % (
-            len(step.graphs), step.launches_per_step),
+        "launch": "1 CUDA graph replay per step (%d kernels of libp4q per step, programmatic dependent launch)" % (
+            step.launches_per_step),
         "clocks": clk,
     }
     if e2e_ms is not None:

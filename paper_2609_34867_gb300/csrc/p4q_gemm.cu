@@ -214,6 +214,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();  // operands and scales come from the previous kernel
+  pdl_launch_dependents();
   const int per = p.num_m * p.num_n;
 
   if (warp == 0) {
@@ -636,6 +638,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   cluster_sync();  // barriers of both CTAs initialized, TMEM allocated in both
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();  // operands and scales come from the previous kernel
+  pdl_launch_dependents();
 
   if (warp == 0) {
     // ------------------------------------------------------------ MMA issuer (leader)
@@ -1002,8 +1006,7 @@ cudaError_t launch_cfg(const GemmArgs& g, cudaStream_t stream) {
   p.norm_a = g.norm_a;
   p.norm_b = g.norm_b;
   const int grid = p.tiles < num_sms() ? p.tiles : num_sms();
-  w4a4_gemm_kernel<BN, MODE><<<grid, kThreads, C::SMEM, stream>>>(ma, mb, md, p);
-  return cudaGetLastError();
+  return launch_pdl(w4a4_gemm_kernel<BN, MODE>, dim3(grid), dim3(kThreads), C::SMEM, stream, ma, mb, md, p);
 }
 
 template <int MODE>
@@ -1037,8 +1040,8 @@ cudaError_t launch_pair(const GemmArgs& g, cudaStream_t stream) {
   p.norm_a = g.norm_a;
   p.norm_b = g.norm_b;
   const int pairs = p.tiles < num_sms() / 2 ? p.tiles : num_sms() / 2;
-  pair::w4a4_gemm_pair_kernel<MODE><<<2 * pairs, pair::kPairThreads, pair::Lay<MODE>::SMEM, stream>>>(ma, mb, md, p);
-  return cudaGetLastError();
+  return launch_pdl(pair::w4a4_gemm_pair_kernel<MODE>, dim3(2 * pairs), dim3(pair::kPairThreads),
+                    pair::Lay<MODE>::SMEM, stream, ma, mb, md, p);
 }
 
 }  // namespace

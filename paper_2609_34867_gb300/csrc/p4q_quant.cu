@@ -119,6 +119,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   if (threadIdx.x < kGroups) aborts[threadIdx.x] = 0;
   fence_barrier_init();
   __syncthreads();
+  pdl_wait();  // rows (and kept indices) come from the previous kernel
+  pdl_launch_dependents();
 
   unsigned char* ring = smem + static_cast<size_t>(grp) * S * stage_bytes;
   uint64_t* full = bars + grp * S;
@@ -269,8 +271,8 @@ cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out,
                       2 * kWarps * 4 + kGroups * 4;
   const int need = (rows + kGroups - 1) / kGroups;
   const int grid = std::min(need, kCtasPerSm * sm_count());
-  quant_rows_kernel<G, NORM><<<grid, kThreads, smem, stream>>>(src, rows, L, out, p.S, p.stage_bytes);
-  return cudaGetLastError();
+  return launch_pdl(quant_rows_kernel<G, NORM>, dim3(grid), dim3(kThreads), smem, stream, src, rows, L, out, p.S,
+                    p.stage_bytes);
 }
 
 template <bool NORM>

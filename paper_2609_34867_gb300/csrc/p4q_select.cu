@@ -61,6 +61,8 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
     query_scores_kernel(const uint8_t* __restrict__ vcodes, const int32_t* __restrict__ vnorm,
                         const uint8_t* __restrict__ qcodes, const int32_t* __restrict__ qnorm, int B, int N, int d,
                         int J, float* __restrict__ scores) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tok = blockIdx.x * kScoreWarps + warp;
   if (tok >= B * N) return;
@@ -219,6 +221,8 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     select_stages_kernel(const float* __restrict__ scores, const float* __restrict__ A_cls,
                          const float* __restrict__ gram, int gp, int N, int J, int K, int Kq, int Ks,
                          int Kd, int32_t* __restrict__ idx) {
+  pdl_wait();
+  pdl_launch_dependents();
   extern __shared__ uint8_t smem_raw[];
   BlockScratch& s = *reinterpret_cast<BlockScratch*>(smem_raw);
   const int b = blockIdx.x;
@@ -366,9 +370,8 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
 
 cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
   const int toks = p.B * p.N;
-  query_scores_kernel<<<(toks + kScoreWarps - 1) / kScoreWarps, kScoreWarps * 32, 0, stream>>>(
-      ws.vcodes, ws.vnorm, ws.qcodes, ws.qnorm, p.B, p.N, p.d, p.J, ws.scores);
-  return cudaGetLastError();
+  return launch_pdl(query_scores_kernel, dim3((toks + kScoreWarps - 1) / kScoreWarps), dim3(kScoreWarps * 32), 0,
+                    stream, ws.vcodes, ws.vnorm, ws.qcodes, ws.qnorm, p.B, p.N, p.d, p.J, ws.scores);
 }
 
 namespace {
@@ -377,6 +380,8 @@ namespace {
 // in, the cosines out (same bits as the cosine epilogue of the GEMM).
 __global__ void __launch_bounds__(128) gram_cos_kernel(float* __restrict__ gram, const int32_t* __restrict__ norm,
                                                        int N, int gp) {
+  pdl_wait();
+  pdl_launch_dependents();
   const int row = blockIdx.x;  // b * N + i
   const int j0 = 4 * (blockIdx.y * blockDim.x + threadIdx.x);
   if (j0 >= N) return;
@@ -398,8 +403,7 @@ __global__ void __launch_bounds__(128) gram_cos_kernel(float* __restrict__ gram,
 cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
   const int per_row = (p.N + 3) / 4;
   const dim3 grid(p.B * p.N, (per_row + 127) / 128);
-  gram_cos_kernel<<<grid, 128, 0, stream>>>(ws.gram, ws.vnorm, p.N, ws.gram_pitch);
-  return cudaGetLastError();
+  return launch_pdl(gram_cos_kernel, grid, dim3(128), 0, stream, ws.gram, ws.vnorm, p.N, ws.gram_pitch);
 }
 
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls, int32_t* idx,
@@ -413,9 +417,8 @@ cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws,
   }
   // one thread per kPer tokens: idle threads would only add instructions to every round
   const int threads = std::min(kSelThreads, ((p.N + kPer - 1) / kPer + 31) / 32 * 32);
-  select_stages_kernel<<<p.B, threads, smem, stream>>>(ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J,
-                                                           p.K, p.Kq, p.Ks, p.Kd, idx);
-  return cudaGetLastError();
+  return launch_pdl(select_stages_kernel, dim3(p.B), dim3(threads), static_cast<size_t>(smem), stream, ws.scores,
+                    A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx);
 }
 
 }  // namespace p4q
