@@ -536,6 +536,19 @@ namespace pair {
 #ifndef P4Q_PAIR_PACK
 #define P4Q_PAIR_PACK 4
 #endif
+#ifndef P4Q_PAIR_SPIN
+#define P4Q_PAIR_SPIN 2
+#endif
+#if P4Q_PAIR_SPIN & 1
+#define PAIR_WAIT_MMA mbar_wait_spin
+#else
+#define PAIR_WAIT_MMA mbar_wait
+#endif
+#if P4Q_PAIR_SPIN & 2
+#define PAIR_WAIT_CONV mbar_wait_spin_warp
+#else
+#define PAIR_WAIT_CONV mbar_wait_warp
+#endif
 #ifndef P4Q_PAIR_PREFETCH
 #define P4Q_PAIR_PREFETCH 6
 #endif
@@ -654,7 +667,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         const uint32_t d = tmem_base + static_cast<uint32_t>(ab * BN);
         for (int kb = 0; kb < KB; ++kb, ++g) {
           const int s = g % SC;
-          if (!mbar_wait(&full_c[s], (g / SC) & 1, abort_flag, &g_gemm_err)) {
+          if (!PAIR_WAIT_MMA(&full_c[s], (g / SC) & 1, abort_flag, &g_gemm_err)) {
             ok = false;
             break;
           }
@@ -691,7 +704,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         const int g = gbase + kb;
         const int ps = g % P, c = g % SC;
         // the packed k-block (TMA, this CTA's 128 A rows then 128 B rows of 64 bytes)
-        if (!mbar_wait_warp(&pack_full[ps], (g / P) & 1, abort_flag, &g_gemm_err)) {
+        if (!PAIR_WAIT_CONV(&pack_full[ps], (g / P) & 1, abort_flag, &g_gemm_err)) {
           ok = false;
           break;
         }
@@ -709,7 +722,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         for (int j = 0; j < NA; ++j) u[j] = unpack_chunk(v[j], accA[j]);
 #pragma unroll
         for (int j = 0; j < NB; ++j) u[NA + j] = unpack_chunk(v[NA + j], accB[j]);
-        if (!mbar_wait_warp(&empty_c[c], ((g / SC) & 1) ^ 1, abort_flag, &g_gemm_err)) {
+        if (!PAIR_WAIT_CONV(&empty_c[c], ((g / SC) & 1) ^ 1, abort_flag, &g_gemm_err)) {
           ok = false;
           break;
         }
