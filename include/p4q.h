@@ -88,9 +88,12 @@ uint64_t p4q_launch_count(void);
  *   0 automatic (default): CTA-pair kernel for fp16 outputs with M >= 256 and
  *     N >= 256, single-CTA kernel otherwise;
  *   1 single-CTA kernel only;
- *   2 CTA-pair kernel whenever N >= 256 (also for int32 outputs).
- * Returns P4Q_ERR_INVALID_ARG for other values. Not thread-safe against
- * concurrent launches. */
+ *   2 CTA-pair kernel whenever N >= 256 (also for int32 outputs);
+ *   3 like 0, and the workspace entry points take the expanded-operand path
+ *     whenever a workspace is given (also below M = 512).
+ * Variants 1 and 2 also keep the workspace entry points on the in-kernel
+ * unpack. Returns P4Q_ERR_INVALID_ARG for other values. Not thread-safe
+ * against concurrent launches. */
 p4q_status p4q_set_gemm_variant(int variant);
 
 /* Test of the bounded-wait path: launches one warp that waits on an mbarrier
@@ -159,6 +162,32 @@ p4q_status p4q_w4a4_linear(const uint8_t* Xq, const float* s_a, int M, int Kin,
  * acc [M, N] int32 row-major (device, written). Same limits as above. */
 p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N,
                              int32_t* acc, p4q_stream_t stream);
+
+/* Workspace bytes for p4q_w4a4_linear_ws / p4q_w4a4_gemm_s32_ws on an
+ * M x N x Kin linear: both operands as one byte per code plus their row
+ * sums. 0 for sizes the linear rejects. */
+size_t p4q_w4a4_linear_workspace_bytes(int M, int N, int Kin);
+
+/* p4q_w4a4_linear with a caller workspace (App. B.3; same results bit for
+ * bit). With a workspace, large linears (M >= 512 and N >= 256) first expand
+ * both packed operands into it, one byte per code (u = v + 8) with the row
+ * sums of u, and then run a GEMM whose operands reach the tensor cores by
+ * TMA alone (no unpacking on the SMs that run the MMAs); other shapes, or
+ * ws == NULL, run exactly as p4q_w4a4_linear. The paper has no counterpart:
+ * this is a deployment choice for GPUs without 4-bit integer MMAs.
+ *   ws        device workspace, 16-byte aligned, or NULL
+ *   ws_bytes  >= p4q_w4a4_linear_workspace_bytes(M, N, Kin) when ws != NULL,
+ *             else P4Q_ERR_WORKSPACE_TOO_SMALL (P4Q_ERR_MISALIGNED if unaligned)
+ * The workspace is scratch overwritten by every call: calls sharing one must
+ * be ordered (same stream). Other arguments and rules as p4q_w4a4_linear. */
+p4q_status p4q_w4a4_linear_ws(const uint8_t* Xq, const float* s_a, int M, int Kin, const uint8_t* Wq,
+                              const float* s_w, int N, uint16_t* Y, void* ws, size_t ws_bytes,
+                              p4q_stream_t stream);
+
+/* Test view of the same path: the exact int32 accumulators (as
+ * p4q_w4a4_gemm_s32). */
+p4q_status p4q_w4a4_gemm_s32_ws(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,
+                                void* ws, size_t ws_bytes, p4q_stream_t stream);
 
 /* ---------------------------------------------------------------------- */
 /* Quantization-aware visual-token selector (Sec. 3.2, Eq. 4)               */

@@ -19,8 +19,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 std::atomic<uint64_t> g_launches{0};
 
 // Counts one kernel launch when `e` reports success.
-cudaError_t counted(cudaError_t e) {
-  if (e == cudaSuccess) g_launches.fetch_add(1, std::memory_order_relaxed);
+cudaError_t counted(cudaError_t e, unsigned int kernels = 1) {
+  if (e == cudaSuccess) g_launches.fetch_add(kernels, std::memory_order_relaxed);
   return e;
 }
 
@@ -160,14 +160,15 @@ const char* p4q_status_string(p4q_status s) {
 uint64_t p4q_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 p4q_status p4q_set_gemm_variant(int variant) {
-  if (variant < 0 || variant > 2) return P4Q_ERR_INVALID_ARG;
-  set_gemm_pair_mode(variant == 0 ? -1 : variant == 1 ? 0 : 1);
+  if (variant < 0 || variant > 3) return P4Q_ERR_INVALID_ARG;
+  set_gemm_pair_mode(variant == 0 || variant == 3 ? -1 : variant == 1 ? 0 : 1);
+  set_gemm8_mode(variant == 0 ? 0 : variant == 3 ? 2 : 1);
   return P4Q_OK;
 }
 
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
-  const unsigned int g = gemm_read_and_clear_error() | quant_read_and_clear_error();
+  const unsigned int g = gemm_read_and_clear_error() | gemm8_read_and_clear_error() | quant_read_and_clear_error();
   if (cudaGetLastError() != cudaSuccess) return P4Q_ERR_CUDA;
   return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
 }
@@ -222,6 +223,62 @@ p4q_status p4q_w4a4_linear(const uint8_t* Xq, const float* s_a, int M, int Kin, 
   g.s_a = s_a;
   g.s_b = s_w;
   return from_cuda(counted(launch_w4a4_gemm(g, reinterpret_cast<cudaStream_t>(stream))));
+}
+
+size_t p4q_w4a4_linear_workspace_bytes(int M, int N, int Kin) {
+  if (M < 0 || N < 1 || Kin < 1 || Kin % 128 != 0 || Kin > P4Q_MAX_ROW || N % 8 != 0) return 0;
+  return gemm8_workspace_bytes(M, N, Kin);
+}
+
+namespace {
+
+// The workspace entry points: the expanded-operand path when a workspace is
+// given and the shape qualifies, else the in-kernel unpack.
+p4q_status run_linear_ws(const GemmArgs& g, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  if (ws) {
+    if (!aligned16(ws)) return P4Q_ERR_MISALIGNED;
+    if (ws_bytes < gemm8_workspace_bytes(g.M, g.N, g.K)) return P4Q_ERR_WORKSPACE_TOO_SMALL;
+    if (gemm8_applies(g)) return from_cuda(counted(launch_w4a4_gemm8(g, ws, ws_bytes, stream), 3));
+  }
+  return from_cuda(counted(launch_w4a4_gemm(g, stream)));
+}
+
+}  // namespace
+
+p4q_status p4q_w4a4_linear_ws(const uint8_t* Xq, const float* s_a, int M, int Kin, const uint8_t* Wq,
+                              const float* s_w, int N, uint16_t* Y, void* ws, size_t ws_bytes, p4q_stream_t stream) {
+  p4q_status st = check_gemm(Xq, M, Kin, Wq, N, Y);
+  if (st != P4Q_OK) return st;
+  if (!s_w || (M > 0 && !s_a)) return P4Q_ERR_INVALID_ARG;
+  if (M == 0) return P4Q_OK;
+  if ((st = check_device()) != P4Q_OK) return st;
+  GemmArgs g;
+  g.A = Xq;
+  g.B = Wq;
+  g.M = M;
+  g.N = N;
+  g.K = Kin;
+  g.out = GemmOut::kHalf;
+  g.D = Y;
+  g.s_a = s_a;
+  g.s_b = s_w;
+  return run_linear_ws(g, ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+p4q_status p4q_w4a4_gemm_s32_ws(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc, void* ws,
+                                size_t ws_bytes, p4q_stream_t stream) {
+  p4q_status st = check_gemm(Xq, M, Kin, Wq, N, acc);
+  if (st != P4Q_OK || M == 0) return st;
+  if ((st = check_device()) != P4Q_OK) return st;
+  GemmArgs g;
+  g.A = Xq;
+  g.B = Wq;
+  g.M = M;
+  g.N = N;
+  g.K = Kin;
+  g.out = GemmOut::kS32;
+  g.D = acc;
+  return run_linear_ws(g, ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
 p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,

@@ -928,6 +928,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 
 }  // namespace pair
 
+}  // namespace
+
 PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
   static std::once_flag once;
@@ -986,6 +988,8 @@ int num_sms() {
   }
   return n;
 }
+
+namespace {
 
 template <int BN, int MODE>
 cudaError_t launch_cfg(const GemmArgs& g, cudaStream_t stream) {

@@ -3,6 +3,8 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <utility>
@@ -76,6 +78,8 @@ cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream);
 // kernel for large fp16 linears), 0 single-CTA only, 1 CTA-pair whenever the
 // shape allows (N >= 256).
 void set_gemm_pair_mode(int mode);
+// Expanded-operand path: 0 automatic (M >= 512), 1 never, 2 whenever a workspace is given.
+void set_gemm8_mode(int mode);
 
 // ------------------------------------------------------------ selector
 struct SelectPlan {
@@ -102,9 +106,27 @@ cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cuda
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls,
                                  int32_t* idx, cudaStream_t stream);
 
-// Device error words of the kernels with bounded waits (GEMM, quantizer).
+// Device error words of the kernels with bounded waits (GEMMs, quantizer).
 unsigned int gemm_read_and_clear_error();
+unsigned int gemm8_read_and_clear_error();
 unsigned int quant_read_and_clear_error();
+
+// ------------------------------------------------------------ shared GEMM helpers (p4q_gemm.cu)
+int num_sms();
+// 3-D map over the output [batch][rows][cols] with row pitch `pitch` elements;
+// 32 x 32 boxes in the swizzle the epilogues write.
+bool make_output_map(CUtensorMap* map, void* base, GemmOut out, int rows, int cols, int pitch, int batch);
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn();
+
+// ------------------------------------------------------------ expanded-operand GEMM (p4q_gemm8.cu)
+// Bytes of the workspace the expanded-operand path needs for an M x N x K
+// linear: both operands as one byte per code (u = v + 8) and their row sums.
+size_t gemm8_workspace_bytes(int M, int N, int K);
+// Whether the expanded-operand path serves this shape (large enough that the
+// expansion pays for itself).
+bool gemm8_applies(const GemmArgs& g);
+// Expands both operands into the workspace, then runs the FP8 GEMM.
+cudaError_t launch_w4a4_gemm8(const GemmArgs& g, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 // One bounded wait that nothing completes: times out after limit_ns and sets
 // the GEMM's device error word (tests the time-out path).

@@ -61,6 +61,12 @@ def lib() -> ctypes.CDLL:
         L.p4q_w4a4_linear.restype = st
         L.p4q_w4a4_gemm_s32.argtypes = [P, I, I, P, I, P, P]
         L.p4q_w4a4_gemm_s32.restype = st
+        L.p4q_w4a4_linear_workspace_bytes.argtypes = [I, I, I]
+        L.p4q_w4a4_linear_workspace_bytes.restype = S
+        L.p4q_w4a4_linear_ws.argtypes = [P, P, I, I, P, P, I, P, P, S, P]
+        L.p4q_w4a4_linear_ws.restype = st
+        L.p4q_w4a4_gemm_s32_ws.argtypes = [P, I, I, P, I, P, P, S, P]
+        L.p4q_w4a4_gemm_s32_ws.restype = st
         L.p4q_select_workspace_bytes.argtypes = [I, I, I, I, ctypes.POINTER(SelectParams)]
         L.p4q_select_workspace_bytes.restype = S
         L.p4q_select.argtypes = [P, I, I, I, P, I, P, ctypes.POINTER(SelectParams), P, P, S, P]
@@ -104,7 +110,8 @@ def p4q_launch_count() -> int:
 
 
 def p4q_set_gemm_variant(variant: int):
-    """0 automatic, 1 single-CTA GEMM only, 2 CTA-pair GEMM whenever N >= 256."""
+    """0 automatic, 1 single-CTA GEMM only, 2 CTA-pair GEMM whenever N >= 256,
+    3 automatic with the expanded-operand path whenever a workspace is given."""
     _check(lib().p4q_set_gemm_variant(int(variant)), "p4q_set_gemm_variant")
 
 
@@ -206,6 +213,35 @@ def w4a4_linear(Xq, s_a, Wq, s_w, stream=None):
     Y = torch.empty((Xq.shape[0], Wq.shape[0]), dtype=torch.float16, device=Xq.device)
     p4q_w4a4_linear(Xq, s_a, Wq, s_w, Y, stream)
     return Y
+
+
+def linear_workspace(M, N, K, device):
+    """A device workspace large enough for p4q_w4a4_linear_ws on M x N x K."""
+    n = int(lib().p4q_w4a4_linear_workspace_bytes(int(M), int(N), int(K)))
+    if n == 0:
+        raise P4QError(1, "p4q_w4a4_linear_workspace_bytes")
+    return torch.empty((n,), dtype=torch.uint8, device=device)
+
+
+def p4q_w4a4_linear_ws(Xq, s_a, Wq, s_w, Y, ws, stream=None):
+    """p4q_w4a4_linear with a caller workspace (None: no workspace)."""
+    _need(Xq, torch.uint8, 2, "Xq"); _need(Wq, torch.uint8, 2, "Wq"); _need(Y, torch.float16, 2, "Y")
+    M, K = Xq.shape[0], Xq.shape[1] * 2
+    N = Wq.shape[0]
+    wp, wn = (None, 0) if ws is None else (_ptr(ws), ws.numel() * ws.element_size())
+    _check(lib().p4q_w4a4_linear_ws(_ptr(Xq), _ptr(s_a), M, K, _ptr(Wq), _ptr(s_w), N, _ptr(Y), wp, wn,
+                                    _stream(stream)), "p4q_w4a4_linear_ws")
+
+
+def w4a4_gemm_s32_ws(Xq, Wq, ws, stream=None):
+    """Allocating wrapper of p4q_w4a4_gemm_s32_ws: returns the int32 accumulators."""
+    M, K = Xq.shape[0], Xq.shape[1] * 2
+    N = Wq.shape[0]
+    acc = torch.empty((M, N), dtype=torch.int32, device=Xq.device)
+    wp, wn = (None, 0) if ws is None else (_ptr(ws), ws.numel() * ws.element_size())
+    _check(lib().p4q_w4a4_gemm_s32_ws(_ptr(Xq), M, K, _ptr(Wq), N, _ptr(acc), wp, wn, _stream(stream)),
+           "p4q_w4a4_gemm_s32_ws")
+    return acc
 
 
 def w4a4_gemm_s32(Xq, Wq, stream=None):

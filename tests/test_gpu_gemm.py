@@ -75,3 +75,68 @@ def test_linear_fp16_within_tolerance(p4q, dev, variant, M, N, K):
     err = np.abs(y - ref)
     lim = np.maximum(1e-3 * np.abs(ref), 2e-3)
     assert np.all(err <= lim), f"max err {err.max()} at {np.unravel_index(np.argmax(err - lim), err.shape)}"
+
+
+# ---------------------------------------------------------------- expanded-operand path (workspace entry points)
+@pytest.fixture
+def expanded(p4q):
+    """Forces the expanded-operand path of the workspace entry points (also below 512 rows)."""
+    p4q.p4q_set_gemm_variant(3)
+    yield
+    p4q.p4q_set_gemm_variant(0)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 256, 128), (200, 264, 256), (256, 256, 128), (257, 264, 256),
+                                   (600, 1032, 384), (2048, 4096, 512), (1100, 2056, 4096), (64, 2048, 11008)])
+def test_expanded_gemm_s32_bit_exact(p4q, dev, expanded, M, N, K):
+    rng = np.random.default_rng(M * 13 + N + 5)
+    a, w = _packed(rng, M, K), _packed(rng, N, K)
+    ws = p4q.linear_workspace(M, N, K, dev)
+    acc = p4q.w4a4_gemm_s32_ws(torch.from_numpy(a).to(dev), torch.from_numpy(w).to(dev), ws)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    ref = oracle.gemm_s32(oracle.unpack_codes(a), oracle.unpack_codes(w))
+    assert np.array_equal(acc.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("K", [13824, 16384])
+def test_expanded_gemm_extreme_codes_exact(p4q, dev, expanded, K):
+    pat = {"p7": 0x77, "m7": 0x99, "m8": 0x88, "alt": 0x97, "zero": 0x00}
+    names = list(pat)
+    a = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 26)[:128]
+    w = np.stack([np.full(K // 2, pat[n], np.uint8) for n in names] * 52)[:256]
+    ws = p4q.linear_workspace(128, 256, K, dev)
+    acc = p4q.w4a4_gemm_s32_ws(torch.from_numpy(a).to(dev), torch.from_numpy(w).to(dev), ws)
+    torch.cuda.synchronize()
+    ref = oracle.gemm_s32(oracle.unpack_codes(a), oracle.unpack_codes(w))
+    assert np.array_equal(acc.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("M,N,K", [(2048, 4096, 4096), (512, 264, 128), (1024, 13824, 5120), (700, 4096, 11008)])
+def test_expanded_linear_fp16_within_tolerance(p4q, dev, M, N, K):
+    """Automatic dispatch (M >= 512 takes the expanded path) through p4q_w4a4_linear_ws."""
+    rng = np.random.default_rng(K + M + 1)
+    a, w = _packed(rng, M, K), _packed(rng, N, K)
+    sa = (rng.random(M) * 0.5 + 0.01).astype(np.float32)
+    sw = (rng.random(N) * 0.002 + 1e-4).astype(np.float32)
+    ws = p4q.linear_workspace(M, N, K, dev)
+    Y = torch.empty((M, N), dtype=torch.float16, device=dev)
+    p4q.p4q_w4a4_linear_ws(torch.from_numpy(a).to(dev), torch.from_numpy(sa).to(dev), torch.from_numpy(w).to(dev),
+                           torch.from_numpy(sw).to(dev), Y, ws)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    y = Y.float().cpu().numpy()
+    ref = oracle.linear(oracle.unpack_codes(a), sa, oracle.unpack_codes(w), sw)
+    err = np.abs(y - ref)
+    lim = np.maximum(1e-3 * np.abs(ref), 2e-3)
+    assert np.all(err <= lim), f"max err {err.max()}"
+
+
+def test_expanded_linear_rejects_a_short_workspace(p4q, dev):
+    Xq = torch.zeros((1024, 2048), dtype=torch.uint8, device=dev)
+    Wq = torch.zeros((512, 2048), dtype=torch.uint8, device=dev)
+    s = torch.ones((1024,), dtype=torch.float32, device=dev)
+    Y = torch.empty((1024, 512), dtype=torch.float16, device=dev)
+    short = torch.empty((1024,), dtype=torch.uint8, device=dev)
+    with pytest.raises(p4q.P4QError):
+        p4q.p4q_w4a4_linear_ws(Xq, s, Wq, s[:512], Y, short)
