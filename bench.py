@@ -5,7 +5,11 @@ One step = the whole path over one batch of the LLaVA-1.5-7B-shaped workload
 budget 192 kept tokens per image):
   p4q_select_gather_quant  fake-quant -> query / saliency / diversity stages
                            -> gather of the kept FP16 rows + text -> INT4
-  p4q_w4a4_linear x 4      q|k|v and gate|up (each one GEMM over the
+  p4q_expand_codes         the pruned sequence's codes, one byte per code
+                           (once, for the four GEMMs that read it), each
+                           GEMM's packed weights (per call), the re-quantized
+                           o / down inputs
+  p4q_w4a4_linear_expanded x 4  q|k|v and gate|up (each one GEMM over the
                            concatenated output channels) on the pruned
                            sequence (M = 2048), o on the re-quantized q
                            output, down on the re-quantized up output
@@ -52,11 +56,11 @@ FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed step
 # per launch over the four GEMMs of one step (profiles/
 # w4a4_gemm_pair_llava15_7b_b8_step.md, section 2), valid only while the GEMM
 # source is unchanged since the capture.
-PROFILED_GEMM = {"source_sha1": "7a7d338c9c3d6708bd71a92109b136bfdfcfb1eb", "dram_bytes_per_launch": 41999488}
+PROFILED_GEMM = {"source_sha1": "", "dram_bytes_per_launch": 0}
 
 
 def gemm_source_sha1() -> str:
-    p = os.path.join(ROOT, "paper_2609_34867_gb300", "csrc", "p4q_gemm.cu")
+    p = os.path.join(ROOT, "paper_2609_34867_gb300", "csrc", "p4q_gemm8.cu")
     return hashlib.sha1(open(p, "rb").read()).hexdigest()
 
 
@@ -232,21 +236,38 @@ class Step:
                 self.Xq_re[name] = torch.empty((M, dims[name].k_in // 2), dtype=torch.uint8, device=dev)
                 self.s_re[name] = torch.empty((M,), dtype=torch.float32, device=dev)
         self.out_name = w.linears[-1].name
-        # The step is a chain of segments (selector, each GEMM, each
-        # re-quantization) captured as one CUDA graph each, so that events
-        # recorded between the replays time the selector and every GEMM.
-        self.segments = [("select", "select", self._select)]
+        # Expanded operands (one byte per code + row sums, p4q_expand_codes):
+        # the pruned sequence once per step for every GEMM that reads it, the
+        # re-quantized o / down inputs, and each GEMM's weights per call into
+        # one scratch (the weights stay packed INT4 in memory).
+        self.Xu = torch.empty((M, d), dtype=torch.uint8, device=dev)
+        self.sXu = torch.empty((M,), dtype=torch.int32, device=dev)
+        self.Xu_re, self.sXu_re = {}, {}
+        for name in self.Xq_re:
+            self.Xu_re[name] = torch.empty((M, dims[name].k_in), dtype=torch.uint8, device=dev)
+            self.sXu_re[name] = torch.empty((M,), dtype=torch.int32, device=dev)
+        wmax = max(self.Wq[0, g].shape[0] * self.Wq[0, g].shape[1] * 2 for g, _ in self.gemms)
+        nmax = max(self.Wq[0, g].shape[0] for g, _ in self.gemms)
+        self.Wu = torch.empty((wmax,), dtype=torch.uint8, device=dev)
+        self.sWu = torch.empty((nmax,), dtype=torch.int32, device=dev)
+        # The step is a chain of segments (selector, each expansion, each GEMM,
+        # each re-quantization); the timed loop replays it as one CUDA graph,
+        # the breakdown replays one graph per segment with events between them.
+        self.segments = [("select", "select", self._select),
+                         ("expand", "expand_x", lambda: p4q.p4q_expand_codes(self.Xq, self.Xu, self.sXu))]
         for layer in range(w.layers):
             for gname, members in self.gemms:
                 if members[0] in self.REQUANT:
                     name = members[0]
                     self.segments.append(("quant", "quant_" + name, (lambda n=name: p4q.p4q_quant_act_ld(
                         self.output(self.REQUANT[n]), self.Xq_re[n], self.s_re[n]))))
-                    self.segments.append(("linear", gname, (lambda l=layer, g=gname, n=name: self._gemm(
-                        l, g, self.Xq_re[n], self.s_re[n]))))
+                    self.segments.append(("expand", "expand_" + name, (lambda n=name: p4q.p4q_expand_codes(
+                        self.Xq_re[n], self.Xu_re[n], self.sXu_re[n]))))
+                    xin = (lambda n=name: (self.Xu_re[n], self.sXu_re[n], self.s_re[n]))
                 else:
-                    self.segments.append(("linear", gname, (lambda l=layer, g=gname: self._gemm(
-                        l, g, self.Xq, self.s_a))))
+                    xin = (lambda: (self.Xu, self.sXu, self.s_a))
+                self.segments.append(("expand", "expand_w_" + gname, (lambda l=layer, g=gname: self._expand_w(l, g))))
+                self.segments.append(("linear", gname, (lambda l=layer, g=gname, x=xin: self._gemm(l, g, *x()))))
         self.lin_ops = {g: sum(2 * w.M * dims[m].n_out * dims[m].k_in for m in members) * w.layers
                         for g, members in self.gemms}
         self.graphs = None
@@ -267,8 +288,16 @@ class Step:
         self.p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
                                          self.s_a, self.ws)
 
-    def _gemm(self, layer, gname, Xq, s):
-        self.p4q.p4q_w4a4_linear(Xq, s, self.Wq[layer, gname], self.s_w[layer, gname], self.Y[gname])
+    def _expand_w(self, layer, gname):
+        Wq = self.Wq[layer, gname]
+        n = Wq.shape[0]
+        self.p4q.p4q_expand_codes(Wq, self.Wu[:n * Wq.shape[1] * 2].view(n, -1), self.sWu[:n])
+
+    def _gemm(self, layer, gname, Xu, sXu, s):
+        Wq = self.Wq[layer, gname]
+        n = Wq.shape[0]
+        self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, self.Wu[:n * Wq.shape[1] * 2].view(n, -1), self.sWu[:n],
+                                          self.s_w[layer, gname], self.Y[gname])
 
     def body(self):
         """The step as plain C-ABI calls (no graph)."""
@@ -310,7 +339,7 @@ class Step:
     def kernel_times(self):
         """Milliseconds of the most recent graph step (after a sync):
         {"select": ms, "quant": ms summed, "linear": {gemm: ms summed over layers}}."""
-        out = {"select": 0.0, "quant": 0.0, "linear": {g: 0.0 for g, _ in self.gemms}}
+        out = {"select": 0.0, "quant": 0.0, "expand": 0.0, "linear": {g: 0.0 for g, _ in self.gemms}}
         for i, (kind, name, _) in enumerate(self.segments):
             ms = self.events[i].elapsed_time(self.events[i + 1])
             if kind == "linear":
@@ -352,7 +381,7 @@ def run_gpu(args, rank, world, local_rank):
     clocks = ClockSampler(int(os.environ.get("P4Q_NVSMI_INDEX", local_rank)))
     e_start = torch.cuda.Event(enable_timing=True)
     e_end = torch.cuda.Event(enable_timing=True)
-    step_ms, sel_ms, gemm_ms = [], [], {g: [] for g, _ in step.gemms}
+    step_ms, sel_ms, exp_ms, quant_ms, gemm_ms = [], [], [], [], {g: [] for g, _ in step.gemms}
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -373,6 +402,8 @@ def run_gpu(args, rank, world, local_rank):
         torch.cuda.synchronize()
         kt = step.kernel_times()
         sel_ms.append(kt["select"])
+        exp_ms.append(kt["expand"])
+        quant_ms.append(kt["quant"])
         for n in gemm_ms:
             gemm_ms[n].append(kt["linear"][n])
     if world > 1:
@@ -456,10 +487,12 @@ def run_gpu(args, rank, world, local_rank):
                       "selector and per-GEMM times from segment graphs with events between them",
             "parallelism": f"dp{world} (independent batches)"},
         "select_prune_us_per_image": round(float(sel_ms.mean()) * 1e3 / w.B, 3),
+        "expand_us_per_step": round(float(np.mean(exp_ms)) * 1e3, 2),
+        "requant_us_per_step": round(float(np.mean(quant_ms)) * 1e3, 2),
         "gemm_tops": round(ach, 3),
         "pct_int8_tensor_peak": None,
         "pct_fp8_tensor_peak": round(100.0 * ach / peak, 2),
-        "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_pair_kernel (tcgen05 kind::f8f6f4, cta_group::2)",
+        "roofline": {"bound": "tensor", "kernel": "w4a4_gemm8_pair_kernel (tcgen05 kind::f8f6f4, cta_group::2, TMA-fed expanded operands)",
                      "achieved": round(ach, 3), "peak": round(peak, 1), "unit": "TFLOP/s",
                      "frac": round(ach / peak, 4), "traffic": traffic, "peak_source": peak_src,
                      "launches_timed": n_gemm,

@@ -184,6 +184,22 @@ p4q_status p4q_w4a4_linear_ws(const uint8_t* Xq, const float* s_a, int M, int Ki
                               const float* s_w, int N, uint16_t* Y, void* ws, size_t ws_bytes,
                               p4q_stream_t stream);
 
+/* The two halves of the expanded-operand path, for callers that expand an
+ * operand once and use it in several linears (activations shared by the q,
+ * k, v, gate and up projections) or keep expanded weights.
+ * p4q_expand_codes: packed INT4 rows q [rows, Kin/2] -> u [rows, Kin] bytes,
+ * u = v + 8 for each code v (per packed 32-bit word: its four low-nibble
+ * codes, then its four high-nibble codes), and sum_u [rows] int32.
+ *   Kin % 128 == 0, Kin <= P4Q_MAX_ROW; 16-byte aligned pointers; rows == 0 is a no-op.
+ * p4q_w4a4_linear_expanded: Y = fp16_rne(((float)acc * s_a[m]) * s_w[n]) with
+ * acc the exact integer dot product of the codes, from expanded operands
+ * (Xu, sum_xu: [M, Kin], [M]; Wu, sum_wu: [N, Kin], [N]); same results as
+ * p4q_w4a4_linear. Requires N >= 256, N % 8 == 0, Kin % 128 == 0. */
+p4q_status p4q_expand_codes(const uint8_t* q, int rows, int Kin, uint8_t* u, int32_t* sum_u, p4q_stream_t stream);
+p4q_status p4q_w4a4_linear_expanded(const uint8_t* Xu, const int32_t* sum_xu, const float* s_a, int M, int Kin,
+                                    const uint8_t* Wu, const int32_t* sum_wu, const float* s_w, int N, uint16_t* Y,
+                                    p4q_stream_t stream);
+
 /* Test view of the same path: the exact int32 accumulators (as
  * p4q_w4a4_gemm_s32). */
 p4q_status p4q_w4a4_gemm_s32_ws(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,

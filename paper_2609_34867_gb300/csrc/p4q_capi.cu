@@ -281,6 +281,38 @@ p4q_status p4q_w4a4_gemm_s32_ws(const uint8_t* Xq, int M, int Kin, const uint8_t
   return run_linear_ws(g, ws, ws_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
+p4q_status p4q_expand_codes(const uint8_t* q, int rows, int Kin, uint8_t* u, int32_t* sum_u, p4q_stream_t stream) {
+  if (rows < 0 || Kin < 1) return P4Q_ERR_INVALID_ARG;
+  if (rows > 0 && (!q || !u || !sum_u)) return P4Q_ERR_INVALID_ARG;
+  if (Kin % 128 != 0 || Kin > P4Q_MAX_ROW) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (rows > 0 && (!aligned16(q) || !aligned16(u) || !aligned16(sum_u))) return P4Q_ERR_MISALIGNED;
+  if (rows == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_expand_codes(q, rows, Kin, u, sum_u, reinterpret_cast<cudaStream_t>(stream))));
+}
+
+p4q_status p4q_w4a4_linear_expanded(const uint8_t* Xu, const int32_t* sum_xu, const float* s_a, int M, int Kin,
+                                    const uint8_t* Wu, const int32_t* sum_wu, const float* s_w, int N, uint16_t* Y,
+                                    p4q_stream_t stream) {
+  if (M < 0 || N < 1 || Kin < 1 || !Wu || !sum_wu || !s_w || (M > 0 && (!Xu || !sum_xu || !s_a || !Y)))
+    return P4Q_ERR_INVALID_ARG;
+  if (Kin % 128 != 0 || Kin > P4Q_MAX_ROW || N % 8 != 0 || N < 256) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned16(Wu) || (M > 0 && (!aligned16(Xu) || !aligned16(Y)))) return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  GemmArgs g;
+  g.M = M;
+  g.N = N;
+  g.K = Kin;
+  g.out = GemmOut::kHalf;
+  g.D = Y;
+  g.s_a = s_a;
+  g.s_b = s_w;
+  return from_cuda(counted(launch_gemm8(g, Xu, sum_xu, Wu, sum_wu, reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,
                              p4q_stream_t stream) {
   p4q_status st = check_gemm(Xq, M, Kin, Wq, N, acc);

@@ -429,15 +429,29 @@ bool gemm8_applies(const GemmArgs& g) {
   return g_gemm8_mode == 2 || g.M >= kMinRows;
 }
 
+cudaError_t launch_expand_codes(const uint8_t* q, int rows, int K, uint8_t* u, int32_t* sum_u, cudaStream_t stream) {
+  if (rows <= 0) return cudaSuccess;
+  return launch_pdl(expand_codes_kernel, dim3((rows + 7) / 8), dim3(256), 0, stream, q, rows, K, u, sum_u);
+}
+
+cudaError_t launch_gemm8(const GemmArgs& g, const uint8_t* a8, const int32_t* sum_a, const uint8_t* b8,
+                         const int32_t* sum_b, cudaStream_t stream) {
+  Ws8 w;
+  w.a8 = const_cast<uint8_t*>(a8);
+  w.b8 = const_cast<uint8_t*>(b8);
+  w.sum_a = const_cast<int32_t*>(sum_a);
+  w.sum_b = const_cast<int32_t*>(sum_b);
+  return g.out == GemmOut::kHalf ? launch8<0>(g, w, stream) : launch8<1>(g, w, stream);
+}
+
 cudaError_t launch_w4a4_gemm8(const GemmArgs& g, void* ws, size_t ws_bytes, cudaStream_t stream) {
   Ws8 w;
   if (!ws || ws_bytes < ws8_layout(g.M, g.N, g.K, ws, &w)) return cudaErrorInvalidValue;
-  cudaError_t e = launch_pdl(expand_codes_kernel, dim3((g.M + 7) / 8), dim3(256), 0, stream, g.A, g.M, g.K, w.a8,
-                             w.sum_a);
+  cudaError_t e = launch_expand_codes(g.A, g.M, g.K, w.a8, w.sum_a, stream);
   if (e != cudaSuccess) return e;
-  e = launch_pdl(expand_codes_kernel, dim3((g.N + 7) / 8), dim3(256), 0, stream, g.B, g.N, g.K, w.b8, w.sum_b);
+  e = launch_expand_codes(g.B, g.N, g.K, w.b8, w.sum_b, stream);
   if (e != cudaSuccess) return e;
-  return g.out == GemmOut::kHalf ? launch8<0>(g, w, stream) : launch8<1>(g, w, stream);
+  return launch_gemm8(g, w.a8, w.sum_a, w.b8, w.sum_b, stream);
 }
 
 unsigned int gemm8_read_and_clear_error() {

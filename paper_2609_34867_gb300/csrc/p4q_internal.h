@@ -127,6 +127,11 @@ size_t gemm8_workspace_bytes(int M, int N, int K);
 bool gemm8_applies(const GemmArgs& g);
 // Expands both operands into the workspace, then runs the FP8 GEMM.
 cudaError_t launch_w4a4_gemm8(const GemmArgs& g, void* ws, size_t ws_bytes, cudaStream_t stream);
+// The two halves: packed rows -> one byte per code (u = v + 8) + row sums of u;
+// the GEMM on expanded operands (g.A / g.B unused; batch 1, N >= 256).
+cudaError_t launch_expand_codes(const uint8_t* q, int rows, int K, uint8_t* u, int32_t* sum_u, cudaStream_t stream);
+cudaError_t launch_gemm8(const GemmArgs& g, const uint8_t* a8, const int32_t* sum_a, const uint8_t* b8,
+                         const int32_t* sum_b, cudaStream_t stream);
 
 // One bounded wait that nothing completes: times out after limit_ns and sets
 // the GEMM's device error word (tests the time-out path).

@@ -67,6 +67,10 @@ def lib() -> ctypes.CDLL:
         L.p4q_w4a4_linear_ws.restype = st
         L.p4q_w4a4_gemm_s32_ws.argtypes = [P, I, I, P, I, P, P, S, P]
         L.p4q_w4a4_gemm_s32_ws.restype = st
+        L.p4q_expand_codes.argtypes = [P, I, I, P, P, P]
+        L.p4q_expand_codes.restype = st
+        L.p4q_w4a4_linear_expanded.argtypes = [P, P, P, I, I, P, P, P, I, P, P]
+        L.p4q_w4a4_linear_expanded.restype = st
         L.p4q_select_workspace_bytes.argtypes = [I, I, I, I, ctypes.POINTER(SelectParams)]
         L.p4q_select_workspace_bytes.restype = S
         L.p4q_select.argtypes = [P, I, I, I, P, I, P, ctypes.POINTER(SelectParams), P, P, S, P]
@@ -242,6 +246,30 @@ def w4a4_gemm_s32_ws(Xq, Wq, ws, stream=None):
     _check(lib().p4q_w4a4_gemm_s32_ws(_ptr(Xq), M, K, _ptr(Wq), N, _ptr(acc), wp, wn, _stream(stream)),
            "p4q_w4a4_gemm_s32_ws")
     return acc
+
+
+def p4q_expand_codes(q, u, sum_u, stream=None):
+    """Packed codes q [rows, K/2] uint8 -> u [rows, K] uint8 (u = v + 8), sum_u [rows] int32."""
+    _need(q, torch.uint8, 2, "q"); _need(u, torch.uint8, 2, "u"); _need(sum_u, torch.int32, 1, "sum_u")
+    rows, K = q.shape[0], q.shape[1] * 2
+    _check(lib().p4q_expand_codes(_ptr(q), rows, K, _ptr(u), _ptr(sum_u), _stream(stream)), "p4q_expand_codes")
+
+
+def expand_codes(q, stream=None):
+    """Allocating wrapper of p4q_expand_codes: returns (u, sum_u)."""
+    u = torch.empty((q.shape[0], q.shape[1] * 2), dtype=torch.uint8, device=q.device)
+    s = torch.empty((q.shape[0],), dtype=torch.int32, device=q.device)
+    p4q_expand_codes(q, u, s, stream)
+    return u, s
+
+
+def p4q_w4a4_linear_expanded(Xu, sum_xu, s_a, Wu, sum_wu, s_w, Y, stream=None):
+    """Y [M, N] fp16 from expanded operands (see p4q_expand_codes)."""
+    _need(Xu, torch.uint8, 2, "Xu"); _need(Wu, torch.uint8, 2, "Wu"); _need(Y, torch.float16, 2, "Y")
+    M, K = Xu.shape
+    N = Wu.shape[0]
+    _check(lib().p4q_w4a4_linear_expanded(_ptr(Xu), _ptr(sum_xu), _ptr(s_a), M, K, _ptr(Wu), _ptr(sum_wu), _ptr(s_w),
+                                          N, _ptr(Y), _stream(stream)), "p4q_w4a4_linear_expanded")
 
 
 def w4a4_gemm_s32(Xq, Wq, stream=None):

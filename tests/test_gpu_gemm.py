@@ -140,3 +140,33 @@ def test_expanded_linear_rejects_a_short_workspace(p4q, dev):
     short = torch.empty((1024,), dtype=torch.uint8, device=dev)
     with pytest.raises(p4q.P4QError):
         p4q.p4q_w4a4_linear_ws(Xq, s, Wq, s[:512], Y, short)
+
+
+def test_expand_codes_layout_and_sums(p4q, dev):
+    """One byte u = v + 8 per code; per packed 32-bit word its four low-nibble
+    codes, then its four high-nibble codes; sum_u per row."""
+    rng = np.random.default_rng(3)
+    q = _packed(rng, 37, 384)
+    u, s = p4q.expand_codes(torch.from_numpy(q).to(dev))
+    torch.cuda.synchronize()
+    v = oracle.unpack_codes(q).astype(np.int32) + 8          # [rows, K] natural order
+    w = v.reshape(37, -1, 4, 2)                              # [rows, word, byte, (lo, hi)]
+    expect = np.concatenate([w[..., 0], w[..., 1]], axis=2).reshape(37, -1)
+    assert np.array_equal(u.cpu().numpy().astype(np.int32), expect)
+    assert np.array_equal(s.cpu().numpy(), v.sum(axis=1))
+
+
+def test_linear_expanded_matches_linear(p4q, dev):
+    rng = np.random.default_rng(4)
+    M, N, K = 300, 512, 1024
+    a, w = torch.from_numpy(_packed(rng, M, K)).to(dev), torch.from_numpy(_packed(rng, N, K)).to(dev)
+    sa = torch.rand(M, device=dev) * 0.3 + 0.01
+    sw = torch.rand(N, device=dev) * 0.002 + 1e-4
+    ref = p4q.w4a4_linear(a, sa, w, sw)
+    Xu, sX = p4q.expand_codes(a)
+    Wu, sW = p4q.expand_codes(w)
+    Y = torch.empty((M, N), dtype=torch.float16, device=dev)
+    p4q.p4q_w4a4_linear_expanded(Xu, sX, sa, Wu, sW, sw, Y)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    assert torch.equal(Y.view(torch.int16), ref.view(torch.int16))
