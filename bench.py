@@ -248,13 +248,17 @@ class Step:
             self.sXu_re[name] = torch.empty((M,), dtype=torch.int32, device=dev)
         wmax = max(self.Wq[0, g].shape[0] * self.Wq[0, g].shape[1] * 2 for g, _ in self.gemms)
         nmax = max(self.Wq[0, g].shape[0] for g, _ in self.gemms)
-        self.Wu = torch.empty((wmax,), dtype=torch.uint8, device=dev)
-        self.sWu = torch.empty((nmax,), dtype=torch.int32, device=dev)
+        # two weight scratches: the next GEMM's weights expand on a side stream
+        # while the current GEMM (or the selector, for the first) runs
+        self.Wu = [torch.empty((wmax,), dtype=torch.uint8, device=dev) for _ in range(2)]
+        self.sWu = [torch.empty((nmax,), dtype=torch.int32, device=dev) for _ in range(2)]
+        self.side = torch.cuda.Stream(device=dev)
         # The step is a chain of segments (selector, each expansion, each GEMM,
         # each re-quantization); the timed loop replays it as one CUDA graph,
         # the breakdown replays one graph per segment with events between them.
         self.segments = [("select", "select", self._select),
                          ("expand", "expand_x", lambda: p4q.p4q_expand_codes(self.Xq, self.Xu, self.sXu))]
+        self.gemm_calls = []  # (layer, gemm, input) in step order
         for layer in range(w.layers):
             for gname, members in self.gemms:
                 if members[0] in self.REQUANT:
@@ -266,8 +270,9 @@ class Step:
                     xin = (lambda n=name: (self.Xu_re[n], self.sXu_re[n], self.s_re[n]))
                 else:
                     xin = (lambda: (self.Xu, self.sXu, self.s_a))
-                self.segments.append(("expand", "expand_w_" + gname, (lambda l=layer, g=gname: self._expand_w(l, g))))
-                self.segments.append(("linear", gname, (lambda l=layer, g=gname, x=xin: self._gemm(l, g, *x()))))
+                self.segments.append(("expand", "expand_w_" + gname, (lambda l=layer, g=gname: self._expand_w(l, g, 0))))
+                self.segments.append(("linear", gname, (lambda l=layer, g=gname, x=xin: self._gemm(l, g, 0, *x()))))
+                self.gemm_calls.append((layer, gname, xin))
         self.lin_ops = {g: sum(2 * w.M * dims[m].n_out * dims[m].k_in for m in members) * w.layers
                         for g, members in self.gemms}
         self.graphs = None
@@ -288,21 +293,62 @@ class Step:
         self.p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
                                          self.s_a, self.ws)
 
-    def _expand_w(self, layer, gname):
+    def _wu(self, layer, gname, slot):
         Wq = self.Wq[layer, gname]
         n = Wq.shape[0]
-        self.p4q.p4q_expand_codes(Wq, self.Wu[:n * Wq.shape[1] * 2].view(n, -1), self.sWu[:n])
+        return self.Wu[slot][:n * Wq.shape[1] * 2].view(n, -1), self.sWu[slot][:n]
 
-    def _gemm(self, layer, gname, Xu, sXu, s):
-        Wq = self.Wq[layer, gname]
-        n = Wq.shape[0]
-        self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, self.Wu[:n * Wq.shape[1] * 2].view(n, -1), self.sWu[:n],
-                                          self.s_w[layer, gname], self.Y[gname])
+    def _expand_w(self, layer, gname, slot, stream=None):
+        u, su = self._wu(layer, gname, slot)
+        self.p4q.p4q_expand_codes(self.Wq[layer, gname], u, su, stream)
 
-    def body(self):
-        """The step as plain C-ABI calls (no graph)."""
+    def _gemm(self, layer, gname, slot, Xu, sXu, s):
+        u, su = self._wu(layer, gname, slot)
+        self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, u, su, self.s_w[layer, gname], self.Y[gname])
+
+    def body_serial(self):
+        """The step's segments one after another on the current stream."""
         for _, _, fn in self.segments:
             fn()
+
+    def body(self):
+        """The step as plain C-ABI calls (no graph). Weight expansions run on a
+        side stream one GEMM ahead, into two alternating scratches: the first
+        overlaps the selector, each later one the previous GEMM."""
+        torch = self.torch
+        main = torch.cuda.current_stream()
+        self.side.wait_stream(main)  # fork: inputs of this step are in place
+        ready = [torch.cuda.Event() for _ in self.gemm_calls]
+        freed = [torch.cuda.Event() for _ in self.gemm_calls]
+
+        def expand(i):
+            layer, gname, _ = self.gemm_calls[i]
+            with torch.cuda.stream(self.side):
+                if i >= 2:
+                    self.side.wait_event(freed[i - 2])  # the scratch's previous GEMM is done
+                self._expand_w(layer, gname, i % 2, self.side)
+                ready[i].record(self.side)
+
+        n = len(self.gemm_calls)
+        if n:
+            expand(0)
+        if n > 1:
+            expand(1)
+        gi = 0
+        for kind, _, fn in self.segments:
+            if kind == "expand" and _.startswith("expand_w_"):
+                continue  # done on the side stream
+            if kind == "linear":
+                layer, gname, xin = self.gemm_calls[gi]
+                main.wait_event(ready[gi])
+                self._gemm(layer, gname, gi % 2, *xin())
+                freed[gi].record(main)
+                if gi + 2 < n:
+                    expand(gi + 2)
+                gi += 1
+            else:
+                fn()
+        main.wait_stream(self.side)  # join
 
     def capture(self):
         """Captures the whole step into one CUDA graph (consecutive kernels
@@ -316,6 +362,8 @@ class Step:
             with torch.cuda.graph(g):
                 fn()
             self.graphs.append(g)
+        self.body()  # warm the side-stream path before capturing it
+        torch.cuda.synchronize()
         n0 = self.p4q.p4q_launch_count()
         self.full = torch.cuda.CUDAGraph()
         with torch.cuda.graph(self.full):
