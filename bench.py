@@ -52,11 +52,11 @@ METRIC = "W4A4 prefill linear TOPS (% INT8 tensor peak); select+prune µs/image"
 WORKLOAD = wl.LLAVA15_7B
 FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed steps
 
-# Latest ncu capture of the dominant kernel: mean DRAM bytes (read + write)
-# per launch over the four GEMMs of one step (profiles/
-# w4a4_gemm_pair_llava15_7b_b8_step.md, section 2), valid only while the GEMM
-# source is unchanged since the capture.
-PROFILED_GEMM = {"source_sha1": "", "dram_bytes_per_launch": 0}
+# Latest ncu capture of the dominant kernel (the expanded-operand GEMM): mean
+# DRAM bytes (read + write) per launch over the four GEMMs of one step
+# (profiles/w4a4_gemm_llava15_7b_b8_step.md, section 2), valid only while the
+# GEMM source is unchanged since the capture.
+PROFILED_GEMM = {"source_sha1": "609f6df13de63f704fd7dc885994a527d6ed8a2c", "dram_bytes_per_launch": 80020672}
 
 
 def gemm_source_sha1() -> str:

@@ -1,6 +1,7 @@
 """Single-call cases of the hot path, for profiling and microbenchmarks.
 
   python -m paper_2609_34867_gb300.kernel_cases gemm M N K [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases gemm8 M N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases quant M K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [--reps R]
 
@@ -13,6 +14,8 @@ selects the first replayed launch.
 
   gemm    p4q_w4a4_linear on random packed codes: M x K activations,
           N x K weights, fp16 output (2 M N K integer ops per call);
+  gemm8   p4q_w4a4_linear_expanded on the same operands expanded once by
+          p4q_expand_codes before timing (the GEMM kernel alone);
   quant   p4q_quant_act on M x K fp16 activations with the outlier channels
           (bytes: 2 M K in, M K / 2 + 4 M out);
   select  p4q_select_gather_quant on one of the LLaVA-shaped workloads.
@@ -58,14 +61,14 @@ def _timed(fn, reps, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "quant", "select"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "select"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
     dev = torch.device("cuda:0")
     torch.cuda.set_device(dev)
     p4q.lib()
-    if a.case == "gemm":
+    if a.case in ("gemm", "gemm8"):
         M, N, K = (int(x) for x in a.args)
         g = torch.Generator(device=dev).manual_seed(0)
         Xq = torch.randint(0, 256, (M, K // 2), dtype=torch.uint8, device=dev, generator=g)
@@ -73,8 +76,13 @@ def main(argv=None):
         s_a = torch.rand(M, device=dev, generator=g)
         s_w = torch.rand(N, device=dev, generator=g) * 0.01
         Y = torch.empty((M, N), dtype=torch.float16, device=dev)
-        ms = _timed(lambda: p4q.p4q_w4a4_linear(Xq, s_a, Wq, s_w, Y), a.reps, dev)
-        print(f"gemm {M}x{N}x{K}: {ms * 1e3:.1f} us/call, {2 * M * N * K / ms / 1e9:.1f} TOPS")
+        if a.case == "gemm":
+            ms = _timed(lambda: p4q.p4q_w4a4_linear(Xq, s_a, Wq, s_w, Y), a.reps, dev)
+        else:
+            Xu, sX = p4q.expand_codes(Xq)
+            Wu, sW = p4q.expand_codes(Wq)
+            ms = _timed(lambda: p4q.p4q_w4a4_linear_expanded(Xu, sX, s_a, Wu, sW, s_w, Y), a.reps, dev)
+        print(f"{a.case} {M}x{N}x{K}: {ms * 1e3:.1f} us/call, {2 * M * N * K / ms / 1e9:.1f} TOPS")
     elif a.case == "quant":
         M, K = (int(x) for x in a.args)
         X = torch.from_numpy(wl.activations(M, K, seed=wl.SWEEP_SEED)).to(dev)
