@@ -5,10 +5,10 @@ One step = the whole path over one batch of the LLaVA-1.5-7B-shaped workload
 budget 192 kept tokens per image):
   p4q_select_gather_quant  fake-quant -> query / saliency / diversity stages
                            -> gather of the kept FP16 rows + text -> INT4
-  p4q_expand_codes         the pruned sequence's codes, one byte per code
-                           (once, for the four GEMMs that read it), each
-                           GEMM's packed weights (per call), the re-quantized
-                           o / down inputs
+  (the selector's gather and the two re-quantizations also write their
+  codes in the expanded form, one byte per code, that the GEMMs read)
+  p4q_expand_codes         each GEMM's packed INT4 weights, per call, on a
+                           side stream one GEMM ahead
   p4q_w4a4_linear_expanded x 4  q|k|v and gate|up (each one GEMM over the
                            concatenated output channels) on the pruned
                            sequence (M = 2048), o on the re-quantized q
@@ -56,7 +56,7 @@ FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed step
 # DRAM bytes (read + write) per launch over the four GEMMs of one step
 # (profiles/w4a4_gemm_llava15_7b_b8_step.md, section 2), valid only while the
 # GEMM source is unchanged since the capture.
-PROFILED_GEMM = {"source_sha1": "609f6df13de63f704fd7dc885994a527d6ed8a2c", "dram_bytes_per_launch": 80020672}
+PROFILED_GEMM = {"source_sha1": "4e651cb373181f70736026a123aaa3ea35814df5", "dram_bytes_per_launch": 80020672}
 
 
 def gemm_source_sha1() -> str:
@@ -256,17 +256,14 @@ class Step:
         # The step is a chain of segments (selector, each expansion, each GEMM,
         # each re-quantization); the timed loop replays it as one CUDA graph,
         # the breakdown replays one graph per segment with events between them.
-        self.segments = [("select", "select", self._select),
-                         ("expand", "expand_x", lambda: p4q.p4q_expand_codes(self.Xq, self.Xu, self.sXu))]
+        self.segments = [("select", "select", self._select)]
         self.gemm_calls = []  # (layer, gemm, input) in step order
         for layer in range(w.layers):
             for gname, members in self.gemms:
                 if members[0] in self.REQUANT:
                     name = members[0]
-                    self.segments.append(("quant", "quant_" + name, (lambda n=name: p4q.p4q_quant_act_ld(
-                        self.output(self.REQUANT[n]), self.Xq_re[n], self.s_re[n]))))
-                    self.segments.append(("expand", "expand_" + name, (lambda n=name: p4q.p4q_expand_codes(
-                        self.Xq_re[n], self.Xu_re[n], self.sXu_re[n]))))
+                    self.segments.append(("quant", "quant_" + name, (lambda n=name: p4q.p4q_quant_act_expanded(
+                        self.output(self.REQUANT[n]), self.Xq_re[n], self.s_re[n], self.Xu_re[n], self.sXu_re[n]))))
                     xin = (lambda n=name: (self.Xu_re[n], self.sXu_re[n], self.s_re[n]))
                 else:
                     xin = (lambda: (self.Xu, self.sXu, self.s_a))
@@ -290,8 +287,8 @@ class Step:
         return self.Wq[layer, g][off:off + n], self.s_w[layer, g][off:off + n]
 
     def _select(self):
-        self.p4q.p4q_select_gather_quant(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X, self.Xq,
-                                         self.s_a, self.ws)
+        self.p4q.p4q_select_gather_quant_expanded(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X,
+                                                  self.Xq, self.s_a, self.Xu, self.sXu, self.ws)
 
     def _wu(self, layer, gname, slot):
         Wq = self.Wq[layer, gname]

@@ -132,6 +132,13 @@ p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* 
 p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
                             p4q_stream_t stream);
 
+/* p4q_quant_act_ld that also writes the codes in the expanded form of
+ * p4q_expand_codes (Xu [M, Kin] bytes, sum_xu [M] int32), for
+ * p4q_w4a4_linear_expanded, without a second pass. The paper has no
+ * counterpart. */
+p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a, uint8_t* Xu,
+                                  int32_t* sum_xu, p4q_stream_t stream);
+
 /* Per-output-channel weight quantization (App. B.3: symmetric, per output
  * channel, then round-to-nearest): the same per-row quantizer applied to each
  * output row of W.
@@ -274,6 +281,16 @@ p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const
                                    const p4q_select_params* params, int32_t* idx, uint16_t* X,
                                    uint8_t* Xq, float* s_a, void* ws, size_t ws_bytes,
                                    p4q_stream_t stream);
+
+/* p4q_select_gather_quant that also writes the pruned sequence's codes in
+ * the expanded form of p4q_expand_codes (Xu [B*(K+T), d] bytes, sum_xu
+ * [B*(K+T)] int32; both NULL or both set), for p4q_w4a4_linear_expanded,
+ * without a second pass over the codes. The paper has no counterpart. */
+p4q_status p4q_select_gather_quant_expanded(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
+                                            const float* A_cls, const uint16_t* text, int T,
+                                            const p4q_select_params* params, int32_t* idx, uint16_t* X,
+                                            uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, void* ws,
+                                            size_t ws_bytes, p4q_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -184,6 +184,25 @@ p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* 
   return p4q_quant_act_ld(X, Kin, M, Kin, Xq, s_a, stream);
 }
 
+p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a, uint8_t* Xu,
+                                  int32_t* sum_xu, p4q_stream_t stream) {
+  p4q_status st = check_rows(X, M, Kin, Xq, s_a);
+  if (st != P4Q_OK) return st;
+  if (ldx < Kin || (M > 0 && (!Xu || !sum_xu))) return P4Q_ERR_INVALID_ARG;
+  if (ldx % 8 != 0 || (M > 0 && (!aligned16(Xu) || !aligned16(sum_xu)))) return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
+  if ((st = check_device()) != P4Q_OK) return st;
+  RowSource src;
+  src.X = X;
+  src.ldx = ldx;
+  RowSinks o;
+  o.codes = Xq;
+  o.scale = s_a;
+  o.u = Xu;
+  o.sum_u = sum_xu;
+  return from_cuda(counted(launch_quant_rows(src, M, Kin, o, reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
                             p4q_stream_t stream) {
   p4q_status st = check_rows(X, M, Kin, Xq, s_a);
@@ -349,10 +368,20 @@ p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const
                                    const float* A_cls, const uint16_t* text, int T,
                                    const p4q_select_params* params, int32_t* idx, uint16_t* X, uint8_t* Xq,
                                    float* s_a, void* ws, size_t ws_bytes, p4q_stream_t stream) {
+  return p4q_select_gather_quant_expanded(V, B, N, d, Q, J, A_cls, text, T, params, idx, X, Xq, s_a, nullptr,
+                                          nullptr, ws, ws_bytes, stream);
+}
+
+p4q_status p4q_select_gather_quant_expanded(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
+                                            const float* A_cls, const uint16_t* text, int T,
+                                            const p4q_select_params* params, int32_t* idx, uint16_t* X,
+                                            uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, void* ws,
+                                            size_t ws_bytes, p4q_stream_t stream) {
   p4q_status st = check_select_args(V, B, N, d, J, params, idx);
   if (st != P4Q_OK) return st;
-  if (T < 0 || (T > 0 && !text) || !X || !Xq || !s_a) return P4Q_ERR_INVALID_ARG;
+  if (T < 0 || (T > 0 && !text) || !X || !Xq || !s_a || (!Xu != !sum_xu)) return P4Q_ERR_INVALID_ARG;
   if ((T > 0 && !aligned16(text)) || !aligned16(X) || !aligned16(Xq) || !aligned16(s_a)) return P4Q_ERR_MISALIGNED;
+  if (Xu && (!aligned16(Xu) || !aligned16(sum_xu))) return P4Q_ERR_MISALIGNED;
   if ((st = check_device()) != P4Q_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   st = run_select(V, B, N, d, Q, J, A_cls, params, idx, ws, ws_bytes, s);
@@ -370,6 +399,8 @@ p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const
   o.codes = Xq;
   o.scale = s_a;
   o.copy = X;
+  o.u = Xu;
+  o.sum_u = sum_xu;
   return from_cuda(counted(launch_quant_rows(src, B * (params->K + T), d, o, s)));
 }
 

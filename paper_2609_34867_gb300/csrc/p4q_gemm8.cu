@@ -11,9 +11,9 @@
 // alone, already in the 128-byte-swizzled K-major layout the MMAs read.
 //
 // Byte order inside each 16-byte packed chunk (32 codes): for each packed
-// 32-bit word, its four low-nibble codes, then its four high-nibble codes.
-// The permutation is the same for both operands, so every dot product is
-// unchanged.
+// 32-bit word, its four low-nibble codes, then its four high-nibble codes
+// (p4q_expand.cu). The permutation is the same for both operands, so every
+// dot product is unchanged.
 //
 // Kernel: persistent, one cluster of two CTAs per 256 x 256 output tile,
 //   warp 0    MMA issuer (leader CTA): 4 x tcgen05.mma (M 256, N 256, K 32)
@@ -310,46 +310,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
 }
 
-// One warp per row: packed codes [rows, K/2] -> one byte per code u = v + 8
-// [rows, K] (per packed 32-bit word: its four low-nibble codes, then its four
-// high-nibble codes) and sum_u[row]. All of a lane's 16-byte loads of the row
-// are issued before the first store (MAXC chunks per lane).
-template <int MAXC>
-__global__ void __launch_bounds__(256) expand_codes_kernel(const uint8_t* __restrict__ src, int rows, int K,
-                                                           uint8_t* __restrict__ dst, int32_t* __restrict__ sums) {
-  pdl_wait();
-  pdl_launch_dependents();
-  const int row = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (row >= rows) return;
-  const uint4* s4 = reinterpret_cast<const uint4*>(src + static_cast<size_t>(row) * (K >> 1));
-  uint4* d4 = reinterpret_cast<uint4*>(dst + static_cast<size_t>(row) * K);
-  const int nch = K >> 5;  // 16-byte packed chunks per row
-  uint4 w[MAXC];
-#pragma unroll
-  for (int i = 0; i < MAXC; ++i) {
-    const int c = lane + 32 * i;
-    if (c < nch) w[i] = ldg_stream16(s4 + c);
-  }
-  constexpr uint32_t ones = 0x01010101u;
-  uint32_t acc = 0;
-#pragma unroll
-  for (int i = 0; i < MAXC; ++i) {
-    const int c = lane + 32 * i;
-    if (c < nch) {
-      const uint32_t l0 = (w[i].x & 0x0F0F0F0Fu) ^ 0x08080808u, h0 = ((w[i].x >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
-      const uint32_t l1 = (w[i].y & 0x0F0F0F0Fu) ^ 0x08080808u, h1 = ((w[i].y >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
-      const uint32_t l2 = (w[i].z & 0x0F0F0F0Fu) ^ 0x08080808u, h2 = ((w[i].z >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
-      const uint32_t l3 = (w[i].w & 0x0F0F0F0Fu) ^ 0x08080808u, h3 = ((w[i].w >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
-      d4[2 * c] = make_uint4(l0, h0, l1, h1);
-      d4[2 * c + 1] = make_uint4(l2, h2, l3, h3);
-      // byte-wise sum of the eight words first (each byte <= 8 x 15 < 256), then one dp4a
-      acc = __dp4a(l0 + h0 + l1 + h1 + l2 + h2 + l3 + h3, ones, acc);
-    }
-  }
-  acc = __reduce_add_sync(0xFFFFFFFFu, acc);
-  if (lane == 0) sums[row] = static_cast<int32_t>(acc);
-}
-
 // 3-D map over expanded codes: dims (K bytes, rows, 1), 128 x box_rows boxes,
 // 128-byte swizzle (the K-major layout the MMA descriptors describe).
 bool make_expanded_map(CUtensorMap* map, const uint8_t* base, int K, int rows, int box_rows) {
@@ -431,15 +391,6 @@ bool gemm8_applies(const GemmArgs& g) {
   if (g_gemm8_mode == 1) return false;
   if (g.batch != 1 || g.M <= 0 || g.N < 256 || (g.out != GemmOut::kHalf && g.out != GemmOut::kS32)) return false;
   return g_gemm8_mode == 2 || g.M >= kMinRows;
-}
-
-cudaError_t launch_expand_codes(const uint8_t* q, int rows, int K, uint8_t* u, int32_t* sum_u, cudaStream_t stream) {
-  if (rows <= 0) return cudaSuccess;
-  const dim3 grid((rows + 7) / 8), block(256);
-  const int nch = K >> 5;
-  if (nch <= 32 * 4) return launch_pdl(expand_codes_kernel<4>, grid, block, 0, stream, q, rows, K, u, sum_u);
-  if (nch <= 32 * 8) return launch_pdl(expand_codes_kernel<8>, grid, block, 0, stream, q, rows, K, u, sum_u);
-  return launch_pdl(expand_codes_kernel<16>, grid, block, 0, stream, q, rows, K, u, sum_u);
 }
 
 cudaError_t launch_gemm8(const GemmArgs& g, const uint8_t* a8, const int32_t* sum_a, const uint8_t* b8,

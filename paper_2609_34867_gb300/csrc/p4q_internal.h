@@ -47,6 +47,8 @@ struct RowSinks {
   float* scale = nullptr;     // [rows] (required)
   int32_t* norm2 = nullptr;   // [rows] sum of squared codes
   uint16_t* copy = nullptr;   // [rows, L] fp16 copy of the source row (gather mode)
+  uint8_t* u = nullptr;       // [rows, L] codes expanded to one byte each (u = v + 8, the GEMM's order)
+  int32_t* sum_u = nullptr;   // [rows] sum of u (with u)
 };
 
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,

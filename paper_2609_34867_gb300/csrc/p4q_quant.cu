@@ -114,7 +114,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(kGroups) * S * stage_bytes);
   uint32_t* red = reinterpret_cast<uint32_t*>(bars + kGroups * kMaxStages);
   int* red_n = reinterpret_cast<int*>(red + kWarps);
-  int* aborts = red_n + kWarps;
+  int* red_u = red_n + kWarps;
+  int* aborts = red_u + kWarps;
   if (threadIdx.x < kGroups * S) mbar_init(&bars[threadIdx.x], 1);
   if (threadIdx.x < kGroups) aborts[threadIdx.x] = 0;
   fence_barrier_init();
@@ -174,20 +175,33 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
 
     float2 n2 = make_float2(0.0f, 0.0f);  // exact: sums of squared codes <= 49 * 16384 < 2^24
+    uint32_t su = 0;                      // sum of the expanded codes u = v + 8 (expanded output)
     if (!failed) {
       uint32_t* q4 = reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(row) * (L >> 1));
       uint4* cp = out.copy ? reinterpret_cast<uint4*>(out.copy + static_cast<size_t>(row) * L) : nullptr;
+      uint2* up = out.u ? reinterpret_cast<uint2*>(out.u + static_cast<size_t>(row) * L) : nullptr;
 #pragma unroll 4
       for (int c = gt; c < nch; c += kGroupThreads) {
         const uint4 v = v4[c];
-        q4[c] = (a != 0.0f) ? quant_chunk<NORM>(v, s, inv, n2) : 0u;
+        const uint32_t pw = (a != 0.0f) ? quant_chunk<NORM>(v, s, inv, n2) : 0u;
+        q4[c] = pw;
         if (cp) cp[c] = v;
+        if (up) {
+          // one byte per code, u = v + 8: the word's four low-nibble codes, then its four high-nibble codes
+          const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+          up[c] = make_uint2(eu, ou);
+          su = __dp4a(eu + ou, 0x01010101u, su);
+        }
       }
     }
-    int wn = 0;
+    int wn = 0, wu = 0;
     if (NORM) {
       wn = __reduce_add_sync(0xFFFFFFFFu, static_cast<int>(n2.x + n2.y));
       if (G > 1 && lane == 0) red_n[warp] = wn;
+    }
+    if (out.sum_u) {
+      wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
+      if (G > 1 && lane == 0) red_u[warp] = wu;
     }
     // every warp of the group is done with buffer st (and has published red_n)
     if (G > 1)
@@ -199,10 +213,16 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 #pragma unroll
       for (int w = 0; w < G; ++w) wn += red_n[grp * G + w];
     }
+    if (out.sum_u && G > 1) {
+      wu = 0;
+#pragma unroll
+      for (int w = 0; w < G; ++w) wu += red_u[grp * G + w];
+    }
     if (leader) {
       if (!failed) {
         out.scale[row] = (a != 0.0f) ? s : 0.0f;
         if (NORM) out.norm2[row] = wn;
+        if (out.sum_u) out.sum_u[row] = wu;
         if (issued < mine) {
           mbar_arrive_expect_tx(&full[st], row_bytes);
           bulk_load(ring + static_cast<size_t>(st) * stage_bytes, row_ptr(src, first + issued * total, L), row_bytes,
@@ -268,7 +288,7 @@ cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out,
   }
   constexpr int kGroups = kWarps / G;
   const size_t smem = static_cast<size_t>(kGroups) * p.S * p.stage_bytes + kGroups * kMaxStages * 8 +
-                      2 * kWarps * 4 + kGroups * 4;
+                      3 * kWarps * 4 + kGroups * 4;
   const int need = (rows + kGroups - 1) / kGroups;
   const int grid = std::min(need, kCtasPerSm * sm_count());
   return launch_pdl(quant_rows_kernel<G, NORM>, dim3(grid), dim3(kThreads), smem, stream, src, rows, L, out, p.S,

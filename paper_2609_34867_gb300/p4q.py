@@ -55,6 +55,11 @@ def lib() -> ctypes.CDLL:
         L.p4q_quant_act.restype = st
         L.p4q_quant_act_ld.argtypes = [P, I, I, I, P, P, P]
         L.p4q_quant_act_ld.restype = st
+        L.p4q_quant_act_expanded.argtypes = [P, I, I, I, P, P, P, P, P]
+        L.p4q_quant_act_expanded.restype = st
+        L.p4q_select_gather_quant_expanded.argtypes = [P, I, I, I, P, I, P, P, I, ctypes.POINTER(SelectParams), P,
+                                                       P, P, P, P, P, P, S, P]
+        L.p4q_select_gather_quant_expanded.restype = st
         L.p4q_quant_weight.argtypes = [P, I, I, P, P, P]
         L.p4q_quant_weight.restype = st
         L.p4q_w4a4_linear.argtypes = [P, P, I, I, P, P, I, P, P]
@@ -141,6 +146,17 @@ def p4q_quant_act_ld(X, Xq, s_a, stream=None):
            "p4q_quant_act_ld")
 
 
+def p4q_quant_act_expanded(X, Xq, s_a, Xu, sum_xu, stream=None):
+    """p4q_quant_act_ld plus the expanded codes (see p4q_expand_codes)."""
+    if not isinstance(X, torch.Tensor) or X.dtype != torch.float16 or X.dim() != 2 or X.stride(1) != 1 or not X.is_cuda:
+        raise TypeError("X: expected a CUDA fp16 2-D tensor with unit column stride")
+    _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    _need(Xu, torch.uint8, 2, "Xu"); _need(sum_xu, torch.int32, 1, "sum_xu")
+    M, K = X.shape
+    _check(lib().p4q_quant_act_expanded(_ptr(X), X.stride(0), M, K, _ptr(Xq), _ptr(s_a), _ptr(Xu), _ptr(sum_xu),
+                                        _stream(stream)), "p4q_quant_act_expanded")
+
+
 def p4q_quant_weight(W, Wq, s_w, stream=None):
     """W [N, Kin] fp16 -> Wq [N, Kin/2] uint8, s_w [N] fp32 (one scale per output channel)."""
     _need(W, torch.float16, 2, "W"); _need(Wq, torch.uint8, 2, "Wq"); _need(s_w, torch.float32, 1, "s_w")
@@ -193,6 +209,22 @@ def p4q_select_gather_quant(V, Q, A_cls, text, K, idx, X, Xq, s_a, ws, alpha_per
     _check(lib().p4q_select_gather_quant(_ptr(V), B, N, d, _ptr(Q), J, _ptr(A_cls), _ptr(text), T,
                                          ctypes.byref(p), _ptr(idx), _ptr(X), _ptr(Xq), _ptr(s_a), _ptr(ws),
                                          ws.numel(), _stream(stream)), "p4q_select_gather_quant")
+
+
+def p4q_select_gather_quant_expanded(V, Q, A_cls, text, K, idx, X, Xq, s_a, Xu, sum_xu, ws, alpha_permille=300,
+                                     beta_permille=200, stream=None):
+    """p4q_select_gather_quant plus the pruned sequence's expanded codes (see p4q_expand_codes)."""
+    _need(V, torch.float16, 3, "V"); _need(idx, torch.int32, 2, "idx"); _need(ws, torch.uint8, 1, "ws")
+    _need(X, torch.float16, 3, "X"); _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    _need(Xu, torch.uint8, 2, "Xu"); _need(sum_xu, torch.int32, 1, "sum_xu")
+    B, N, d = V.shape
+    J = 0 if Q is None else Q.shape[1]
+    T = 0 if text is None else text.shape[1]
+    p = SelectParams(K, alpha_permille, beta_permille)
+    _check(lib().p4q_select_gather_quant_expanded(_ptr(V), B, N, d, _ptr(Q), J, _ptr(A_cls), _ptr(text), T,
+                                                  ctypes.byref(p), _ptr(idx), _ptr(X), _ptr(Xq), _ptr(s_a), _ptr(Xu),
+                                                  _ptr(sum_xu), _ptr(ws), ws.numel(), _stream(stream)),
+           "p4q_select_gather_quant_expanded")
 
 
 # ---------------------------------------------------------------- helpers

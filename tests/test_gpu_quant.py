@@ -92,3 +92,21 @@ def test_quant_act_on_a_column_block_matches_dense(p4q, dev):
     assert torch.equal(Xq, ref_q) and torch.equal(s.view(torch.int32), ref_s.view(torch.int32))
     c, sc = oracle.quantize_rows(block.cpu().numpy())
     assert np.array_equal(oracle.unpack_codes(Xq.cpu().numpy()), c)
+
+
+def test_quant_act_expanded_matches_quant_then_expand(p4q, dev):
+    """The quantizer's expanded output equals p4q_expand_codes of its packed
+    codes (bytes and row sums), for one-warp and multi-warp row lengths."""
+    for M, K, seed in [(300, 1024, 31), (77, 11008, 32), (129, 5120, 33)]:
+        X = torch.from_numpy(wl.activations(M, K, seed=seed)).to(dev)
+        X[3].zero_()
+        Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+        s = torch.empty((M,), dtype=torch.float32, device=dev)
+        Xu = torch.empty((M, K), dtype=torch.uint8, device=dev)
+        su = torch.empty((M,), dtype=torch.int32, device=dev)
+        p4q.p4q_quant_act_expanded(X, Xq, s, Xu, su)
+        ref_q, ref_s = p4q.quant_act(X)
+        ref_u, ref_su = p4q.expand_codes(ref_q)
+        torch.cuda.synchronize()
+        assert torch.equal(Xq, ref_q) and torch.equal(s.view(torch.int32), ref_s.view(torch.int32))
+        assert torch.equal(Xu, ref_u) and torch.equal(su, ref_su)

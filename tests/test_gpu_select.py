@@ -88,3 +88,23 @@ def test_select_gather_quant_without_text(p4q, dev):
     ref_idx = oracle.select_batch(x.V, w.K, x.Q, x.A)
     assert np.array_equal(idx.cpu().numpy(), ref_idx)
     assert np.array_equal(X.cpu().numpy().astype(np.float32), oracle.gather(x.V, ref_idx))
+
+
+def test_select_gather_quant_expanded_matches(p4q, dev):
+    w = wl.Workload("t", B=2, N=300, d=512, K=40, T=8, J=3, seed=17, heavy_tail=False, linears=())
+    x = wl.selector_inputs(w)
+    V, Q, A, T = (_t(a, dev) for a in (x.V, x.Q, x.A, x.text))
+    ws = p4q.select_workspace(w.B, w.N, w.d, w.J, w.K, dev)
+    M = w.B * (w.K + w.T)
+    idx = torch.empty((w.B, w.K), dtype=torch.int32, device=dev)
+    X = torch.empty((w.B, w.K + w.T, w.d), dtype=torch.float16, device=dev)
+    Xq = torch.empty((M, w.d // 2), dtype=torch.uint8, device=dev)
+    s = torch.empty((M,), dtype=torch.float32, device=dev)
+    Xu = torch.empty((M, w.d), dtype=torch.uint8, device=dev)
+    su = torch.empty((M,), dtype=torch.int32, device=dev)
+    p4q.p4q_select_gather_quant_expanded(V, Q, A, T, w.K, idx, X, Xq, s, Xu, su, ws)
+    ref_idx, ref_X, ref_q, ref_s = p4q.select_gather_quant(V, Q, A, T, w.K)
+    ref_u, ref_su = p4q.expand_codes(ref_q)
+    torch.cuda.synchronize()
+    assert torch.equal(idx, ref_idx) and torch.equal(X.view(torch.int16), ref_X.view(torch.int16))
+    assert torch.equal(Xq, ref_q) and torch.equal(Xu, ref_u) and torch.equal(su, ref_su)
