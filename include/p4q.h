@@ -260,7 +260,7 @@ p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
  * All calls on a device share the one array: calls whose work overlaps on the
  * GPU (other streams, or several host threads) race and give undefined
  * results, so serialize them. */
-#define P4Q_NOALLOC_SCRATCH_BYTES (32u << 20)
+#define P4Q_NOALLOC_SCRATCH_BYTES (48u << 20)
 p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
                               const float* A_cls, const p4q_select_params* params, int32_t* idx,
                               p4q_stream_t stream);

@@ -84,6 +84,8 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   sv.codes = w.vcodes;
   sv.scale = w.vscale;
   sv.norm2 = w.vnorm;
+  sv.u = w.vu;  // the expanded codes the cosine-matrix GEMM reads (large token sets)
+  sv.sum_u = w.vsum;
   cudaError_t e = counted(launch_quant_rows(src, B * N, d, sv, stream));
   if (e != cudaSuccess) return from_cuda(e);
   if (bud.Kq > 0) {
@@ -111,13 +113,15 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     g.d_pitch = w.gram_pitch;
     g.norm_a = w.vnorm;
     g.norm_b = w.vnorm;
-    // Large token sets: exact int32 dot products on the CTA-pair GEMM, then
-    // the cosine of every entry by a full-GPU elementwise pass (the division
-    // and square root would otherwise serialize in the GEMM's four epilogue
-    // warps). Small ones: the cosine epilogue of the single-CTA GEMM.
-    const bool split = N >= 256;
+    // Then the cosine of every entry by a full-GPU elementwise pass (the
+    // division and square root would otherwise serialize in the GEMM's four
+    // epilogue warps). Small token sets: the cosine epilogue of the
+    // single-CTA GEMM on the packed codes.
+    // Large token sets: exact int32 dot products of the expanded codes (written
+    // by the fake-quantization above) on the TMA-fed CTA-pair GEMM.
+    const bool split = w.vu != nullptr;
     g.out = split ? GemmOut::kS32 : GemmOut::kCos;
-    e = counted(launch_w4a4_gemm(g, stream));
+    e = counted(split ? launch_gemm8(g, w.vu, w.vsum, w.vu, w.vsum, stream) : launch_w4a4_gemm(g, stream));
     if (e != cudaSuccess) return from_cuda(e);
     if (split && (e = counted(launch_gram_cos(plan, w, stream))) != cudaSuccess) return from_cuda(e);
   }

@@ -15,6 +15,9 @@
 // (p4q_expand.cu). The permutation is the same for both operands, so every
 // dot product is unchanged.
 //
+// Operands [batch][rows][K] (row-contiguous, batch entries back to back),
+// row sums [batch][rows], output [batch][M][pitch].
+//
 // Kernel: persistent, one cluster of two CTAs per 256 x 256 output tile,
 //   warp 0    MMA issuer (leader CTA): 4 x tcgen05.mma (M 256, N 256, K 32)
 //             per 128-deep k-block into one of two TMEM accumulators;
@@ -50,12 +53,12 @@ constexpr uint32_t TMEM_COLS = 2 * BN;
 constexpr int kMinRows = 512;           // smaller M: the in-kernel unpack path is cheaper than the expansion
 
 struct Params8 {
-  int M, N, K;
-  int num_m, num_n, tiles;
+  int M, N, K, batch;
+  int num_m, num_n, per, tiles;  // per: tiles per batch entry
   const float* s_a;
   const float* s_b;
-  const int32_t* sum_a;  // [M] sum of u over each A row
-  const int32_t* sum_b;  // [N]
+  const int32_t* sum_a;  // [batch, M] sum of u over each A row
+  const int32_t* sum_b;  // [batch, N]
 };
 
 template <int MODE>  // GemmOut::kHalf or kS32
@@ -174,8 +177,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int g = 0;
       bool ok = true;
       for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x()) {
-        const int nb = t / p.num_m;
-        const int m0 = (t - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
+        const int bz = t / p.per, r = t - bz * p.per, nb = r / p.num_m;
+        const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
         const int n0 = nb * BN + static_cast<int>(rank) * HB;                       // this CTA's B rows
         for (int kb = 0; kb < KB; ++kb, ++g) {
           const int s = g % S;
@@ -185,8 +188,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           }
           if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * STAGE_BYTES);
           uint8_t* st = smem + s * STAGE_BYTES;
-          tma_load_3d_pair(&tmA, full_leader + 8u * s, st, kb * BK, m0, 0);
-          tma_load_3d_pair(&tmB, full_leader + 8u * s, st + A_BYTES, kb * BK, n0, 0);
+          tma_load_3d_pair(&tmA, full_leader + 8u * s, st, kb * BK, m0, bz);
+          tma_load_3d_pair(&tmB, full_leader + 8u * s, st + A_BYTES, kb * BK, n0, bz);
         }
       }
       if (!ok && rank == 0) {
@@ -206,8 +209,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     int it = 0, nbox = 0;
     bool failed = false;
     for (int t = cluster_id_x(); t < p.tiles; t += nclusters_x(), ++it) {
-      const int nb = t / p.num_m;
-      const int m0 = (t - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;
+      const int bz = t / p.per, r = t - bz * p.per, nb = r / p.num_m;
+      const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;
       const int n0 = nb * BN;
       const int ab = it & 1;
       if (!failed && !mbar_wait_warp(&acc_full[ab], (it >> 1) & 1, abort_flag, &g_gemm8_err)) failed = true;
@@ -218,7 +221,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (!failed) {
         for (int i = ew * 32 + lane; i < BN; i += kEpiWarps * 32) {
           const int n = n0 + i;
-          sbw[i] = (n < p.N) ? static_cast<float>(-8 * p.sum_b[n]) : 0.0f;
+          sbw[i] = (n < p.N) ? static_cast<float>(-8 * p.sum_b[static_cast<size_t>(bz) * p.N + n]) : 0.0f;
           if (MODE == static_cast<int>(GemmOut::kHalf)) colv[i] = (n < p.N) ? p.s_b[n] : 0.0f;
         }
       }
@@ -226,7 +229,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (failed) continue;
       // acc = P - 8 sum u_a - 8 sum u_b + 64 K in fp32: every term and partial
       // result is an integer of magnitude < 2^24, so the fused multiply-add is exact.
-      const float corrA = (m < p.M) ? static_cast<float>(64 * p.K - 8 * p.sum_a[m]) : 0.0f;
+      const float corrA = (m < p.M) ? static_cast<float>(64 * p.K - 8 * p.sum_a[static_cast<size_t>(bz) * p.M + m]) : 0.0f;
       const float sa = (MODE == static_cast<int>(GemmOut::kHalf) && m < p.M) ? p.s_a[m] : 0.0f;
 #pragma unroll 1
       for (int cc = 0; cc < BN / 32; ++cc) {
@@ -282,7 +285,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) {
-          tma_store_3d(&tmD, box, n0 + cc * 32, m0 + q * 32, 0);
+          tma_store_3d(&tmD, box, n0 + cc * 32, m0 + q * 32, bz);
           bulk_commit_group();
         }
         ++nbox;
@@ -310,12 +313,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   }
 }
 
-// 3-D map over expanded codes: dims (K bytes, rows, 1), 128 x box_rows boxes,
-// 128-byte swizzle (the K-major layout the MMA descriptors describe).
-bool make_expanded_map(CUtensorMap* map, const uint8_t* base, int K, int rows, int box_rows) {
+// 3-D map over expanded codes: dims (K bytes, rows, batch), 128 x box_rows
+// boxes, 128-byte swizzle (the K-major layout the MMA descriptors describe).
+bool make_expanded_map(CUtensorMap* map, const uint8_t* base, int K, int rows, int batch, int box_rows) {
   auto enc = get_encode_fn();
   if (!enc) return false;
-  cuuint64_t dims[3] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows), 1};
+  cuuint64_t dims[3] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows), static_cast<cuuint64_t>(batch)};
   cuuint64_t strides[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(K) * rows};
   cuuint32_t box[3] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows), 1};
   cuuint32_t estr[3] = {1, 1, 1};
@@ -359,17 +362,20 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
     attr_set = true;
   }
   CUtensorMap ma, mb, md;
-  if (!make_expanded_map(&ma, w.a8, g.K, g.M, BM)) return cudaErrorInvalidValue;
-  if (!make_expanded_map(&mb, w.b8, g.K, g.N, HB)) return cudaErrorInvalidValue;
+  const int batch = g.batch > 0 ? g.batch : 1;
+  if (!make_expanded_map(&ma, w.a8, g.K, g.M, batch, BM)) return cudaErrorInvalidValue;
+  if (!make_expanded_map(&mb, w.b8, g.K, g.N, batch, HB)) return cudaErrorInvalidValue;
   const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
-  if (!make_output_map(&md, g.D, g.out, g.M, g.N, pitch, 1)) return cudaErrorInvalidValue;
+  if (!make_output_map(&md, g.D, g.out, g.M, g.N, pitch, batch)) return cudaErrorInvalidValue;
   Params8 p;
   p.M = g.M;
   p.N = g.N;
   p.K = g.K;
+  p.batch = batch;
   p.num_m = (g.M + 2 * BM - 1) / (2 * BM);
   p.num_n = (g.N + BN - 1) / BN;
-  p.tiles = p.num_m * p.num_n;
+  p.per = p.num_m * p.num_n;
+  p.tiles = p.per * batch;
   p.s_a = g.s_a;
   p.s_b = g.s_b;
   p.sum_a = w.sum_a;

@@ -98,7 +98,12 @@ struct SelectWorkspace {
   float* scores;     // [B, J, N] query cosines
   float* gram;       // [B, N, gram_pitch] cosine of every token pair
   int gram_pitch;    // N rounded up to a multiple of 4
+  uint8_t* vu;       // [B*N, d] codes, one byte each (tokens >= kGramExpandedMin), else null
+  int32_t* vsum;     // [B*N] sum of those bytes
 };
+
+// Token count from which the cosine matrix runs on the expanded-operand GEMM.
+constexpr int kGramExpandedMin = 256;
 
 size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, void* base);
 

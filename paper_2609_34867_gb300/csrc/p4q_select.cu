@@ -353,6 +353,8 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
   const size_t o_qc = take(BJ * (d / 2)), o_qs = take(BJ * 4), o_qn = take(BJ * 4);
   const int gp = (N + 3) & ~3;
   const size_t o_sc = take(BJ * N * 4), o_g = take(BN * gp * 4);
+  const bool expanded = N >= kGramExpandedMin;
+  const size_t o_vu = expanded ? take(BN * d) : 0, o_vsum = expanded ? take(BN * 4) : 0;
   if (ws && base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     ws->vcodes = p + o_vc;
@@ -364,6 +366,8 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
     ws->scores = reinterpret_cast<float*>(p + o_sc);
     ws->gram = reinterpret_cast<float*>(p + o_g);
     ws->gram_pitch = gp;
+    ws->vu = expanded ? p + o_vu : nullptr;
+    ws->vsum = expanded ? reinterpret_cast<int32_t*>(p + o_vsum) : nullptr;
   }
   return off;
 }
