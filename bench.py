@@ -246,13 +246,14 @@ class Step:
         for name in self.Xq_re:
             self.Xu_re[name] = torch.empty((M, dims[name].k_in), dtype=torch.uint8, device=dev)
             self.sXu_re[name] = torch.empty((M,), dtype=torch.int32, device=dev)
-        wmax = max(self.Wq[0, g].shape[0] * self.Wq[0, g].shape[1] * 2 for g, _ in self.gemms)
-        nmax = max(self.Wq[0, g].shape[0] for g, _ in self.gemms)
-        # two weight scratches: the next GEMM's weights expand on a side stream
-        # while the current GEMM (or the selector, for the first) runs
-        self.Wu = [torch.empty((wmax,), dtype=torch.uint8, device=dev) for _ in range(2)]
-        self.sWu = [torch.empty((nmax,), dtype=torch.int32, device=dev) for _ in range(2)]
+        # one weight scratch per GEMM of a layer: the weights expand on a side
+        # stream, ahead of the GEMMs that read them (see body)
+        self.slot = {g: i for i, (g, _) in enumerate(self.gemms)}
+        self.Wu = [torch.empty((self.Wq[0, g].shape[0], self.Wq[0, g].shape[1] * 2), dtype=torch.uint8, device=dev)
+                   for g, _ in self.gemms]
+        self.sWu = [torch.empty((self.Wq[0, g].shape[0],), dtype=torch.int32, device=dev) for g, _ in self.gemms]
         self.side = torch.cuda.Stream(device=dev)
+        self.aux = torch.cuda.Stream(device=dev)
         # The step is a chain of segments (selector, each expansion, each GEMM,
         # each re-quantization); the timed loop replays it as one CUDA graph,
         # the breakdown replays one graph per segment with events between them.
@@ -267,8 +268,8 @@ class Step:
                     xin = (lambda n=name: (self.Xu_re[n], self.sXu_re[n], self.s_re[n]))
                 else:
                     xin = (lambda: (self.Xu, self.sXu, self.s_a))
-                self.segments.append(("expand", "expand_w_" + gname, (lambda l=layer, g=gname: self._expand_w(l, g, 0))))
-                self.segments.append(("linear", gname, (lambda l=layer, g=gname, x=xin: self._gemm(l, g, 0, *x()))))
+                self.segments.append(("expand", "expand_w_" + gname, (lambda l=layer, g=gname: self._expand_w(l, g))))
+                self.segments.append(("linear", gname, (lambda l=layer, g=gname, x=xin: self._gemm(l, g, *x()))))
                 self.gemm_calls.append((layer, gname, xin))
         self.lin_ops = {g: sum(2 * w.M * dims[m].n_out * dims[m].k_in for m in members) * w.layers
                         for g, members in self.gemms}
@@ -290,18 +291,13 @@ class Step:
         self.p4q.p4q_select_gather_quant_expanded(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X,
                                                   self.Xq, self.s_a, self.Xu, self.sXu, self.ws)
 
-    def _wu(self, layer, gname, slot):
-        Wq = self.Wq[layer, gname]
-        n = Wq.shape[0]
-        return self.Wu[slot][:n * Wq.shape[1] * 2].view(n, -1), self.sWu[slot][:n]
+    def _expand_w(self, layer, gname, stream=None):
+        k = self.slot[gname]
+        self.p4q.p4q_expand_codes(self.Wq[layer, gname], self.Wu[k], self.sWu[k], stream)
 
-    def _expand_w(self, layer, gname, slot, stream=None):
-        u, su = self._wu(layer, gname, slot)
-        self.p4q.p4q_expand_codes(self.Wq[layer, gname], u, su, stream)
-
-    def _gemm(self, layer, gname, slot, Xu, sXu, s):
-        u, su = self._wu(layer, gname, slot)
-        self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, u, su, self.s_w[layer, gname], self.Y[gname])
+    def _gemm(self, layer, gname, Xu, sXu, s):
+        k = self.slot[gname]
+        self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, self.Wu[k], self.sWu[k], self.s_w[layer, gname], self.Y[gname])
 
     def body_serial(self):
         """The step's segments one after another on the current stream."""
@@ -309,43 +305,60 @@ class Step:
             fn()
 
     def body(self):
-        """The step as plain C-ABI calls (no graph). Weight expansions run on a
-        side stream one GEMM ahead, into two alternating scratches: the first
-        overlaps the selector, each later one the previous GEMM."""
+        """The step as plain C-ABI calls (no graph), on three streams:
+        - side: every GEMM's weight expansion, into that GEMM's scratch, in
+          step order (a later layer's waits until the previous layer's GEMM
+          has read the scratch), overlapping the selector and the GEMMs;
+        - aux: the o chain (re-quantization of the q block, o GEMM), which
+          only needs the q|k|v GEMM and so overlaps the gate|up GEMM;
+        - the current stream: everything else."""
         torch = self.torch
         main = torch.cuda.current_stream()
-        self.side.wait_stream(main)  # fork: inputs of this step are in place
-        ready = [torch.cuda.Event() for _ in self.gemm_calls]
-        freed = [torch.cuda.Event() for _ in self.gemm_calls]
-
-        def expand(i):
-            layer, gname, _ = self.gemm_calls[i]
-            with torch.cuda.stream(self.side):
-                if i >= 2:
-                    self.side.wait_event(freed[i - 2])  # the scratch's previous GEMM is done
-                self._expand_w(layer, gname, i % 2, self.side)
-                ready[i].record(self.side)
-
+        self.side.wait_stream(main)  # fork: the inputs of this step are in place
+        self.aux.wait_stream(main)
         n = len(self.gemm_calls)
-        if n:
-            expand(0)
-        if n > 1:
-            expand(1)
-        gi = 0
-        for kind, _, fn in self.segments:
-            if kind == "expand" and _.startswith("expand_w_"):
-                continue  # done on the side stream
-            if kind == "linear":
-                layer, gname, xin = self.gemm_calls[gi]
-                main.wait_event(ready[gi])
-                self._gemm(layer, gname, gi % 2, *xin())
-                freed[gi].record(main)
-                if gi + 2 < n:
-                    expand(gi + 2)
-                gi += 1
-            else:
-                fn()
+        ngemm = len(self.gemms)
+        ready = [torch.cuda.Event() for _ in range(n)]
+        freed = [torch.cuda.Event() for _ in range(n)]
+        with torch.cuda.stream(self.side):
+            for i, (layer, gname, _) in enumerate(self.gemm_calls):
+                if i >= ngemm:
+                    self.side.wait_event(freed[i - ngemm])
+                self._expand_w(layer, gname, self.side)
+                ready[i].record(self.side)
+        self._select()
+        members = dict(self.gemms)
+        o_src = self.col[self.REQUANT["o"]][0] if "o" in self.Xq_re else None
+        src_done, o_read = None, None
+        for i, (layer, gname, xin) in enumerate(self.gemm_calls):
+            first = members[gname][0]
+            if first == "o":
+                with torch.cuda.stream(self.aux):
+                    if src_done is not None:
+                        self.aux.wait_event(src_done)
+                    self.p4q.p4q_quant_act_expanded(self.output("q"), self.Xq_re["o"], self.s_re["o"],
+                                                    self.Xu_re["o"], self.sXu_re["o"], self.aux)
+                    o_read = torch.cuda.Event()
+                    o_read.record(self.aux)
+                    self.aux.wait_event(ready[i])
+                    self.p4q.p4q_w4a4_linear_expanded(*xin(), self.Wu[self.slot[gname]], self.sWu[self.slot[gname]],
+                                                      self.s_w[layer, gname], self.Y[gname], self.aux)
+                    freed[i].record(self.aux)
+                continue
+            if first in self.REQUANT:
+                src = self.REQUANT[first]
+                self.p4q.p4q_quant_act_expanded(self.output(src), self.Xq_re[first], self.s_re[first],
+                                                self.Xu_re[first], self.sXu_re[first])
+            if gname == o_src and o_read is not None:
+                main.wait_event(o_read)  # the previous layer's o chain has read this GEMM's output
+            main.wait_event(ready[i])
+            self._gemm(layer, gname, *xin())
+            freed[i].record(main)
+            if gname == o_src:
+                src_done = torch.cuda.Event()
+                src_done.record(main)
         main.wait_stream(self.side)  # join
+        main.wait_stream(self.aux)
 
     def capture(self):
         """Captures the whole step into one CUDA graph (consecutive kernels
