@@ -7,13 +7,15 @@ budget 192 kept tokens per image):
                            -> gather of the kept FP16 rows + text -> INT4
   (the selector's gather and the two re-quantizations also write their
   codes in the expanded form, one byte per code, that the GEMMs read)
-  p4q_expand_codes         each GEMM's packed INT4 weights, per call, on a
-                           side stream one GEMM ahead
+  p4q_expand_codes         each GEMM's packed INT4 weights, per call, into
+                           that GEMM's scratch, on a side stream from the
+                           start of the step
   p4q_w4a4_linear_expanded x 4  q|k|v and gate|up (each one GEMM over the
                            concatenated output channels) on the pruned
                            sequence (M = 2048), o on the re-quantized q
                            output, down on the re-quantized up output
-                           (2 x p4q_quant_act_ld on column blocks).
+                           (2 x p4q_quant_act_expanded on column blocks;
+                           the o chain on a third stream beside gate|up).
 The metric is W4A4 linear TOPS: 2 * M * N * K integer ops of the seven linears
 per step divided by the step time (the selector's time included); the
 selector's share is also reported as microseconds per image.
@@ -56,7 +58,7 @@ FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed step
 # DRAM bytes (read + write) per launch over the four GEMMs of one step
 # (profiles/w4a4_gemm_llava15_7b_b8_step.md, section 2), valid only while the
 # GEMM source is unchanged since the capture.
-PROFILED_GEMM = {"source_sha1": "4e651cb373181f70736026a123aaa3ea35814df5", "dram_bytes_per_launch": 80020672}
+PROFILED_GEMM = {"source_sha1": "a5aabe263180372449196085094568fbaf61e0c2", "dram_bytes_per_launch": 79060224}
 
 
 def gemm_source_sha1() -> str:
