@@ -101,16 +101,27 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
   }
 }
 
-constexpr int kSelThreads = 1024;  // upper bound; launches use ceil(N / kPer) threads rounded to warps
-constexpr int kPer = 4;  // tokens per thread: token i = kPer * threadIdx.x + e
+constexpr int kSelThreads = 1024;  // upper bound on the block
+constexpr int kPer = 4;  // tokens per thread of group 0: token i = kPer * threadIdx.x + e
+// Diversity stage: a pool of the kPool smallest free (m, token) pairs is
+// iterated by one warp (kPool / 32 entries per lane) with the pool's cosine
+// block in shared memory; at most kPick picks per iteration.
+constexpr int kPool = 128, kPick = 16;
+constexpr int kPoolPer = kPool / 32;
+static_assert(kPoolPer == 4, "pool warp layout: four slots per lane");
 
 struct BlockScratch {
   unsigned int hist[256];
   unsigned int wsum[32];
-  unsigned int wkey[2][32];  // per-warp minimum keys of a greedy round (double buffered)
-  unsigned int widx[2][32];  // and the lowest token index holding that key
   int digit, above;
-  int list[P4Q_MAX_TOKENS];
+  int t, npend;                              // greedy picks so far; pending rows in list
+  int pick[kPick];                           // pool slots of this iteration's candidates, ascending
+  int ptok[kPool];                           // pool slot -> token (ascending)
+  float pm[kPool];                           // m of the pool tokens when the pool was built
+  unsigned int keptbits[P4Q_MAX_TOKENS / 32];
+  int list[P4Q_MAX_TOKENS];                  // rows still to apply to m (the kept set, then picks)
+  __align__(16) float part[P4Q_MAX_TOKENS];  // partial maxima of the row groups other than group 0
+  __align__(16) float cp[kPool][kPool];      // cos(ptok[i], ptok[j])
 };
 
 // Exclusive prefix sum over the block of per-thread counts (thread order).
@@ -217,6 +228,163 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
   __syncthreads();
 }
 
+// Sorts four 64-bit values ascending (five compare-exchanges).
+__device__ __forceinline__ void sort4(unsigned long long (&h)[kPoolPer]) {
+  auto cx = [](unsigned long long& x, unsigned long long& y) {
+    const unsigned long long lo = x < y ? x : y, hi = x < y ? y : x;
+    x = lo;
+    y = hi;
+  };
+  cx(h[0], h[1]);
+  cx(h[2], h[3]);
+  cx(h[0], h[2]);
+  cx(h[1], h[3]);
+  cx(h[1], h[2]);
+}
+
+// m <- max(m, row r of the image's cosine matrix) for the n rows listed in
+// s.list, on all row groups of the block: group g takes chunks of eight rows
+// g, g + groups, ...; every thread loads 16 bytes per row (its group-0
+// thread's four tokens), so the loads of different groups overlap (one SM
+// keeps few row loads of one warp in flight). Group 0 then merges the other
+// groups' partial maxima. Ends with the block synchronized.
+__device__ void apply_rows(float (&m)[kPer], const float* __restrict__ G, int gp, int N, int n, int tpg, int groups,
+                           BlockScratch& s) {
+  const int g = threadIdx.x / tpg;
+  const int tb = kPer * (threadIdx.x - g * tpg);  // first token of this thread's slice
+  float p[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) p[e] = -INFINITY;
+  if (tb < N) {  // tb + kPer <= gp: the 16-byte load stays inside the row's pitch
+    for (int j0 = 8 * g; j0 < n; j0 += 8 * groups) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        v[u] = (j0 + u < n) ? *reinterpret_cast<const float4*>(G + static_cast<size_t>(s.list[j0 + u]) * gp + tb)
+                            : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        p[0] = fmaxf(p[0], v[u].x); p[1] = fmaxf(p[1], v[u].y);
+        p[2] = fmaxf(p[2], v[u].z); p[3] = fmaxf(p[3], v[u].w);
+      }
+    }
+    if (g > 0) *reinterpret_cast<float4*>(&s.part[(g - 1) * kPer * tpg + tb]) = make_float4(p[0], p[1], p[2], p[3]);
+  }
+  __syncthreads();
+  if (g == 0 && tb < N) {
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) m[e] = fmaxf(m[e], p[e]);
+    for (int h = 1; h < groups; ++h) {
+      const float4 q = *reinterpret_cast<const float4*>(&s.part[(h - 1) * kPer * tpg + tb]);
+      m[0] = fmaxf(m[0], q.x); m[1] = fmaxf(m[1], q.y); m[2] = fmaxf(m[2], q.z); m[3] = fmaxf(m[3], q.w);
+    }
+  }
+  __syncthreads();
+}
+
+// One phase of greedy rounds on the pool, by warp 0 (lane l holds slots
+// 4l .. 4l + 3, in token order). The next pick is the smallest free
+// (m, token) pair. A pool entry is certain to be in order while its pair is
+// at most tau, the largest pair at the pool's construction: every token
+// outside the pool was above tau then and m only grows. Per iteration the r
+// smallest certain entries c_0 < c_1 < ... are taken by r rounds of a warp
+// minimum; c_0 is the next pick, and c_a the pick after c_0 .. c_{a-1}
+// whenever none of their cosines exceeds m(c_a) (nothing else can pass it).
+// The longest such prefix is picked, the pool's m absorbs the picks' cosines,
+// and the picked tokens are appended to s.list as rows still to apply to the
+// tokens outside the pool. Ends when Kd picks are made or no entry is
+// certain; s.t and s.npend hold the counts.
+__device__ void pool_rounds(int npool, int Kd, BlockScratch& s) {
+  const int lane = threadIdx.x & 31;
+  constexpr unsigned long long kNone = ~0ull;
+  float pm[kPoolPer];
+  unsigned int alive = 0;
+  unsigned long long mx = 0;
+#pragma unroll
+  for (int k = 0; k < kPoolPer; ++k) {
+    const int slot = kPoolPer * lane + k;
+    pm[k] = slot < npool ? s.pm[slot] : 0.0f;
+    if (slot < npool) {
+      alive |= 1u << k;
+      const unsigned long long pr = (static_cast<unsigned long long>(float_order_key(pm[k])) << 32) | slot;
+      mx = pr > mx ? pr : mx;
+    }
+  }
+  const uint32_t thi = __reduce_max_sync(0xFFFFFFFFu, static_cast<uint32_t>(mx >> 32));
+  const uint32_t tlo = __reduce_max_sync(0xFFFFFFFFu, static_cast<uint32_t>(mx >> 32) == thi ? static_cast<uint32_t>(mx) : 0u);
+  const unsigned long long tau = (static_cast<unsigned long long>(thi) << 32) | tlo;
+  int t = s.t, npend = 0;
+  while (t < Kd) {
+    unsigned long long h[kPoolPer];
+    int nv = 0;
+#pragma unroll
+    for (int k = 0; k < kPoolPer; ++k) {
+      const unsigned long long pr =
+          (static_cast<unsigned long long>(float_order_key(pm[k])) << 32) | (kPoolPer * lane + k);
+      h[k] = ((alive >> k) & 1u) && pr <= tau ? pr : kNone;
+      nv += h[k] != kNone;
+    }
+    nv = __reduce_add_sync(0xFFFFFFFFu, nv);
+    const int r = min(min(kPick, Kd - t), nv);
+    if (r == 0) break;
+    sort4(h);
+    int rk[kPoolPer];  // position among the candidates of each of this lane's slots, or -1
+#pragma unroll
+    for (int k = 0; k < kPoolPer; ++k) rk[k] = -1;
+#pragma unroll
+    for (int a = 0; a < kPick; ++a) {
+      if (a < r) {
+        const uint32_t hk = static_cast<uint32_t>(h[0] >> 32);
+        const uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, hk);
+        // tied heads: the lowest lane holds the lowest slot
+        const bool mine = lane == __ffs(__ballot_sync(0xFFFFFFFFu, hk == wk)) - 1;
+        if (mine) {
+          const int slot = static_cast<int>(static_cast<uint32_t>(h[0]));
+          s.pick[a] = slot;
+#pragma unroll
+          for (int k = 0; k < kPoolPer; ++k)
+            if (slot == kPoolPer * lane + k) rk[k] = a;
+        }
+#pragma unroll
+        for (int k = 0; k + 1 < kPoolPer; ++k) h[k] = mine ? h[k + 1] : h[k];
+        h[kPoolPer - 1] = mine ? kNone : h[kPoolPer - 1];
+      }
+    }
+    __syncwarp();
+    unsigned int fail = 0;
+#pragma unroll
+    for (int k = 0; k < kPoolPer; ++k) {
+      if (rk[k] >= 1) {
+        const float* row = s.cp[kPoolPer * lane + k];
+        for (int b2 = 0; b2 < rk[k]; ++b2)
+          if (row[s.pick[b2]] > pm[k]) fail |= 1u << rk[k];
+      }
+    }
+    fail = __reduce_or_sync(0xFFFFFFFFu, fail);
+    const int L = fail ? __ffs(fail) - 1 : r;  // bit 0 is never set
+    for (int b2 = 0; b2 < L; ++b2) {
+      const float4 c = *reinterpret_cast<const float4*>(&s.cp[s.pick[b2]][kPoolPer * lane]);
+      pm[0] = fmaxf(pm[0], c.x); pm[1] = fmaxf(pm[1], c.y); pm[2] = fmaxf(pm[2], c.z); pm[3] = fmaxf(pm[3], c.w);
+    }
+#pragma unroll
+    for (int k = 0; k < kPoolPer; ++k) {
+      if (rk[k] >= 0 && rk[k] < L) {
+        alive &= ~(1u << k);
+        const int tok = s.ptok[kPoolPer * lane + k];
+        s.list[npend + rk[k]] = tok;
+        atomicOr(&s.keptbits[tok >> 5], 1u << (tok & 31));
+      }
+    }
+    npend += L;
+    t += L;
+    __syncwarp();
+  }
+  if (lane == 0) {
+    s.t = t;
+    s.npend = npend;
+  }
+}
+
 __global__ void __launch_bounds__(kSelThreads, 1)
     select_stages_kernel(const float* __restrict__ scores, const float* __restrict__ A_cls,
                          const float* __restrict__ gram, int gp, int N, int J, int K, int Kq, int Ks,
@@ -227,7 +395,6 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   BlockScratch& s = *reinterpret_cast<BlockScratch*>(smem_raw);
   const int b = blockIdx.x;
   const int base = kPer * threadIdx.x;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   bool kept[kPer];
 #pragma unroll
   for (int e = 0; e < kPer; ++e) kept[e] = false;
@@ -248,82 +415,86 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(a[base + e]) : 0u;
     block_take_top(key, kept, base, N, Ks, s);
   }
-  // Stage 3: greedy max-min diversity on the cosine matrix G of the image.
+  // Stage 3: greedy max-min diversity on the cosine matrix G of the image:
+  // m_i = max over the kept set of cos(i, r) (-inf while it is empty); each
+  // round keeps the free token with the smallest m (lower index on ties) and
+  // m absorbs its cosines. Rounds run in phases on a pool of the smallest
+  // free (m, token) pairs (pool_rounds); between phases the whole block
+  // applies the pending rows and rebuilds the pool.
   if (Kd > 0) {
     const float* G = gram + static_cast<size_t>(b) * N * gp;
+    const int tpg = ((N + kPer - 1) / kPer + 31) / 32 * 32, groups = blockDim.x / tpg;
+    for (int w = threadIdx.x; w < P4Q_MAX_TOKENS / 32; w += blockDim.x) s.keptbits[w] = 0u;
     int cnt = 0;
 #pragma unroll
     for (int e = 0; e < kPer; ++e) cnt += (base + e < N && kept[e]) ? 1 : 0;
-    int total;
-    int pos = block_exclusive_scan(cnt, &total, s);
+    int nkept;
+    int pos = block_exclusive_scan(cnt, &nkept, s);
 #pragma unroll
     for (int e = 0; e < kPer; ++e)
       if (base + e < N && kept[e]) s.list[pos++] = base + e;
+    if (threadIdx.x == 0) {
+      s.t = 0;
+      s.npend = nkept;  // the kept set's rows come first
+    }
     __syncthreads();
-    // m_i = max over the kept set R0 of cos(i, r); -inf when R0 is empty.
     float m[kPer];
 #pragma unroll
     for (int e = 0; e < kPer; ++e) m[e] = -INFINITY;
-    const bool full4 = (base + kPer <= N);  // rows start 16-byte aligned (pitch % 4 == 0)
-    auto take_row = [&](int r) {
-      const float* row = G + static_cast<size_t>(r) * gp;
-      if (full4) {
-        const float4 g = *reinterpret_cast<const float4*>(row + base);
-        m[0] = fmaxf(m[0], g.x); m[1] = fmaxf(m[1], g.y); m[2] = fmaxf(m[2], g.z); m[3] = fmaxf(m[3], g.w);
-      } else {
+    for (int last = -1;;) {
+      const int t = s.t;
 #pragma unroll
-        for (int e = 0; e < kPer; ++e)
-          if (base + e < N) m[e] = fmaxf(m[e], row[base + e]);
-      }
-    };
-    // The kept rows are independent: fetch them eight at a time so their
-    // L2 latencies overlap.
-    int r = 0;
-    if (full4) {
-      for (; r + 8 <= total; r += 8) {
-        float4 g[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-          g[u] = *reinterpret_cast<const float4*>(G + static_cast<size_t>(s.list[r + u]) * gp + base);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          m[0] = fmaxf(m[0], g[u].x); m[1] = fmaxf(m[1], g[u].y);
-          m[2] = fmaxf(m[2], g[u].z); m[3] = fmaxf(m[3], g[u].w);
-        }
-      }
-    }
-    for (; r < total; ++r) take_row(s.list[r]);
-    // Greedy rounds: argmin of m over the free tokens (lower index on ties),
-    // one block barrier per round.
-    for (int t = 0; t < Kd; ++t) {
-      uint32_t bk = 0xFFFFFFFFu, bi = 0xFFFFFFFFu;
+      for (int e = 0; e < kPer; ++e)
+        if (base + e < N && ((s.keptbits[(base + e) >> 5] >> ((base + e) & 31)) & 1u)) kept[e] = true;
+      // every phase picks at least once (right after a rebuild the whole pool
+      // is certain); the progress check only guards the loop
+      if (t >= Kd || t == last) break;
+      last = t;
+      apply_rows(m, G, gp, N, s.npend, tpg, groups, s);
+      // pool: the q smallest free (m, token) pairs (radix select on inverted keys)
+      const int q = min(kPool, N - nkept - t);
+      bool member[kPer];
 #pragma unroll
       for (int e = 0; e < kPer; ++e) {
-        if (base + e < N && !kept[e]) {
-          const uint32_t k = float_order_key(m[e]);
-          if (k < bk) {  // strictly smaller: the lower index of this thread wins ties
-            bk = k;
-            bi = static_cast<uint32_t>(base + e);
+        member[e] = kept[e];
+        key[e] = (base + e < N) ? ~float_order_key(m[e]) : 0u;
+      }
+      block_take_top(key, member, base, N, q, s);
+      cnt = 0;
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) cnt += (base + e < N && member[e] && !kept[e]) ? 1 : 0;
+      int npool;
+      pos = block_exclusive_scan(cnt, &npool, s);
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) {
+        if (base + e < N && member[e] && !kept[e]) {
+          s.ptok[pos] = base + e;
+          s.pm[pos] = m[e];
+          ++pos;
+        }
+      }
+      __syncthreads();
+      // the pool's cosine block (symmetric: the upper triangle is loaded)
+      for (int x0 = threadIdx.x; x0 < kPool * kPool; x0 += 8 * blockDim.x) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int x = x0 + u * blockDim.x, i = x / kPool, j = x % kPool;
+          v[u] = (x < kPool * kPool && i < npool && j < npool && j >= i)
+                     ? G[static_cast<size_t>(s.ptok[i]) * gp + s.ptok[j]] : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int x = x0 + u * blockDim.x, i = x / kPool, j = x % kPool;
+          if (x < kPool * kPool && i < npool && j < npool && j >= i) {
+            s.cp[i][j] = v[u];
+            s.cp[j][i] = v[u];
           }
         }
       }
-      uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, bk);
-      uint32_t wi = __reduce_min_sync(0xFFFFFFFFu, bk == wk ? bi : 0xFFFFFFFFu);
-      const int slot = t & 1;
-      if (lane == 0) {
-        s.wkey[slot][warp] = wk;
-        s.widx[slot][warp] = wi;
-      }
       __syncthreads();
-      const bool have = lane < static_cast<int>(blockDim.x >> 5);
-      const uint32_t ck = have ? s.wkey[slot][lane] : 0xFFFFFFFFu, ci = have ? s.widx[slot][lane] : 0xFFFFFFFFu;
-      wk = __reduce_min_sync(0xFFFFFFFFu, ck);
-      wi = __reduce_min_sync(0xFFFFFFFFu, ck == wk ? ci : 0xFFFFFFFFu);
-      const int pick = static_cast<int>(wi);
-#pragma unroll
-      for (int e = 0; e < kPer; ++e)
-        if (base + e == pick) kept[e] = true;
-      take_row(pick);
+      if (threadIdx.x < 32) pool_rounds(npool, Kd, s);
+      __syncthreads();
     }
   }
   // Output: the kept set in ascending index order.
@@ -419,8 +590,10 @@ cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws,
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  // one thread per kPer tokens: idle threads would only add instructions to every round
-  const int threads = std::min(kSelThreads, ((p.N + kPer - 1) / kPer + 31) / 32 * 32);
+  // group 0: one thread per kPer tokens (idle threads would only add
+  // instructions to every ranking); as many row groups as fit the block
+  const int tpg = ((p.N + kPer - 1) / kPer + 31) / 32 * 32;
+  const int threads = tpg * std::max(1, kSelThreads / tpg);
   return launch_pdl(select_stages_kernel, dim3(p.B), dim3(threads), static_cast<size_t>(smem), stream, ws.scores,
                     A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx);
 }
