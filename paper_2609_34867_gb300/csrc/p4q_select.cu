@@ -102,6 +102,9 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
 }
 
 constexpr int kSelThreads = 1024;  // upper bound on the block
+// Smaller blocks get more registers per thread: 512 threads for N <= 2048,
+// 768 for N <= 3072, 1024 above.
+constexpr int kSelThreadsSmall = 512, kSelThreadsMid = 768;
 constexpr int kPer = 4;  // tokens per thread of group 0: token i = kPer * threadIdx.x + e
 // Diversity stage: a pool of the kPool smallest free (m, token) pairs is
 // iterated by one warp (kPool / 32 entries per lane) with the pool's cosine
@@ -115,17 +118,22 @@ struct BlockScratch {
   unsigned int wsum[32];
   int digit, above;
   int t, npend;                              // greedy picks so far; pending rows in list
-  int pick[kPick];                           // pool slots of this iteration's candidates, ascending
+  __align__(16) int pick[kPick];             // pool slots of this iteration's candidates, ascending
   int ptok[kPool];                           // pool slot -> token (ascending)
   float pm[kPool];                           // m of the pool tokens when the pool was built
   unsigned int keptbits[P4Q_MAX_TOKENS / 32];
   int list[P4Q_MAX_TOKENS];                  // rows still to apply to m (the kept set, then picks)
   __align__(16) float part[P4Q_MAX_TOKENS];  // partial maxima of the row groups other than group 0
+  int slotof[P4Q_MAX_TOKENS];                // token -> pool slot, -1 outside the pool
   __align__(16) float cp[kPool][kPool];      // cos(ptok[i], ptok[j])
 };
 
-// Exclusive prefix sum over the block of per-thread counts (thread order).
-__device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
+// Barrier of the first nt threads of the block (group 0, the token owners);
+// the other row groups do not take part in the rankings.
+__device__ __forceinline__ void group_sync(int nt) { named_bar_sync(1, static_cast<uint32_t>(nt)); }
+
+// Exclusive prefix sum of per-thread counts over the first nt threads (thread order).
+__device__ int block_exclusive_scan(int v, int* total, int nt, BlockScratch& s) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int x = v;
 #pragma unroll
@@ -134,9 +142,9 @@ __device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
     if (lane >= o) x += y;
   }
   if (lane == 31) s.wsum[warp] = x;
-  __syncthreads();
+  group_sync(nt);
   if (warp == 0) {
-    int w = lane < static_cast<int>(blockDim.x >> 5) ? s.wsum[lane] : 0;
+    int w = lane < (nt >> 5) ? s.wsum[lane] : 0;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xFFFFFFFFu, w, o);
@@ -144,10 +152,10 @@ __device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
     }
     s.wsum[lane] = w;  // inclusive
   }
-  __syncthreads();
+  group_sync(nt);
   const int before = (warp ? s.wsum[warp - 1] : 0) + x - v;
-  *total = s.wsum[(blockDim.x >> 5) - 1];
-  __syncthreads();
+  *total = s.wsum[(nt >> 5) - 1];
+  group_sync(nt);
   return before;
 }
 
@@ -156,7 +164,7 @@ __device__ int block_exclusive_scan(int v, int* total, BlockScratch& s) {
 // Radix select, 8 bits per pass, from the most significant byte; the
 // histogram updates are aggregated per warp over equal digits, since scores
 // of similar magnitude share their leading bytes.
-__device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], int base, int N, int q,
+__device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], int base, int N, int q, int nt,
                                BlockScratch& s) {
   if (q <= 0) return;
   const int lane = threadIdx.x & 31;
@@ -164,8 +172,8 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
   int need = q;
   for (int pass = 0; pass < 4; ++pass) {
     const int shift = 24 - 8 * pass;
-    for (int h = threadIdx.x; h < 256; h += blockDim.x) s.hist[h] = 0;
-    __syncthreads();
+    for (int h = threadIdx.x; h < 256; h += nt) s.hist[h] = 0;
+    group_sync(nt);
 #pragma unroll
     for (int e = 0; e < kPer; ++e) {
       const bool live = (base + e < N) && !kept[e] && (key[e] & mask) == prefix;
@@ -173,7 +181,7 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
       const unsigned peers = __match_any_sync(0xFFFFFFFFu, dig);
       if (live && (__ffs(peers) - 1) == lane) atomicAdd(&s.hist[dig], static_cast<unsigned>(__popc(peers)));
     }
-    __syncthreads();
+    group_sync(nt);
     if (threadIdx.x < 32) {
       // lane l owns digits [8l, 8l+8); find the digit where the count from the top reaches need
       unsigned int c[8], own = 0;
@@ -201,11 +209,11 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
         }
       }
     }
-    __syncthreads();
+    group_sync(nt);
     need -= s.above;
     prefix |= static_cast<uint32_t>(s.digit) << shift;
     mask |= 255u << shift;
-    __syncthreads();
+    group_sync(nt);
   }
   // keys > prefix are taken; among keys == prefix the first `need` in index order
   int eq = 0;
@@ -213,7 +221,7 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
   for (int e = 0; e < kPer; ++e)
     if (base + e < N && !kept[e] && key[e] == prefix) ++eq;
   int total;
-  int rank = block_exclusive_scan(eq, &total, s);
+  int rank = block_exclusive_scan(eq, &total, nt, s);
 #pragma unroll
   for (int e = 0; e < kPer; ++e) {
     if (base + e < N && !kept[e]) {
@@ -225,7 +233,7 @@ __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], 
       }
     }
   }
-  __syncthreads();
+  group_sync(nt);
 }
 
 // Sorts four 64-bit values ascending (five compare-exchanges).
@@ -331,40 +339,54 @@ __device__ void pool_rounds(int npool, int Kd, BlockScratch& s) {
     int rk[kPoolPer];  // position among the candidates of each of this lane's slots, or -1
 #pragma unroll
     for (int k = 0; k < kPoolPer; ++k) rk[k] = -1;
+    // (branch-free: r is uniform over the warp, rounds past it change nothing)
 #pragma unroll
     for (int a = 0; a < kPick; ++a) {
-      if (a < r) {
-        const uint32_t hk = static_cast<uint32_t>(h[0] >> 32);
-        const uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, hk);
-        // tied heads: the lowest lane holds the lowest slot
-        const bool mine = lane == __ffs(__ballot_sync(0xFFFFFFFFu, hk == wk)) - 1;
-        if (mine) {
-          const int slot = static_cast<int>(static_cast<uint32_t>(h[0]));
-          s.pick[a] = slot;
+      const uint32_t hk = static_cast<uint32_t>(h[0] >> 32);
+      const uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, hk);
+      // tied heads: the lowest lane holds the lowest slot
+      const unsigned int tied = __ballot_sync(0xFFFFFFFFu, hk == wk);
+      const bool mine = a < r && lane == __ffs(tied) - 1;
+      const int slot = static_cast<int>(static_cast<uint32_t>(h[0]));
+      if (mine) s.pick[a] = slot;
 #pragma unroll
-          for (int k = 0; k < kPoolPer; ++k)
-            if (slot == kPoolPer * lane + k) rk[k] = a;
-        }
+      for (int k = 0; k < kPoolPer; ++k) rk[k] = (mine && slot == kPoolPer * lane + k) ? a : rk[k];
 #pragma unroll
-        for (int k = 0; k + 1 < kPoolPer; ++k) h[k] = mine ? h[k + 1] : h[k];
-        h[kPoolPer - 1] = mine ? kNone : h[kPoolPer - 1];
-      }
+      for (int k = 0; k + 1 < kPoolPer; ++k) h[k] = mine ? h[k + 1] : h[k];
+      h[kPoolPer - 1] = mine ? kNone : h[kPoolPer - 1];
     }
     __syncwarp();
+    // cos(c_a, c_b) for this lane's slots from row c_b (the block is
+    // symmetric): one conflict-free 16-byte read per earlier candidate
+    // (loads unconditional: every entry of s.pick is a valid slot, stale past r)
     unsigned int fail = 0;
 #pragma unroll
-    for (int k = 0; k < kPoolPer; ++k) {
-      if (rk[k] >= 1) {
-        const float* row = s.cp[kPoolPer * lane + k];
-        for (int b2 = 0; b2 < rk[k]; ++b2)
-          if (row[s.pick[b2]] > pm[k]) fail |= 1u << rk[k];
+    for (int c0 = 0; c0 < kPick; c0 += 4) {  // four reads in flight
+      float4 c[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) c[u] = *reinterpret_cast<const float4*>(&s.cp[s.pick[c0 + u]][kPoolPer * lane]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int b2 = c0 + u;
+        fail |= (b2 < rk[0] && c[u].x > pm[0]) ? 1u << rk[0] : 0u;
+        fail |= (b2 < rk[1] && c[u].y > pm[1]) ? 1u << rk[1] : 0u;
+        fail |= (b2 < rk[2] && c[u].z > pm[2]) ? 1u << rk[2] : 0u;
+        fail |= (b2 < rk[3] && c[u].w > pm[3]) ? 1u << rk[3] : 0u;
       }
     }
     fail = __reduce_or_sync(0xFFFFFFFFu, fail);
     const int L = fail ? __ffs(fail) - 1 : r;  // bit 0 is never set
-    for (int b2 = 0; b2 < L; ++b2) {
-      const float4 c = *reinterpret_cast<const float4*>(&s.cp[s.pick[b2]][kPoolPer * lane]);
-      pm[0] = fmaxf(pm[0], c.x); pm[1] = fmaxf(pm[1], c.y); pm[2] = fmaxf(pm[2], c.z); pm[3] = fmaxf(pm[3], c.w);
+#pragma unroll
+    for (int c0 = 0; c0 < kPick; c0 += 4) {
+      float4 c[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) c[u] = *reinterpret_cast<const float4*>(&s.cp[s.pick[c0 + u]][kPoolPer * lane]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const bool use = c0 + u < L;
+        pm[0] = use ? fmaxf(pm[0], c[u].x) : pm[0]; pm[1] = use ? fmaxf(pm[1], c[u].y) : pm[1];
+        pm[2] = use ? fmaxf(pm[2], c[u].z) : pm[2]; pm[3] = use ? fmaxf(pm[3], c[u].w) : pm[3];
+      }
     }
 #pragma unroll
     for (int k = 0; k < kPoolPer; ++k) {
@@ -385,7 +407,8 @@ __device__ void pool_rounds(int npool, int Kd, BlockScratch& s) {
   }
 }
 
-__global__ void __launch_bounds__(kSelThreads, 1)
+template <int kMaxThreads>
+__global__ void __launch_bounds__(kMaxThreads, 1)
     select_stages_kernel(const float* __restrict__ scores, const float* __restrict__ A_cls,
                          const float* __restrict__ gram, int gp, int N, int J, int K, int Kq, int Ks,
                          int Kd, int32_t* __restrict__ idx) {
@@ -394,26 +417,30 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   BlockScratch& s = *reinterpret_cast<BlockScratch*>(smem_raw);
   const int b = blockIdx.x;
-  const int base = kPer * threadIdx.x;
+  const int base = kPer * threadIdx.x;  // tokens of a group-0 thread (none for the other groups)
+  const int tpg = ((N + kPer - 1) / kPer + 31) / 32 * 32, groups = blockDim.x / tpg;
+  const bool g0 = threadIdx.x < tpg;
   bool kept[kPer];
 #pragma unroll
   for (int e = 0; e < kPer; ++e) kept[e] = false;
   uint32_t key[kPer];
 
-  // Stage 1: query relevance, one ranking per concept, quota floor(Kq/J) + (j < Kq % J).
-  for (int j = 0; j < J && Kq > 0; ++j) {
-    const int quota = Kq / J + (j < Kq % J ? 1 : 0);
-    const float* sc = scores + (static_cast<size_t>(b) * J + j) * N;
+  if (g0) {
+    // Stage 1: query relevance, one ranking per concept, quota floor(Kq/J) + (j < Kq % J).
+    for (int j = 0; j < J && Kq > 0; ++j) {
+      const int quota = Kq / J + (j < Kq % J ? 1 : 0);
+      const float* sc = scores + (static_cast<size_t>(b) * J + j) * N;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(sc[base + e]) : 0u;
-    block_take_top(key, kept, base, N, quota, s);
-  }
-  // Stage 2: visual saliency on the tokens not kept.
-  if (Ks > 0) {
-    const float* a = A_cls + static_cast<size_t>(b) * N;
+      for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(sc[base + e]) : 0u;
+      block_take_top(key, kept, base, N, quota, tpg, s);
+    }
+    // Stage 2: visual saliency on the tokens not kept.
+    if (Ks > 0) {
+      const float* a = A_cls + static_cast<size_t>(b) * N;
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(a[base + e]) : 0u;
-    block_take_top(key, kept, base, N, Ks, s);
+      for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(a[base + e]) : 0u;
+      block_take_top(key, kept, base, N, Ks, tpg, s);
+    }
   }
   // Stage 3: greedy max-min diversity on the cosine matrix G of the image:
   // m_i = max over the kept set of cos(i, r) (-inf while it is empty); each
@@ -423,19 +450,20 @@ __global__ void __launch_bounds__(kSelThreads, 1)
   // applies the pending rows and rebuilds the pool.
   if (Kd > 0) {
     const float* G = gram + static_cast<size_t>(b) * N * gp;
-    const int tpg = ((N + kPer - 1) / kPer + 31) / 32 * 32, groups = blockDim.x / tpg;
     for (int w = threadIdx.x; w < P4Q_MAX_TOKENS / 32; w += blockDim.x) s.keptbits[w] = 0u;
-    int cnt = 0;
+    if (threadIdx.x < kPick) s.pick[threadIdx.x] = 0;
+    int nkept = 0, cnt = 0, pos = 0;
+    if (g0) {
 #pragma unroll
-    for (int e = 0; e < kPer; ++e) cnt += (base + e < N && kept[e]) ? 1 : 0;
-    int nkept;
-    int pos = block_exclusive_scan(cnt, &nkept, s);
+      for (int e = 0; e < kPer; ++e) cnt += (base + e < N && kept[e]) ? 1 : 0;
+      pos = block_exclusive_scan(cnt, &nkept, tpg, s);
 #pragma unroll
-    for (int e = 0; e < kPer; ++e)
-      if (base + e < N && kept[e]) s.list[pos++] = base + e;
-    if (threadIdx.x == 0) {
-      s.t = 0;
-      s.npend = nkept;  // the kept set's rows come first
+      for (int e = 0; e < kPer; ++e)
+        if (base + e < N && kept[e]) s.list[pos++] = base + e;
+      if (threadIdx.x == 0) {
+        s.t = 0;
+        s.npend = nkept;  // the kept set's rows come first
+      }
     }
     __syncthreads();
     float m[kPer];
@@ -450,45 +478,61 @@ __global__ void __launch_bounds__(kSelThreads, 1)
       // is certain); the progress check only guards the loop
       if (t >= Kd || t == last) break;
       last = t;
+      for (int i = threadIdx.x; i < N; i += blockDim.x) s.slotof[i] = -1;
       apply_rows(m, G, gp, N, s.npend, tpg, groups, s);
-      // pool: the q smallest free (m, token) pairs (radix select on inverted keys)
-      const int q = min(kPool, N - nkept - t);
-      bool member[kPer];
+      int npool = 0;
+      if (g0) {
+        // pool: the q smallest free (m, token) pairs (radix select on inverted keys), in token order
+        const int q = min(kPool, N - nkept - t);
+        bool member[kPer];
 #pragma unroll
-      for (int e = 0; e < kPer; ++e) {
-        member[e] = kept[e];
-        key[e] = (base + e < N) ? ~float_order_key(m[e]) : 0u;
-      }
-      block_take_top(key, member, base, N, q, s);
-      cnt = 0;
-#pragma unroll
-      for (int e = 0; e < kPer; ++e) cnt += (base + e < N && member[e] && !kept[e]) ? 1 : 0;
-      int npool;
-      pos = block_exclusive_scan(cnt, &npool, s);
-#pragma unroll
-      for (int e = 0; e < kPer; ++e) {
-        if (base + e < N && member[e] && !kept[e]) {
-          s.ptok[pos] = base + e;
-          s.pm[pos] = m[e];
-          ++pos;
+        for (int e = 0; e < kPer; ++e) {
+          member[e] = kept[e];
+          key[e] = (base + e < N) ? ~float_order_key(m[e]) : 0u;
         }
+        block_take_top(key, member, base, N, q, tpg, s);
+        cnt = 0;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) cnt += (base + e < N && member[e] && !kept[e]) ? 1 : 0;
+        pos = block_exclusive_scan(cnt, &npool, tpg, s);
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) {
+          if (base + e < N && member[e] && !kept[e]) {
+            s.ptok[pos] = base + e;
+            s.pm[pos] = m[e];
+            s.slotof[base + e] = pos;
+            ++pos;
+          }
+        }
+        if (threadIdx.x == 0) s.npend = npool;  // rows of the pool tokens, for the cosine block
       }
       __syncthreads();
-      // the pool's cosine block (symmetric: the upper triangle is loaded)
-      for (int x0 = threadIdx.x; x0 < kPool * kPool; x0 += 8 * blockDim.x) {
-        float v[8];
+      npool = s.npend;
+      // the pool's cosine block from whole rows of the pool tokens (coalesced):
+      // each thread keeps the columns of its four tokens that are in the pool
+      {
+        const int g = threadIdx.x / tpg;
+        const int tb = kPer * (threadIdx.x - g * tpg);
+        int sl[kPer];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int x = x0 + u * blockDim.x, i = x / kPool, j = x % kPool;
-          v[u] = (x < kPool * kPool && i < npool && j < npool && j >= i)
-                     ? G[static_cast<size_t>(s.ptok[i]) * gp + s.ptok[j]] : 0.0f;
-        }
+        for (int e = 0; e < kPer; ++e) sl[e] = (tb + e < N) ? s.slotof[tb + e] : -1;
+        if (tb < N && (sl[0] >= 0 || sl[1] >= 0 || sl[2] >= 0 || sl[3] >= 0)) {
+          for (int i0 = 8 * g; i0 < npool; i0 += 8 * groups) {
+            float4 v[8];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int x = x0 + u * blockDim.x, i = x / kPool, j = x % kPool;
-          if (x < kPool * kPool && i < npool && j < npool && j >= i) {
-            s.cp[i][j] = v[u];
-            s.cp[j][i] = v[u];
+            for (int u = 0; u < 8; ++u)
+              v[u] = (i0 + u < npool) ? *reinterpret_cast<const float4*>(G + static_cast<size_t>(s.ptok[i0 + u]) * gp + tb)
+                                      : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+              if (i0 + u < npool) {
+                float* row = s.cp[i0 + u];
+                if (sl[0] >= 0) row[sl[0]] = v[u].x;
+                if (sl[1] >= 0) row[sl[1]] = v[u].y;
+                if (sl[2] >= 0) row[sl[2]] = v[u].z;
+                if (sl[3] >= 0) row[sl[3]] = v[u].w;
+              }
+            }
           }
         }
       }
@@ -498,14 +542,16 @@ __global__ void __launch_bounds__(kSelThreads, 1)
     }
   }
   // Output: the kept set in ascending index order.
-  int cnt = 0;
+  if (g0) {
+    int cnt = 0;
 #pragma unroll
-  for (int e = 0; e < kPer; ++e) cnt += (base + e < N && kept[e]) ? 1 : 0;
-  int total;
-  int pos = block_exclusive_scan(cnt, &total, s);
+    for (int e = 0; e < kPer; ++e) cnt += (base + e < N && kept[e]) ? 1 : 0;
+    int total;
+    int pos = block_exclusive_scan(cnt, &total, tpg, s);
 #pragma unroll
-  for (int e = 0; e < kPer; ++e)
-    if (base + e < N && kept[e] && pos < K) idx[static_cast<size_t>(b) * K + pos++] = base + e;
+    for (int e = 0; e < kPer; ++e)
+      if (base + e < N && kept[e] && pos < K) idx[static_cast<size_t>(b) * K + pos++] = base + e;
+  }
 }
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
@@ -586,16 +632,29 @@ cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws,
   static bool attr_set = false;
   const int smem = static_cast<int>(sizeof(BlockScratch));
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(select_stages_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    cudaError_t e = cudaFuncSetAttribute(select_stages_kernel<kSelThreadsSmall>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(select_stages_kernel<kSelThreadsMid>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               smem);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(select_stages_kernel<kSelThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
   // group 0: one thread per kPer tokens (idle threads would only add
   // instructions to every ranking); as many row groups as fit the block
   const int tpg = ((p.N + kPer - 1) / kPer + 31) / 32 * 32;
-  const int threads = tpg * std::max(1, kSelThreads / tpg);
-  return launch_pdl(select_stages_kernel, dim3(p.B), dim3(threads), static_cast<size_t>(smem), stream, ws.scores,
-                    A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx);
+  if (tpg <= kSelThreadsSmall)
+    return launch_pdl(select_stages_kernel<kSelThreadsSmall>, dim3(p.B), dim3(tpg * (kSelThreadsSmall / tpg)),
+                      static_cast<size_t>(smem), stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K,
+                      p.Kq, p.Ks, p.Kd, idx);
+  if (tpg <= kSelThreadsMid)
+    return launch_pdl(select_stages_kernel<kSelThreadsMid>, dim3(p.B), dim3(tpg * (kSelThreadsMid / tpg)),
+                      static_cast<size_t>(smem), stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K,
+                      p.Kq, p.Ks, p.Kd, idx);
+  return launch_pdl(select_stages_kernel<kSelThreads>, dim3(p.B), dim3(tpg), static_cast<size_t>(smem), stream,
+                    ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx);
 }
 
 }  // namespace p4q
