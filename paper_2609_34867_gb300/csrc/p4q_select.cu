@@ -304,6 +304,7 @@ __device__ void apply_rows(float (&m)[kPer], const float* __restrict__ G, int gp
 // certain; s.t and s.npend hold the counts.
 __device__ void pool_rounds(int npool, int Kd, BlockScratch& s) {
   const int lane = threadIdx.x & 31;
+  const unsigned int lanes_below = (1u << lane) - 1u;
   constexpr unsigned long long kNone = ~0ull;
   float pm[kPoolPer];
   unsigned int alive = 0;
@@ -336,24 +337,44 @@ __device__ void pool_rounds(int npool, int Kd, BlockScratch& s) {
     const int r = min(min(kPick, Kd - t), nv);
     if (r == 0) break;
     sort4(h);
+    // The lane's sorted entries as 32-bit keys (the pair order is the key
+    // order, ties between lanes resolving to the lower lane) and their slots
+    // as a queue of 2-bit indices into the lane's four slots.
+    uint32_t hk[kPoolPer];
+    uint32_t perm = 0;
+#pragma unroll
+    for (int k = 0; k < kPoolPer; ++k) {
+      hk[k] = static_cast<uint32_t>(h[k] >> 32);
+      perm |= (static_cast<uint32_t>(h[k]) & 3u) << (2 * k);
+    }
+    // r rounds of the warp minimum (branch-free: r is uniform over the warp,
+    // later rounds change nothing); a lane records the rounds of its pops
+    uint32_t rks = 0, pks = 0;
+    int np = 0;
+#pragma unroll
+    for (int a = 0; a < kPick; ++a) {
+      const uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, hk[0]);
+      const unsigned int tied = __ballot_sync(0xFFFFFFFFu, hk[0] == wk);
+      const bool mine = a < r && hk[0] == wk && (tied & lanes_below) == 0u;
+      if (mine) {
+        s.pick[a] = kPoolPer * lane + static_cast<int>(perm & 3u);
+        rks |= static_cast<uint32_t>(a) << (4 * np);
+        pks |= (perm & 3u) << (2 * np);
+        ++np;
+        perm >>= 2;
+#pragma unroll
+        for (int k = 0; k + 1 < kPoolPer; ++k) hk[k] = hk[k + 1];
+        hk[kPoolPer - 1] = 0xFFFFFFFFu;
+      }
+    }
     int rk[kPoolPer];  // position among the candidates of each of this lane's slots, or -1
 #pragma unroll
     for (int k = 0; k < kPoolPer; ++k) rk[k] = -1;
-    // (branch-free: r is uniform over the warp, rounds past it change nothing)
 #pragma unroll
-    for (int a = 0; a < kPick; ++a) {
-      const uint32_t hk = static_cast<uint32_t>(h[0] >> 32);
-      const uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, hk);
-      // tied heads: the lowest lane holds the lowest slot
-      const unsigned int tied = __ballot_sync(0xFFFFFFFFu, hk == wk);
-      const bool mine = a < r && lane == __ffs(tied) - 1;
-      const int slot = static_cast<int>(static_cast<uint32_t>(h[0]));
-      if (mine) s.pick[a] = slot;
+    for (int j = 0; j < kPoolPer; ++j) {
+      const int kj = static_cast<int>((pks >> (2 * j)) & 3u), aj = static_cast<int>((rks >> (4 * j)) & 15u);
 #pragma unroll
-      for (int k = 0; k < kPoolPer; ++k) rk[k] = (mine && slot == kPoolPer * lane + k) ? a : rk[k];
-#pragma unroll
-      for (int k = 0; k + 1 < kPoolPer; ++k) h[k] = mine ? h[k + 1] : h[k];
-      h[kPoolPer - 1] = mine ? kNone : h[kPoolPer - 1];
+      for (int k = 0; k < kPoolPer; ++k) rk[k] = (j < np && kj == k) ? aj : rk[k];
     }
     __syncwarp();
     // cos(c_a, c_b) for this lane's slots from row c_b (the block is
