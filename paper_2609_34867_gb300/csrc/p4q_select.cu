@@ -42,61 +42,73 @@ __device__ __forceinline__ int sext_nibbles(uint32_t n) {
   return static_cast<int>((n & 0x0F0F0F0Fu) | ((n & 0x08080808u) * 0x1Eu));
 }
 
-// Signed dot product of 32 packed codes (one 16-byte chunk) of two rows.
-__device__ __forceinline__ int dot32(const uint4& x, const uint4& y, int acc) {
-  acc = __dp4a(sext_nibbles(x.x), sext_nibbles(y.x), acc);
-  acc = __dp4a(sext_nibbles(x.x >> 4), sext_nibbles(y.x >> 4), acc);
-  acc = __dp4a(sext_nibbles(x.y), sext_nibbles(y.y), acc);
-  acc = __dp4a(sext_nibbles(x.y >> 4), sext_nibbles(y.y >> 4), acc);
-  acc = __dp4a(sext_nibbles(x.z), sext_nibbles(y.z), acc);
-  acc = __dp4a(sext_nibbles(x.z >> 4), sext_nibbles(y.z >> 4), acc);
-  acc = __dp4a(sext_nibbles(x.w), sext_nibbles(y.w), acc);
-  acc = __dp4a(sext_nibbles(x.w >> 4), sext_nibbles(y.w >> 4), acc);
-  return acc;
-}
-
-// scores[b, j, i] = cos(concept j of image b, token i of image b); one warp
-// per token, the token's packed codes loaded with 16-byte loads by all lanes.
+// scores[b, j, i] = cos(concept j of image b, token i of image b). One CTA
+// per kScoreWarps tokens of one image, one warp per token (many warps in
+// flight: the kernel is latency-bound): the image's J concept codes are
+// staged in shared memory, every lane loads 16-byte chunks of the token's
+// packed codes and sign-extends each chunk once for all J concepts (dp4a on
+// the sign-extended nibbles); lane j then finishes the cosine of concept j.
+// kJ bounds J (the concept loops unroll to kJ: a small kJ keeps the code in
+// the instruction cache).
+template <int kJ>
 __global__ void __launch_bounds__(kScoreWarps * 32)
     query_scores_kernel(const uint8_t* __restrict__ vcodes, const int32_t* __restrict__ vnorm,
                         const uint8_t* __restrict__ qcodes, const int32_t* __restrict__ qnorm, int B, int N, int d,
                         int J, float* __restrict__ scores) {
   pdl_wait();
   pdl_launch_dependents();
+  extern __shared__ uint4 qs[];  // [J][d/32] chunks of 32 packed codes
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tok = blockIdx.x * kScoreWarps + warp;
-  if (tok >= B * N) return;
-  const int b = tok / N, i = tok - b * N;
-  const int nvec = d >> 5;  // 16-byte chunks (32 codes) per row
-  const uint4* tv = reinterpret_cast<const uint4*>(vcodes + static_cast<size_t>(tok) * (d >> 1));
+  const int b = blockIdx.y, i = blockIdx.x * kScoreWarps + warp;
+  const int nvec = d >> 5;
   const uint4* tq = reinterpret_cast<const uint4*>(qcodes + static_cast<size_t>(b) * J * (d >> 1));
-  int acc[P4Q_MAX_CONCEPTS];
+  const uint4* tv = reinterpret_cast<const uint4*>(vcodes + (static_cast<size_t>(b) * N + (i < N ? i : 0)) * (d >> 1));
+  uint4 x[4];  // the first chunks of the token, loaded before the barrier
 #pragma unroll
-  for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) acc[j] = 0;
+  for (int u = 0; u < 4; ++u) x[u] = (i < N && u * 32 + lane < nvec) ? __ldg(tv + u * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+  for (int c = threadIdx.x; c < J * nvec; c += blockDim.x) qs[c] = tq[c];
+  __syncthreads();
+  if (i >= N) return;
+  int acc[kJ];
+#pragma unroll
+  for (int j = 0; j < kJ; ++j) acc[j] = 0;
   for (int c0 = 0; c0 < nvec; c0 += 4 * 32) {
-    uint4 x[4];
+    if (c0 > 0) {
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + u * 32 + lane;
+        x[u] = c < nvec ? __ldg(tv + c) : make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int c = c0 + u * 32 + lane;
-      x[u] = c < nvec ? __ldg(tv + c) : make_uint4(0u, 0u, 0u, 0u);
-    }
+      if (c >= nvec) continue;
+      int e[4][2];  // sign-extended nibbles of the chunk: [word][low / high]
+      const uint32_t w[4] = {x[u].x, x[u].y, x[u].z, x[u].w};
 #pragma unroll
-    for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) {
-      if (j < J) {
+      for (int k = 0; k < 4; ++k) {
+        e[k][0] = sext_nibbles(w[k]);
+        e[k][1] = sext_nibbles(w[k] >> 4);
+      }
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int c = c0 + u * 32 + lane;
-          if (c < nvec) acc[j] = dot32(x[u], __ldg(tq + static_cast<size_t>(j) * nvec + c), acc[j]);
+      for (int j = 0; j < kJ; ++j) {
+        if (j < J) {
+          const uint4 y = qs[j * nvec + c];
+          const uint32_t wy[4] = {y.x, y.y, y.z, y.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            acc[j] = __dp4a(e[k][1], sext_nibbles(wy[k] >> 4), __dp4a(e[k][0], sext_nibbles(wy[k]), acc[j]));
         }
       }
     }
   }
-  const int nv = vnorm[tok];
+  const int nv = vnorm[static_cast<size_t>(b) * N + i];
 #pragma unroll
-  for (int j = 0; j < P4Q_MAX_CONCEPTS; ++j) {
+  for (int j = 0; j < kJ; ++j) {
     if (j < J) {
       const int dot = __reduce_add_sync(0xFFFFFFFFu, acc[j]);
-      if (lane == 0) scores[(static_cast<size_t>(b) * J + j) * N + i] = code_cosine(dot, qnorm[b * J + j], nv);
+      if (lane == j) scores[(static_cast<size_t>(b) * J + j) * N + i] = code_cosine(dot, qnorm[b * J + j], nv);
     }
   }
 }
@@ -611,41 +623,67 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
 }
 
 cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
-  const int toks = p.B * p.N;
-  return launch_pdl(query_scores_kernel, dim3((toks + kScoreWarps - 1) / kScoreWarps), dim3(kScoreWarps * 32), 0,
-                    stream, ws.vcodes, ws.vnorm, ws.qcodes, ws.qnorm, p.B, p.N, p.d, p.J, ws.scores);
+  const size_t smem = static_cast<size_t>(p.J) * (p.d / 2);
+  static size_t smem_set = 48u << 10;
+  if (smem > smem_set) {
+    cudaError_t e = cudaFuncSetAttribute(query_scores_kernel<P4Q_MAX_CONCEPTS>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    smem_set = smem;
+  }
+  const dim3 grid((p.N + kScoreWarps - 1) / kScoreWarps, p.B);
+  if (p.J <= 4)  // J * d / 2 <= 32 KB: no attribute needed
+    return launch_pdl(query_scores_kernel<4>, grid, dim3(kScoreWarps * 32), smem, stream, ws.vcodes, ws.vnorm,
+                      ws.qcodes, ws.qnorm, p.B, p.N, p.d, p.J, ws.scores);
+  return launch_pdl(query_scores_kernel<P4Q_MAX_CONCEPTS>, grid, dim3(kScoreWarps * 32), smem, stream, ws.vcodes,
+                    ws.vnorm, ws.qcodes, ws.qnorm, p.B, p.N, p.d, p.J, ws.scores);
 }
 
 namespace {
 
-// Row (b, i) of the Gram buffer, four entries per thread: int32 dot products
-// in, the cosines out (same bits as the cosine epilogue of the GEMM).
-__global__ void __launch_bounds__(128) gram_cos_kernel(float* __restrict__ gram, const int32_t* __restrict__ norm,
-                                                       int N, int gp) {
+// The Gram buffer in place: int32 dot products in, the cosines out (same
+// bits as the cosine epilogue of the GEMM). One warp per row at a time
+// (grid-stride over rows), each lane two 16-byte chunks of four entries in
+// flight; the IEEE division and square root make this instruction-bound.
+__global__ void __launch_bounds__(256) gram_cos_kernel(float* __restrict__ gram, const int32_t* __restrict__ norm,
+                                                       int N, int gp, int rows) {
   pdl_wait();
   pdl_launch_dependents();
-  const int row = blockIdx.x;  // b * N + i
-  const int j0 = 4 * (blockIdx.y * blockDim.x + threadIdx.x);
-  if (j0 >= N) return;
-  const int b = row / N;
-  const int na = norm[row];
-  int4* cell = reinterpret_cast<int4*>(gram + static_cast<size_t>(row) * gp + j0);
-  const int4 d = *cell;
-  const int32_t* nr = norm + static_cast<size_t>(b) * N;
-  float4 c;
-  c.x = code_cosine(d.x, na, nr[j0]);
-  c.y = (j0 + 1 < N) ? code_cosine(d.y, na, nr[j0 + 1]) : 0.0f;
-  c.z = (j0 + 2 < N) ? code_cosine(d.z, na, nr[j0 + 2]) : 0.0f;
-  c.w = (j0 + 3 < N) ? code_cosine(d.w, na, nr[j0 + 3]) : 0.0f;
-  *reinterpret_cast<float4*>(cell) = c;
+  const int lane = threadIdx.x & 31;
+  const int nwarps = gridDim.x * (blockDim.x >> 5);
+  const int cpr = gp >> 2;  // chunks per row
+  for (int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows; row += nwarps) {
+    const int na = norm[row];
+    const int32_t* nr = norm + (row / N) * N;  // norms of the image's tokens
+    float* g = gram + static_cast<size_t>(row) * gp;
+    for (int c0 = lane; c0 < cpr; c0 += 64) {
+      int4 dv[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int c = c0 + 32 * u;
+        dv[u] = c < cpr ? *reinterpret_cast<const int4*>(g + 4 * c) : make_int4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int j = 4 * (c0 + 32 * u);
+        if (j >= N) continue;
+        float4 c;
+        c.x = code_cosine(dv[u].x, na, nr[j]);
+        c.y = (j + 1 < N) ? code_cosine(dv[u].y, na, nr[j + 1]) : 0.0f;
+        c.z = (j + 2 < N) ? code_cosine(dv[u].z, na, nr[j + 2]) : 0.0f;
+        c.w = (j + 3 < N) ? code_cosine(dv[u].w, na, nr[j + 3]) : 0.0f;
+        *reinterpret_cast<float4*>(g + j) = c;
+      }
+    }
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
-  const int per_row = (p.N + 3) / 4;
-  const dim3 grid(p.B * p.N, (per_row + 127) / 128);
-  return launch_pdl(gram_cos_kernel, grid, dim3(128), 0, stream, ws.gram, ws.vnorm, p.N, ws.gram_pitch);
+  const int rows = p.B * p.N;
+  const int blocks = std::min((rows + 7) / 8, 8 * num_sms());
+  return launch_pdl(gram_cos_kernel, dim3(blocks), dim3(256), 0, stream, ws.gram, ws.vnorm, p.N, ws.gram_pitch, rows);
 }
 
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls, int32_t* idx,
