@@ -86,17 +86,19 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   sv.norm2 = w.vnorm;
   sv.u = w.vu;  // the expanded codes the cosine-matrix GEMM reads (large token sets)
   sv.sum_u = w.vsum;
-  cudaError_t e = counted(launch_quant_rows(src, B * N, d, sv, stream));
+  // the concept rows ride in the same launch, after the visual tokens
+  RowSinks oq;
+  oq.codes = w.qcodes;
+  oq.scale = w.qscale;
+  oq.norm2 = w.qnorm;
+  if (bud.Kq > 0) {
+    src.X2 = Q;
+    src.split = B * N;
+  }
+  cudaError_t e = counted(launch_quant_rows(src, B * N + (bud.Kq > 0 ? B * Jeff : 0), d, sv, stream, &oq));
   if (e != cudaSuccess) return from_cuda(e);
   if (bud.Kq > 0) {
-    RowSource sq;
-    sq.X = Q;
-    RowSinks oq;
-    oq.codes = w.qcodes;
-    oq.scale = w.qscale;
-    oq.norm2 = w.qnorm;
-    e = counted(launch_quant_rows(sq, B * Jeff, d, oq, stream));
-    if (e == cudaSuccess) e = counted(launch_query_scores(plan, w, stream));
+    e = counted(launch_query_scores(plan, w, stream));
     if (e != cudaSuccess) return from_cuda(e);
   }
   if (bud.Kd > 0) {

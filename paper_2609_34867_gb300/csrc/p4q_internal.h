@@ -39,6 +39,8 @@ struct RowSource {
   const int32_t* idx = nullptr;    // [B, K] kept indices (gather mode)
   const uint16_t* text = nullptr;  // [B, T, L] (gather mode)
   int N = 0, K = 0, T = 0;         // gather mode sizes
+  const uint16_t* X2 = nullptr;    // dense rows split, split + 1, ... (the second sinks; dense mode)
+  int split = 0;
 };
 
 // Outputs of the per-row quantizer. Optional pointers may be null.
@@ -51,8 +53,10 @@ struct RowSinks {
   int32_t* sum_u = nullptr;   // [rows] sum of u (with u)
 };
 
+// Rows at or past src.split (when src.X2 is set) come from X2 and go to
+// *out2, renumbered from 0: two row sets quantized by one launch.
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
-                              cudaStream_t stream);
+                              cudaStream_t stream, const RowSinks* out2 = nullptr);
 
 // ------------------------------------------------------------ GEMM
 enum class GemmOut { kHalf = 0, kS32 = 1, kCos = 2 };

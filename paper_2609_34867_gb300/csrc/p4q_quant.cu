@@ -88,6 +88,7 @@ __device__ __forceinline__ uint32_t quant_chunk(const uint4 v, float s, float in
 }
 
 __device__ __forceinline__ const uint16_t* row_ptr(const RowSource& src, int row, int L) {
+  if (src.X2 != nullptr && row >= src.split) return src.X2 + static_cast<size_t>(row - src.split) * L;
   if (src.idx == nullptr) return src.X + static_cast<size_t>(row) * (src.ldx > 0 ? src.ldx : L);
   const int per = src.K + src.T;
   const int b = row / per, r = row - b * per;
@@ -104,7 +105,7 @@ __device__ __forceinline__ const uint16_t* row_ptr(const RowSource& src, int row
 // in flight before the CTA exits.
 template <int G, bool NORM>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
-    quant_rows_kernel(RowSource src, int rows, int L, RowSinks out, int S, uint32_t stage_bytes) {
+    quant_rows_kernel(RowSource src, int rows, int L, RowSinks out1, RowSinks out2, int S, uint32_t stage_bytes) {
   constexpr int kGroups = kWarps / G;
   constexpr int kGroupThreads = 32 * G;
   extern __shared__ __align__(128) unsigned char smem[];
@@ -145,7 +146,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   int consumed = 0;  // rows whose buffer this warp has seen complete
   for (int j = 0; j < mine; ++j) {
     const int st = j % S;
-    const int row = first + j * total;
+    const bool second = src.X2 != nullptr && first + j * total >= src.split;
+    const RowSinks& out = second ? out2 : out1;
+    const int row = second ? first + j * total - src.split : first + j * total;  // row of its sinks
     if (!failed) {
       failed = !mbar_wait_warp(&full[st], (j / S) & 1, abort, &g_quant_err);
       if (!failed) consumed = j + 1;
@@ -277,7 +280,7 @@ int sm_count() {
 }
 
 template <int G, bool NORM>
-cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out, const Plan& p,
+cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out, const RowSinks& out2, const Plan& p,
                      cudaStream_t stream) {
   static bool attr_set = false;
   if (!attr_set) {
@@ -291,27 +294,33 @@ cudaError_t launch_g(const RowSource& src, int rows, int L, const RowSinks& out,
                       3 * kWarps * 4 + kGroups * 4;
   const int need = (rows + kGroups - 1) / kGroups;
   const int grid = std::min(need, kCtasPerSm * sm_count());
-  return launch_pdl(quant_rows_kernel<G, NORM>, dim3(grid), dim3(kThreads), smem, stream, src, rows, L, out, p.S,
-                    p.stage_bytes);
+  return launch_pdl(quant_rows_kernel<G, NORM>, dim3(grid), dim3(kThreads), smem, stream, src, rows, L, out, out2,
+                    p.S, p.stage_bytes);
 }
 
 template <bool NORM>
-cudaError_t launch_norm(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
+cudaError_t launch_norm(const RowSource& src, int rows, int L, const RowSinks& out, const RowSinks& out2,
+                        cudaStream_t stream) {
   const Plan p = plan_for(L);
   switch (p.G) {
-    case 1: return launch_g<1, NORM>(src, rows, L, out, p, stream);
-    case 2: return launch_g<2, NORM>(src, rows, L, out, p, stream);
-    case 4: return launch_g<4, NORM>(src, rows, L, out, p, stream);
-    default: return launch_g<8, NORM>(src, rows, L, out, p, stream);
+    case 1: return launch_g<1, NORM>(src, rows, L, out, out2, p, stream);
+    case 2: return launch_g<2, NORM>(src, rows, L, out, out2, p, stream);
+    case 4: return launch_g<4, NORM>(src, rows, L, out, out2, p, stream);
+    default: return launch_g<8, NORM>(src, rows, L, out, out2, p, stream);
   }
 }
 
 }  // namespace
 
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
-                              cudaStream_t stream) {
+                              cudaStream_t stream, const RowSinks* out2) {
   if (rows <= 0) return cudaSuccess;
-  return out.norm2 ? launch_norm<true>(src, rows, L, out, stream) : launch_norm<false>(src, rows, L, out, stream);
+  if (src.X2 != nullptr && (out2 == nullptr || out2->codes == nullptr || out2->scale == nullptr || src.idx != nullptr ||
+                            src.ldx != 0 || (out.norm2 == nullptr) != (out2->norm2 == nullptr)))
+    return cudaErrorInvalidValue;
+  const RowSinks& o2 = out2 ? *out2 : out;
+  return out.norm2 ? launch_norm<true>(src, rows, L, out, o2, stream)
+                   : launch_norm<false>(src, rows, L, out, o2, stream);
 }
 
 unsigned int quant_read_and_clear_error() {
