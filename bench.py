@@ -10,12 +10,13 @@ budget 192 kept tokens per image):
   p4q_expand_codes         each GEMM's packed INT4 weights, per call, into
                            that GEMM's scratch, on a side stream from the
                            start of the step
-  p4q_w4a4_linear_expanded x 4  q|k|v and gate|up (each one GEMM over the
+  p4q_w4a4_linear_expanded x 3  q|k|v|gate|up (one GEMM over the
                            concatenated output channels) on the pruned
                            sequence (M = 2048), o on the re-quantized q
                            output, down on the re-quantized up output
                            (2 x p4q_quant_act_expanded on column blocks;
-                           the o chain on a third stream beside gate|up).
+                           the o chain on a third stream beside the
+                           down chain).
 The metric is W4A4 linear TOPS: 2 * M * N * K integer ops of the seven linears
 per step divided by the step time (the selector's time included); the
 selector's share is also reported as microseconds per image.
@@ -181,11 +182,13 @@ class Step:
     weights, independent batches). Every layer runs on the pruned sequence:
     q, k, v, gate, up on its INT4 codes, o on the re-quantized q output, down
     on the re-quantized up output. Linears that read the same input run as one
-    GEMM over their concatenated output channels (q|k|v and gate|up), which
+    GEMM over their concatenated output channels (q|k|v|gate|up), which
     computes exactly the same outputs (the weight quantizer works per output
-    channel) with fewer launches and fuller waves of tiles."""
+    channel) with fewer launches and fuller waves of tiles: 1072 tiles of
+    256 x 256 take 15 rounds of the 76 CTA pairs, where q|k|v and gate|up
+    apart take 6 + 10."""
 
-    FUSE = (("qkv", ("q", "k", "v")), ("gate_up", ("gate", "up")))
+    FUSE = (("qkv_gate_up", ("q", "k", "v", "gate", "up")),)
     REQUANT = {"o": "q", "down": "up"}  # linear -> the linear whose output it re-quantizes
 
     def __init__(self, w: wl.Workload, dev, seed: int):
