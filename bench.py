@@ -314,8 +314,8 @@ class Step:
         - side: every GEMM's weight expansion, into that GEMM's scratch, in
           step order (a later layer's waits until the previous layer's GEMM
           has read the scratch), overlapping the selector and the GEMMs;
-        - aux: the o chain (re-quantization of the q block, o GEMM), which
-          only needs the q|k|v GEMM and so overlaps the gate|up GEMM;
+        - aux: the o chain (re-quantization of the q block, o GEMM), beside
+          the down chain (re-quantization of the up block, down GEMM);
         - the current stream: everything else."""
         torch = self.torch
         main = torch.cuda.current_stream()
