@@ -3,6 +3,7 @@
   python -m paper_2609_34867_gb300.kernel_cases gemm M N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases gemm8 M N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases quant M K [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases requant M L LD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
@@ -18,6 +19,9 @@ selects the first replayed launch.
           p4q_expand_codes before timing (the GEMM kernel alone);
   quant   p4q_quant_act on M x K fp16 activations with the outlier channels
           (bytes: 2 M K in, M K / 2 + 4 M out);
+  requant p4q_quant_act_expanded on the last L columns of an M x LD fp16
+          matrix (a linear's output block inside a fused GEMM's output), with
+          the expanded codes (bytes: 2 M L in, 3 M L / 2 + 8 M out);
   select  p4q_select_gather_quant on one of the LLaVA-shaped workloads.
 """
 from __future__ import annotations
@@ -61,7 +65,7 @@ def _timed(fn, reps, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "select"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -91,6 +95,18 @@ def main(argv=None):
         ms = _timed(lambda: p4q.p4q_quant_act(X, Xq, s), a.reps, dev)
         nbytes = 2 * M * K + M * K // 2 + 4 * M
         print(f"quant {M}x{K}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "requant":
+        M, L, LD = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        Y = (torch.randn((M, LD), generator=g, device=dev) * 4.0).to(torch.float16)
+        X = Y[:, LD - L:]
+        Xq = torch.empty((M, L // 2), dtype=torch.uint8, device=dev)
+        s = torch.empty((M,), dtype=torch.float32, device=dev)
+        Xu = torch.empty((M, L), dtype=torch.uint8, device=dev)
+        su = torch.empty((M,), dtype=torch.int32, device=dev)
+        ms = _timed(lambda: p4q.p4q_quant_act_expanded(X, Xq, s, Xu, su), a.reps, dev)
+        nbytes = 2 * M * L + 3 * M * L // 2 + 8 * M
+        print(f"requant {M}x{L} of {LD}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
     else:
         w = wl.WORKLOADS[a.args[0]]
         x = wl.selector_inputs(w)
