@@ -369,21 +369,33 @@ class Step:
         """Captures the whole step into one CUDA graph (consecutive kernels
         overlap their launch and set-up with the previous kernel's tail), and
         every segment into its own graph for per-segment timing (after warm-up
-        calls have set up the kernels' attributes)."""
+        calls have set up the kernels' attributes). Garbage collection is
+        done before and held off during the captures: a collected object that
+        owns a CUDA graph (a Step lives in a reference cycle through its
+        segment closures) would destroy it mid-capture, which invalidates the
+        capture."""
+        import gc
         torch = self.torch
-        self.graphs = []
-        for _, _, fn in self.segments:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g):
-                fn()
-            self.graphs.append(g)
-        self.body()  # warm the side-stream path before capturing it
-        torch.cuda.synchronize()
-        n0 = self.p4q.p4q_launch_count()
-        self.full = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(self.full):
-            self.body()
-        self.launches_per_step = self.p4q.p4q_launch_count() - n0
+        gc.collect()
+        was_enabled = gc.isenabled()
+        gc.disable()
+        try:
+            self.graphs = []
+            for _, _, fn in self.segments:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    fn()
+                self.graphs.append(g)
+            self.body()  # warm the side-stream path before capturing it
+            torch.cuda.synchronize()
+            n0 = self.p4q.p4q_launch_count()
+            self.full = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(self.full):
+                self.body()
+            self.launches_per_step = self.p4q.p4q_launch_count() - n0
+        finally:
+            if was_enabled:
+                gc.enable()
 
     def __call__(self, segments: bool = False):
         """One step: the whole-step graph, or (segments=True) the segment

@@ -23,6 +23,7 @@ Checked against the oracle:
   dequant (App. B.3).
 """
 import dataclasses
+import gc
 
 import numpy as np
 import pytest
@@ -56,6 +57,7 @@ def run_step(p4q, dev):
 
     yield run
     made.clear()
+    gc.collect()  # the steps' CUDA graphs go now, not inside a later capture
     torch.cuda.empty_cache()
 
 
