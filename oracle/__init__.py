@@ -5,7 +5,8 @@ Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``p4q_oracle.c`` (plain C11, compiled with gcc) and shares no code with the
 CUDA library. Every function here marshals numpy arrays; the arithmetic lives
 in the C file, which cites the paper passage each step follows (Sec. 3.2,
-Eq. 4 for the selector; App. A and App. B.3 for the W4A4 quantizer).
+Eq. 4 for the selector and the CLS saliency; App. A and App. B.3 for the
+W4A4 quantizer).
 
 fp16 inputs are widened to fp32 with numpy before the call; that conversion is
 exact, so the oracle sees the same values as the GPU path.
@@ -65,6 +66,8 @@ def _load():
             lib.w4a4_linear.restype = i32
             lib.p4q_gather.argtypes = [P, i32, i32, i32, P, i32, P, i32, P]
             lib.p4q_gather.restype = i32
+            lib.p4q_cls_saliency.argtypes = [P, P, P, i32, i32, i32, i32, i32, P]
+            lib.p4q_cls_saliency.restype = i32
             _lib = lib
     return _lib
 
@@ -194,6 +197,21 @@ def gather(V, idx, text=None):
     if rc != OK:
         raise ValueError(f"oracle gather failed ({rc})")
     return X
+
+
+def cls_saliency(q_cls, k_cls, k):
+    """A_cls [B, N] (fp64) from the vision tower's final-layer attention (Sec. 3.2,
+    Visual Saliency): per crop, the CLS query's softmax over the CLS key and
+    the crop's patch keys, averaged over the heads.
+    q_cls, k_cls: [B, C, H, dh]; k: [B, N, H, dh] (crop c = tokens c*N/C ..)."""
+    q, kc, kp = _f32(q_cls), _f32(k_cls), _f32(k)
+    B, C, H, dh = q.shape
+    N = kp.shape[1]
+    A = np.empty((B, N), np.float64)
+    rc = _load().p4q_cls_saliency(_ptr(q), _ptr(kc), _ptr(kp), B, N, C, H, dh, _ptr(A))
+    if rc != OK:
+        raise ValueError(f"oracle cls_saliency failed ({rc})")
+    return A
 
 
 def pack_codes(codes):

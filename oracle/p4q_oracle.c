@@ -41,6 +41,11 @@
  *      times. Updating m_i with the newest pick equals recomputing the max
  *      over the whole kept set, because max is associative.
  *   R8 output indices are sorted ascending.
+ *   R9 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
+ *      self-attention, each crop's [CLS] token is the query; its attention
+ *      row is the softmax, over the CLS key and the crop's patch keys, of
+ *      q . k / sqrt(d_h); A_cls of a patch is that weight averaged over the
+ *      heads. One CLS per crop (crops of N / C consecutive tokens). fp64.
  *
  * Build: plain C11, -O2 -ffp-contract=off (no fused multiply-add, no
  * fast-math), optional OpenMP over independent rows / images.
@@ -327,5 +332,47 @@ int p4q_gather(const float* V, int B, int N, int d, const int32_t* idx, int K, c
     for (int t = 0; t < T; ++t)
       memcpy(xb + (int64_t)(K + t) * d, text + ((int64_t)b * T + t) * d, sizeof(float) * d);
   }
+  return ORACLE_OK;
+}
+
+/* CLS-to-patch saliency A_cls (Sec. 3.2, Visual Saliency; reading R9):
+ *   q_cls, k_cls: [B, C, H, dh] (the final layer's CLS query and key of each
+ *   crop, per head); k: [B, N, H, dh] (patch keys; crop c holds tokens
+ *   [c * N / C, (c + 1) * N / C)); out A: [B, N]. For each image b, crop c,
+ *   head h: logits l_0 = q . k_cls / sqrt(dh) and l_i = q . k_i / sqrt(dh)
+ *   for the crop's patches, p = softmax over {l_0, l_i}, then
+ *   A[b, i] = (1 / H) sum_h p_i. fp64 throughout. */
+int p4q_cls_saliency(const float* q_cls, const float* k_cls, const float* k, int B, int N, int C, int H, int dh,
+                     double* A) {
+  if (!q_cls || !k_cls || !k || !A || B < 0 || N < 1 || C < 1 || N % C != 0 || H < 1 || dh < 1)
+    return ORACLE_BAD_ARG;
+  const int n = N / C;
+  const double inv_sqrt = 1.0 / sqrt((double)dh);
+  double* l = (double*)malloc(sizeof(double) * (size_t)(n + 1));
+  if (!l) return ORACLE_BAD_ARG;
+  for (int64_t i = 0; i < (int64_t)B * N; ++i) A[i] = 0.0;
+  for (int b = 0; b < B; ++b) {
+    for (int c = 0; c < C; ++c) {
+      for (int h = 0; h < H; ++h) {
+        const float* q = q_cls + (((int64_t)b * C + c) * H + h) * dh;
+        const float* kc = k_cls + (((int64_t)b * C + c) * H + h) * dh;
+        double dot = 0.0;
+        for (int e = 0; e < dh; ++e) dot += (double)q[e] * (double)kc[e];
+        l[0] = dot * inv_sqrt;
+        for (int i = 0; i < n; ++i) {
+          const float* ki = k + (((int64_t)b * N + (int64_t)c * n + i) * H + h) * dh;
+          dot = 0.0;
+          for (int e = 0; e < dh; ++e) dot += (double)q[e] * (double)ki[e];
+          l[1 + i] = dot * inv_sqrt;
+        }
+        double mx = l[0];
+        for (int i = 1; i <= n; ++i) mx = l[i] > mx ? l[i] : mx;
+        double z = 0.0;
+        for (int i = 0; i <= n; ++i) z += exp(l[i] - mx);
+        for (int i = 0; i < n; ++i) A[(int64_t)b * N + (int64_t)c * n + i] += exp(l[1 + i] - mx) / z / (double)H;
+      }
+    }
+  }
+  free(l);
   return ORACLE_OK;
 }
