@@ -216,6 +216,27 @@ p4q_status p4q_w4a4_gemm_s32_ws(const uint8_t* Xq, int M, int Kin, const uint8_t
 /* Quantization-aware visual-token selector (Sec. 3.2, Eq. 4)               */
 /* ---------------------------------------------------------------------- */
 
+/* CLS-to-patch saliency A_cls, the input of the selector's stage 2 (Sec. 3.2,
+ * Visual Saliency: in the vision tower's final self-attention layer each
+ * crop's [CLS] token is the query; the attention weights of the patch keys
+ * are averaged across the heads). Per image b, crop c and head h:
+ *   l_0 = q . k_cls / sqrt(dh), l_i = q . k_i / sqrt(dh) for the crop's
+ *   patches i; p = softmax over {l_0, l_i} (the CLS key is part of the
+ *   attention row); A_cls[b, i] = (1 / H) sum_h p_i.
+ * fp16 inputs, fp32 arithmetic (products accumulated in fp32, expf, one
+ * division per head), heads summed in order (deterministic).
+ *   q_cls [B, C, H, dh] fp16  final-layer CLS query of each crop, per head
+ *   k_cls [B, C, H, dh] fp16  final-layer CLS key of each crop, per head
+ *   k     [B, N, H, dh] fp16  patch keys; crop c holds tokens
+ *                             [c * N / C, (c + 1) * N / C)
+ *   A_cls [B, N] fp32         written
+ * Requires 1 <= B <= 65535, 1 <= C, N % C == 0, 1 <= N / C <= P4Q_MAX_TOKENS,
+ * dh in {32, 64, 80, 128}, 1 <= H <= 32, H * (N / C) * 4 <= 227 KB (one
+ * crop's weights in shared memory), 16-byte aligned pointers. All device
+ * pointers; asynchronous on `stream`. */
+p4q_status p4q_cls_saliency(const uint16_t* q_cls, const uint16_t* k_cls, const uint16_t* k, int B, int N, int C,
+                            int H, int dh, float* A_cls, p4q_stream_t stream);
+
 /* Device workspace needed by p4q_select / p4q_select_gather_quant for these
  * sizes (bytes, a multiple of 256). Returns 0 if the sizes are invalid. */
 size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_params* params);

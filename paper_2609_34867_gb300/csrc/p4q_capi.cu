@@ -165,6 +165,19 @@ const char* p4q_status_string(p4q_status s) {
 
 uint64_t p4q_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+p4q_status p4q_cls_saliency(const uint16_t* q_cls, const uint16_t* k_cls, const uint16_t* k, int B, int N, int C,
+                            int H, int dh, float* A_cls, p4q_stream_t stream) {
+  if (!q_cls || !k_cls || !k || !A_cls || B < 1 || N < 1 || C < 1 || H < 1) return P4Q_ERR_INVALID_ARG;
+  if (B > 65535 || N % C != 0 || N / C > P4Q_MAX_TOKENS || (dh != 32 && dh != 64 && dh != 80 && dh != 128) ||
+      H > cls_saliency_max_heads(dh) || cls_saliency_smem_bytes(N, C, H) > 227u * 1024u)
+    return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned16(q_cls) || !aligned16(k_cls) || !aligned16(k) || !aligned16(A_cls)) return P4Q_ERR_MISALIGNED;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_cls_saliency(q_cls, k_cls, k, B, N, C, H, dh, A_cls,
+                                               reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_set_gemm_variant(int variant) {
   if (variant < 0 || variant > 3) return P4Q_ERR_INVALID_ARG;
   set_gemm_pair_mode(variant == 0 || variant == 3 ? -1 : variant == 1 ? 0 : 1);

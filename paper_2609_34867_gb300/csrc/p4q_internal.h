@@ -87,6 +87,15 @@ void set_gemm_pair_mode(int mode);
 // Expanded-operand path: 0 automatic (M >= 512), 1 never, 2 whenever a workspace is given.
 void set_gemm8_mode(int mode);
 
+// ------------------------------------------------------------ CLS saliency
+// Shared memory of one (image, crop) CTA: H x (N / C) fp32 weights.
+size_t cls_saliency_smem_bytes(int N, int C, int H);
+// Heads one CTA takes for this head dimension (one warp each).
+int cls_saliency_max_heads(int dh);
+// dh in {32, 64, 80, 128}; else cudaErrorInvalidValue.
+cudaError_t launch_cls_saliency(const uint16_t* q_cls, const uint16_t* k_cls, const uint16_t* k, int B, int N,
+                                int C, int H, int dh, float* A, cudaStream_t stream);
+
 // ------------------------------------------------------------ selector
 struct SelectPlan {
   int B, N, d, J, K, Kq, Ks, Kd;

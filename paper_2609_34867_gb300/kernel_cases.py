@@ -5,6 +5,7 @@
   python -m paper_2609_34867_gb300.kernel_cases quant M K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases requant M L LD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases saliency B N [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -22,7 +23,10 @@ selects the first replayed launch.
   requant p4q_quant_act_expanded on the last L columns of an M x LD fp16
           matrix (a linear's output block inside a fused GEMM's output), with
           the expanded codes (bytes: 2 M L in, 3 M L / 2 + 8 M out);
-  select  p4q_select_gather_quant on one of the LLaVA-shaped workloads.
+  select  p4q_select_gather_quant on one of the LLaVA-shaped workloads;
+  saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
+          heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
+          fp16 keys and queries in, 4 B N out).
 """
 from __future__ import annotations
 
@@ -65,7 +69,7 @@ def _timed(fn, reps, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -107,6 +111,14 @@ def main(argv=None):
         ms = _timed(lambda: p4q.p4q_quant_act_expanded(X, Xq, s, Xu, su), a.reps, dev)
         nbytes = 2 * M * L + 3 * M * L // 2 + 8 * M
         print(f"requant {M}x{L} of {LD}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "saliency":
+        B, N = (int(x) for x in a.args)
+        v = wl.vision_attention(B, N, seed=0)
+        q, kc, k = (torch.from_numpy(t).to(dev) for t in (v.q_cls, v.k_cls, v.k))
+        A = torch.empty((B, N), dtype=torch.float32, device=dev)
+        ms = _timed(lambda: p4q.p4q_cls_saliency(q, kc, k, A), a.reps, dev)
+        nbytes = 2 * (q.numel() + kc.numel() + k.numel()) + 4 * A.numel()
+        print(f"saliency {B}x{N}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
     else:
         w = wl.WORKLOADS[a.args[0]]
         x = wl.selector_inputs(w)

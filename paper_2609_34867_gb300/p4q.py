@@ -47,6 +47,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_launch_count.restype = ctypes.c_uint64
         L.p4q_set_gemm_variant.argtypes = [I]
         L.p4q_set_gemm_variant.restype = st
+        L.p4q_cls_saliency.argtypes = [P, P, P, I, I, I, I, I, P, P]
+        L.p4q_cls_saliency.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
@@ -225,6 +227,24 @@ def p4q_select_gather_quant_expanded(V, Q, A_cls, text, K, idx, X, Xq, s_a, Xu, 
                                                   ctypes.byref(p), _ptr(idx), _ptr(X), _ptr(Xq), _ptr(s_a), _ptr(Xu),
                                                   _ptr(sum_xu), _ptr(ws), ws.numel(), _stream(stream)),
            "p4q_select_gather_quant_expanded")
+
+
+def p4q_cls_saliency(q_cls, k_cls, k, A_cls, stream=None):
+    """A_cls [B, N] fp32 from the final-layer CLS query/key [B, C, H, dh] and
+    patch keys [B, N, H, dh] (fp16, contiguous)."""
+    _need(q_cls, torch.float16, 4, "q_cls"); _need(k_cls, torch.float16, 4, "k_cls")
+    _need(k, torch.float16, 4, "k"); _need(A_cls, torch.float32, 2, "A_cls")
+    B, C, H, dh = q_cls.shape
+    N = k.shape[1]
+    _check(lib().p4q_cls_saliency(_ptr(q_cls), _ptr(k_cls), _ptr(k), B, N, C, H, dh, _ptr(A_cls), _stream(stream)),
+           "p4q_cls_saliency")
+
+
+def cls_saliency(q_cls, k_cls, k, stream=None):
+    """Allocating wrapper of p4q_cls_saliency."""
+    A = torch.empty((q_cls.shape[0], k.shape[1]), dtype=torch.float32, device=k.device)
+    p4q_cls_saliency(q_cls, k_cls, k, A, stream)
+    return A
 
 
 # ---------------------------------------------------------------- helpers

@@ -129,6 +129,31 @@ def cls_saliency(rng: np.random.Generator, B: int, N: int) -> np.ndarray:
     return out.astype(np.float32)
 
 
+VIT_HEADS, VIT_HEAD_DIM = 16, 64  # CLIP ViT-L/14 vision tower: 1024 wide = 16 heads x 64
+
+
+@dataclasses.dataclass
+class VisionAttention:
+    q_cls: np.ndarray  # [B, C, H, dh] fp16, the final layer's CLS query of each crop
+    k_cls: np.ndarray  # [B, C, H, dh] fp16, its CLS key
+    k: np.ndarray      # [B, N, H, dh] fp16, the patch keys (crop c = tokens c*CROP ..)
+
+
+def vision_attention(B: int, N: int, seed: int, H: int = VIT_HEADS, dh: int = VIT_HEAD_DIM,
+                     crop: int = CROP) -> VisionAttention:
+    """Synthetic final-layer attention inputs of the vision tower, one CLS per
+    crop of `crop` tokens (N a multiple of it): N(0, 1) keys, the CLS query
+    N(0, 1) x 2 so that each head's attention row is peaked (logit spread
+    about 2) like a trained ViT's."""
+    assert N % crop == 0
+    rng = np.random.default_rng(seed)
+    C = N // crop
+    q = (rng.standard_normal(size=(B, C, H, dh), dtype=np.float32) * np.float32(2.0)).astype(np.float16)
+    kc = rng.standard_normal(size=(B, C, H, dh), dtype=np.float32).astype(np.float16)
+    k = rng.standard_normal(size=(B, N, H, dh), dtype=np.float32).astype(np.float16)
+    return VisionAttention(q, kc, k)
+
+
 @dataclasses.dataclass
 class SelectorInputs:
     V: np.ndarray      # [B, N, d] fp16

@@ -58,6 +58,20 @@ def test_invalid_arguments_are_rejected_before_any_launch(lib):
     assert lib.p4q_w4a4_linear(P(16), P(16), 4, 128, None, P(16), 8, P(16), None) == 1
 
 
+def test_cls_saliency_validates_shapes(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_cls_saliency.argtypes = [P, P, P, I, I, I, I, I, P, P]
+    f = lib.p4q_cls_saliency
+    ok = (P(16), P(16), P(16))
+    assert f(None, P(16), P(16), 1, 576, 1, 16, 64, P(16), None) == 1   # null pointer
+    assert f(*ok, 0, 576, 1, 16, 64, P(16), None) == 1                  # B < 1
+    assert f(*ok, 1, 577, 2, 16, 64, P(16), None) == 2                  # N % C
+    assert f(*ok, 1, 576, 1, 16, 48, P(16), None) == 2                  # head dim
+    assert f(*ok, 1, 576, 1, 33, 64, P(16), None) == 2                  # heads
+    assert f(*ok, 1, 4096, 1, 32, 64, P(16), None) == 2                 # one crop's weights exceed shared memory
+    assert f(P(8), P(16), P(16), 1, 576, 1, 16, 64, P(16), None) == 3   # misaligned
+
+
 class Params(ctypes.Structure):
     _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
 
