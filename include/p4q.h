@@ -85,8 +85,10 @@ uint64_t p4q_launch_count(void);
 
 /* GEMM kernel variant used by p4q_w4a4_linear and p4q_w4a4_gemm_s32, for all
  * later calls in the process (for tests and tuning; results are identical):
- *   0 automatic (default): CTA-pair kernel for fp16 outputs with M >= 256 and
- *     N >= 256, single-CTA kernel otherwise;
+ *   0 automatic (default): for M <= 8 rows a weight-streaming kernel (dp4a
+ *     on the CUDA cores: the packed weights are read once); CTA-pair kernel
+ *     for fp16 outputs with M >= 256 and N >= 256; single-CTA kernel
+ *     otherwise;
  *   1 single-CTA kernel only;
  *   2 CTA-pair kernel whenever N >= 256 (also for int32 outputs);
  *   3 like 0, and the workspace entry points take the expanded-operand path

@@ -1069,6 +1069,8 @@ static int g_pair_mode = -1;  // -1: automatic, 0: never, 1: whenever the shape 
 void set_gemm_pair_mode(int mode) { g_pair_mode = mode; }
 
 cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream) {
+  // a few rows (decode): weight streaming on the CUDA cores (automatic mode only)
+  if (g_pair_mode == -1 && gemv_applies(g)) return launch_gemv(g, stream);
   const bool pair_ok = g.M > 0 && g.N >= 256 && g.batch > 0 && g_pair_mode != 0 &&
                        (g_pair_mode == 1 || (g.M >= 256 && g.out == GemmOut::kHalf));
   if (pair_ok && g.out == GemmOut::kHalf) return launch_pair<0>(g, stream);

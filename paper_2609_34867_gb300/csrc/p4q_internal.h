@@ -80,9 +80,14 @@ struct GemmArgs {
 // cannot run on this kernel.
 cudaError_t launch_w4a4_gemm(const GemmArgs& g, cudaStream_t stream);
 
-// Which GEMM kernel serves fp16 / int32 outputs: -1 automatic (the CTA-pair
-// kernel for large fp16 linears), 0 single-CTA only, 1 CTA-pair whenever the
-// shape allows (N >= 256).
+// W4A4 linear / int32 accumulators for M <= 8 rows (decode): streams the
+// packed weights, dp4a against the activation rows staged in shared memory.
+bool gemv_applies(const GemmArgs& g);
+cudaError_t launch_gemv(const GemmArgs& g, cudaStream_t stream);
+
+// Which GEMM kernel serves fp16 / int32 outputs: -1 automatic (the
+// weight-streaming kernel for M <= 8, the CTA-pair kernel for large fp16
+// linears), 0 single-CTA only, 1 CTA-pair whenever the shape allows (N >= 256).
 void set_gemm_pair_mode(int mode);
 // Expanded-operand path: 0 automatic (M >= 512), 1 never, 2 whenever a workspace is given.
 void set_gemm8_mode(int mode);
