@@ -68,6 +68,10 @@ def _load():
             lib.p4q_gather.restype = i32
             lib.p4q_cls_saliency.argtypes = [P, P, P, i32, i32, i32, i32, i32, P]
             lib.p4q_cls_saliency.restype = i32
+            lib.oracle_exp32_array.argtypes = [P, i64, P]
+            lib.oracle_exp32_array.restype = i32
+            lib.p4q_swiglu_quantize_rows.argtypes = [P, P, i64, i64, P, P]
+            lib.p4q_swiglu_quantize_rows.restype = i32
             _lib = lib
     return _lib
 
@@ -212,6 +216,32 @@ def cls_saliency(q_cls, k_cls, k):
     if rc != OK:
         raise ValueError(f"oracle cls_saliency failed ({rc})")
     return A
+
+
+def exp32(x):
+    """The oracle's own fp32 exponential (Cody-Waite reduction, degree-7
+    Taylor polynomial, ldexp), elementwise; the CUDA path evaluates the same
+    function bit for bit."""
+    a = _f32(x)
+    y = np.empty_like(a)
+    rc = _load().oracle_exp32_array(_ptr(a), a.size, _ptr(y))
+    if rc != OK:
+        raise ValueError("oracle exp32 failed")
+    return y
+
+
+def swiglu_quantize_rows(gate, up):
+    """h = silu(gate) * up (silu(g) = g / (1 + exp32(-g)), fp32), then the per-row
+    4-bit quantizer: returns (codes int8 [rows, cols], scale fp32 [rows])."""
+    g, u = _f32(gate), _f32(up)
+    assert g.shape == u.shape and g.ndim == 2
+    rows, cols = g.shape
+    codes = np.empty((rows, cols), np.int8)
+    scale = np.empty((rows,), np.float32)
+    rc = _load().p4q_swiglu_quantize_rows(_ptr(g), _ptr(u), rows, cols, _ptr(codes), _ptr(scale))
+    if rc != OK:
+        raise ValueError(f"oracle swiglu_quantize_rows failed ({rc})")
+    return codes, scale
 
 
 def pack_codes(codes):

@@ -41,6 +41,14 @@
  *      times. Updating m_i with the newest pick equals recomputing the max
  *      over the whole kept set, because max is associative.
  *   R8 output indices are sorted ascending.
+ *   R10 SwiGLU before down_proj (the decoder's MLP; the paper quantizes every
+ *      linear's input per token): h = silu(gate) * up, silu(g) =
+ *      g / (1 + exp32(-g)), then h quantized by R1. exp32 is this file's own
+ *      fp32 exponential (Cody-Waite range reduction with ln 2 split as
+ *      355/512 + a low part, degree-7 Taylor polynomial by Horner's rule with
+ *      fused multiply-adds, ldexp; 0 below -87.33655, inf above 88.72284):
+ *      every step is one correctly rounded fp32 operation, so the CUDA path
+ *      evaluates the same function bit for bit and the codes match exactly.
  *   R9 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
  *      self-attention, each crop's [CLS] token is the query; its attention
  *      row is the softmax, over the CLS key and the crop's patch keys, of
@@ -375,4 +383,57 @@ int p4q_cls_saliency(const float* q_cls, const float* k_cls, const float* k, int
   }
   free(l);
   return ORACLE_OK;
+}
+
+/* Own fp32 exponential (reading R10): n = rint(x * log2 e); r = x - n ln2 in
+ * two fused steps (ln2 = 355/512 + LN2_LO; n * 355/512 is exact for the n
+ * that occur); e^r by the degree-7 Taylor polynomial (|r| <= ln2 / 2: the
+ * truncation is below 2e-8 relative); times 2^n. Results that would be
+ * subnormal are 0 (they vanish in 1 + e anyway). */
+float oracle_exp32(float x) {
+  if (x > 0x1.62e430p+6f) return INFINITY;
+  if (x < -0x1.5d58a0p+6f) return 0.0f;
+  const float n = nearbyintf(x * 0x1.715476p+0f);
+  float r = fmaf(-n, 0x1.630000p-1f, x);
+  r = fmaf(-n, -0x1.bd0106p-13f, r);
+  float p = 0x1.a01a02p-13f;
+  p = fmaf(p, r, 0x1.6c16c2p-10f);
+  p = fmaf(p, r, 0x1.111112p-7f);
+  p = fmaf(p, r, 0x1.555556p-5f);
+  p = fmaf(p, r, 0x1.555556p-3f);
+  p = fmaf(p, r, 0.5f);
+  p = fmaf(p, r, 1.0f);
+  p = fmaf(p, r, 1.0f);
+  return ldexpf(p, (int)n);
+}
+
+int oracle_exp32_array(const float* x, int64_t n, float* y) {
+  if (!x || !y || n < 0) return ORACLE_BAD_ARG;
+  for (int64_t i = 0; i < n; ++i) y[i] = oracle_exp32(x[i]);
+  return ORACLE_OK;
+}
+
+/* SwiGLU then the per-token quantizer (reading R10): h = silu(g) * u with
+ * silu(g) = g / (1 + exp32(-g)), every operation one rounded fp32 step, then
+ * quantize_row on h. gate, up, h: [rows, cols]. */
+int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, int64_t cols, int8_t* code,
+                             float* scale) {
+  if (!gate || !up || !code || !scale || rows < 0 || cols <= 0) return ORACLE_BAD_ARG;
+  int rc = ORACLE_OK;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r) {
+    float* h = (float*)malloc(sizeof(float) * (size_t)cols);
+    if (!h) {
+      rc = ORACLE_BAD_ARG;
+      continue;
+    }
+    for (int64_t k = 0; k < cols; ++k) {
+      const float g = gate[r * cols + k];
+      const float silu = g / (1.0f + oracle_exp32(-g));
+      h[k] = silu * up[r * cols + k];
+    }
+    quantize_row(h, cols, code + r * cols, scale + r);
+    free(h);
+  }
+  return rc;
 }
