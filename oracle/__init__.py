@@ -220,8 +220,8 @@ def cls_saliency(q_cls, k_cls, k):
 
 def exp32(x):
     """The oracle's own fp32 exponential (Cody-Waite reduction, degree-7
-    Taylor polynomial, ldexp), elementwise; the CUDA path evaluates the same
-    function bit for bit."""
+    Taylor polynomial, power-of-two scaling; 0 below -87), elementwise; the
+    CUDA path evaluates the same function bit for bit."""
     a = _f32(x)
     y = np.empty_like(a)
     rc = _load().oracle_exp32_array(_ptr(a), a.size, _ptr(y))

@@ -46,7 +46,8 @@
  *      g / (1 + exp32(-g)), then h quantized by R1. exp32 is this file's own
  *      fp32 exponential (Cody-Waite range reduction with ln 2 split as
  *      355/512 + a low part, degree-7 Taylor polynomial by Horner's rule with
- *      fused multiply-adds, ldexp; 0 below -87.33655, inf above 88.72284):
+ *      fused multiply-adds, two exact power-of-two scalings; 0 below -87,
+ *      inf above 88.72284):
  *      every step is one correctly rounded fp32 operation, so the CUDA path
  *      evaluates the same function bit for bit and the codes match exactly.
  *   R9 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
@@ -385,14 +386,23 @@ int p4q_cls_saliency(const float* q_cls, const float* k_cls, const float* k, int
   return ORACLE_OK;
 }
 
+/* 2^k as an fp32 bit pattern, -126 <= k <= 127. */
+static float pow2f(int k) {
+  const uint32_t b = (uint32_t)(k + 127) << 23;
+  float f;
+  memcpy(&f, &b, sizeof f);
+  return f;
+}
+
 /* Own fp32 exponential (reading R10): n = rint(x * log2 e); r = x - n ln2 in
  * two fused steps (ln2 = 355/512 + LN2_LO; n * 355/512 is exact for the n
  * that occur); e^r by the degree-7 Taylor polynomial (|r| <= ln2 / 2: the
- * truncation is below 2e-8 relative); times 2^n. Results that would be
- * subnormal are 0 (they vanish in 1 + e anyway). */
+ * truncation is below 2e-8 relative); times 2^n as two exact multiplications
+ * by powers of two. Below -87 the result is 0 (so every other result is a
+ * normal number; such values vanish in 1 + e anyway), above 88.72284 inf. */
 float oracle_exp32(float x) {
   if (x > 0x1.62e430p+6f) return INFINITY;
-  if (x < -0x1.5d58a0p+6f) return 0.0f;
+  if (x < -87.0f) return 0.0f;
   const float n = nearbyintf(x * 0x1.715476p+0f);
   float r = fmaf(-n, 0x1.630000p-1f, x);
   r = fmaf(-n, -0x1.bd0106p-13f, r);
@@ -404,7 +414,8 @@ float oracle_exp32(float x) {
   p = fmaf(p, r, 0.5f);
   p = fmaf(p, r, 1.0f);
   p = fmaf(p, r, 1.0f);
-  return ldexpf(p, (int)n);
+  const int k = (int)n, a = k / 2;
+  return (p * pow2f(a)) * pow2f(k - a);
 }
 
 int oracle_exp32_array(const float* x, int64_t n, float* y) {
