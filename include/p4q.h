@@ -141,6 +141,27 @@ p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t*
 p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a, uint8_t* Xu,
                                   int32_t* sum_xu, p4q_stream_t stream);
 
+/* SwiGLU before down_proj fused with the per-token quantizer of its input
+ * (App. A quantizes every linear's input per token; the decoder's MLP feeds
+ * down_proj with silu(gate) * up). For each row m:
+ *   h_k = silu(g_k) * u_k with silu(g) = g * (1 / (1 + exp32(-g))), each
+ *   operation one rounded fp32 step (the reciprocal correctly rounded), where
+ *   exp32 is this library's own fp32 exponential: n = rint(x * log2 e),
+ *   r = x - n * ln2 by two fused multiply-adds (ln2 = 355/512 + a low part),
+ *   e^r by the degree-7 Taylor polynomial (Horner, fused multiply-adds),
+ *   times 2^n by two exact power-of-two multiplications; 0 for x < -87, inf
+ *   for x > 88.72284 (within 1 ulp of e^x in between);
+ *   then the codes and scale of h as p4q_quant_act.
+ *   gate, up [M, Kin] fp16, rows ld_gate / ld_up elements apart (column
+ *              blocks of a fused gate|up output; device, read)
+ *   Xq [M, Kin/2], s_a [M]           written
+ *   Xu [M, Kin], sum_xu [M]          the expanded codes (p4q_expand_codes
+ *                                    form) or both NULL
+ * Requires M >= 0, 16 <= Kin <= P4Q_MAX_ROW, Kin % 16 == 0, ld >= Kin,
+ * ld % 8 == 0, 16-byte aligned pointers. M == 0 is a no-op. */
+p4q_status p4q_swiglu_quant_expanded(const uint16_t* gate, int ld_gate, const uint16_t* up, int ld_up, int M, int Kin,
+                                     uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, p4q_stream_t stream);
+
 /* Per-output-channel weight quantization (App. B.3: symmetric, per output
  * channel, then round-to-nearest): the same per-row quantizer applied to each
  * output row of W.

@@ -231,7 +231,7 @@ def exp32(x):
 
 
 def swiglu_quantize_rows(gate, up):
-    """h = silu(gate) * up (silu(g) = g / (1 + exp32(-g)), fp32), then the per-row
+    """h = silu(gate) * up (silu(g) = g * (1 / (1 + exp32(-g))), fp32), then the per-row
     4-bit quantizer: returns (codes int8 [rows, cols], scale fp32 [rows])."""
     g, u = _f32(gate), _f32(up)
     assert g.shape == u.shape and g.ndim == 2

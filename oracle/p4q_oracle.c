@@ -43,7 +43,8 @@
  *   R8 output indices are sorted ascending.
  *   R10 SwiGLU before down_proj (the decoder's MLP; the paper quantizes every
  *      linear's input per token): h = silu(gate) * up, silu(g) =
- *      g / (1 + exp32(-g)), then h quantized by R1. exp32 is this file's own
+ *      g * (1 / (1 + exp32(-g))) (four rounded fp32 steps), then h quantized
+ *      by R1. exp32 is this file's own
  *      fp32 exponential (Cody-Waite range reduction with ln 2 split as
  *      355/512 + a low part, degree-7 Taylor polynomial by Horner's rule with
  *      fused multiply-adds, two exact power-of-two scalings; 0 below -87,
@@ -425,7 +426,7 @@ int oracle_exp32_array(const float* x, int64_t n, float* y) {
 }
 
 /* SwiGLU then the per-token quantizer (reading R10): h = silu(g) * u with
- * silu(g) = g / (1 + exp32(-g)), every operation one rounded fp32 step, then
+ * silu(g) = g * (1 / (1 + exp32(-g))), every operation one rounded fp32 step, then
  * quantize_row on h. gate, up, h: [rows, cols]. */
 int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, int64_t cols, int8_t* code,
                              float* scale) {
@@ -440,7 +441,8 @@ int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, i
     }
     for (int64_t k = 0; k < cols; ++k) {
       const float g = gate[r * cols + k];
-      const float silu = g / (1.0f + oracle_exp32(-g));
+      const float sig = 1.0f / (1.0f + oracle_exp32(-g));
+      const float silu = g * sig;
       h[k] = silu * up[r * cols + k];
     }
     quantize_row(h, cols, code + r * cols, scale + r);

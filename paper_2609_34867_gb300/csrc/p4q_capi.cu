@@ -222,6 +222,22 @@ p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, ui
   return from_cuda(counted(launch_quant_rows(src, M, Kin, o, reinterpret_cast<cudaStream_t>(stream))));
 }
 
+p4q_status p4q_swiglu_quant_expanded(const uint16_t* gate, int ld_gate, const uint16_t* up, int ld_up, int M, int Kin,
+                                     uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, p4q_stream_t stream) {
+  if (M < 0 || Kin < 16 || ld_gate < Kin || ld_up < Kin || (!Xu) != (!sum_xu)) return P4Q_ERR_INVALID_ARG;
+  if (M > 0 && (!gate || !up || !Xq || !s_a)) return P4Q_ERR_INVALID_ARG;
+  if (Kin % 16 != 0 || Kin > P4Q_MAX_ROW) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (ld_gate % 8 != 0 || ld_up % 8 != 0) return P4Q_ERR_MISALIGNED;
+  if (M > 0 && (!aligned16(gate) || !aligned16(up) || !aligned16(Xq) || !aligned16(s_a) ||
+                (Xu && (!aligned16(Xu) || !aligned16(sum_xu)))))
+    return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_swiglu_quant(gate, ld_gate, up, ld_up, M, Kin, Xq, s_a, Xu, sum_xu,
+                                               reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
                             p4q_stream_t stream) {
   p4q_status st = check_rows(X, M, Kin, Xq, s_a);

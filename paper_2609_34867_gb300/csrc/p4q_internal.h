@@ -92,6 +92,12 @@ void set_gemm_pair_mode(int mode);
 // Expanded-operand path: 0 automatic (M >= 512), 1 never, 2 whenever a workspace is given.
 void set_gemm8_mode(int mode);
 
+// ------------------------------------------------------------ SwiGLU -> quantizer
+// Rows of gate / up (fp16, row pitches ldg / ldu in elements): codes of
+// h = silu(gate) * up per row (packed; expanded + row sums when Xu != null).
+cudaError_t launch_swiglu_quant(const uint16_t* gate, long long ldg, const uint16_t* up, long long ldu, int M, int K,
+                                uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, cudaStream_t stream);
+
 // ------------------------------------------------------------ CLS saliency
 // Shared memory of one (image, crop) CTA: H x (N / C) fp32 weights.
 size_t cls_saliency_smem_bytes(int N, int C, int H);

@@ -49,6 +49,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_set_gemm_variant.restype = st
         L.p4q_cls_saliency.argtypes = [P, P, P, I, I, I, I, I, P, P]
         L.p4q_cls_saliency.restype = st
+        L.p4q_swiglu_quant_expanded.argtypes = [P, I, P, I, I, I, P, P, P, P, P]
+        L.p4q_swiglu_quant_expanded.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
@@ -157,6 +159,23 @@ def p4q_quant_act_expanded(X, Xq, s_a, Xu, sum_xu, stream=None):
     M, K = X.shape
     _check(lib().p4q_quant_act_expanded(_ptr(X), X.stride(0), M, K, _ptr(Xq), _ptr(s_a), _ptr(Xu), _ptr(sum_xu),
                                         _stream(stream)), "p4q_quant_act_expanded")
+
+
+def p4q_swiglu_quant_expanded(gate, up, Xq, s_a, Xu=None, sum_xu=None, stream=None):
+    """Codes of silu(gate) * up per row (gate, up: [M, Kin] fp16 views with unit
+    column stride, e.g. column blocks of a fused gate|up output); Xu / sum_xu
+    optional (both or neither)."""
+    for t, name in ((gate, "gate"), (up, "up")):
+        if not isinstance(t, torch.Tensor) or t.dtype != torch.float16 or t.dim() != 2 or t.stride(1) != 1 or \
+                not t.is_cuda:
+            raise TypeError(f"{name}: expected a CUDA fp16 2-D tensor with unit column stride")
+    _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    if Xu is not None:
+        _need(Xu, torch.uint8, 2, "Xu"); _need(sum_xu, torch.int32, 1, "sum_xu")
+    M, K = gate.shape
+    _check(lib().p4q_swiglu_quant_expanded(_ptr(gate), gate.stride(0), _ptr(up), up.stride(0), M, K, _ptr(Xq),
+                                           _ptr(s_a), _ptr(Xu), _ptr(sum_xu), _stream(stream)),
+           "p4q_swiglu_quant_expanded")
 
 
 def p4q_quant_weight(W, Wq, s_w, stream=None):

@@ -72,6 +72,19 @@ def test_cls_saliency_validates_shapes(lib):
     assert f(P(8), P(16), P(16), 1, 576, 1, 16, 64, P(16), None) == 3   # misaligned
 
 
+def test_swiglu_quant_validates_arguments(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_swiglu_quant_expanded.argtypes = [P, I, P, I, I, I, P, P, P, P, P]
+    f = lib.p4q_swiglu_quant_expanded
+    assert f(P(16), 4096, P(16), 4096, 0, 4096, P(16), P(16), None, None, None) == 0     # empty is a no-op
+    assert f(P(16), 4096, P(16), 4096, 4, 4096, P(16), P(16), P(16), None, None) == 1    # Xu without sum_xu
+    assert f(P(16), 100, P(16), 4096, 4, 4096, P(16), P(16), None, None, None) == 1      # pitch < Kin
+    assert f(P(16), 4096, P(16), 4096, 4, 4100, P(16), P(16), None, None, None) == 1     # pitch < Kin
+    assert f(P(16), 4104, P(16), 4104, 4, 4100, P(16), P(16), None, None, None) == 2     # Kin % 16
+    assert f(P(16), 4100, P(16), 4104, 4, 4096, P(16), P(16), None, None, None) == 3     # pitch % 8
+    assert f(P(8), 4096, P(16), 4096, 4, 4096, P(16), P(16), None, None, None) == 3      # misaligned gate
+
+
 class Params(ctypes.Structure):
     _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
 
