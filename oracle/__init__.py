@@ -72,6 +72,12 @@ def _load():
             lib.oracle_exp32_array.restype = i32
             lib.p4q_swiglu_quantize_rows.argtypes = [P, P, i64, i64, P, P]
             lib.p4q_swiglu_quantize_rows.restype = i32
+            lib.oracle_sumsq32.argtypes = [P, i64]
+            lib.oracle_sumsq32.restype = f32
+            lib.p4q_rmsnorm_rows.argtypes = [P, P, f32, i64, i64, P]
+            lib.p4q_rmsnorm_rows.restype = i32
+            lib.p4q_rmsnorm_quantize_rows.argtypes = [P, P, f32, i64, i64, P, P]
+            lib.p4q_rmsnorm_quantize_rows.restype = i32
             _lib = lib
     return _lib
 
@@ -241,6 +247,40 @@ def swiglu_quantize_rows(gate, up):
     rc = _load().p4q_swiglu_quantize_rows(_ptr(g), _ptr(u), rows, cols, _ptr(codes), _ptr(scale))
     if rc != OK:
         raise ValueError(f"oracle swiglu_quantize_rows failed ({rc})")
+    return codes, scale
+
+
+def sumsq32(x) -> np.float32:
+    """The exact sum of squares of fp16 values, rounded once to fp32."""
+    a = _f32(x).ravel()
+    v = _load().oracle_sumsq32(_ptr(a), a.size)
+    if v < 0:
+        raise ValueError("oracle sumsq32: input is not fp16-valued")
+    return np.float32(v)
+
+
+def rmsnorm_rows(x, w, eps):
+    """RMSNorm of each row of fp16 values x [rows, cols] with gain w [cols]
+    (fp16 values): returns y as float32 [rows, cols] holding fp16 values."""
+    a, g = _f32(x), _f32(w)
+    assert a.ndim == 2 and g.shape == (a.shape[1],)
+    y = np.empty_like(a)
+    rc = _load().p4q_rmsnorm_rows(_ptr(a), _ptr(g), float(eps), a.shape[0], a.shape[1], _ptr(y))
+    if rc != OK:
+        raise ValueError(f"oracle rmsnorm_rows failed ({rc})")
+    return y
+
+
+def rmsnorm_quantize_rows(x, w, eps):
+    """RMSNorm then the per-row 4-bit quantizer: (codes int8 [rows, cols], scale fp32 [rows])."""
+    a, g = _f32(x), _f32(w)
+    assert a.ndim == 2 and g.shape == (a.shape[1],)
+    rows, cols = a.shape
+    codes = np.empty((rows, cols), np.int8)
+    scale = np.empty((rows,), np.float32)
+    rc = _load().p4q_rmsnorm_quantize_rows(_ptr(a), _ptr(g), float(eps), rows, cols, _ptr(codes), _ptr(scale))
+    if rc != OK:
+        raise ValueError(f"oracle rmsnorm_quantize_rows failed ({rc})")
     return codes, scale
 
 

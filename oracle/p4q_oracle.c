@@ -41,7 +41,7 @@
  *      times. Updating m_i with the newest pick equals recomputing the max
  *      over the whole kept set, because max is associative.
  *   R8 output indices are sorted ascending.
- *   R10 SwiGLU before down_proj (the decoder's MLP; the paper quantizes every
+ *   R12 SwiGLU before down_proj (the decoder's MLP; the paper quantizes every
  *      linear's input per token): h = silu(gate) * up, silu(g) =
  *      g * (1 / (1 + exp32(-g))) (four rounded fp32 steps), then h quantized
  *      by R1. exp32 is this file's own
@@ -51,7 +51,14 @@
  *      inf above 88.72284):
  *      every step is one correctly rounded fp32 operation, so the CUDA path
  *      evaluates the same function bit for bit and the codes match exactly.
- *   R9 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
+ *   R13 RMSNorm before the quantized linears (the decoder's input norms feed
+ *      q/k/v/gate/up; the paper quantizes every linear's input per token):
+ *      S = sum x^2 exactly (fp16 squares are multiples of 2^-48; the sum is
+ *      held as a 128-bit integer), rounded once to fp32; ms = S / d;
+ *      r = 1 / sqrt(ms + eps) (r = 0 when ms + eps == 0); t = fp16(x * r);
+ *      y = fp16(t * w) (every step one rounded fp32 or fp16 operation), then
+ *      y quantized by R1.
+ *   R11 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
  *      self-attention, each crop's [CLS] token is the query; its attention
  *      row is the softmax, over the CLS key and the crop's patch keys, of
  *      q . k / sqrt(d_h); A_cls of a patch is that weight averaged over the
@@ -345,7 +352,7 @@ int p4q_gather(const float* V, int B, int N, int d, const int32_t* idx, int K, c
   return ORACLE_OK;
 }
 
-/* CLS-to-patch saliency A_cls (Sec. 3.2, Visual Saliency; reading R9):
+/* CLS-to-patch saliency A_cls (Sec. 3.2, Visual Saliency; reading R11):
  *   q_cls, k_cls: [B, C, H, dh] (the final layer's CLS query and key of each
  *   crop, per head); k: [B, N, H, dh] (patch keys; crop c holds tokens
  *   [c * N / C, (c + 1) * N / C)); out A: [B, N]. For each image b, crop c,
@@ -395,7 +402,7 @@ static float pow2f(int k) {
   return f;
 }
 
-/* Own fp32 exponential (reading R10): n = rint(x * log2 e); r = x - n ln2 in
+/* Own fp32 exponential (reading R12): n = rint(x * log2 e); r = x - n ln2 in
  * two fused steps (ln2 = 355/512 + LN2_LO; n * 355/512 is exact for the n
  * that occur); e^r by the degree-7 Taylor polynomial (|r| <= ln2 / 2: the
  * truncation is below 2e-8 relative); times 2^n as two exact multiplications
@@ -425,7 +432,7 @@ int oracle_exp32_array(const float* x, int64_t n, float* y) {
   return ORACLE_OK;
 }
 
-/* SwiGLU then the per-token quantizer (reading R10): h = silu(g) * u with
+/* SwiGLU then the per-token quantizer (reading R12): h = silu(g) * u with
  * silu(g) = g * (1 / (1 + exp32(-g))), every operation one rounded fp32 step, then
  * quantize_row on h. gate, up, h: [rows, cols]. */
 int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, int64_t cols, int8_t* code,
@@ -447,6 +454,86 @@ int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, i
     }
     quantize_row(h, cols, code + r * cols, scale + r);
     free(h);
+  }
+  return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* RMSNorm then the per-token quantizer (reading R13).                   */
+/* ------------------------------------------------------------------ */
+
+/* fl32 of the exact sum of squares of fp16 values: |x| = k * 2^-24 with an
+ * integer k < 2^40, so the sum is an integer count of 2^-48 held in 128 bits,
+ * rounded once to 24 significant bits (to nearest, ties to even). Writes
+ * ORACLE_BAD_ARG to *rc when some x is not an fp16 value. */
+static float sumsq32(const float* x, int64_t n, int* rc) {
+  unsigned __int128 S = 0;
+  for (int64_t i = 0; i < n; ++i) {
+    const double k = fabs((double)x[i]) * 16777216.0;
+    if (!(k < 1099511627776.0) || k != floor(k)) {
+      *rc = ORACLE_BAD_ARG;
+      return 0.0f;
+    }
+    const uint64_t ki = (uint64_t)k;
+    S += (unsigned __int128)ki * ki;
+  }
+  int L = 0;
+  for (unsigned __int128 t = S; t != 0; t >>= 1) ++L;
+  if (L <= 24) return ldexpf((float)(uint64_t)S, -48);
+  const int sh = L - 24;
+  uint64_t q = (uint64_t)(S >> sh);
+  const unsigned __int128 rem = S - ((unsigned __int128)q << sh);
+  const unsigned __int128 half = (unsigned __int128)1 << (sh - 1);
+  if (rem > half || (rem == half && (q & 1u))) ++q;
+  return ldexpf((float)q, sh - 48);
+}
+
+float oracle_sumsq32(const float* x, int64_t n) {
+  int rc = ORACLE_OK;
+  const float s = sumsq32(x, n, &rc);
+  return rc == ORACLE_OK ? s : -1.0f;
+}
+
+static int rmsnorm_row(const float* x, const float* w, float eps, int64_t cols, float* y) {
+  int rc = ORACLE_OK;
+  const float S = sumsq32(x, cols, &rc);
+  if (rc != ORACLE_OK) return rc;
+  const float ms = S / (float)cols;
+  const float den = ms + eps;
+  const float r = den == 0.0f ? 0.0f : 1.0f / sqrtf(den);
+  for (int64_t k = 0; k < cols; ++k) {
+    const float t = (float)(_Float16)(x[k] * r);
+    y[k] = (float)(_Float16)(t * w[k]);
+  }
+  return ORACLE_OK;
+}
+
+/* The normalized rows y (fp16 values, returned as fp32). x: [rows, cols] fp16
+ * values, w: [cols] fp16 values (the norm's gain), eps >= 0. */
+int p4q_rmsnorm_rows(const float* x, const float* w, float eps, int64_t rows, int64_t cols, float* y) {
+  if (!x || !w || !y || rows < 0 || cols <= 0 || !(eps >= 0.0f)) return ORACLE_BAD_ARG;
+  int rc = ORACLE_OK;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r)
+    if (rmsnorm_row(x + r * cols, w, eps, cols, y + r * cols) != ORACLE_OK) rc = ORACLE_BAD_ARG;
+  return rc;
+}
+
+/* RMSNorm then quantize_row on y: codes [rows, cols], scale [rows]. */
+int p4q_rmsnorm_quantize_rows(const float* x, const float* w, float eps, int64_t rows, int64_t cols, int8_t* code,
+                              float* scale) {
+  if (!x || !w || !code || !scale || rows < 0 || cols <= 0 || !(eps >= 0.0f)) return ORACLE_BAD_ARG;
+  int rc = ORACLE_OK;
+#pragma omp parallel for schedule(static)
+  for (int64_t r = 0; r < rows; ++r) {
+    float* y = (float*)malloc(sizeof(float) * (size_t)cols);
+    if (!y || rmsnorm_row(x + r * cols, w, eps, cols, y) != ORACLE_OK) {
+      rc = ORACLE_BAD_ARG;
+      free(y);
+      continue;
+    }
+    quantize_row(y, cols, code + r * cols, scale + r);
+    free(y);
   }
   return rc;
 }
