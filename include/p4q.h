@@ -162,6 +162,27 @@ p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, ui
 p4q_status p4q_swiglu_quant_expanded(const uint16_t* gate, int ld_gate, const uint16_t* up, int ld_up, int M, int Kin,
                                      uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, p4q_stream_t stream);
 
+/* RMSNorm before the quantized linears fused with the per-token quantizer of
+ * its output (App. A quantizes every linear's input per token; the decoder's
+ * input norms feed q/k/v/gate/up). For each row m of X (d = Kin values):
+ *   S = sum_k x_k^2 computed exactly (fp16 squares are integer multiples of
+ *       2^-48; the sum is held in 128 bits), rounded once to fp32 (to
+ *       nearest, ties to even);
+ *   ms = S / d; r = 1 / sqrt(ms + eps), r = 0 when ms + eps == 0;
+ *   t_k = fp16(x_k * r); y_k = fp16(t_k * w_k) (each step one correctly
+ *   rounded operation);
+ *   then the codes and scale of y as p4q_quant_act.
+ *   X [M, Kin] fp16, rows ldx elements apart (device, read); finite values
+ *   w [Kin] fp16 gain (device, read); y must stay finite
+ *   eps >= 0
+ *   Xq [M, Kin/2], s_a [M]           written
+ *   Xu [M, Kin], sum_xu [M]          the expanded codes (p4q_expand_codes
+ *                                    form) or both NULL
+ * Requires M >= 0, 16 <= Kin <= P4Q_MAX_ROW, Kin % 16 == 0, ldx >= Kin,
+ * ldx % 8 == 0, 16-byte aligned pointers. M == 0 is a no-op. */
+p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t* w, float eps, int M, int Kin,
+                                      uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, p4q_stream_t stream);
+
 /* Per-output-channel weight quantization (App. B.3: symmetric, per output
  * channel, then round-to-nearest): the same per-row quantizer applied to each
  * output row of W.

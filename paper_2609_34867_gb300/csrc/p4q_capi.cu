@@ -238,6 +238,23 @@ p4q_status p4q_swiglu_quant_expanded(const uint16_t* gate, int ld_gate, const ui
                                                reinterpret_cast<cudaStream_t>(stream))));
 }
 
+p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t* w, float eps, int M, int Kin,
+                                      uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, p4q_stream_t stream) {
+  if (M < 0 || Kin < 16 || ldx < Kin || (!Xu) != (!sum_xu) || !(eps >= 0.0f) || !(eps < INFINITY))
+    return P4Q_ERR_INVALID_ARG;
+  if (M > 0 && (!X || !w || !Xq || !s_a)) return P4Q_ERR_INVALID_ARG;
+  if (Kin % 16 != 0 || Kin > P4Q_MAX_ROW) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (ldx % 8 != 0) return P4Q_ERR_MISALIGNED;
+  if (M > 0 && (!aligned16(X) || !aligned16(w) || !aligned16(Xq) || !aligned16(s_a) ||
+                (Xu && (!aligned16(Xu) || !aligned16(sum_xu)))))
+    return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_rmsnorm_quant(X, ldx, w, eps, M, Kin, Xq, s_a, Xu, sum_xu,
+                                                reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
                             p4q_stream_t stream) {
   p4q_status st = check_rows(X, M, Kin, Xq, s_a);

@@ -34,6 +34,19 @@ __device__ __forceinline__ unsigned long long globaltimer() {
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// ---------------------------------------------------------------- 4-bit code of one value
+// clamp(round_half_even(fl32(h / s)), -8, 7) for a row scale s = fl32(a / 7),
+// |h| <= a, inv = fl32(1 / s): h * inv rounded by the magic constant, recomputed
+// with the correctly rounded quotient near a .5 boundary (the two quotients
+// differ by less than 2^-19 there).
+__device__ __forceinline__ int q4_code(float h, float s, float inv) {
+  const float q = __fmul_rn(h, inv);
+  const float c = __fsub_rn(__fadd_rn(q, 12582912.0f), 12582912.0f);
+  float r = c;
+  if (fabsf(__fsub_rn(q, c)) > 0.5f - 0x1p-17f) r = rintf(__fdiv_rn(h, s));
+  return max(-8, min(7, static_cast<int>(r)));
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

@@ -98,6 +98,12 @@ void set_gemm8_mode(int mode);
 cudaError_t launch_swiglu_quant(const uint16_t* gate, long long ldg, const uint16_t* up, long long ldu, int M, int K,
                                 uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, cudaStream_t stream);
 
+// ------------------------------------------------------------ RMSNorm -> quantizer
+// Rows of X (fp16, row pitch ldx elements), gain w [K] fp16: codes of the
+// RMSNorm of each row (packed; expanded + row sums when Xu != null).
+cudaError_t launch_rmsnorm_quant(const uint16_t* X, long long ldx, const uint16_t* w, float eps, int M, int K,
+                                 uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, cudaStream_t stream);
+
 // ------------------------------------------------------------ CLS saliency
 // Shared memory of one (image, crop) CTA: H x (N / C) fp32 weights.
 size_t cls_saliency_smem_bytes(int N, int C, int H);

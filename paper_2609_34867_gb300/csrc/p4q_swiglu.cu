@@ -54,17 +54,6 @@ __device__ __forceinline__ float swiglu(float g, float u) {
   return __fmul_rn(__fmul_rn(g, sig), u);
 }
 
-// round_half_even(h / s) for |h| <= 7 s: h * inv rounded by the magic constant,
-// recomputed with the exact quotient near a .5 boundary (the two quotients
-// differ by less than 2^-19 there).
-__device__ __forceinline__ int code_of(float h, float s, float inv) {
-  const float q = __fmul_rn(h, inv);
-  const float c = __fsub_rn(__fadd_rn(q, 12582912.0f), 12582912.0f);
-  float r = c;
-  if (fabsf(__fsub_rn(q, c)) > 0.5f - 0x1p-17f) r = rintf(__fdiv_rn(h, s));
-  return max(-8, min(7, static_cast<int>(r)));
-}
-
 template <int MAXC, bool EXPANDED>
 __global__ void __launch_bounds__(kSwThreads)
     swiglu_quant_kernel(const __half* __restrict__ gate, long long ldg, const __half* __restrict__ up, long long ldu,
@@ -122,7 +111,7 @@ __global__ void __launch_bounds__(kSwThreads)
       uint32_t pw = 0;
       if (a != 0.0f) {
 #pragma unroll
-        for (int e = 0; e < 8; ++e) pw |= (static_cast<uint32_t>(code_of(h[j][e], s, inv)) & 0xFu) << (4 * e);
+        for (int e = 0; e < 8; ++e) pw |= (static_cast<uint32_t>(q4_code(h[j][e], s, inv)) & 0xFu) << (4 * e);
       }
       q4[c] = pw;
       if (EXPANDED) {

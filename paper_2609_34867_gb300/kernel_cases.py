@@ -7,6 +7,7 @@
   python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases saliency B N [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases swiglu M K LD [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases rmsnorm M K [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -27,6 +28,8 @@ selects the first replayed launch.
   select  p4q_select_gather_quant on one of the LLaVA-shaped workloads;
   swiglu  p4q_swiglu_quant_expanded on gate / up, the last 2 K columns of an
           M x LD fp16 matrix (bytes: 4 M K in, 3 M K / 2 + 8 M out);
+  rmsnorm p4q_rmsnorm_quant_expanded on M x K fp16 rows with a K-value gain
+          (bytes: 2 M K + 2 K in, 3 M K / 2 + 8 M out);
   saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
           heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
           fp16 keys and queries in, 4 B N out).
@@ -72,7 +75,7 @@ def _timed(fn, reps, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -126,6 +129,18 @@ def main(argv=None):
         ms = _timed(lambda: p4q.p4q_swiglu_quant_expanded(G, U, Xq, s, Xu, su), a.reps, dev)
         nbytes = 4 * M * K + 3 * M * K // 2 + 8 * M
         print(f"swiglu {M}x{K} of {LD}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "rmsnorm":
+        M, K = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        X = (torch.randn((M, K), generator=g, device=dev) * 2.0).to(torch.float16)
+        w = (1.0 + 0.2 * torch.randn((K,), generator=g, device=dev)).to(torch.float16)
+        Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+        s = torch.empty((M,), dtype=torch.float32, device=dev)
+        Xu = torch.empty((M, K), dtype=torch.uint8, device=dev)
+        su = torch.empty((M,), dtype=torch.int32, device=dev)
+        ms = _timed(lambda: p4q.p4q_rmsnorm_quant_expanded(X, w, 1e-6, Xq, s, Xu, su), a.reps, dev)
+        nbytes = 2 * M * K + 2 * K + 3 * M * K // 2 + 8 * M
+        print(f"rmsnorm {M}x{K}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
     elif a.case == "saliency":
         B, N = (int(x) for x in a.args)
         v = wl.vision_attention(B, N, seed=0)

@@ -51,6 +51,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_cls_saliency.restype = st
         L.p4q_swiglu_quant_expanded.argtypes = [P, I, P, I, I, I, P, P, P, P, P]
         L.p4q_swiglu_quant_expanded.restype = st
+        L.p4q_rmsnorm_quant_expanded.argtypes = [P, I, P, ctypes.c_float, I, I, P, P, P, P, P]
+        L.p4q_rmsnorm_quant_expanded.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
@@ -176,6 +178,24 @@ def p4q_swiglu_quant_expanded(gate, up, Xq, s_a, Xu=None, sum_xu=None, stream=No
     _check(lib().p4q_swiglu_quant_expanded(_ptr(gate), gate.stride(0), _ptr(up), up.stride(0), M, K, _ptr(Xq),
                                            _ptr(s_a), _ptr(Xu), _ptr(sum_xu), _stream(stream)),
            "p4q_swiglu_quant_expanded")
+
+
+def p4q_rmsnorm_quant_expanded(X, w, eps, Xq, s_a, Xu=None, sum_xu=None, stream=None):
+    """Codes of the RMSNorm of each row of X ([M, Kin] fp16 view with unit
+    column stride) with gain w ([Kin] fp16) and epsilon eps; Xu / sum_xu
+    optional (both or neither)."""
+    if not isinstance(X, torch.Tensor) or X.dtype != torch.float16 or X.dim() != 2 or X.stride(1) != 1 or \
+            not X.is_cuda:
+        raise TypeError("X: expected a CUDA fp16 2-D tensor with unit column stride")
+    _need(w, torch.float16, 1, "w"); _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    if Xu is not None:
+        _need(Xu, torch.uint8, 2, "Xu"); _need(sum_xu, torch.int32, 1, "sum_xu")
+    M, K = X.shape
+    if w.shape[0] != K:
+        raise ValueError(f"w has {w.shape[0]} values, X rows have {K}")
+    _check(lib().p4q_rmsnorm_quant_expanded(_ptr(X), X.stride(0), _ptr(w), float(eps), M, K, _ptr(Xq), _ptr(s_a),
+                                            _ptr(Xu), _ptr(sum_xu), _stream(stream)),
+           "p4q_rmsnorm_quant_expanded")
 
 
 def p4q_quant_weight(W, Wq, s_w, stream=None):

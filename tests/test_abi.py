@@ -85,6 +85,22 @@ def test_swiglu_quant_validates_arguments(lib):
     assert f(P(8), 4096, P(16), 4096, 4, 4096, P(16), P(16), None, None, None) == 3      # misaligned gate
 
 
+def test_rmsnorm_quant_validates_arguments(lib):
+    P, I, F = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    lib.p4q_rmsnorm_quant_expanded.argtypes = [P, I, P, F, I, I, P, P, P, P, P]
+    f = lib.p4q_rmsnorm_quant_expanded
+    assert f(P(16), 4096, P(16), 1e-6, 0, 4096, P(16), P(16), None, None, None) == 0     # empty is a no-op
+    assert f(P(16), 4096, P(16), 1e-6, 4, 4096, P(16), P(16), P(16), None, None) == 1    # Xu without sum_xu
+    assert f(P(16), 4096, P(16), -1.0, 4, 4096, P(16), P(16), None, None, None) == 1     # eps < 0
+    assert f(P(16), 4096, P(16), float("nan"), 4, 4096, P(16), P(16), None, None, None) == 1
+    assert f(P(16), 4096, P(16), float("inf"), 4, 4096, P(16), P(16), None, None, None) == 1
+    assert f(P(16), 4096, None, 1e-6, 4, 4096, P(16), P(16), None, None, None) == 1      # no gain
+    assert f(P(16), 100, P(16), 1e-6, 4, 4096, P(16), P(16), None, None, None) == 1      # pitch < Kin
+    assert f(P(16), 4104, P(16), 1e-6, 4, 4100, P(16), P(16), None, None, None) == 2     # Kin % 16
+    assert f(P(16), 4100, P(16), 1e-6, 4, 4096, P(16), P(16), None, None, None) == 3     # pitch % 8
+    assert f(P(16), 4096, P(8), 1e-6, 4, 4096, P(16), P(16), None, None, None) == 3      # misaligned gain
+
+
 class Params(ctypes.Structure):
     _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
 
