@@ -36,15 +36,16 @@ __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepc
 
 // ---------------------------------------------------------------- 4-bit code of one value
 // clamp(round_half_even(fl32(h / s)), -8, 7) for a row scale s = fl32(a / 7),
-// |h| <= a, inv = fl32(1 / s): h * inv rounded by the magic constant, recomputed
-// with the correctly rounded quotient near a .5 boundary (the two quotients
-// differ by less than 2^-19 there).
+// |h| <= a, inv = fl32(1 / s): h * inv rounded to an integer by adding
+// 1.5 * 2^23 (whose bits then hold the integer in the low mantissa bits),
+// recomputed with the correctly rounded quotient near a .5 boundary (the two
+// quotients differ by less than 2^-19 there).
 __device__ __forceinline__ int q4_code(float h, float s, float inv) {
   const float q = __fmul_rn(h, inv);
-  const float c = __fsub_rn(__fadd_rn(q, 12582912.0f), 12582912.0f);
-  float r = c;
-  if (fabsf(__fsub_rn(q, c)) > 0.5f - 0x1p-17f) r = rintf(__fdiv_rn(h, s));
-  return max(-8, min(7, static_cast<int>(r)));
+  const float qm = __fadd_rn(q, 12582912.0f);
+  int r = __float_as_int(qm) - 0x4B400000;
+  if (fabsf(__fsub_rn(q, __fsub_rn(qm, 12582912.0f))) > 0.5f - 0x1p-17f) r = __float2int_rn(__fdiv_rn(h, s));
+  return max(-8, min(7, r));
 }
 
 // ---------------------------------------------------------------- mbarrier

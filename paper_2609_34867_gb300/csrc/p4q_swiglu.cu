@@ -30,7 +30,11 @@ __device__ __forceinline__ float pow2f(int k) { return __int_as_float((k + 127) 
 __device__ __forceinline__ float exp32(float x) {
   if (x > 0x1.62e430p+6f) return __int_as_float(0x7f800000);
   if (x < -87.0f) return 0.0f;
-  const float n = rintf(__fmul_rn(x, 0x1.715476p+0f));
+  // n = round_half_even(x * log2 e) by adding 1.5 * 2^23 (|n| <= 128); its
+  // bits hold n in the low mantissa bits
+  const float nm = __fadd_rn(__fmul_rn(x, 0x1.715476p+0f), 12582912.0f);
+  const float n = __fsub_rn(nm, 12582912.0f);
+  const int k = __float_as_int(nm) - 0x4B400000;
   float r = __fmaf_rn(-n, 0x1.630000p-1f, x);
   r = __fmaf_rn(-n, -0x1.bd0106p-13f, r);
   float p = 0x1.a01a02p-13f;
@@ -43,7 +47,6 @@ __device__ __forceinline__ float exp32(float x) {
   p = __fmaf_rn(p, r, 1.0f);
   // p * 2^n is exact (a normal result): one multiplication, two when 2^n
   // itself overflows (n = 128)
-  const int k = static_cast<int>(n);
   if (k <= 127) return __fmul_rn(p, pow2f(k));
   return __fmul_rn(__fmul_rn(p, pow2f(64)), pow2f(k - 64));
 }
