@@ -72,6 +72,8 @@ def _load():
             lib.oracle_exp32_array.restype = i32
             lib.p4q_swiglu_quantize_rows.argtypes = [P, P, i64, i64, P, P]
             lib.p4q_swiglu_quantize_rows.restype = i32
+            lib.p4q_causal_attention.argtypes = [P, P, P, i32, i32, i32, i32, i32, P]
+            lib.p4q_causal_attention.restype = i32
             lib.oracle_sumsq32.argtypes = [P, i64]
             lib.oracle_sumsq32.restype = f32
             lib.p4q_rmsnorm_rows.argtypes = [P, P, f32, i64, i64, P]
@@ -282,6 +284,18 @@ def rmsnorm_quantize_rows(x, w, eps):
     if rc != OK:
         raise ValueError(f"oracle rmsnorm_quantize_rows failed ({rc})")
     return codes, scale
+
+
+def causal_attention(q, k, v, B, m, H, Hkv, dh):
+    """Causal softmax attention per sample and head (fp64): q [B*m, H*dh],
+    k, v [B*m, Hkv*dh] (fp16 values); returns o float64 [B*m, H*dh]."""
+    q, k, v = _f32(q), _f32(k), _f32(v)
+    assert q.shape == (B * m, H * dh) and k.shape == (B * m, Hkv * dh) and v.shape == k.shape
+    o = np.empty((B * m, H * dh), np.float64)
+    rc = _load().p4q_causal_attention(_ptr(q), _ptr(k), _ptr(v), B, m, H, Hkv, dh, _ptr(o))
+    if rc != OK:
+        raise ValueError(f"oracle causal_attention failed ({rc})")
+    return o
 
 
 def pack_codes(codes):

@@ -58,6 +58,12 @@
  *      r = 1 / sqrt(ms + eps) (r = 0 when ms + eps == 0); t = fp16(x * r);
  *      y = fp16(t * w) (every step one rounded fp32 or fp16 operation), then
  *      y quantized by R1.
+ *   R14 attention on the pruned sequence (App. B: the key and value caches
+ *      stay in FP16 while the linears run in W4A4): causal softmax attention
+ *      of each of the m positions of a sample over positions 0..i, logits
+ *      q . k / sqrt(d_h), heads sharing key/value heads in groups of H / H_kv
+ *      (H_kv = H: one key/value head per head). Position encodings are
+ *      applied by the caller. fp64 throughout.
  *   R11 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
  *      self-attention, each crop's [CLS] token is the query; its attention
  *      row is the softmax, over the CLS key and the crop's patch keys, of
@@ -534,6 +540,58 @@ int p4q_rmsnorm_quantize_rows(const float* x, const float* w, float eps, int64_t
     }
     quantize_row(y, cols, code + r * cols, scale + r);
     free(y);
+  }
+  return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* Causal attention on the pruned sequence (reading R14).                 */
+/* ------------------------------------------------------------------ */
+
+/* q [B*m, H*dh], k and v [B*m, Hkv*dh] (rows of consecutive positions of one
+ * sample, head h in columns h*dh .. h*dh + dh - 1), o [B*m, H*dh]:
+ *   o_i = sum_{j <= i} p_ij v_j, p_i. = softmax_j(q_i . k_j / sqrt(dh)),
+ * with key/value head h / (H / Hkv) for head h. fp64. */
+int p4q_causal_attention(const float* q, const float* k, const float* v, int B, int m, int H, int Hkv, int dh,
+                         double* o) {
+  if (!q || !k || !v || !o || B < 0 || m < 1 || H < 1 || Hkv < 1 || H % Hkv != 0 || dh < 1) return ORACLE_BAD_ARG;
+  const double inv_sqrt = 1.0 / sqrt((double)dh);
+  const int64_t ldq = (int64_t)H * dh, ldk = (int64_t)Hkv * dh;
+  int rc = ORACLE_OK;
+#pragma omp parallel for collapse(2) schedule(static)
+  for (int b = 0; b < B; ++b) {
+    for (int h = 0; h < H; ++h) {
+      const int hk = h / (H / Hkv);
+      double* l = (double*)malloc(sizeof(double) * (size_t)m);
+      if (!l) {
+        rc = ORACLE_BAD_ARG;
+        continue;
+      }
+      for (int i = 0; i < m; ++i) {
+        const float* qi = q + ((int64_t)b * m + i) * ldq + (int64_t)h * dh;
+        double mx = -INFINITY;
+        for (int j = 0; j <= i; ++j) {
+          const float* kj = k + ((int64_t)b * m + j) * ldk + (int64_t)hk * dh;
+          double dot = 0.0;
+          for (int e = 0; e < dh; ++e) dot += (double)qi[e] * (double)kj[e];
+          l[j] = dot * inv_sqrt;
+          if (l[j] > mx) mx = l[j];
+        }
+        double z = 0.0;
+        for (int j = 0; j <= i; ++j) {
+          l[j] = exp(l[j] - mx);
+          z += l[j];
+        }
+        double* oi = o + ((int64_t)b * m + i) * ldq + (int64_t)h * dh;
+        for (int e = 0; e < dh; ++e) oi[e] = 0.0;
+        for (int j = 0; j <= i; ++j) {
+          const float* vj = v + ((int64_t)b * m + j) * ldk + (int64_t)hk * dh;
+          const double p = l[j] / z;
+          for (int e = 0; e < dh; ++e) oi[e] += p * (double)vj[e];
+        }
+      }
+      free(l);
+    }
   }
   return rc;
 }
