@@ -187,7 +187,8 @@ p4q_status p4q_set_gemm_variant(int variant) {
 
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
-  const unsigned int g = gemm_read_and_clear_error() | gemm8_read_and_clear_error() | quant_read_and_clear_error();
+  const unsigned int g = gemm_read_and_clear_error() | gemm8_read_and_clear_error() | quant_read_and_clear_error() |
+                         attn_read_and_clear_error();
   if (cudaGetLastError() != cudaSuccess) return P4Q_ERR_CUDA;
   return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
 }
@@ -253,6 +254,22 @@ p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t
   if (st != P4Q_OK) return st;
   return from_cuda(counted(launch_rmsnorm_quant(X, ldx, w, eps, M, Kin, Xq, s_a, Xu, sum_xu,
                                                 reinterpret_cast<cudaStream_t>(stream))));
+}
+
+p4q_status p4q_causal_attention(const uint16_t* q, int ldq, const uint16_t* k, int ldk, const uint16_t* v, int ldv,
+                                int B, int m, int H, int Hkv, int dh, uint16_t* o, int ldo, p4q_stream_t stream) {
+  if (B < 0 || m < 1 || H < 1 || Hkv < 1 || H % Hkv != 0) return P4Q_ERR_INVALID_ARG;
+  if (ldq < H * dh || ldk < Hkv * dh || ldv < Hkv * dh || ldo < H * dh) return P4Q_ERR_INVALID_ARG;
+  if (B > 0 && (!q || !k || !v || !o)) return P4Q_ERR_INVALID_ARG;
+  if (dh != 128 || m > kAttnMaxLen || B > 65535 || H > 65535 || static_cast<long long>(B) * m > (1ll << 31) - 1)
+    return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (ldq % 8 != 0 || ldk % 8 != 0 || ldv % 8 != 0 || ldo % 8 != 0) return P4Q_ERR_MISALIGNED;
+  if (B > 0 && (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o))) return P4Q_ERR_MISALIGNED;
+  if (B == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_causal_attention(q, ldq, k, ldk, v, ldv, B, m, H, Hkv, o, ldo,
+                                                   reinterpret_cast<cudaStream_t>(stream))));
 }
 
 p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,

@@ -104,6 +104,17 @@ cudaError_t launch_swiglu_quant(const uint16_t* gate, long long ldg, const uint1
 cudaError_t launch_rmsnorm_quant(const uint16_t* X, long long ldx, const uint16_t* w, float eps, int M, int K,
                                  uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, cudaStream_t stream);
 
+// ------------------------------------------------------------ causal attention (FP16 K/V)
+// Longest sample the kernel takes (keys of one sample in shared memory and TMEM).
+constexpr int kAttnMaxLen = 384;
+// Dynamic shared memory of one CTA for samples of m positions.
+size_t causal_attention_smem_bytes(int m);
+// q [B*m, ldq], k / v [B*m, ldk / ldv], o [B*m, ldo] fp16 rows; head dim 128.
+cudaError_t launch_causal_attention(const uint16_t* q, long long ldq, const uint16_t* k, long long ldk,
+                                    const uint16_t* v, long long ldv, int B, int m, int H, int Hkv, uint16_t* o,
+                                    long long ldo, cudaStream_t stream);
+unsigned int attn_read_and_clear_error();
+
 // ------------------------------------------------------------ CLS saliency
 // Shared memory of one (image, crop) CTA: H x (N / C) fp32 weights.
 size_t cls_saliency_smem_bytes(int N, int C, int H);

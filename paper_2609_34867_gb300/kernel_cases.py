@@ -8,6 +8,7 @@
   python -m paper_2609_34867_gb300.kernel_cases saliency B N [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases swiglu M K LD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases rmsnorm M K [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases attn B M H [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -30,6 +31,9 @@ selects the first replayed launch.
           M x LD fp16 matrix (bytes: 4 M K in, 3 M K / 2 + 8 M out);
   rmsnorm p4q_rmsnorm_quant_expanded on M x K fp16 rows with a K-value gain
           (bytes: 2 M K + 2 K in, 3 M K / 2 + 8 M out);
+  attn    p4q_causal_attention on B samples of M positions, H heads of 128
+          (flops: 2 x 2 x 128 x M (M + 1) / 2 per sample and head, the
+          causal Q K^T and P V; bytes: q, k, v in, o out, fp16);
   saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
           heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
           fp16 keys and queries in, 4 B N out).
@@ -75,7 +79,7 @@ def _timed(fn, reps, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -141,6 +145,17 @@ def main(argv=None):
         ms = _timed(lambda: p4q.p4q_rmsnorm_quant_expanded(X, w, 1e-6, Xq, s, Xu, su), a.reps, dev)
         nbytes = 2 * M * K + 2 * K + 3 * M * K // 2 + 8 * M
         print(f"rmsnorm {M}x{K}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "attn":
+        B, M, H = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        qkv = torch.randn((B * M, 3 * H * 128), generator=g, device=dev).to(torch.float16)
+        Q, K, V = qkv[:, :H * 128], qkv[:, H * 128:2 * H * 128], qkv[:, 2 * H * 128:]
+        O = torch.empty((B * M, H * 128), dtype=torch.float16, device=dev)
+        ms = _timed(lambda: p4q.p4q_causal_attention(Q, K, V, O, B, M, H, H), a.reps, dev)
+        flops = 2 * 2 * 128 * M * (M + 1) / 2 * B * H
+        nbytes = 4 * B * M * H * 128 * 2
+        print(f"attn {B}x{M} H={H}: {ms * 1e3:.1f} us/call, {flops / ms / 1e9:.1f} TFLOP/s, "
+              f"{nbytes / ms / 1e6:.1f} GB/s")
     elif a.case == "saliency":
         B, N = (int(x) for x in a.args)
         v = wl.vision_attention(B, N, seed=0)

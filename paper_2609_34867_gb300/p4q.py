@@ -53,6 +53,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_swiglu_quant_expanded.restype = st
         L.p4q_rmsnorm_quant_expanded.argtypes = [P, I, P, ctypes.c_float, I, I, P, P, P, P, P]
         L.p4q_rmsnorm_quant_expanded.restype = st
+        L.p4q_causal_attention.argtypes = [P, I, P, I, P, I, I, I, I, I, I, P, I, P]
+        L.p4q_causal_attention.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
@@ -196,6 +198,18 @@ def p4q_rmsnorm_quant_expanded(X, w, eps, Xq, s_a, Xu=None, sum_xu=None, stream=
     _check(lib().p4q_rmsnorm_quant_expanded(_ptr(X), X.stride(0), _ptr(w), float(eps), M, K, _ptr(Xq), _ptr(s_a),
                                             _ptr(Xu), _ptr(sum_xu), _stream(stream)),
            "p4q_rmsnorm_quant_expanded")
+
+
+def p4q_causal_attention(q, k, v, o, B, m, H, Hkv, stream=None):
+    """Causal attention per sample and head on fp16 rows (head dim 128): q, o
+    [B*m, >= H*128], k, v [B*m, >= Hkv*128], 2-D views with unit column stride
+    (e.g. column blocks of a fused projection output)."""
+    for t, name in ((q, "q"), (k, "k"), (v, "v"), (o, "o")):
+        if not isinstance(t, torch.Tensor) or t.dtype != torch.float16 or t.dim() != 2 or t.stride(1) != 1 or \
+                not t.is_cuda or t.shape[0] != B * m:
+            raise TypeError(f"{name}: expected a CUDA fp16 2-D tensor of B*m rows with unit column stride")
+    _check(lib().p4q_causal_attention(_ptr(q), q.stride(0), _ptr(k), k.stride(0), _ptr(v), v.stride(0), B, m, H,
+                                      Hkv, 128, _ptr(o), o.stride(0), _stream(stream)), "p4q_causal_attention")
 
 
 def p4q_quant_weight(W, Wq, s_w, stream=None):

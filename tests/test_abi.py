@@ -101,6 +101,22 @@ def test_rmsnorm_quant_validates_arguments(lib):
     assert f(P(16), 4096, P(8), 1e-6, 4, 4096, P(16), P(16), None, None, None) == 3      # misaligned gain
 
 
+def test_causal_attention_validates_arguments(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_causal_attention.argtypes = [P, I, P, I, P, I, I, I, I, I, I, P, I, P]
+    f = lib.p4q_causal_attention
+    ok = (P(16), 4096, P(16), 4096, P(16), 4096)
+    assert f(*ok, 0, 256, 32, 32, 128, P(16), 4096, None) == 0        # empty is a no-op
+    assert f(*ok, 2, 0, 32, 32, 128, P(16), 4096, None) == 1          # m < 1
+    assert f(*ok, 2, 256, 32, 5, 128, P(16), 4096, None) == 1         # H % Hkv
+    assert f(*ok, 2, 256, 32, 32, 128, P(16), 2048, None) == 1        # ldo < H dh
+    assert f(*ok, 2, 256, 32, 32, 128, None, 4096, None) == 1         # no output
+    assert f(*ok, 2, 256, 32, 32, 64, P(16), 4096, None) == 2         # dh != 128
+    assert f(*ok, 2, 385, 32, 32, 128, P(16), 4096, None) == 2        # m > 384
+    assert f(P(16), 4100, P(16), 4096, P(16), 4096, 2, 256, 32, 32, 128, P(16), 4096, None) == 3  # pitch % 8
+    assert f(P(8), 4096, P(16), 4096, P(16), 4096, 2, 256, 32, 32, 128, P(16), 4096, None) == 3   # misaligned
+
+
 class Params(ctypes.Structure):
     _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
 
