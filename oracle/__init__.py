@@ -74,6 +74,10 @@ def _load():
             lib.p4q_swiglu_quantize_rows.restype = i32
             lib.p4q_causal_attention.argtypes = [P, P, P, i32, i32, i32, i32, i32, P]
             lib.p4q_causal_attention.restype = i32
+            lib.p4q_block_mse.argtypes = [P, P, P, i32, i32, P, P]
+            lib.p4q_block_mse.restype = i32
+            lib.p4q_topk_replacement.argtypes = [P, P, i32, i32, i32, P, P]
+            lib.p4q_topk_replacement.restype = i32
             lib.oracle_sumsq32.argtypes = [P, i64]
             lib.oracle_sumsq32.restype = f32
             lib.p4q_rmsnorm_rows.argtypes = [P, P, f32, i64, i64, P]
@@ -296,6 +300,35 @@ def causal_attention(q, k, v, B, m, H, Hkv, dh):
     if rc != OK:
         raise ValueError(f"oracle causal_attention failed ({rc})")
     return o
+
+
+def block_mse(Yq, Yf, offsets):
+    """Eq. 5's block objective: per-sample ||Yq - Yf||_F^2 / (m_n d) over rows
+    offsets[n] .. offsets[n+1]-1, and their mean. Returns (e float64 [B], L)."""
+    a, f = _f32(Yq), _f32(Yf)
+    off = np.ascontiguousarray(offsets, np.int32)
+    assert a.ndim == 2 and a.shape == f.shape and off[-1] == a.shape[0]
+    B = off.size - 1
+    e = np.empty(B, np.float64)
+    L = np.empty(1, np.float64)
+    rc = _load().p4q_block_mse(_ptr(a), _ptr(f), _ptr(off), B, a.shape[1], _ptr(e), _ptr(L))
+    if rc != OK:
+        raise ValueError(f"oracle block_mse failed ({rc})")
+    return e, float(L[0])
+
+
+def topk_replacement(s_ref, s_alt, K):
+    """Eq. 9's replacement ratio per sample (Top-K sets, ties to the lower
+    index): returns (intersection int32 [B], rho float32 [B])."""
+    r, a = _f32(s_ref), _f32(s_alt)
+    assert r.ndim == 2 and r.shape == a.shape
+    B, N = r.shape
+    inter = np.empty(B, np.int32)
+    rho = np.empty(B, np.float32)
+    rc = _load().p4q_topk_replacement(_ptr(r), _ptr(a), B, N, int(K), _ptr(inter), _ptr(rho))
+    if rc != OK:
+        raise ValueError(f"oracle topk_replacement failed ({rc})")
+    return inter, rho
 
 
 def pack_codes(codes):

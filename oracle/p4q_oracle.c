@@ -64,6 +64,13 @@
  *      q . k / sqrt(d_h), heads sharing key/value heads in groups of H / H_kv
  *      (H_kv = H: one key/value head per head). Position encodings are
  *      applied by the caller. fp64 throughout.
+ *   R15 calibration data path (Sec. 3.3, Eq. 5; App. A, Eq. 9): the block
+ *      objective of a sample is the squared Frobenius distance of the W4A4 and
+ *      full-precision block outputs over its m_n rows, divided by m_n d, and
+ *      the batch objective their mean; the Top-K set of a score vector takes
+ *      the K largest scores, ties to the lower index (as R8), and the
+ *      replacement ratio is 1 - |T_ref & T_alt| / K, evaluated in fp32 from
+ *      the integer intersection. fp64 sums.
  *   R11 CLS saliency (Sec. 3.2, Visual Saliency): in the vision tower's final
  *      self-attention, each crop's [CLS] token is the query; its attention
  *      row is the softmax, over the CLS key and the crop's patch keys, of
@@ -594,4 +601,56 @@ int p4q_causal_attention(const float* q, const float* k, const float* v, int B, 
     }
   }
   return rc;
+}
+
+/* ------------------------------------------------------------------ */
+/* Pruning-aware calibration data path (reading R15).                   */
+/* ------------------------------------------------------------------ */
+
+/* Eq. 5's block objective: sample n owns rows off[n] .. off[n+1]-1 of the
+ * W4A4 block output Yq and the full-precision output Yf (d columns each);
+ * e[n] = sum (Yq - Yf)^2 / (m_n d), *L = (1/B) sum_n e[n]. fp64. */
+int p4q_block_mse(const float* Yq, const float* Yf, const int32_t* off, int B, int d, double* e, double* L) {
+  if (!Yq || !Yf || !off || !e || !L || B < 1 || d < 1 || off[0] != 0) return ORACLE_BAD_ARG;
+  double tot = 0.0;
+  for (int n = 0; n < B; ++n) {
+    const int64_t r0 = off[n], r1 = off[n + 1];
+    if (r1 <= r0) return ORACLE_BAD_ARG;
+    double acc = 0.0;
+    for (int64_t i = r0 * d; i < r1 * d; ++i) {
+      const double diff = (double)Yq[i] - (double)Yf[i];
+      acc += diff * diff;
+    }
+    e[n] = acc / ((double)(r1 - r0) * (double)d);
+    tot += e[n];
+  }
+  *L = tot / (double)B;
+  return ORACLE_OK;
+}
+
+/* Token i belongs to the Top-K set of s when fewer than K tokens rank above
+ * it: a larger score, or an equal score at a lower index. */
+static int in_topk(const float* s, int N, int K, int i) {
+  int above = 0;
+  for (int j = 0; j < N; ++j)
+    if (s[j] > s[i] || (s[j] == s[i] && j < i)) ++above;
+  return above < K;
+}
+
+/* Eq. 9's replacement ratio per sample: s_ref, s_alt [B, N] scores of the
+ * same tokens under two precisions; inter[b] = |T_ref & T_alt|,
+ * rho[b] = 1 - inter[b] / K (fp32 division and subtraction). */
+int p4q_topk_replacement(const float* s_ref, const float* s_alt, int B, int N, int K, int32_t* inter, float* rho) {
+  if (!s_ref || !s_alt || !inter || !rho || B < 0 || N < 1 || K < 1 || K > N) return ORACLE_BAD_ARG;
+#pragma omp parallel for schedule(static)
+  for (int b = 0; b < B; ++b) {
+    const float* r = s_ref + (int64_t)b * N;
+    const float* a = s_alt + (int64_t)b * N;
+    int c = 0;
+    for (int i = 0; i < N; ++i)
+      if (in_topk(r, N, K, i) && in_topk(a, N, K, i)) ++c;
+    inter[b] = c;
+    rho[b] = 1.0f - (float)c / (float)K;
+  }
+  return ORACLE_OK;
 }
