@@ -200,6 +200,40 @@ p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t
 p4q_status p4q_causal_attention(const uint16_t* q, int ldq, const uint16_t* k, int ldk, const uint16_t* v, int ldv,
                                 int B, int m, int H, int Hkv, int dh, uint16_t* o, int ldo, p4q_stream_t stream);
 
+/* ---------------------------------------------------------------------- */
+/* Pruning-aware calibration data path (Sec. 3.3, Eq. 5; App. A, Eq. 9)     */
+/* ---------------------------------------------------------------------- */
+
+/* Workspace of p4q_block_mse for B samples (fp64 partial sums); 0 when B is
+ * outside 1 .. 1024. */
+size_t p4q_block_mse_workspace_bytes(int B);
+
+/* Eq. 5's block objective. Sample n owns rows offsets[n] .. offsets[n+1]-1 of
+ * the W4A4 block output Yq and of the full-precision block output Yf (both
+ * computed on the same pruned input H^{FP,keep}, e.g. the X of
+ * p4q_select_gather_quant):
+ *   e[n] = ||Yq_n - Yf_n||_F^2 / (m_n d),   *L = (1/B) sum_n e[n].
+ * Squares summed in fp32 per thread over a few hundred values, combined in
+ * fp64 in a fixed order (the result does not depend on the launch).
+ *   Yq, Yf  [offsets[B], ld] fp16 (device, read), d columns used
+ *   offsets HOST array of B + 1 ints, offsets[0] = 0, strictly increasing
+ *   e [B], L [1] fp32 (device, written)
+ *   ws      device workspace of p4q_block_mse_workspace_bytes(B) bytes
+ * Requires 1 <= B <= 1024, d % 8 == 0, ld >= d, ld % 8 == 0, 16-byte aligned
+ * Yq, Yf and ws. */
+p4q_status p4q_block_mse(const uint16_t* Yq, int ldq, const uint16_t* Yf, int ldf, const int32_t* offsets, int B,
+                         int d, float* e, float* L, void* ws, size_t ws_bytes, p4q_stream_t stream);
+
+/* Eq. 9's Top-K replacement ratio per sample: the Top-K sets of the scores
+ * of the same N tokens under a reference and an alternative precision (the K
+ * largest scores; ties, with -0 equal to +0, to the lower index) and
+ *   inter[b] = |T_ref & T_alt|,   rho[b] = fl32(1 - fl32(inter[b] / K)).
+ *   s_ref, s_alt [B, N] fp32 finite (device, read)
+ *   inter [B] int32, rho [B] fp32 (device, written)
+ * Requires 1 <= K <= N <= P4Q_MAX_TOKENS, 0 <= B <= 65535 (0: no-op). */
+p4q_status p4q_topk_replacement(const float* s_ref, const float* s_alt, int B, int N, int K, int32_t* inter,
+                                float* rho, p4q_stream_t stream);
+
 /* Per-output-channel weight quantization (App. B.3: symmetric, per output
  * channel, then round-to-nearest): the same per-row quantizer applied to each
  * output row of W.

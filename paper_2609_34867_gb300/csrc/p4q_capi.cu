@@ -272,6 +272,38 @@ p4q_status p4q_causal_attention(const uint16_t* q, int ldq, const uint16_t* k, i
                                                    reinterpret_cast<cudaStream_t>(stream))));
 }
 
+size_t p4q_block_mse_workspace_bytes(int B) {
+  return (B < 1 || B > kMseMaxSamples) ? 0 : block_mse_workspace_bytes(B);
+}
+
+p4q_status p4q_block_mse(const uint16_t* Yq, int ldq, const uint16_t* Yf, int ldf, const int32_t* offsets, int B,
+                         int d, float* e, float* L, void* ws, size_t ws_bytes, p4q_stream_t stream) {
+  if (!Yq || !Yf || !offsets || !e || !L || B < 1 || d < 8 || ldq < d || ldf < d) return P4Q_ERR_INVALID_ARG;
+  if (B > kMseMaxSamples) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (offsets[0] != 0) return P4Q_ERR_INVALID_ARG;
+  for (int n = 0; n < B; ++n)
+    if (offsets[n + 1] <= offsets[n]) return P4Q_ERR_INVALID_ARG;
+  if (d % 8 != 0) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (ldq % 8 != 0 || ldf % 8 != 0 || !aligned16(Yq) || !aligned16(Yf) || !aligned16(ws)) return P4Q_ERR_MISALIGNED;
+  if (!ws || ws_bytes < block_mse_workspace_bytes(B)) return P4Q_ERR_WORKSPACE_TOO_SMALL;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return from_cuda(counted(launch_block_mse(Yq, ldq, Yf, ldf, offsets, B, d, static_cast<double*>(ws), e, L, s), 2));
+}
+
+p4q_status p4q_topk_replacement(const float* s_ref, const float* s_alt, int B, int N, int K, int32_t* inter,
+                                float* rho, p4q_stream_t stream) {
+  if (B < 0 || N < 1 || K < 1 || K > N) return P4Q_ERR_INVALID_ARG;
+  if (B > 0 && (!s_ref || !s_alt || !inter || !rho)) return P4Q_ERR_INVALID_ARG;
+  if (N > P4Q_MAX_TOKENS || B > 65535) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (B == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(
+      counted(launch_topk_replacement(s_ref, s_alt, B, N, K, inter, rho, reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_quant_act_ld(const uint16_t* X, int ldx, int M, int Kin, uint8_t* Xq, float* s_a,
                             p4q_stream_t stream) {
   p4q_status st = check_rows(X, M, Kin, Xq, s_a);

@@ -115,6 +115,18 @@ cudaError_t launch_causal_attention(const uint16_t* q, long long ldq, const uint
                                     long long ldo, cudaStream_t stream);
 unsigned int attn_read_and_clear_error();
 
+// ------------------------------------------------------------ calibration data path
+constexpr int kMseMaxSamples = 1024;
+// CTAs per sample of the block-objective reduction, and its workspace (fp64 partials).
+int block_mse_chunks(int B);
+size_t block_mse_workspace_bytes(int B);
+// off: host array of B + 1 row offsets (validated by the caller).
+cudaError_t launch_block_mse(const uint16_t* Yq, long long ldq, const uint16_t* Yf, long long ldf, const int32_t* off,
+                             int B, int d, double* partial, float* e, float* L, cudaStream_t stream);
+// Top-K sets of two score rows per sample and their intersection (selector's radix select).
+cudaError_t launch_topk_replacement(const float* s_ref, const float* s_alt, int B, int N, int K, int32_t* inter,
+                                    float* rho, cudaStream_t stream);
+
 // ------------------------------------------------------------ CLS saliency
 // Shared memory of one (image, crop) CTA: H x (N / C) fp32 weights.
 size_t cls_saliency_smem_bytes(int N, int C, int H);

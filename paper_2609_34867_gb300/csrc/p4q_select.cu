@@ -145,7 +145,8 @@ struct BlockScratch {
 __device__ __forceinline__ void group_sync(int nt) { named_bar_sync(1, static_cast<uint32_t>(nt)); }
 
 // Exclusive prefix sum of per-thread counts over the first nt threads (thread order).
-__device__ int block_exclusive_scan(int v, int* total, int nt, BlockScratch& s) {
+template <class Scratch>
+__device__ int block_exclusive_scan(int v, int* total, int nt, Scratch& s) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int x = v;
 #pragma unroll
@@ -176,8 +177,9 @@ __device__ int block_exclusive_scan(int v, int* total, int nt, BlockScratch& s) 
 // Radix select, 8 bits per pass, from the most significant byte; the
 // histogram updates are aggregated per warp over equal digits, since scores
 // of similar magnitude share their leading bytes.
+template <class Scratch>
 __device__ void block_take_top(const uint32_t (&key)[kPer], bool (&kept)[kPer], int base, int N, int q, int nt,
-                               BlockScratch& s) {
+                               Scratch& s) {
   if (q <= 0) return;
   const int lane = threadIdx.x & 31;
   uint32_t prefix = 0, mask = 0;
@@ -589,7 +591,59 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
+// ---------------------------------------------------------------- Top-K replacement ratio
+// App. A, Eq. 9: per sample, the Top-K sets of two score rows over the same N
+// tokens (ties to the lower index, the selector's radix select) and the size
+// of their intersection; rho = 1 - |T_ref & T_alt| / K. One CTA per sample,
+// token i = kPer * threadIdx.x + e.
+// Order key of a score with -0 and +0 equal (they tie, and the lower index wins).
+__device__ __forceinline__ uint32_t score_key(float v) { return float_order_key(v == 0.0f ? 0.0f : v); }
+
+struct TopkScratch {
+  unsigned int hist[256];
+  unsigned int wsum[32];
+  int digit, above;
+};
+
+__global__ void __launch_bounds__(kSelThreads)
+    topk_replacement_kernel(const float* __restrict__ s_ref, const float* __restrict__ s_alt, int N, int K,
+                            int32_t* __restrict__ inter, float* __restrict__ rho) {
+  pdl_wait();
+  pdl_launch_dependents();
+  __shared__ TopkScratch s;
+  const int b = blockIdx.x, nt = blockDim.x, base = kPer * threadIdx.x;
+  uint32_t key[kPer];
+  bool in_ref[kPer], in_alt[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) {
+    key[e] = base + e < N ? score_key(s_ref[static_cast<size_t>(b) * N + base + e]) : 0u;
+    in_ref[e] = false;
+    in_alt[e] = false;
+  }
+  block_take_top(key, in_ref, base, N, K, nt, s);
+#pragma unroll
+  for (int e = 0; e < kPer; ++e)
+    key[e] = base + e < N ? score_key(s_alt[static_cast<size_t>(b) * N + base + e]) : 0u;
+  block_take_top(key, in_alt, base, N, K, nt, s);
+  int c = 0;
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) c += (in_ref[e] && in_alt[e]) ? 1 : 0;
+  int total;
+  block_exclusive_scan(c, &total, nt, s);
+  if (threadIdx.x == 0) {
+    inter[b] = total;
+    rho[b] = __fsub_rn(1.0f, __fdiv_rn(static_cast<float>(total), static_cast<float>(K)));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_topk_replacement(const float* s_ref, const float* s_alt, int B, int N, int K, int32_t* inter,
+                                    float* rho, cudaStream_t stream) {
+  if (B <= 0) return cudaSuccess;
+  const int nt = ((N + kPer - 1) / kPer + 31) / 32 * 32;
+  return launch_pdl(topk_replacement_kernel, dim3(B), dim3(nt), 0, stream, s_ref, s_alt, N, K, inter, rho);
+}
 
 size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, void* base) {
   const size_t BN = static_cast<size_t>(B) * N, BJ = static_cast<size_t>(B) * J;

@@ -9,6 +9,8 @@
   python -m paper_2609_34867_gb300.kernel_cases swiglu M K LD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases rmsnorm M K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases attn B M H [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases mse B M D [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases topk B N K [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -34,6 +36,8 @@ selects the first replayed launch.
   attn    p4q_causal_attention on B samples of M positions, H heads of 128
           (flops: 2 x 2 x 128 x M (M + 1) / 2 per sample and head, the
           causal Q K^T and P V; bytes: q, k, v in, o out, fp16);
+  mse     p4q_block_mse on B samples of M rows x D fp16 (bytes: 4 B M D in);
+  topk    p4q_topk_replacement on B x N fp32 score pairs (bytes: 8 B N in);
   saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
           heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
           fp16 keys and queries in, 4 B N out).
@@ -79,7 +83,7 @@ def _timed(fn, reps, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn", "mse", "topk"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -156,6 +160,27 @@ def main(argv=None):
         nbytes = 4 * B * M * H * 128 * 2
         print(f"attn {B}x{M} H={H}: {ms * 1e3:.1f} us/call, {flops / ms / 1e9:.1f} TFLOP/s, "
               f"{nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "mse":
+        B, M, D = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        Yq = torch.randn((B * M, D), generator=g, device=dev).to(torch.float16)
+        Yf = torch.randn((B * M, D), generator=g, device=dev).to(torch.float16)
+        e = torch.empty((B,), dtype=torch.float32, device=dev)
+        L = torch.empty((1,), dtype=torch.float32, device=dev)
+        ws = torch.empty((p4q.p4q_block_mse_workspace_bytes(B),), dtype=torch.uint8, device=dev)
+        off = [n * M for n in range(B + 1)]
+        ms = _timed(lambda: p4q.p4q_block_mse(Yq, Yf, off, e, L, ws), a.reps, dev)
+        nbytes = 4 * B * M * D
+        print(f"mse {B}x{M}x{D}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "topk":
+        B, N, K = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        s1 = torch.randn((B, N), generator=g, device=dev)
+        s2 = torch.randn((B, N), generator=g, device=dev)
+        inter = torch.empty((B,), dtype=torch.int32, device=dev)
+        rho = torch.empty((B,), dtype=torch.float32, device=dev)
+        ms = _timed(lambda: p4q.p4q_topk_replacement(s1, s2, K, inter, rho), a.reps, dev)
+        print(f"topk {B}x{N} K={K}: {ms * 1e3:.1f} us/call, {8 * B * N / ms / 1e6:.1f} GB/s")
     elif a.case == "saliency":
         B, N = (int(x) for x in a.args)
         v = wl.vision_attention(B, N, seed=0)

@@ -55,6 +55,12 @@ def lib() -> ctypes.CDLL:
         L.p4q_rmsnorm_quant_expanded.restype = st
         L.p4q_causal_attention.argtypes = [P, I, P, I, P, I, I, I, I, I, I, P, I, P]
         L.p4q_causal_attention.restype = st
+        L.p4q_block_mse_workspace_bytes.argtypes = [I]
+        L.p4q_block_mse_workspace_bytes.restype = S
+        L.p4q_block_mse.argtypes = [P, I, P, I, P, I, I, P, P, P, S, P]
+        L.p4q_block_mse.restype = st
+        L.p4q_topk_replacement.argtypes = [P, P, I, I, I, P, P, P]
+        L.p4q_topk_replacement.restype = st
         L.p4q_device_status.argtypes = [P]
         L.p4q_device_status.restype = st
         L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
@@ -210,6 +216,40 @@ def p4q_causal_attention(q, k, v, o, B, m, H, Hkv, stream=None):
             raise TypeError(f"{name}: expected a CUDA fp16 2-D tensor of B*m rows with unit column stride")
     _check(lib().p4q_causal_attention(_ptr(q), q.stride(0), _ptr(k), k.stride(0), _ptr(v), v.stride(0), B, m, H,
                                       Hkv, 128, _ptr(o), o.stride(0), _stream(stream)), "p4q_causal_attention")
+
+
+def p4q_block_mse_workspace_bytes(B):
+    return int(lib().p4q_block_mse_workspace_bytes(int(B)))
+
+
+def p4q_block_mse(Yq, Yf, offsets, e, L, ws, stream=None):
+    """Eq. 5's block objective: Yq, Yf [rows, d] fp16 2-D views with unit column
+    stride; offsets a host sequence of B + 1 row offsets; e [B], L [1] fp32;
+    ws a uint8 device buffer of p4q_block_mse_workspace_bytes(B) bytes."""
+    for t, name in ((Yq, "Yq"), (Yf, "Yf")):
+        if not isinstance(t, torch.Tensor) or t.dtype != torch.float16 or t.dim() != 2 or t.stride(1) != 1 or \
+                not t.is_cuda:
+            raise TypeError(f"{name}: expected a CUDA fp16 2-D tensor with unit column stride")
+    if Yq.shape != Yf.shape:
+        raise ValueError("Yq and Yf differ in shape")
+    off = (ctypes.c_int32 * len(offsets))(*[int(x) for x in offsets])
+    B = len(offsets) - 1
+    if B >= 1 and int(offsets[-1]) > Yq.shape[0]:
+        raise ValueError("offsets run past the rows of Yq")
+    _need(e, torch.float32, 1, "e"); _need(L, torch.float32, 1, "L"); _need(ws, torch.uint8, 1, "ws")
+    _check(lib().p4q_block_mse(_ptr(Yq), Yq.stride(0), _ptr(Yf), Yf.stride(0), off, B, Yq.shape[1], _ptr(e), _ptr(L),
+                               _ptr(ws), ws.numel(), _stream(stream)), "p4q_block_mse")
+
+
+def p4q_topk_replacement(s_ref, s_alt, K, inter, rho, stream=None):
+    """Eq. 9's replacement ratio: s_ref, s_alt [B, N] fp32 -> inter [B] int32, rho [B] fp32."""
+    _need(s_ref, torch.float32, 2, "s_ref"); _need(s_alt, torch.float32, 2, "s_alt")
+    _need(inter, torch.int32, 1, "inter"); _need(rho, torch.float32, 1, "rho")
+    if s_ref.shape != s_alt.shape:
+        raise ValueError("score rows differ in shape")
+    B, N = s_ref.shape
+    _check(lib().p4q_topk_replacement(_ptr(s_ref), _ptr(s_alt), B, N, int(K), _ptr(inter), _ptr(rho),
+                                      _stream(stream)), "p4q_topk_replacement")
 
 
 def p4q_quant_weight(W, Wq, s_w, stream=None):

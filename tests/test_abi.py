@@ -117,6 +117,33 @@ def test_causal_attention_validates_arguments(lib):
     assert f(P(8), 4096, P(16), 4096, P(16), 4096, 2, 256, 32, 32, 128, P(16), 4096, None) == 3   # misaligned
 
 
+def test_calibration_entries_validate_arguments(lib):
+    P, I, S = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+    lib.p4q_block_mse_workspace_bytes.argtypes = [I]
+    lib.p4q_block_mse_workspace_bytes.restype = S
+    assert lib.p4q_block_mse_workspace_bytes(0) == 0 and lib.p4q_block_mse_workspace_bytes(1025) == 0
+    assert lib.p4q_block_mse_workspace_bytes(8) >= 8 * 8
+    lib.p4q_block_mse.argtypes = [P, I, P, I, P, I, I, P, P, P, S, P]
+    f = lib.p4q_block_mse
+    off = (ctypes.c_int32 * 3)(0, 10, 20)
+    bad = (ctypes.c_int32 * 3)(0, 10, 10)
+    first = (ctypes.c_int32 * 3)(1, 10, 20)
+    big = 1 << 20
+    assert f(P(16), 64, P(16), 64, bad, 2, 64, P(16), P(16), P(16), big, None) == 1    # empty sample
+    assert f(P(16), 64, P(16), 64, first, 2, 64, P(16), P(16), P(16), big, None) == 1  # offsets[0] != 0
+    assert f(P(16), 64, P(16), 64, None, 2, 64, P(16), P(16), P(16), big, None) == 1   # no offsets
+    assert f(P(16), 64, P(16), 64, off, 2, 60, P(16), P(16), P(16), big, None) == 2    # d % 8
+    assert f(P(16), 68, P(16), 64, off, 2, 64, P(16), P(16), P(16), big, None) == 3    # pitch % 8
+    assert f(P(16), 64, P(16), 64, off, 2, 64, P(16), P(16), P(16), 8, None) == 4      # workspace
+    lib.p4q_topk_replacement.argtypes = [P, P, I, I, I, P, P, P]
+    g = lib.p4q_topk_replacement
+    assert g(P(16), P(16), 0, 576, 64, P(16), P(16), None) == 0       # empty is a no-op
+    assert g(P(16), P(16), 2, 576, 577, P(16), P(16), None) == 1      # K > N
+    assert g(P(16), P(16), 2, 576, 0, P(16), P(16), None) == 1        # K < 1
+    assert g(None, P(16), 2, 576, 64, P(16), P(16), None) == 1        # no scores
+    assert g(P(16), P(16), 2, 4097, 64, P(16), P(16), None) == 2      # N > P4Q_MAX_TOKENS
+
+
 class Params(ctypes.Structure):
     _fields_ = [("K", ctypes.c_int32), ("alpha_permille", ctypes.c_int32), ("beta_permille", ctypes.c_int32)]
 
