@@ -356,7 +356,13 @@ size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_p
  *         256-byte aligned; its contents are scratch.
  * Requires 1 <= B, 1 <= K <= N <= P4Q_MAX_TOKENS, 0 <= J <= P4Q_MAX_CONCEPTS,
  * d % 128 == 0, 128 <= d <= P4Q_MAX_ROW, 0 <= alpha, beta and
- * alpha + beta <= 1000. */
+ * alpha + beta <= 1000.
+ * All work is ordered on `stream`. When the cosine-matrix GEMM leaves an SM
+ * per image free, stages 1-2 run beside it on a second stream the library
+ * owns (one per device, created on the first call that is not being captured
+ * into a CUDA graph), forked from and joined back into `stream` by events
+ * inside the call, so a graph captured from `stream` contains both branches;
+ * a host lock keeps concurrent callers' fork/join pairs apart. */
 p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
                       const float* A_cls, const p4q_select_params* params, int32_t* idx,
                       void* ws, size_t ws_bytes, p4q_stream_t stream);

@@ -62,6 +62,36 @@ p4q_status check_select_args(const uint16_t* V, int B, int N, int d, int J, cons
   return P4Q_OK;
 }
 
+// A second stream of the library per device, with a fork and a join event,
+// for the stage-1/2 launch of the selector beside the cosine matrix; created
+// on the first call that is not being captured into a graph.
+struct SideStream {
+  cudaStream_t s = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+  bool failed = false;
+};
+std::mutex g_side_mutex;
+SideStream g_side[64];
+
+SideStream* side_stream(cudaStream_t stream) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  SideStream& r = g_side[dev];
+  if (r.s) return &r;
+  if (r.failed) return nullptr;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return nullptr;
+  if (cudaStreamCreateWithFlags(&r.s, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&r.fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&r.join, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    r.failed = true;  // the serial order is used from now on
+    r.s = nullptr;
+    return nullptr;
+  }
+  return &r;
+}
+
 p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
                       const p4q_select_params* params, int32_t* idx, void* ws, size_t ws_bytes,
                       cudaStream_t stream) {
@@ -101,6 +131,25 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     e = counted(launch_query_scores(plan, w, stream));
     if (e != cudaSuccess) return from_cuda(e);
   }
+  // Stages 1-2 (query relevance, saliency) need only the scores and A_cls:
+  // when the cosine-matrix GEMM leaves an SM per image free, they run on the
+  // side stream beside it and stage 3 starts from their kept set.
+  std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
+  SideStream* side = nullptr;
+  if (bud.Kd > 0 && (bud.Kq > 0 || bud.Ks > 0) && w.vu != nullptr && select_split_applies(N)) {
+    if (num_sms() - 2 * gemm8_pairs(N, N, B, num_sms()) >= B) {
+      side_lock.lock();
+      side = side_stream(stream);
+      if (!side) side_lock.unlock();
+    }
+  }
+  if (side) {
+    cudaError_t se = cudaEventRecord(side->fork, stream);
+    if (se == cudaSuccess) se = cudaStreamWaitEvent(side->s, side->fork, 0);
+    if (se == cudaSuccess) se = counted(launch_select_stages(plan, w, A_cls, idx, side->s, 1));
+    if (se == cudaSuccess) se = cudaEventRecord(side->join, side->s);
+    if (se != cudaSuccess) return from_cuda(se);
+  }
   if (bud.Kd > 0) {
     GemmArgs g;
     g.A = w.vcodes;
@@ -126,6 +175,11 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     e = counted(split ? launch_gemm8(g, w.vu, w.vsum, w.vu, w.vsum, stream) : launch_w4a4_gemm(g, stream));
     if (e != cudaSuccess) return from_cuda(e);
     if (split && (e = counted(launch_gram_cos(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+  }
+  if (side) {
+    e = cudaStreamWaitEvent(stream, side->join, 0);
+    if (e != cudaSuccess) return from_cuda(e);
+    return from_cuda(counted(launch_select_stages(plan, w, A_cls, idx, stream, 2)));
   }
   return from_cuda(counted(launch_select_stages(plan, w, A_cls, idx, stream)));
 }

@@ -153,6 +153,7 @@ struct SelectWorkspace {
   int gram_pitch;    // N rounded up to a multiple of 4
   uint8_t* vu;       // [B*N, d] codes, one byte each (tokens >= kGramExpandedMin), else null
   int32_t* vsum;     // [B*N] sum of those bytes
+  uint32_t* kept12;  // [B, ceil(N/32)] kept set after stages 1-2, as bits (split launches)
 };
 
 // Token count from which the cosine matrix runs on the expanded-operand GEMM.
@@ -163,8 +164,17 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
 cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
 // In place: the int32 dot products of ws.gram become the cosines of Eq. 4.
 cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+// mode 0: stages 1-3; 1: stages 1-2 into ws.kept12; 2: stage 3 from ws.kept12
+// (modes 1 and 2 for N where select_split_applies).
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls,
-                                 int32_t* idx, cudaStream_t stream);
+                                 int32_t* idx, cudaStream_t stream, int mode = 0);
+bool select_split_applies(int N);
+// CTA pairs the expanded-operand GEMM launches: one per 256 x 256 output
+// tile (two 128-row CTAs), at most one pair per two SMs.
+inline int gemm8_pairs(int M, int N, int batch, int sms) {
+  const int tiles = ((M + 255) / 256) * ((N + 255) / 256) * (batch > 0 ? batch : 1);
+  return tiles < sms / 2 ? tiles : sms / 2;
+}
 
 // Device error words of the kernels with bounded waits (GEMMs, quantizer).
 unsigned int gemm_read_and_clear_error();

@@ -442,11 +442,17 @@ __device__ void pool_rounds(int npool, int Kd, BlockScratch& s) {
   }
 }
 
-template <int kMaxThreads>
+// kMode: kStagesAll runs stages 1-3 and writes idx; kStages12 runs stages 1-2
+// and writes the kept set as bits (token t: bit t % 32 of word t / 32 of the
+// image's row of kept12) so that it can run beside the cosine matrix; kStage3
+// starts from those bits.
+enum { kStagesAll = 0, kStages12 = 1, kStage3 = 2 };
+
+template <int kMaxThreads, int kMode>
 __global__ void __launch_bounds__(kMaxThreads, 1)
     select_stages_kernel(const float* __restrict__ scores, const float* __restrict__ A_cls,
                          const float* __restrict__ gram, int gp, int N, int J, int K, int Kq, int Ks,
-                         int Kd, int32_t* __restrict__ idx) {
+                         int Kd, int32_t* __restrict__ idx, uint32_t* __restrict__ kept12) {
   pdl_wait();
   pdl_launch_dependents();
   extern __shared__ uint8_t smem_raw[];
@@ -459,8 +465,17 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 #pragma unroll
   for (int e = 0; e < kPer; ++e) kept[e] = false;
   uint32_t key[kPer];
+  const int words = (N + 31) / 32;
 
-  if (g0) {
+  if (kMode == kStage3) {
+    if (g0) {
+#pragma unroll
+      for (int e = 0; e < kPer; ++e) {
+        const int i = base + e;
+        kept[e] = i < N && ((kept12[static_cast<size_t>(b) * words + (i >> 5)] >> (i & 31)) & 1u);
+      }
+    }
+  } else if (g0) {
     // Stage 1: query relevance, one ranking per concept, quota floor(Kq/J) + (j < Kq % J).
     for (int j = 0; j < J && Kq > 0; ++j) {
       const int quota = Kq / J + (j < Kq % J ? 1 : 0);
@@ -476,6 +491,18 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
       for (int e = 0; e < kPer; ++e) key[e] = (base + e < N) ? float_order_key(a[base + e]) : 0u;
       block_take_top(key, kept, base, N, Ks, tpg, s);
     }
+  }
+  if (kMode == kStages12) {
+    for (int w = threadIdx.x; w < words; w += blockDim.x) s.keptbits[w] = 0u;
+    __syncthreads();
+    if (g0) {
+#pragma unroll
+      for (int e = 0; e < kPer; ++e)
+        if (base + e < N && kept[e]) atomicOr(&s.keptbits[(base + e) >> 5], 1u << ((base + e) & 31));
+    }
+    __syncthreads();
+    for (int w = threadIdx.x; w < words; w += blockDim.x) kept12[static_cast<size_t>(b) * words + w] = s.keptbits[w];
+    return;
   }
   // Stage 3: greedy max-min diversity on the cosine matrix G of the image:
   // m_i = max over the kept set of cos(i, r) (-inf while it is empty); each
@@ -659,6 +686,7 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
   const size_t o_sc = take(BJ * N * 4), o_g = take(BN * gp * 4);
   const bool expanded = N >= kGramExpandedMin;
   const size_t o_vu = expanded ? take(BN * d) : 0, o_vsum = expanded ? take(BN * 4) : 0;
+  const size_t o_k12 = take(static_cast<size_t>(B) * ((N + 31) / 32) * 4);
   if (ws && base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     ws->vcodes = p + o_vc;
@@ -672,6 +700,7 @@ size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, 
     ws->gram_pitch = gp;
     ws->vu = expanded ? p + o_vu : nullptr;
     ws->vsum = expanded ? reinterpret_cast<int32_t*>(p + o_vsum) : nullptr;
+    ws->kept12 = reinterpret_cast<uint32_t*>(p + o_k12);
   }
   return off;
 }
@@ -741,33 +770,48 @@ cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cuda
 }
 
 cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls, int32_t* idx,
-                                 cudaStream_t stream) {
+                                 cudaStream_t stream, int mode) {
   static bool attr_set = false;
   const int smem = static_cast<int>(sizeof(BlockScratch));
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(select_stages_kernel<kSelThreadsSmall>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(select_stages_kernel<kSelThreadsMid>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               smem);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(select_stages_kernel<kSelThreads>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
+    const void* fns[] = {reinterpret_cast<const void*>(select_stages_kernel<kSelThreadsSmall, kStagesAll>),
+                         reinterpret_cast<const void*>(select_stages_kernel<kSelThreadsSmall, kStages12>),
+                         reinterpret_cast<const void*>(select_stages_kernel<kSelThreadsSmall, kStage3>),
+                         reinterpret_cast<const void*>(select_stages_kernel<kSelThreadsMid, kStagesAll>),
+                         reinterpret_cast<const void*>(select_stages_kernel<kSelThreads, kStagesAll>)};
+    for (const void* f : fns) {
+      cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      if (e != cudaSuccess) return e;
+    }
     attr_set = true;
   }
   // group 0: one thread per kPer tokens (idle threads would only add
   // instructions to every ranking); as many row groups as fit the block
   const int tpg = ((p.N + kPer - 1) / kPer + 31) / 32 * 32;
-  if (tpg <= kSelThreadsSmall)
-    return launch_pdl(select_stages_kernel<kSelThreadsSmall>, dim3(p.B), dim3(tpg * (kSelThreadsSmall / tpg)),
+  if (tpg <= kSelThreadsSmall) {
+    const dim3 block(tpg * (kSelThreadsSmall / tpg));
+    if (mode == kStages12)
+      return launch_pdl(select_stages_kernel<kSelThreadsSmall, kStages12>, dim3(p.B), dim3(tpg),
+                        static_cast<size_t>(smem), stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K,
+                        p.Kq, p.Ks, p.Kd, idx, ws.kept12);
+    if (mode == kStage3)
+      return launch_pdl(select_stages_kernel<kSelThreadsSmall, kStage3>, dim3(p.B), block, static_cast<size_t>(smem),
+                        stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx,
+                        ws.kept12);
+    return launch_pdl(select_stages_kernel<kSelThreadsSmall, kStagesAll>, dim3(p.B), block,
                       static_cast<size_t>(smem), stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K,
-                      p.Kq, p.Ks, p.Kd, idx);
+                      p.Kq, p.Ks, p.Kd, idx, ws.kept12);
+  }
+  if (mode != kStagesAll) return cudaErrorInvalidValue;  // split launches serve N <= 2048
   if (tpg <= kSelThreadsMid)
-    return launch_pdl(select_stages_kernel<kSelThreadsMid>, dim3(p.B), dim3(tpg * (kSelThreadsMid / tpg)),
+    return launch_pdl(select_stages_kernel<kSelThreadsMid, kStagesAll>, dim3(p.B), dim3(tpg * (kSelThreadsMid / tpg)),
                       static_cast<size_t>(smem), stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K,
-                      p.Kq, p.Ks, p.Kd, idx);
-  return launch_pdl(select_stages_kernel<kSelThreads>, dim3(p.B), dim3(tpg), static_cast<size_t>(smem), stream,
-                    ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx);
+                      p.Kq, p.Ks, p.Kd, idx, ws.kept12);
+  return launch_pdl(select_stages_kernel<kSelThreads, kStagesAll>, dim3(p.B), dim3(tpg), static_cast<size_t>(smem),
+                    stream, ws.scores, A_cls, ws.gram, ws.gram_pitch, p.N, p.J, p.K, p.Kq, p.Ks, p.Kd, idx,
+                    ws.kept12);
 }
+
+bool select_split_applies(int N) { return ((N + kPer - 1) / kPer + 31) / 32 * 32 <= kSelThreadsSmall; }
 
 }  // namespace p4q
