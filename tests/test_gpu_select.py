@@ -108,3 +108,44 @@ def test_select_gather_quant_expanded_matches(p4q, dev):
     torch.cuda.synchronize()
     assert torch.equal(idx, ref_idx) and torch.equal(X.view(torch.int16), ref_X.view(torch.int16))
     assert torch.equal(Xq, ref_q) and torch.equal(Xu, ref_u) and torch.equal(su, ref_su)
+
+
+def test_select_from_two_host_threads_on_two_streams(p4q, dev):
+    """Concurrent calls on two streams share the library's second stream and
+    its fork / join events (stages 1-2 beside the cosine matrix): each call
+    must still see its own stages 1-2, call after call."""
+    import threading
+
+    cases = []
+    for seed in (40, 41):
+        w = wl.Workload("t", B=4, N=576, d=512, K=96, T=0, J=3, seed=seed, heavy_tail=False, linears=())
+        x = wl.selector_inputs(w)
+        ref = oracle.select_batch(x.V, w.K, x.Q, x.A)
+        ins = (_t(x.V, dev), _t(x.Q, dev), _t(x.A, dev))
+        cases.append((ins, w.K, ref))
+    errors = []
+
+    def run(i):
+        try:
+            (V, Q, A), K, ref = cases[i]
+            stream = torch.cuda.Stream(device=dev)
+            ws = p4q.select_workspace(V.shape[0], V.shape[1], V.shape[2], Q.shape[1], K, dev)
+            for _ in range(20):
+                with torch.cuda.stream(stream):
+                    idx = torch.full((V.shape[0], K), -1, dtype=torch.int32, device=dev)
+                    p4q.p4q_select(V, Q, A, K, idx, ws, stream=stream)
+                stream.synchronize()
+                if not np.array_equal(idx.cpu().numpy(), ref):
+                    errors.append(i)
+                    return
+        except Exception as e:  # surfaced below
+            errors.append(repr(e))
+
+    torch.cuda.synchronize()  # the inputs are in place before either thread starts
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert p4q.p4q_device_status() == 0
+    assert not errors, errors
