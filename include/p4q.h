@@ -189,13 +189,15 @@ p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t
  *   o_i = sum_{j <= i} p_ij v_j, p_i. = softmax_j(q_i . k_j / sqrt(dh)),
  * with key/value head h / (H / Hkv). Position encodings are applied by the
  * caller. fp16 inputs, products accumulated in fp32, p rounded to fp16 before
- * the product with v, fp32 row sums, fp16 output.
+ * the product with v (keys taken 256 at a time with running row maxima: p is
+ * relative to the maximum so far, the earlier partial sums and products
+ * rescaled when it moves), fp32 row sums, fp16 output.
  *   q [B*m, ldq] fp16: row b*m + i holds position i of sample b, head h in
  *                      columns h*dh .. h*dh + dh - 1   (device, read)
  *   k, v [B*m, ldk / ldv] fp16, Hkv heads likewise   (device, read; rows may
  *                      be column blocks of a fused projection output)
  *   o [B*m, ldo] fp16, columns 0 .. H*dh - 1 written (device)
- * Requires dh == 128, 1 <= m <= 384, H % Hkv == 0, ld >= the row's heads *
+ * Requires dh == 128, 1 <= m <= 8192, H % Hkv == 0, ld >= the row's heads *
  * dh, every ld % 8 == 0, 16-byte aligned pointers. B == 0 is a no-op. */
 p4q_status p4q_causal_attention(const uint16_t* q, int ldq, const uint16_t* k, int ldk, const uint16_t* v, int ldv,
                                 int B, int m, int H, int Hkv, int dh, uint16_t* o, int ldo, p4q_stream_t stream);

@@ -112,7 +112,7 @@ def test_causal_attention_validates_arguments(lib):
     assert f(*ok, 2, 256, 32, 32, 128, P(16), 2048, None) == 1        # ldo < H dh
     assert f(*ok, 2, 256, 32, 32, 128, None, 4096, None) == 1         # no output
     assert f(*ok, 2, 256, 32, 32, 64, P(16), 4096, None) == 2         # dh != 128
-    assert f(*ok, 2, 385, 32, 32, 128, P(16), 4096, None) == 2        # m > 384
+    assert f(*ok, 2, 8193, 32, 32, 128, P(16), 4096, None) == 2       # m > 8192
     assert f(P(16), 4100, P(16), 4096, P(16), 4096, 2, 256, 32, 32, 128, P(16), 4096, None) == 3  # pitch % 8
     assert f(P(8), 4096, P(16), 4096, P(16), 4096, 2, 256, 32, 32, 128, P(16), 4096, None) == 3   # misaligned
 

@@ -45,7 +45,8 @@ def _run(p4q, dev, q, k, v, B, m, H, Hkv, ldo=None):
 
 
 @pytest.mark.parametrize("B,m,H,Hkv", [(1, 1, 1, 1), (2, 77, 2, 2), (1, 128, 4, 4), (3, 200, 4, 2),
-                                       (2, 384, 3, 3), (5, 129, 2, 1), (2, 320, 2, 2)])
+                                       (2, 384, 3, 3), (5, 129, 2, 1), (2, 320, 2, 2), (1, 257, 2, 2),
+                                       (2, 700, 2, 1), (1, 1030, 1, 1)])
 def test_attention_matches_oracle(p4q, dev, B, m, H, Hkv):
     q, k, v = _inputs(B, m, H, Hkv, seed=B * 1000 + m)
     got = _run(p4q, dev, q, k, v, B, m, H, Hkv, ldo=H * DH + 64)
@@ -54,9 +55,9 @@ def test_attention_matches_oracle(p4q, dev, B, m, H, Hkv):
 
 
 def test_attention_peaked_rows(p4q, dev):
-    """Large logits (one key dominates most rows) and tiny ones (near-uniform rows)."""
-    B, m, H = 2, 150, 2
-    for scale in (6.0, 0.01):
+    """Large logits (one key dominates most rows) and tiny ones (near-uniform
+    rows), over one key chunk and over three (the running maximum moves)."""
+    for (B, m, H), scale in [((2, 150, 2), 6.0), ((2, 150, 2), 0.01), ((1, 600, 2), 6.0), ((1, 600, 2), 0.01)]:
         q, k, v = _inputs(B, m, H, H, seed=7, qscale=scale)
         got = _run(p4q, dev, q, k, v, B, m, H, H)
         _check(got, oracle.causal_attention(q, k, v, B, m, H, H, DH), v, B, m, H, H)
@@ -77,11 +78,11 @@ def test_attention_on_fused_projection_blocks(p4q, dev):
     _check(O.cpu().numpy(), oracle.causal_attention(q, k, v, B, m, H, H, DH), v, B, m, H, H)
 
 
-@pytest.mark.parametrize("B,m", [(8, 256), (16, 384)])
-def test_attention_fullsize_sampled(p4q, dev, B, m):
-    """The LLaVA-1.5-7B (8 x 256) and LLaVA-NeXT-7B (16 x 384) pruned sequences,
-    32 heads x 128: every output row of sampled (sample, head) pairs."""
-    H = 32
+@pytest.mark.parametrize("B,m,H", [(8, 256, 32), (16, 384, 32), (8, 704, 40)])
+def test_attention_fullsize_sampled(p4q, dev, B, m, H):
+    """The LLaVA-1.5-7B (8 x 256) and LLaVA-NeXT-7B (16 x 384) pruned sequences
+    with 32 heads, and LLaVA-NeXT-13B's (640 + 64 positions, 40 heads; 8 of its
+    32 samples), heads of 128: every output row of sampled (sample, head) pairs."""
     q, k, v = _inputs(B, m, H, H, seed=m)
     got = _run(p4q, dev, q, k, v, B, m, H, H)
     rng = np.random.default_rng(0)
