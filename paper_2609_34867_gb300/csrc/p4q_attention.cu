@@ -42,8 +42,11 @@ namespace {
 constexpr int kBQ = 128;        // query rows per CTA
 constexpr int kDH = 128;        // head dimension
 constexpr int kKeyBlock = 64;   // keys per P / V^T tile
-constexpr int kChunk = 256;     // keys per chunk (S columns in TMEM)
-constexpr int kThreads = 512;
+// 128 keys per chunk and 8 warps: 99 KB of shared memory, 256 TMEM columns
+// and 28 K registers per CTA, so that two CTAs share an SM and one's softmax
+// overlaps the other's loads and MMAs.
+constexpr int kChunk = 128;     // keys per chunk (S columns in TMEM)
+constexpr int kThreads = 256;
 constexpr int kLaneGroups = 4;     // warps w and w + 4k share TMEM lanes 32 (w % 4) ..
 constexpr int kTileBytes = 16384;  // 128 rows x 128 bytes
 
@@ -62,7 +65,8 @@ constexpr int kOffVt = kOffKP + kChunk * 256;
 constexpr int kOffRed = kOffVt + kChunk * 256;
 constexpr int kOffBar = kOffRed + 4 * kBQ * 4;
 constexpr int kSmemBytes = 1024 + kOffBar + 64;
-constexpr uint32_t kTmemCols = 512;  // O: columns 0 .. 127, S: 128 .. 383
+constexpr uint32_t kTmemCols = 128 + kChunk;  // O: columns 0 .. 127, S: 128 .. 128 + kChunk - 1
+static_assert(kTmemCols == 256 || kTmemCols == 512, "TMEM allocations are powers of two");
 
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
@@ -102,7 +106,7 @@ __device__ __forceinline__ uint32_t sw128_off(int r, int c) {
   return static_cast<uint32_t>((r >> 3) * 1024 + (r & 7) * 128 + ((c ^ (r & 7)) << 4));
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, 2)
     causal_attention_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                             const __grid_constant__ CUtensorMap tmV, const AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -292,14 +296,16 @@ __global__ void __launch_bounds__(kThreads, 1)
               make_uint4(hp[4 * u], hp[4 * u + 1], hp[4 * u + 2], hp[4 * u + 3]);
       }
       // O accumulated over the earlier chunks follows the new maximum (this
-      // warp's 32 columns of its lane group's rows)
+      // warp's 32-column chunks of its lane group's rows)
       if (c > 0 && __any_sync(0xFFFFFFFFu, alpha != 1.0f)) {
-        uint32_t r[32];
-        tmem_ld_32x32b_x32(trow + static_cast<uint32_t>(cq * 32), r);
-        tmem_ld_wait();
+        for (int oc = cq; oc < kDH / 32; oc += kStep) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(trow + static_cast<uint32_t>(oc * 32), r);
+          tmem_ld_wait();
 #pragma unroll
-        for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-        tmem_st_32x32b_x32(trow + static_cast<uint32_t>(cq * 32), r);
+          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+          tmem_st_32x32b_x32(trow + static_cast<uint32_t>(oc * 32), r);
+        }
         tmem_st_wait();
       }
       mrow = mnew;
@@ -341,21 +347,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
     for (int k = 1; k < kStep; ++k) sum += red[k * kBQ + row];
     const float inv = 1.0f / sum;
-    const int c0 = cq * 32;  // this warp's 32 head dimensions
-    uint32_t r[32];
-    tmem_ld_32x32b_x32(trow + static_cast<uint32_t>(c0), r);
-    tmem_ld_wait();
-    if (qpos < m) {
-      __half* orow = p.o + (static_cast<size_t>(b) * m + qpos) * p.ldo + h * kDH + c0;
-      uint32_t hv[16];
+    for (int c0 = cq * 32; c0 < kDH; c0 += kStep * 32) {  // this warp's 32-column chunks of head dimensions
+      uint32_t r[32];
+      tmem_ld_32x32b_x32(trow + static_cast<uint32_t>(c0), r);
+      tmem_ld_wait();
+      if (qpos < m) {
+        __half* orow = p.o + (static_cast<size_t>(b) * m + qpos) * p.ldo + h * kDH + c0;
+        uint32_t hv[16];
 #pragma unroll
-      for (int e = 0; e < 32; e += 2) {
-        const __half2 hh = __floats2half2_rn(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv);
-        hv[e >> 1] = *reinterpret_cast<const uint32_t*>(&hh);
+        for (int e = 0; e < 32; e += 2) {
+          const __half2 hh = __floats2half2_rn(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv);
+          hv[e >> 1] = *reinterpret_cast<const uint32_t*>(&hh);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          *reinterpret_cast<uint4*>(orow + 8 * u) =
+              make_uint4(hv[4 * u], hv[4 * u + 1], hv[4 * u + 2], hv[4 * u + 3]);
       }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        *reinterpret_cast<uint4*>(orow + 8 * u) = make_uint4(hv[4 * u], hv[4 * u + 1], hv[4 * u + 2], hv[4 * u + 3]);
     }
   }
   tc_fence_before();
