@@ -560,6 +560,7 @@ def run_gpu(args, rank, world, local_rank):
             torch.cuda.synchronize()
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
+            t_host = time.perf_counter()
             a.record(main)
             copy.wait_event(a)
             h2d(0)
@@ -579,9 +580,11 @@ def run_gpu(args, rank, world, local_rank):
                     copied[i].record(copy)
             main.wait_stream(copy)
             b.record(main)
+            host_ms = (time.perf_counter() - t_host) * 1e3 / E  # enqueueing only: nothing waited on yet
             torch.cuda.synchronize()
         step.V, step.Q, step.A, step.text, step.idx = sets[0]
         e2e_ms = a.elapsed_time(b) / E
+        e2e_host_ms = host_ms
         # every step had the same inputs and the kernels are deterministic: the
         # two result buffers must agree bit for bit (a race in the overlap would not)
         if E >= 2 and not (torch.equal(outYs[0], outYs[1]) and torch.equal(outIs[0], outIs[1])):
@@ -650,6 +653,7 @@ def run_gpu(args, rank, world, local_rank):
                                 "neighbouring steps' compute; total time / steps, no L2 flush (each step moves more "
                                 "than the L2 holds)",
                       "serial_ms_per_step": round(e2e_serial_ms, 4),
+                      "host_enqueue_ms_per_step": round(e2e_host_ms, 4),
                       "serial_value": round(whole_job_tops(ops, world, e2e_serial_ms), 3)}
     if not args.no_cpu_baseline and world == 1:
         rec["cpu_baseline"] = cpu_baseline(w, args.cpu_threads)
