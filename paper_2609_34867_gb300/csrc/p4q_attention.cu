@@ -12,7 +12,8 @@
 //   1. thread 0 loads the query block once, and per key chunk the keys and
 //      values by TMA into 128-byte swizzled tiles (after the previous chunk's
 //      P V has released them), and issues S = Q K^T on the tensor cores
-//      (tcgen05 kind::f16, fp32 accumulators in TMEM columns 128 .. 383);
+//      (tcgen05 kind::f16, N = the chunk's keys, fp32 accumulators in TMEM
+//      columns 128 ..);
 //   2. every thread takes an 8 x 8 block of the staged values into registers
 //      and, after a block-wide barrier, writes it back transposed, so that
 //      each 64-key tile becomes K-major V^T (keys at or past m are zero);
@@ -191,17 +192,16 @@ __global__ void __launch_bounds__(kThreads, 2)
       }
       if (pok) {
         tc_fence_after();
-        constexpr uint32_t idesc = idesc_f16_f32(kBQ, kKeyBlock);
-        for (int n0 = 0; n0 < nc; n0 += kKeyBlock) {
+        // one MMA per 16 head dimensions covers the whole chunk (N = nc keys)
+        const uint32_t idesc = idesc_f16_f32(kBQ, nc);
 #pragma unroll
-          for (int kb = 0; kb < 2; ++kb) {
-            const uint32_t a0 = smem_u32(sQ + kb * kTileBytes);
-            const uint32_t b0 = smem_u32(sKP + kb * (kChunk * 128) + n0 * 128);
+        for (int kb = 0; kb < 2; ++kb) {
+          const uint32_t a0 = smem_u32(sQ + kb * kTileBytes);
+          const uint32_t b0 = smem_u32(sKP + kb * (kChunk * 128));
 #pragma unroll
-            for (int k = 0; k < 4; ++k)
-              mma_f16(tmem + kS + static_cast<uint32_t>(n0), sw128_kmajor_desc(a0 + k * 32),
-                      sw128_kmajor_desc(b0 + k * 32), idesc, (kb | k) != 0 ? 1u : 0u);
-          }
+          for (int k = 0; k < 4; ++k)
+            mma_f16(tmem + kS, sw128_kmajor_desc(a0 + k * 32), sw128_kmajor_desc(b0 + k * 32), idesc,
+                    (kb | k) != 0 ? 1u : 0u);
         }
         mma_commit(s_bar);
       }
