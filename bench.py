@@ -1,8 +1,9 @@
 """Benchmark of the P4Q pruned W4A4 hot path on GB300.
 
-One step = the whole path over one batch of the LLaVA-1.5-7B-shaped workload
-(8 images x 576 visual tokens of 4096 fp16 features + 64 text tokens each,
-budget 192 kept tokens per image):
+One step = the whole path over one batch of the LLaVA-NeXT-13B-shaped workload
+(32 images x 2880 visual tokens of 5120 fp16 features, heavy-tailed outlier
+channels, + 64 text tokens each, budget 640 kept tokens per image; the
+largest of the LLaVA-shaped workloads, and one GPU holds it):
   p4q_select_gather_quant  fake-quant -> query / saliency / diversity stages
                            -> gather of the kept FP16 rows + text -> INT4
   (the selector's gather and the two re-quantizations also write their
@@ -12,7 +13,7 @@ budget 192 kept tokens per image):
                            start of the step
   p4q_w4a4_linear_expanded x 3  q|k|v|gate|up (one GEMM over the
                            concatenated output channels) on the pruned
-                           sequence (M = 2048), o on the re-quantized q
+                           sequence (M = 22528), o on the re-quantized q
                            output, down on the re-quantized up output
                            (2 x p4q_quant_act_expanded on column blocks;
                            the o chain on a third stream beside the
@@ -25,9 +26,9 @@ selector's share is also reported as microseconds per image.
                   [--workload NAME]
 
 --workload runs the same step on another of the LLaVA-shaped workloads (the
-one-image 576-token case, the 16 x 2880-token LLaVA-NeXT-7B batch over 32
-decoder layers, the 32 x 2880-token LLaVA-NeXT-13B batch); the default is the
-8-image batch above.
+one-image 576-token case, the 8 x 576-token LLaVA-1.5-7B batch, the
+16 x 2880-token LLaVA-NeXT-7B batch over 32 decoder layers); the default is
+the 32-image batch above.
 
 --impl reference times the CPU oracle (test infrastructure) on a bounded
 sample of the same workload. Under torchrun each rank runs its own batch
@@ -52,7 +53,7 @@ if ROOT not in sys.path:
 from paper_2609_34867_gb300 import workloads as wl  # noqa: E402
 
 METRIC = "W4A4 prefill linear TOPS (% INT8 tensor peak); select+prune µs/image"
-WORKLOAD = wl.LLAVA15_7B
+WORKLOAD = wl.LLAVANEXT_13B
 FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed steps
 
 # Latest ncu capture of the dominant kernel (the expanded-operand GEMM): mean
@@ -103,13 +104,51 @@ def measured_peaks():
 
 
 def fp8_peak_tops(sustained: bool):
-    """Dense FP8 tensor peak: the measured bf16 peak x the nominal fp8 / bf16 ratio (4.5 / 2.25)."""
+    """Dense FP8 tensor peak derived from the measured bf16 cuBLAS rate: x the
+    nominal fp8 / bf16 ratio (4.5 / 2.25). Reported beside the FP8 rate this
+    run measures itself (p4q_peak_probe), which is the roofline's peak."""
     pk = measured_peaks()
     if pk:
         bf = pk.get("bf16_tflops_sustained" if sustained else "bf16_tflops")
         return 2.0 * bf, ("measured bf16 %s x 2 (nominal fp8/bf16 ratio), MEASURED_PEAKS.json"
                           % ("sustained" if sustained else "burst"))
     return 2.0 * (1700.0 if sustained else 1900.0), "fallback bf16 x 2"
+
+
+def hbm_peak_gbs():
+    pk = measured_peaks()
+    if pk and pk.get("hbm_gbs"):
+        return float(pk["hbm_gbs"]), "measured copy, MEASURED_PEAKS.json"
+    return 6800.0, "fallback 6.8 TB/s"
+
+
+def select_budget(w: wl.Workload):
+    """(K_q, K_s, K_d) of Sec. 3.2's split in integers (concepts and CLS
+    saliency present in every bench workload)."""
+    kq = 300 * w.K // 1000
+    ks = 200 * w.K // 1000
+    return kq, ks, w.K - kq - ks
+
+
+def selector_roofline(w: wl.Workload, us_per_image: float, hbm_gbs: float, f8_tops: float) -> dict:
+    """Select + prune per image against the larger of its two bounds:
+    - HBM: one read of the image's features, its text rows and its kept rows
+      (the gather), and the codes of the pruned sequence written:
+      (N d 2 + T d 2 + K d 2 + (K + T)(d / 2 + 4)) bytes at the measured copy
+      bandwidth;
+    - diversity MACs on the FP8 tensor pipe: (K_q + K_s) N d for the initial
+      maxima plus sum over the K_d greedy rounds of the free tokens' d-long
+      dot products, 2 ops each, at the FP8 rate measured in this run."""
+    kq, ks, kd = select_budget(w)
+    nbytes = w.N * w.d * 2 + w.T * w.d * 2 + w.K * w.d * 2 + (w.K + w.T) * (w.d // 2 + 4)
+    macs = (kq + ks) * w.N * w.d + sum((w.N - kq - ks - t) * w.d for t in range(kd))
+    hbm_us = nbytes / (hbm_gbs * 1e3)
+    mac_us = 2.0 * macs / (f8_tops * 1e6)
+    bound = max(hbm_us, mac_us)
+    return {"bound": "hbm" if hbm_us >= mac_us else "tensor", "achieved_us_per_image": round(us_per_image, 3),
+            "bound_us_per_image": round(bound, 3), "frac": round(bound / us_per_image, 4),
+            "hbm_bytes_per_image": int(nbytes), "hbm_us_per_image": round(hbm_us, 3),
+            "diversity_macs_per_image": int(macs), "diversity_us_per_image": round(mac_us, 3)}
 
 
 # --------------------------------------------------------------------- clocks
@@ -454,6 +493,11 @@ def run_gpu(args, rank, world, local_rank):
         flush()
         step()
     torch.cuda.synchronize()
+    # the pipes' own rates on this GPU (untimed region): the roofline's FP8
+    # peak and the s8 basis of the metric's "% INT8 tensor peak"
+    from paper_2609_34867_gb300 import kernel_cases as kc
+    f8_tops = kc.peak_tops("f8", dev)
+    s8_tops = kc.peak_tops("s8", dev)
 
     # ---- device-timed region: K graph replays, L2 flushed before each, events
     # around each replay; per-kernel times from the events inside the graph
@@ -598,10 +642,16 @@ def run_gpu(args, rank, world, local_rank):
     ops = linear_ops(w)
     ms_per_step = total_ms / args.steps
     value = whole_job_tops(ops, world, ms_per_step)
-    # the burst peak unless the clocks show the power cap throttling the loop
+    # the roofline's peak: the FP8 MMA-only rate measured above; the bf16-derived
+    # figure (burst unless the clocks show the power cap) is reported beside it
     sustained = bool(clk and "sw_power_cap" in clk["reasons"])
-    peak, peak_src = fp8_peak_tops(sustained)
+    peak_bf, peak_bf_src = fp8_peak_tops(sustained)
+    peak = f8_tops
+    hbm_gbs, hbm_src = hbm_peak_gbs()
     ach = gemm_ops / (gemm_time_ms * 1e-3) / 1e12
+    exp_time_ms = float(np.mean(exp_ms))
+    ach_lin = gemm_ops / ((gemm_time_ms + exp_time_ms) * 1e-3) / 1e12
+    sel_us = float(sel_ms.mean()) * 1e3 / w.B
     n_gemm = len(step.gemms) * w.layers * args.steps
     traffic = None
     if PROFILED_GEMM["source_sha1"] == gemm_source_sha1():
@@ -627,15 +677,26 @@ def run_gpu(args, rank, world, local_rank):
             "timing": "CUDA events around each step (one CUDA graph per step), summed over the K steps; "
                       "selector and per-GEMM times from segment graphs with events between them",
             "parallelism": f"dp{world} (independent batches)"},
-        "select_prune_us_per_image": round(float(sel_ms.mean()) * 1e3 / w.B, 3),
-        "expand_us_per_step": round(float(np.mean(exp_ms)) * 1e3, 2),
+        "select_prune_us_per_image": round(sel_us, 3),
+        "select_prune_roofline": selector_roofline(w, sel_us, hbm_gbs, f8_tops),
+        "expand_us_per_step": round(exp_time_ms * 1e3, 2),
         "requant_us_per_step": round(float(np.mean(quant_ms)) * 1e3, 2),
         "gemm_tops": round(ach, 3),
-        "pct_int8_tensor_peak": None,
+        "pct_int8_tensor_peak": round(100.0 * ach / s8_tops, 2),
+        "pct_int8_tensor_peak_basis": "mma.sync m16n8k32 s8 x s8 -> s32 loop measured in this run "
+                                      "(p4q_peak_probe kind 1): %.1f TOPS" % s8_tops,
         "pct_fp8_tensor_peak": round(100.0 * ach / peak, 2),
+        "peaks_measured": {"f8_tcgen05_tops": round(f8_tops, 1), "s8_mma_sync_tops": round(s8_tops, 1),
+                           "fp8_from_bf16_tops": round(peak_bf, 1), "fp8_from_bf16_source": peak_bf_src,
+                           "hbm_gbs": hbm_gbs, "hbm_source": hbm_src},
+        "linear_incl_expand": {"achieved": round(ach_lin, 3), "unit": "TFLOP/s", "frac": round(ach_lin / peak, 4),
+                               "note": "the GEMM kernels' time plus the per-call expansion of their packed "
+                                       "INT4 weights (p4q_expand_codes), as if not overlapped"},
         "roofline": {"bound": "tensor", "kernel": "w4a4_gemm8_pair_kernel (tcgen05 kind::f8f6f4, cta_group::2, TMA-fed expanded operands)",
                      "achieved": round(ach, 3), "peak": round(peak, 1), "unit": "TFLOP/s",
-                     "frac": round(ach / peak, 4), "traffic": traffic, "peak_source": peak_src,
+                     "frac": round(ach / peak, 4), "traffic": traffic,
+                     "peak_source": "measured in this run: tcgen05 kind::f8f6f4 MMA-only loop on operands in "
+                                    "shared memory, 76 CTA pairs (p4q_peak_probe kind 0)",
                      "launches_timed": n_gemm,
                      "note": "integer ops on the FP8 tensor pipe; sm_103a has no integer tcgen05 MMA kind",
                      "per_gemm_us": {n: round(float(np.mean(v)) * 1e3, 2) for n, v in gemm_ms.items()}},
@@ -723,18 +784,23 @@ class OracleSampler:
 
 def cpu_baseline(w: wl.Workload, threads: int, reps: int = 2):
     s = OracleSampler(w, threads)
+    timed = []
     for _ in range(reps):
         for i in range(len(s.pieces)):
-            s.run_piece(i)
+            timed.append(s.run_piece(i))
     est = s.estimate()
     return {"value": round(linear_ops(w) / est / 1e12, 6), "unit": "TOPS", "cores": s.cores, "kind": "oracle",
-            "sample": s.describe(), "est_step_s": round(est, 3)}
+            "sample": s.describe(), "pieces_timed": len(timed),
+            "ms_per_piece": round(float(np.mean(timed)) * 1e3, 3), "est_step_s": round(est, 3)}
 
 
 def run_reference(args, rank):
-    """The oracle as it stands: each step runs one piece of the workload (round
-    robin over the selector and the seven linears); the reported step time is
-    the sum of the pieces' mean times scaled to the full workload."""
+    """The oracle as it stands, on the host cores: W untimed pieces, then
+    exactly K timed pieces, each one bounded piece of the workload (round robin
+    over the selector of one image and the seven linears on a few rows).
+    `steps` and `ms_per_step` describe those pieces as they ran; `value` is the
+    throughput of the full step estimated from each piece's mean time
+    (`est_step_s`, scaled to the whole workload)."""
     if rank != 0:
         return None
     w = wl.WORKLOADS[args.workload]
@@ -742,18 +808,27 @@ def run_reference(args, rank):
     n = len(s.pieces)
     for i in range(args.warmup):
         s.run_piece(i)
+    warm = {i: list(v) for i, v in s.times.items()}
     s.times = {i: [] for i in range(n)}
-    for i in range(max(args.steps, n)):
-        s.run_piece(i)
+    timed = []
+    for i in range(args.steps):
+        timed.append(s.run_piece(args.warmup + i))
+    for i in range(n):  # a piece the timed round robin did not reach: its warm-up time, else one more run
+        if not s.times[i]:
+            s.times[i] = warm[i] or [s.run_piece(i)]
     est = s.estimate()
     value = linear_ops(w) / est / 1e12
+    ms_piece = float(np.mean(timed)) * 1e3
     return {
         "metric": METRIC, "value": round(value, 6), "unit": "TOPS", "n_gpus": args.gpus, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(est * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": round(ms_piece, 3), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int4", "data": "synthetic", "impl": "reference",
         "config": {"workload": w.name, "B": w.B, "N": w.N, "d": w.d, "K": w.K, "T": w.T, "J": w.J, "M": w.M},
+        "est_step_s": round(est, 3),
+        "step_note": "each of the K steps is one piece of the workload (steps and ms_per_step describe the pieces "
+                     "that ran); value = the full step's integer ops / est_step_s",
         "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": s.cores, "kind": "oracle",
-                         "sample": "each step one piece: " + s.describe()},
+                         "sample": "each step one piece: " + s.describe(), "est_step_s": round(est, 3)},
         "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
@@ -765,7 +840,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["p4q", "reference"], default="p4q")
     ap.add_argument("--workload", choices=sorted(wl.WORKLOADS), default=WORKLOAD.name,
-                    help="workload of the step (default: the 8-image LLaVA-1.5-7B batch)")
+                    help="workload of the step (default: the 32-image LLaVA-NeXT-13B batch)")
     ap.add_argument("--e2e-steps", type=int, default=50)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-threads", type=int, default=0, help="oracle threads (0 = all cores)")

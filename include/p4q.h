@@ -109,6 +109,26 @@ p4q_status p4q_set_gemm_variant(int variant);
  * Asynchronous on `stream`. */
 p4q_status p4q_test_wait_timeout(uint32_t limit_us, p4q_stream_t stream);
 
+/* Throughput probe for the roofline denominators of the integer
+ * contractions. The paper has no counterpart: the W4A4 GEMM runs its exact
+ * integer products on the FP8 tensor pipe (sm_103a has no integer tcgen05
+ * MMA kind), and these loops measure what each candidate pipe sustains on
+ * this GPU, with operands that stay on chip:
+ *   kind 0  tcgen05.mma kind::f8f6f4 (E4M3 x E4M3 -> F32, M 256 x N 256 x
+ *           K 32 per instruction, one CTA pair per two SMs), iters x 4 MMAs
+ *           per pair;
+ *   kind 1  mma.sync m16n8k32 s8 x s8 -> s32, 8 independent accumulators per
+ *           warp, 32 warps per SM, iters rounds;
+ *   kind 2  dp4a (s8 x 4 -> s32), 8 chains per thread, iters rounds.
+ *   iters   1 .. 2^24
+ *   sink    device buffer of at least 8192 uint32 (written only by a result
+ *           that never occurs in practice; it keeps the work live)
+ *   ops     HOST pointer: receives the number of operations the launch
+ *           performs (2 per multiply-add)
+ * Time the call with CUDA events on `stream`; ops / time is the rate.
+ * Asynchronous; P4Q_ERR_INVALID_ARG for other kinds or iters. */
+p4q_status p4q_peak_probe(int kind, int iters, uint32_t* sink, double* ops, p4q_stream_t stream);
+
 /* ---------------------------------------------------------------------- */
 /* Per-row 4-bit quantizers (App. A, App. B.3)                             */
 /* ---------------------------------------------------------------------- */

@@ -242,7 +242,7 @@ p4q_status p4q_set_gemm_variant(int variant) {
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
   const unsigned int g = gemm_read_and_clear_error() | gemm8_read_and_clear_error() | quant_read_and_clear_error() |
-                         attn_read_and_clear_error();
+                         attn_read_and_clear_error() | peak_read_and_clear_error();
   if (cudaGetLastError() != cudaSuccess) return P4Q_ERR_CUDA;
   return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
 }
@@ -252,6 +252,15 @@ p4q_status p4q_test_wait_timeout(uint32_t limit_us, p4q_stream_t stream) {
   p4q_status st = check_device();
   if (st != P4Q_OK) return st;
   return from_cuda(counted(launch_expired_wait(1000ull * limit_us, reinterpret_cast<cudaStream_t>(stream))));
+}
+
+p4q_status p4q_peak_probe(int kind, int iters, uint32_t* sink, double* ops, p4q_stream_t stream) {
+  if (kind < 0 || kind > 2 || iters < 1 || iters > (1 << 24) || !sink || !ops) return P4Q_ERR_INVALID_ARG;
+  if (!aligned16(sink)) return P4Q_ERR_MISALIGNED;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  if (static_cast<size_t>(num_sms()) * 4 > peak_probe_sink_words()) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  return from_cuda(counted(launch_peak_probe(kind, iters, sink, ops, reinterpret_cast<cudaStream_t>(stream))));
 }
 
 p4q_status p4q_quant_act(const uint16_t* X, int M, int Kin, uint8_t* Xq, float* s_a, p4q_stream_t stream) {

@@ -203,6 +203,13 @@ cudaError_t launch_expand_codes(const uint8_t* q, int rows, int K, uint8_t* u, i
 cudaError_t launch_gemm8(const GemmArgs& g, const uint8_t* a8, const int32_t* sum_a, const uint8_t* b8,
                          const int32_t* sum_b, cudaStream_t stream);
 
+// Throughput probes of the integer contraction pipes (roofline denominators):
+// kind 0 tcgen05 kind::f8f6f4 MMAs, 1 mma.sync m16n8k32 s8, 2 dp4a; *ops is the
+// number of integer (or FP8) operations the launch performs.
+cudaError_t launch_peak_probe(int kind, int iters, uint32_t* sink, double* ops, cudaStream_t stream);
+size_t peak_probe_sink_words();
+unsigned int peak_read_and_clear_error();
+
 // One bounded wait that nothing completes: times out after limit_ns and sets
 // the GEMM's device error word (tests the time-out path).
 cudaError_t launch_expired_wait(unsigned long long limit_ns, cudaStream_t stream);

@@ -11,6 +11,7 @@
   python -m paper_2609_34867_gb300.kernel_cases attn B M H [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases mse B M D [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases topk B N K [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases peak {f8,s8,dp4a} ITERS [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -38,6 +39,10 @@ selects the first replayed launch.
           causal Q K^T and P V; bytes: q, k, v in, o out, fp16);
   mse     p4q_block_mse on B samples of M rows x D fp16 (bytes: 4 B M D in);
   topk    p4q_topk_replacement on B x N fp32 score pairs (bytes: 8 B N in);
+  peak    p4q_peak_probe: the throughput loop of one integer contraction
+          pipe (f8: tcgen05 kind::f8f6f4 MMAs on operands in shared memory;
+          s8: mma.sync m16n8k32 s8; dp4a), ITERS rounds (ops = 2 per
+          multiply-add, as counted by the probe);
   saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
           heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
           fp16 keys and queries in, 4 B N out).
@@ -81,9 +86,34 @@ def _timed(fn, reps, dev):
     return total / reps
 
 
+PEAK_ITERS = {"f8": 60000, "s8": 20000, "dp4a": 40000}  # a few tens of milliseconds per launch
+
+
+def peak_tops(kind: str, dev, reps: int = 5, iters: int | None = None) -> float:
+    """Best rate in TOPS of `reps` timed launches of one throughput probe
+    (p4q_peak_probe) on `dev`, after one untimed launch."""
+    sink = torch.zeros((8192,), dtype=torch.int32, device=dev)
+    it = iters or PEAK_ITERS[kind]
+    p4q.p4q_peak_probe(kind, it, sink)
+    torch.cuda.synchronize()
+    best = 0.0
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        ops = p4q.p4q_peak_probe(kind, it, sink)
+        b.record()
+        torch.cuda.synchronize()
+        best = max(best, ops / (a.elapsed_time(b) * 1e-3) / 1e12)
+    status = p4q.p4q_device_status()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after the peak probe")
+    return best
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn", "mse", "topk"])
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn",
+                                     "mse", "topk", "peak"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -181,6 +211,12 @@ def main(argv=None):
         rho = torch.empty((B,), dtype=torch.float32, device=dev)
         ms = _timed(lambda: p4q.p4q_topk_replacement(s1, s2, K, inter, rho), a.reps, dev)
         print(f"topk {B}x{N} K={K}: {ms * 1e3:.1f} us/call, {8 * B * N / ms / 1e6:.1f} GB/s")
+    elif a.case == "peak":
+        kind, iters = a.args[0], int(a.args[1])
+        sink = torch.zeros((8192,), dtype=torch.int32, device=dev)
+        ops = p4q.p4q_peak_probe(kind, iters, sink)
+        ms = _timed(lambda: p4q.p4q_peak_probe(kind, iters, sink), a.reps, dev)
+        print(f"peak {kind} x{iters}: {ms * 1e3:.1f} us/call, {ops / ms / 1e9:.1f} TOPS")
     elif a.case == "saliency":
         B, N = (int(x) for x in a.args)
         v = wl.vision_attention(B, N, seed=0)

@@ -65,6 +65,8 @@ def lib() -> ctypes.CDLL:
         L.p4q_device_status.restype = st
         L.p4q_test_wait_timeout.argtypes = [ctypes.c_uint32, P]
         L.p4q_test_wait_timeout.restype = st
+        L.p4q_peak_probe.argtypes = [I, I, P, ctypes.POINTER(ctypes.c_double), P]
+        L.p4q_peak_probe.restype = st
         L.p4q_quant_act.argtypes = [P, I, I, P, P, P]
         L.p4q_quant_act.restype = st
         L.p4q_quant_act_ld.argtypes = [P, I, I, I, P, P, P]
@@ -140,6 +142,22 @@ def p4q_set_gemm_variant(variant: int):
 
 def p4q_device_status(stream=None) -> int:
     return int(lib().p4q_device_status(_stream(stream)))
+
+
+PEAK_KINDS = {"f8": 0, "s8": 1, "dp4a": 2}
+
+
+def p4q_peak_probe(kind: str, iters: int, sink, stream=None) -> float:
+    """Launches one throughput probe (f8: tcgen05 kind::f8f6f4 MMAs, s8:
+    mma.sync m16n8k32 s8, dp4a) on `stream`; returns the operations it performs.
+    sink: a CUDA int32 tensor of at least 8192 elements."""
+    _need(sink, torch.int32, 1, "sink")
+    if sink.numel() < 8192:
+        raise ValueError("sink: at least 8192 elements")
+    ops = ctypes.c_double(0.0)
+    _check(lib().p4q_peak_probe(PEAK_KINDS[kind], iters, _ptr(sink), ctypes.byref(ops), _stream(stream)),
+           "p4q_peak_probe")
+    return ops.value
 
 
 def p4q_quant_act(X, Xq, s_a, stream=None):

@@ -180,6 +180,18 @@ def test_wait_timeout_test_entry_validates_its_limit(lib):
     assert lib.p4q_test_wait_timeout(1000001, None) == 1
 
 
+def test_peak_probe_validates_its_arguments(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    lib.p4q_peak_probe.argtypes = [I, I, P, ctypes.POINTER(ctypes.c_double), P]
+    ops = ctypes.c_double(0.0)
+    assert lib.p4q_peak_probe(3, 10, P(16), ctypes.byref(ops), None) == 1        # unknown kind
+    assert lib.p4q_peak_probe(0, 0, P(16), ctypes.byref(ops), None) == 1         # no iterations
+    assert lib.p4q_peak_probe(1, 1 << 25, P(16), ctypes.byref(ops), None) == 1   # beyond the limit
+    assert lib.p4q_peak_probe(2, 10, None, ctypes.byref(ops), None) == 1         # no sink
+    assert lib.p4q_peak_probe(2, 10, P(16), None, None) == 1                     # no ops pointer
+    assert lib.p4q_peak_probe(2, 10, P(20), ctypes.byref(ops), None) == 3        # sink misaligned
+
+
 def test_strided_quantizer_validates_its_row_pitch(lib):
     P, I = ctypes.c_void_p, ctypes.c_int
     lib.p4q_quant_act_ld.argtypes = [P, I, I, I, P, P, P]
