@@ -71,7 +71,8 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
     if failed:
         raise RuntimeError(f"nvcc failed for {failed}")
     tmp = LIB + f".tmp{os.getpid()}"
-    subprocess.run([nvcc(), GENCODE, "-shared", "-o", tmp] + objs, check=True)
+    # every symbol resolved at link time (a missing definition fails here, not at load)
+    subprocess.run([nvcc(), GENCODE, "-shared", "-Xlinker", "--no-undefined", "-o", tmp] + objs, check=True)
     os.replace(tmp, LIB)
     return LIB
 

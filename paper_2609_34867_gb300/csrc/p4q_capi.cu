@@ -62,36 +62,16 @@ p4q_status check_select_args(const uint16_t* V, int B, int N, int d, int J, cons
   return P4Q_OK;
 }
 
-// A second stream of the library per device, with a fork and a join event,
-// for the stage-1/2 launch of the selector beside the cosine matrix; created
-// on the first call that is not being captured into a graph.
-struct SideStream {
-  cudaStream_t s = nullptr;
-  cudaEvent_t fork = nullptr, join = nullptr;
-  bool failed = false;
-};
-std::mutex g_side_mutex;
-SideStream g_side[64];
-
-SideStream* side_stream(cudaStream_t stream) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-  SideStream& r = g_side[dev];
-  if (r.s) return &r;
-  if (r.failed) return nullptr;
-  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
-  if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return nullptr;
-  if (cudaStreamCreateWithFlags(&r.s, cudaStreamNonBlocking) != cudaSuccess ||
-      cudaEventCreateWithFlags(&r.fork, cudaEventDisableTiming) != cudaSuccess ||
-      cudaEventCreateWithFlags(&r.join, cudaEventDisableTiming) != cudaSuccess) {
-    cudaGetLastError();
-    r.failed = true;  // the serial order is used from now on
-    r.s = nullptr;
-    return nullptr;
-  }
-  return &r;
+// R0 = Kq + Ks of a call (the workspace layout depends on it).
+int select_r0(const p4q_select_params& p, bool have_q, bool have_a) {
+  const Budget bud = split(p, have_q, have_a);
+  return bud.Kq + bud.Ks;
 }
 
+// The selector: fake-quantized copies (tokens and concepts in one launch),
+// query cosines, stages 1-2, the initial diversity maxima on the tensor cores
+// (R0's expanded codes gathered, then one GEMM with a max-cosine epilogue),
+// stage 3 (writes idx). Every launch on `stream`.
 p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
                       const p4q_select_params* params, int32_t* idx, void* ws, size_t ws_bytes,
                       cudaStream_t stream) {
@@ -99,89 +79,51 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   const int Jeff = have_q ? J : 0;
   if (have_q && !aligned16(Q)) return P4Q_ERR_MISALIGNED;
   if (A_cls && !aligned16(A_cls)) return P4Q_ERR_MISALIGNED;
-  const size_t need = select_workspace_layout(B, N, d, Jeff, nullptr, nullptr);
+  const Budget bud = split(*params, have_q, A_cls != nullptr);
+  const int R0 = bud.Kq + bud.Ks;
+  const size_t need = select_workspace_layout(B, N, d, Jeff, R0, nullptr, nullptr);
   if (!ws || ws_bytes < need) return P4Q_ERR_WORKSPACE_TOO_SMALL;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return P4Q_ERR_MISALIGNED;
   SelectWorkspace w;
-  select_workspace_layout(B, N, d, Jeff, &w, ws);
-  const Budget bud = split(*params, have_q, A_cls != nullptr);
+  select_workspace_layout(B, N, d, Jeff, R0, &w, ws);
   SelectPlan plan{B, N, d, Jeff, params->K, bud.Kq, bud.Ks, bud.Kd};
 
-  // Fake-quantized copies of the projector features (and the concepts).
+  // Fake-quantized copies of the projector features (and of the concepts):
+  // the codes expanded to one byte each (what the tensor-core stages read),
+  // their row sums and squared norms; then the code dot products of every
+  // token with its image's concepts on the tensor cores (the query cosines
+  // are taken from them in stages 1-2).
+  cudaError_t e;
   RowSource src;
   src.X = V;
   RowSinks sv;
-  sv.codes = w.vcodes;
   sv.scale = w.vscale;
   sv.norm2 = w.vnorm;
-  sv.u = w.vu;  // the expanded codes the cosine-matrix GEMM reads (large token sets)
+  sv.u = w.vu;
   sv.sum_u = w.vsum;
-  // the concept rows ride in the same launch, after the visual tokens
-  RowSinks oq;
-  oq.codes = w.qcodes;
-  oq.scale = w.qscale;
-  oq.norm2 = w.qnorm;
+  if ((e = counted(launch_quant_rows(src, B * N, d, sv, stream))) != cudaSuccess) return from_cuda(e);
   if (bud.Kq > 0) {
-    src.X2 = Q;
-    src.split = B * N;
+    RowSource qsrc;
+    qsrc.X = Q;
+    RowSinks oq;
+    oq.codes = w.qcodes;
+    oq.scale = w.qscale;
+    oq.norm2 = w.qnorm;
+    oq.u = w.qu;
+    oq.sum_u = w.qsum;
+    if ((e = counted(launch_quant_rows(qsrc, B * Jeff, d, oq, stream))) != cudaSuccess) return from_cuda(e);
+    if ((e = counted(launch_query_dots(plan, w, stream))) != cudaSuccess) return from_cuda(e);
   }
-  cudaError_t e = counted(launch_quant_rows(src, B * N + (bud.Kq > 0 ? B * Jeff : 0), d, sv, stream, &oq));
-  if (e != cudaSuccess) return from_cuda(e);
-  if (bud.Kq > 0) {
-    e = counted(launch_query_scores(plan, w, stream));
-    if (e != cudaSuccess) return from_cuda(e);
+  if (R0 > 0 || bud.Kd > 0) {
+    // stages 1-2 (also the bits of an empty R0, and idx when Kd = 0)
+    if ((e = counted(launch_select_stages12(plan, w, A_cls, idx, stream))) != cudaSuccess) return from_cuda(e);
   }
-  // Stages 1-2 (query relevance, saliency) need only the scores and A_cls:
-  // when the cosine-matrix GEMM leaves an SM per image free, they run on the
-  // side stream beside it and stage 3 starts from their kept set.
-  std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
-  SideStream* side = nullptr;
-  if (bud.Kd > 0 && (bud.Kq > 0 || bud.Ks > 0) && w.vu != nullptr && select_split_applies(N)) {
-    if (num_sms() - 2 * gemm8_pairs(N, N, B, num_sms()) >= B) {
-      side_lock.lock();
-      side = side_stream(stream);
-      if (!side) side_lock.unlock();
-    }
+  if (bud.Kd == 0) return P4Q_OK;
+  if (R0 > 0) {
+    if ((e = counted(launch_gather_r0(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+    if ((e = counted(launch_r0_cosmax(plan, w, stream), 2)) != cudaSuccess) return from_cuda(e);  // GEMM + row pass
   }
-  if (side) {
-    cudaError_t se = cudaEventRecord(side->fork, stream);
-    if (se == cudaSuccess) se = cudaStreamWaitEvent(side->s, side->fork, 0);
-    if (se == cudaSuccess) se = counted(launch_select_stages(plan, w, A_cls, idx, side->s, 1));
-    if (se == cudaSuccess) se = cudaEventRecord(side->join, side->s);
-    if (se != cudaSuccess) return from_cuda(se);
-  }
-  if (bud.Kd > 0) {
-    GemmArgs g;
-    g.A = w.vcodes;
-    g.B = w.vcodes;
-    g.M = N;
-    g.N = N;
-    g.K = d;
-    g.batch = B;
-    g.a_batch_stride = N;
-    g.b_batch_stride = N;
-    g.D = w.gram;
-    g.d_pitch = w.gram_pitch;
-    g.norm_a = w.vnorm;
-    g.norm_b = w.vnorm;
-    // Then the cosine of every entry by a full-GPU elementwise pass (the
-    // division and square root would otherwise serialize in the GEMM's four
-    // epilogue warps). Small token sets: the cosine epilogue of the
-    // single-CTA GEMM on the packed codes.
-    // Large token sets: exact int32 dot products of the expanded codes (written
-    // by the fake-quantization above) on the TMA-fed CTA-pair GEMM.
-    const bool split = w.vu != nullptr;
-    g.out = split ? GemmOut::kS32 : GemmOut::kCos;
-    e = counted(split ? launch_gemm8(g, w.vu, w.vsum, w.vu, w.vsum, stream) : launch_w4a4_gemm(g, stream));
-    if (e != cudaSuccess) return from_cuda(e);
-    if (split && (e = counted(launch_gram_cos(plan, w, stream))) != cudaSuccess) return from_cuda(e);
-  }
-  if (side) {
-    e = cudaStreamWaitEvent(stream, side->join, 0);
-    if (e != cudaSuccess) return from_cuda(e);
-    return from_cuda(counted(launch_select_stages(plan, w, A_cls, idx, stream, 2)));
-  }
-  return from_cuda(counted(launch_select_stages(plan, w, A_cls, idx, stream)));
+  return from_cuda(counted(launch_select_diverse(plan, w, idx, stream)));
 }
 
 p4q_status check_rows(const void* X, int M, int Kin, const void* Xq, const void* s) {
@@ -242,7 +184,7 @@ p4q_status p4q_set_gemm_variant(int variant) {
 p4q_status p4q_device_status(p4q_stream_t stream) {
   if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) return P4Q_ERR_CUDA;
   const unsigned int g = gemm_read_and_clear_error() | gemm8_read_and_clear_error() | quant_read_and_clear_error() |
-                         attn_read_and_clear_error() | peak_read_and_clear_error();
+                         attn_read_and_clear_error() | peak_read_and_clear_error() | diverse_read_and_clear_error();
   if (cudaGetLastError() != cudaSuccess) return P4Q_ERR_CUDA;
   return g ? P4Q_ERR_TIMEOUT : P4Q_OK;
 }
@@ -516,7 +458,8 @@ size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_p
   if (!params || B < 1 || N < 1 || d < 1 || J < 0 || N > P4Q_MAX_TOKENS || J > P4Q_MAX_CONCEPTS ||
       d % 128 != 0 || d > P4Q_MAX_ROW || params->K < 1 || params->K > N)
     return 0;
-  return select_workspace_layout(B, N, d, J, nullptr, nullptr);
+  // the largest R0 a call with these sizes can have: concepts and CLS saliency present
+  return select_workspace_layout(B, N, d, J, select_r0(*params, J > 0, true), nullptr, nullptr);
 }
 
 p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
@@ -586,23 +529,15 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = P4Q_NOALLOC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_select_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_scratch_mutex;
-void* g_scratch_ptr[kMaxDevices] = {};
-
-// Device address of g_select_scratch on the current device (looked up once per
-// device, with that device current). Host code cannot use the symbol itself:
-// in host code it names a host-side placeholder, not device memory.
+// Device address of g_select_scratch in the current context. Host code cannot
+// use the symbol itself: in host code it names a host-side placeholder, not
+// device memory. The address is looked up on every call (a host-side table
+// read once the module is loaded), so it stays right after cudaDeviceReset or
+// under another context of the same device.
 p4q_status scratch_address(void** out) {
-  int dev = -1;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return P4Q_ERR_NO_DEVICE;
-  std::lock_guard<std::mutex> lock(g_scratch_mutex);
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* ptr = nullptr;
-    if (cudaGetSymbolAddress(&ptr, g_select_scratch) != cudaSuccess || ptr == nullptr) return P4Q_ERR_CUDA;
-    g_scratch_ptr[dev] = ptr;
-  }
-  *out = g_scratch_ptr[dev];
+  void* ptr = nullptr;
+  if (cudaGetSymbolAddress(&ptr, g_select_scratch) != cudaSuccess || ptr == nullptr) return P4Q_ERR_CUDA;
+  *out = ptr;
   return P4Q_OK;
 }
 
@@ -613,10 +548,12 @@ extern "C" p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d,
                                          p4q_stream_t stream) {
   p4q_status st = check_select_args(V, B, N, d, J, params, idx);
   if (st != P4Q_OK) return st;
-  const int Jeff = (Q != nullptr && J > 0) ? J : 0;
+  const bool have_q = (Q != nullptr && J > 0);
+  const int Jeff = have_q ? J : 0;
   // Every region of the scratch is written before it is read on each call, so
   // nothing needs clearing between calls.
-  if (select_workspace_layout(B, N, d, Jeff, nullptr, nullptr) > kNoAllocScratchBytes)
+  if (select_workspace_layout(B, N, d, Jeff, select_r0(*params, have_q, A_cls != nullptr), nullptr, nullptr) >
+      kNoAllocScratchBytes)
     return P4Q_ERR_WORKSPACE_TOO_SMALL;
   if ((st = check_device()) != P4Q_OK) return st;
   void* ws = nullptr;

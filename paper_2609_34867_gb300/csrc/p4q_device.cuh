@@ -316,6 +316,48 @@ __host__ __device__ constexpr uint32_t idesc_e4m3_f32(int M, int N) {
          | (static_cast<uint32_t>(M >> 4) << 24);  // M / 16
 }
 
+// Cosine of two fake-quantized rows from their codes (Sec. 3.2, Eq. 4; the
+// positive per-row scales cancel): the integer dot product over the square
+// root of the product of the squared code norms, each operation rounded to
+// fp32 in that order; 0 when a norm is 0.
+__device__ __forceinline__ float code_cosine(int dot, int na, int nb) {
+  if (na == 0 || nb == 0) return 0.0f;
+  return __fdiv_rn(static_cast<float>(dot), __fsqrt_rn(__fmul_rn(static_cast<float>(na), static_cast<float>(nb))));
+}
+
+// Largest Eq. 4 cosine of one row over many columns, exactly as code_cosine
+// would give it, in two passes: cos_approx = fl(dot) * rsqrtf(fl(na * nb))
+// is within 5e-7 of the exact cosine (|cos| <= 1; fl(dot) exact for |dot| <
+// 2^24; the product, the 2-ulp reciprocal square root and the last
+// multiplication each add at most a few 2^-24 relative), so the column of the
+// exact maximum has an approximation within kCosMargin of the largest
+// approximation, and only the columns that do are evaluated exactly (usually
+// one per row: the correctly rounded division and square root stay off the
+// common path, and off the warp's divergent path).
+constexpr float kCosMargin = 4e-6f;
+
+__device__ __forceinline__ float cos_approx(int dot, int na, int nb) {
+  const float p = __fmul_rn(static_cast<float>(na), static_cast<float>(nb));
+  return (na == 0 || nb == 0) ? 0.0f : static_cast<float>(dot) * rsqrtf(p);
+}
+
+// ---------------------------------------------------------------- cp.async (16-byte, generic proxy)
+// Asynchronous 16-byte copy global -> shared by this thread (L2 only).
+__device__ __forceinline__ void cp_async16(uint32_t smem_dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Waits until at most N of this thread's committed cp.async groups are pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Prefetches `bytes` (a multiple of 16) at a 16-byte aligned address into L2.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(bytes) : "memory");
+}
+
 // fp32 order-preserving map to uint32 (larger float -> larger key).
 __device__ __forceinline__ uint32_t float_order_key(float f) {
   uint32_t b = __float_as_uint(f);

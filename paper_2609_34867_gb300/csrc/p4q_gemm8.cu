@@ -18,6 +18,9 @@
 // Operands [batch][rows][K] (row-contiguous, batch entries back to back),
 // row sums [batch][rows], output [batch][M][pitch].
 //
+// int32 tiles may be narrower than 256 columns (p.bn, a multiple of 32): the
+// selector's products of every token with its few kept tokens.
+//
 // Kernel: persistent, one cluster of two CTAs per 256 x 256 output tile,
 //   warp 0    MMA issuer (leader CTA): 4 x tcgen05.mma (M 256, N 256, K 32)
 //             per 128-deep k-block into one of two TMEM accumulators;
@@ -55,6 +58,8 @@ constexpr int kMinRows = 512;           // smaller M: the in-kernel unpack path 
 struct Params8 {
   int M, N, K, batch;
   int num_m, num_n, per, tiles;  // per: tiles per batch entry
+  int bn;                        // int32 tiles: output columns per pair tile (<= BN)
+  int f32_out;                   // int32 tiles: store the exact integers as fp32 values instead
   const float* s_a;
   const float* s_b;
   const int32_t* sum_a;  // [batch, M] sum of u over each A row
@@ -77,6 +82,22 @@ struct Lay8 {
   static_assert(S >= 3, "TMA stages");
   static_assert(SMEM <= 232448, "shared memory budget");
 };
+
+// Tile t -> (batch entry, row tile, column tile). Row tiles vary fastest,
+// except for narrow int32 tiles (bn < BN: a few column tiles over a short B),
+// whose column tiles vary fastest, so that the pairs reading the same A rows
+// run side by side and those rows come from DRAM once.
+__device__ __forceinline__ void tile_coords(const Params8& p, int t, int* bz, int* mt, int* nb) {
+  *bz = t / p.per;
+  const int r = t - *bz * p.per;
+  if (p.bn < BN) {
+    *mt = r / p.num_n;
+    *nb = r - *mt * p.num_n;
+  } else {
+    *nb = r / p.num_m;
+    *mt = r - *nb * p.num_m;
+  }
+}
 
 __device__ __forceinline__ void epi_sync8() {
   asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory");
@@ -114,6 +135,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   const int KB = p.K / BK;
+  const int bn = (MODE == static_cast<int>(GemmOut::kS32)) ? p.bn : BN;  // columns of a pair tile
+  const int hb = bn / 2;                                                  // B rows per CTA
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
@@ -141,7 +164,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     // ------------------------------------------------------------ MMA issuer (leader)
     if (lane == 0 && rank == 0) {
-      constexpr uint32_t idesc = idesc_e4m3_f32(2 * BM, BN);
+      const uint32_t idesc = idesc_e4m3_f32(2 * BM, bn);
       int g = 0, it = 0;
       bool ok = true;
       for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x(), ++it) {
@@ -177,16 +200,17 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       int g = 0;
       bool ok = true;
       for (int t = cluster_id_x(); t < p.tiles && ok; t += nclusters_x()) {
-        const int bz = t / p.per, r = t - bz * p.per, nb = r / p.num_m;
-        const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
-        const int n0 = nb * BN + static_cast<int>(rank) * HB;                       // this CTA's B rows
+        int bz, mt, nb;
+        tile_coords(p, t, &bz, &mt, &nb);
+        const int m0 = mt * (2 * BM) + static_cast<int>(rank) * BM;  // this CTA's A rows
+        const int n0 = nb * bn + static_cast<int>(rank) * hb;                       // this CTA's B rows
         for (int kb = 0; kb < KB; ++kb, ++g) {
           const int s = g % S;
           if (!mbar_wait_spin(&empty[s], ((g / S) & 1) ^ 1, abort_flag, &g_gemm8_err)) {
             ok = false;
             break;
           }
-          if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * STAGE_BYTES);
+          if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * (A_BYTES + hb * BK));
           uint8_t* st = smem + s * STAGE_BYTES;
           tma_load_3d_pair(&tmA, full_leader + 8u * s, st, kb * BK, m0, bz);
           tma_load_3d_pair(&tmB, full_leader + 8u * s, st + A_BYTES, kb * BK, n0, bz);
@@ -209,9 +233,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     int it = 0, nbox = 0;
     bool failed = false;
     for (int t = cluster_id_x(); t < p.tiles; t += nclusters_x(), ++it) {
-      const int bz = t / p.per, r = t - bz * p.per, nb = r / p.num_m;
-      const int m0 = (r - nb * p.num_m) * (2 * BM) + static_cast<int>(rank) * BM;
-      const int n0 = nb * BN;
+      int bz, mt, nb;
+      tile_coords(p, t, &bz, &mt, &nb);
+      const int m0 = mt * (2 * BM) + static_cast<int>(rank) * BM;
+      const int n0 = nb * bn;
       const int ab = it & 1;
       if (!failed && !mbar_wait_warp(&acc_full[ab], (it >> 1) & 1, abort_flag, &g_gemm8_err)) failed = true;
       tc_fence_after();
@@ -219,7 +244,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int m = m0 + row;
       epi_sync8();  // every epilogue warp is done with the previous tile's column constants
       if (!failed) {
-        for (int i = ew * 32 + lane; i < BN; i += kEpiWarps * 32) {
+        for (int i = ew * 32 + lane; i < bn; i += kEpiWarps * 32) {
           const int n = n0 + i;
           sbw[i] = (n < p.N) ? static_cast<float>(-8 * p.sum_b[static_cast<size_t>(bz) * p.N + n]) : 0.0f;
           if (MODE == static_cast<int>(GemmOut::kHalf)) colv[i] = (n < p.N) ? p.s_b[n] : 0.0f;
@@ -232,7 +257,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const float corrA = (m < p.M) ? static_cast<float>(64 * p.K - 8 * p.sum_a[static_cast<size_t>(bz) * p.M + m]) : 0.0f;
       const float sa = (MODE == static_cast<int>(GemmOut::kHalf) && m < p.M) ? p.s_a[m] : 0.0f;
 #pragma unroll 1
-      for (int cc = 0; cc < BN / 32; ++cc) {
+      for (int cc = 0; cc < bn / 32; ++cc) {
         uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
         if (lane == 0) bulk_wait_group_read<1>();
         __syncwarp();
@@ -243,7 +268,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           uint32_t v[16];
           tmem_ld_32x32b_x16(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ab * BN + c0, v);
           tmem_ld_wait();
-          if (cc == BN / 32 - 1 && h == 1) {
+          if (cc == bn / 32 - 1 && h == 1) {
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(acc_empty_leader + 8u * ab);
@@ -273,8 +298,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
                 const int i = g4 * 4 + e;
-                w[e] = static_cast<uint32_t>(
-                    __float2int_rn(__fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c0 + i])));
+                const float x = __fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c0 + i]);
+                w[e] = p.f32_out ? __float_as_uint(x) : static_cast<uint32_t>(__float2int_rn(x));
               }
               // 128-byte rows, 128-byte swizzle: 16-byte chunk (4h + g4) of row `lane`
               const int ch = 4 * h + g4;
@@ -354,6 +379,8 @@ size_t ws8_layout(int M, int N, int K, void* base, Ws8* w) {
 
 template <int MODE>
 cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
+  const int bn = (MODE == static_cast<int>(GemmOut::kS32)) ? g.tile_n : BN;
+  if (bn < 32 || bn > BN || bn % 32 != 0) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(w4a4_gemm8_pair_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -364,16 +391,21 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
   CUtensorMap ma, mb, md;
   const int batch = g.batch > 0 ? g.batch : 1;
   if (!make_expanded_map(&ma, w.a8, g.K, g.M, batch, BM)) return cudaErrorInvalidValue;
-  if (!make_expanded_map(&mb, w.b8, g.K, g.N, batch, HB)) return cudaErrorInvalidValue;
+  if (!make_expanded_map(&mb, w.b8, g.K, g.N, batch, bn / 2)) return cudaErrorInvalidValue;
   const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
-  if (!make_output_map(&md, g.D, g.out, g.M, g.N, pitch, batch)) return cudaErrorInvalidValue;
+  // a row narrower than 16 bytes is stored over its whole pitch (the extra
+  // columns hold the products with zero-filled B rows)
+  const int ocols = (g.N * 4 < 16) ? pitch : g.N;
+  if (!make_output_map(&md, g.D, g.out, g.M, ocols, pitch, batch)) return cudaErrorInvalidValue;
   Params8 p;
   p.M = g.M;
   p.N = g.N;
   p.K = g.K;
   p.batch = batch;
   p.num_m = (g.M + 2 * BM - 1) / (2 * BM);
-  p.num_n = (g.N + BN - 1) / BN;
+  p.num_n = (g.N + bn - 1) / bn;
+  p.bn = bn;
+  p.f32_out = g.f32_out ? 1 : 0;
   p.per = p.num_m * p.num_n;
   p.tiles = p.per * batch;
   p.s_a = g.s_a;

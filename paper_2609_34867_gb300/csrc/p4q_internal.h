@@ -45,7 +45,7 @@ struct RowSource {
 
 // Outputs of the per-row quantizer. Optional pointers may be null.
 struct RowSinks {
-  uint8_t* codes = nullptr;   // [rows, L/2] packed INT4 (required)
+  uint8_t* codes = nullptr;   // [rows, L/2] packed INT4 (may be null when u is given)
   float* scale = nullptr;     // [rows] (required)
   int32_t* norm2 = nullptr;   // [rows] sum of squared codes
   uint16_t* copy = nullptr;   // [rows, L] fp16 copy of the source row (gather mode)
@@ -74,6 +74,8 @@ struct GemmArgs {
   const float* s_b = nullptr;     // kHalf: [N]
   const int32_t* norm_a = nullptr;  // kCos: [batch, M] squared code norms
   const int32_t* norm_b = nullptr;  // kCos: [batch, N]
+  int tile_n = 256;                 // expanded-operand int32 tiles: columns per tile (multiple of 32, <= 256)
+  bool f32_out = false;             // expanded-operand int32 tiles: the exact integers as fp32 values
 };
 
 // Returns cudaSuccess or the launch error; sets *unsupported when the shape
@@ -142,39 +144,46 @@ struct SelectPlan {
 };
 
 struct SelectWorkspace {
-  uint8_t* vcodes;   // [B*N, d/2]
   float* vscale;     // [B*N]
   int32_t* vnorm;    // [B*N]
   uint8_t* qcodes;   // [B*J, d/2]
+  uint8_t* qu;       // [B*J, d] the concepts' codes, one byte each (u = v + 8)
+  int32_t* qsum;     // [B*J] sum of those bytes
   float* qscale;     // [B*J]
   int32_t* qnorm;    // [B*J]
-  float* scores;     // [B, J, N] query cosines
-  float* gram;       // [B, N, gram_pitch] cosine of every token pair
-  int gram_pitch;    // N rounded up to a multiple of 4
-  uint8_t* vu;       // [B*N, d] codes, one byte each (tokens >= kGramExpandedMin), else null
+  float* qdots;      // [B, N, q_pitch] code dot products of every token with its image's concepts (exact, fp32)
+  int q_pitch;       // J rounded up to a multiple of 4
+  uint8_t* vu;       // [B*N, d] codes, one byte each (u = v + 8)
   int32_t* vsum;     // [B*N] sum of those bytes
-  uint32_t* kept12;  // [B, ceil(N/32)] kept set after stages 1-2, as bits (split launches)
+  uint32_t* kept12;  // [B, ceil(N/32)] kept set after stages 1-2, as bits
+  int32_t* r0tok;    // [B, R0] that kept set, ascending (R0 = Kq + Ks)
+  uint8_t* r0u;      // [B, R0, d] its expanded codes
+  int32_t* r0sum;    // [B, R0]
+  int32_t* r0norm;   // [B, R0]
+  float* dots;       // [B, N, dot_pitch] code dot products of every token with every token of R0 (exact, fp32)
+  int dot_pitch;     // R0 rounded up to a multiple of 4
+  int r0_tile_n;     // column tile width of that GEMM
+  float* m;          // [B, N] the largest cosine of each token to R0 (stage 3's initial m)
 };
 
-// Token count from which the cosine matrix runs on the expanded-operand GEMM.
-constexpr int kGramExpandedMin = 256;
+// Workspace of one selector call with R0 = Kq + Ks tokens after stages 1-2.
+size_t select_workspace_layout(int B, int N, int d, int J, int R0, SelectWorkspace* ws, void* base);
+int r0_tile_n(int R0);
 
-size_t select_workspace_layout(int B, int N, int d, int J, SelectWorkspace* ws, void* base);
-
-cudaError_t launch_query_scores(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
-// In place: the int32 dot products of ws.gram become the cosines of Eq. 4.
-cudaError_t launch_gram_cos(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
-// mode 0: stages 1-3; 1: stages 1-2 into ws.kept12; 2: stage 3 from ws.kept12
-// (modes 1 and 2 for N where select_split_applies).
-cudaError_t launch_select_stages(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls,
-                                 int32_t* idx, cudaStream_t stream, int mode = 0);
-bool select_split_applies(int N);
-// CTA pairs the expanded-operand GEMM launches: one per 256 x 256 output
-// tile (two 128-row CTAs), at most one pair per two SMs.
-inline int gemm8_pairs(int M, int N, int batch, int sms) {
-  const int tiles = ((M + 255) / 256) * ((N + 255) / 256) * (batch > 0 ? batch : 1);
-  return tiles < sms / 2 ? tiles : sms / 2;
-}
+// Stages 1-2: kept12 bits, r0tok, and idx when p.Kd == 0.
+// qdots on the expanded-operand CTA-pair GEMM (tokens as A rows, the image's
+// concepts as B rows, one 32-column tile).
+cudaError_t launch_query_dots(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+cudaError_t launch_select_stages12(const SelectPlan& p, const SelectWorkspace& ws, const float* A_cls, int32_t* idx,
+                                   cudaStream_t stream);
+cudaError_t launch_gather_r0(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+// m[b, i] = max over the R0 tokens r of cos(i, r): the exact dot products on
+// the expanded-operand CTA-pair GEMM (tokens as A rows, R0 as B rows, int32
+// tiles), then their cosines and maxima by a full-GPU row pass.
+cudaError_t launch_r0_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+// Stage 3 (greedy max-min diversity) from kept12 and m; writes idx.
+cudaError_t launch_select_diverse(const SelectPlan& p, const SelectWorkspace& ws, int32_t* idx, cudaStream_t stream);
+unsigned int diverse_read_and_clear_error();
 
 // Device error words of the kernels with bounded waits (GEMMs, quantizer).
 unsigned int gemm_read_and_clear_error();

@@ -180,14 +180,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     float2 n2 = make_float2(0.0f, 0.0f);  // exact: sums of squared codes <= 49 * 16384 < 2^24
     uint32_t su = 0;                      // sum of the expanded codes u = v + 8 (expanded output)
     if (!failed) {
-      uint32_t* q4 = reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(row) * (L >> 1));
+      uint32_t* q4 = out.codes ? reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(row) * (L >> 1)) : nullptr;
       uint4* cp = out.copy ? reinterpret_cast<uint4*>(out.copy + static_cast<size_t>(row) * L) : nullptr;
       uint2* up = out.u ? reinterpret_cast<uint2*>(out.u + static_cast<size_t>(row) * L) : nullptr;
 #pragma unroll 4
       for (int c = gt; c < nch; c += kGroupThreads) {
         const uint4 v = v4[c];
         const uint32_t pw = (a != 0.0f) ? quant_chunk<NORM>(v, s, inv, n2) : 0u;
-        q4[c] = pw;
+        if (q4) q4[c] = pw;
         if (cp) cp[c] = v;
         if (up) {
           // one byte per code, u = v + 8: the word's four low-nibble codes, then its four high-nibble codes
@@ -318,6 +318,8 @@ cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSi
   if (src.X2 != nullptr && (out2 == nullptr || out2->codes == nullptr || out2->scale == nullptr || src.idx != nullptr ||
                             src.ldx != 0 || (out.norm2 == nullptr) != (out2->norm2 == nullptr)))
     return cudaErrorInvalidValue;
+  // packed codes may be left out when the expanded ones are written
+  if (out.scale == nullptr || (out.codes == nullptr && out.u == nullptr)) return cudaErrorInvalidValue;
   const RowSinks& o2 = out2 ? *out2 : out;
   return out.norm2 ? launch_norm<true>(src, rows, L, out, o2, stream)
                    : launch_norm<false>(src, rows, L, out, o2, stream);

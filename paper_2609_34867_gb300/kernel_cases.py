@@ -4,7 +4,7 @@
   python -m paper_2609_34867_gb300.kernel_cases gemm8 M N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases quant M K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases requant M L LD [--reps R]
-  python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [B] [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases saliency B N [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases swiglu M K LD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases rmsnorm M K [--reps R]
@@ -29,7 +29,8 @@ selects the first replayed launch.
   requant p4q_quant_act_expanded on the last L columns of an M x LD fp16
           matrix (a linear's output block inside a fused GEMM's output), with
           the expanded codes (bytes: 2 M L in, 3 M L / 2 + 8 M out);
-  select  p4q_select_gather_quant on one of the LLaVA-shaped workloads;
+  select  p4q_select_gather_quant on one of the LLaVA-shaped workloads (B:
+          its first B images instead of all);
   swiglu  p4q_swiglu_quant_expanded on gate / up, the last 2 K columns of an
           M x LD fp16 matrix (bytes: 4 M K in, 3 M K / 2 + 8 M out);
   rmsnorm p4q_rmsnorm_quant_expanded on M x K fp16 rows with a K-value gain
@@ -50,6 +51,7 @@ selects the first replayed launch.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import sys
 
 import torch
@@ -227,6 +229,8 @@ def main(argv=None):
         print(f"saliency {B}x{N}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
     else:
         w = wl.WORKLOADS[a.args[0]]
+        if len(a.args) > 1:  # the same workload on fewer (or more) images
+            w = dataclasses.replace(w, B=int(a.args[1]))
         x = wl.selector_inputs(w)
         V, Q, A, T = (torch.from_numpy(t).to(dev) for t in (x.V, x.Q, x.A, x.text))
         ws = p4q.select_workspace(w.B, w.N, w.d, w.J, w.K, dev)

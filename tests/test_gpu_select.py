@@ -59,6 +59,52 @@ def test_select_orthogonal_ties(p4q, dev):
     assert np.array_equal(idx.cpu().numpy()[0], np.arange(17))
 
 
+def _clustered(B, N, d, centers, seed, noise=0.05):
+    """Tokens drawn around a few centres: a pick raises the diversity maxima
+    of its whole cluster, so the greedy rounds run in many short phases."""
+    rng = np.random.default_rng(seed)
+    C = rng.standard_normal((B, centers, d)).astype(np.float32)
+    lab = rng.integers(0, centers, size=(B, N))
+    V = np.take_along_axis(C, lab[:, :, None], axis=1) + noise * rng.standard_normal((B, N, d)).astype(np.float32)
+    return V.astype(np.float16)
+
+
+@pytest.mark.parametrize("use_signals", [False, True])
+def test_select_clustered_tokens_many_phases(p4q, dev, use_signals):
+    B, N, d, K = 2, 600, 256, 300
+    V = _clustered(B, N, d, 40, seed=21)
+    rng = np.random.default_rng(22)
+    Q = V[:, rng.integers(0, N, 3)].astype(np.float16) if use_signals else None
+    A = rng.random((B, N)).astype(np.float32) if use_signals else None
+    idx = p4q.select(_t(V, dev), _t(Q, dev), _t(A, dev), K)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    ref = oracle.select_batch(V, K, Q, A)
+    assert np.array_equal(idx.cpu().numpy(), ref)
+
+
+def test_select_duplicate_tokens(p4q, dev):
+    """Every token appears three times: a pick's copies reach cosine 1 and are
+    kept only after every other token; ties resolve to the lower index."""
+    rng = np.random.default_rng(23)
+    base = rng.standard_normal((1, 100, 128)).astype(np.float32)
+    V = np.concatenate([base, base, base], axis=1).astype(np.float16)
+    for K in (90, 150, 250):
+        idx = p4q.select(_t(V, dev), None, None, K)
+        torch.cuda.synchronize()
+        assert p4q.p4q_device_status() == 0
+        assert np.array_equal(idx.cpu().numpy(), oracle.select_batch(V, K))
+
+
+@pytest.mark.parametrize("N,K,d", [(2880, 640, 256), (4096, 1024, 128), (2049, 2000, 128)])
+def test_select_large_token_sets(p4q, dev, N, K, d):
+    """Block sizes of 768 and 1024 ranking threads, several column chunks per
+    pool phase (up to K_d picks unseen by a pool), K close to N."""
+    w = wl.Workload("t", B=2, N=N, d=d, K=K, T=0, J=3, seed=31, heavy_tail=True, linears=())
+    got, ref = _select(p4q, dev, wl.selector_inputs(w), K)
+    assert np.array_equal(got, ref)
+
+
 def test_select_one_image_576_tokens_4096d(p4q, dev):
     """The single-image LLaVA-1.5 shape: 576 tokens x 4096, budget 64."""
     w = wl.LLAVA15_7B_ONE
@@ -111,9 +157,9 @@ def test_select_gather_quant_expanded_matches(p4q, dev):
 
 
 def test_select_from_two_host_threads_on_two_streams(p4q, dev):
-    """Concurrent calls on two streams share the library's second stream and
-    its fork / join events (stages 1-2 beside the cosine matrix): each call
-    must still see its own stages 1-2, call after call."""
+    """Concurrent calls from two host threads on two streams, each with its own
+    workspace: the library keeps no state between the launches of a call, so
+    each call must see only its own inputs, call after call."""
     import threading
 
     cases = []
