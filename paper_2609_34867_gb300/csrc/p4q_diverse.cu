@@ -19,10 +19,11 @@
 //      128-byte-swizzled K-major layout),
 //      turned into Eq. 4 cosines in the epilogue: the pool block and, per
 //      pool row, the largest cosine to those picks (the bound becomes m).
-//   3. greedy rounds on the pool by one warp (pool_rounds): a pool entry
+//   3. greedy rounds on the pool by the block (pool_rounds): a pool entry
 //      whose pair is at most tau is below every token outside, so the
-//      smallest such entry is the next pick; its cosines to the pool come
-//      from the block.
+//      smallest such entry is the next pick, and runs of the next smallest
+//      are picked together while no earlier pick raises them; their cosines
+//      to the pool come from the block.
 //   4. the pool's m go back to their tokens (exact up to the picks so far).
 // A phase that picks nothing still makes its pool exact, so phases end.
 #include <cuda_fp16.h>
@@ -38,7 +39,8 @@ __device__ unsigned int g_diverse_err;
 
 namespace {
 
-constexpr int kPool = 128, kPick = 16;
+constexpr int kPool = 128;
+constexpr int kPickMax = 64;  // picks confirmed per pool iteration at most
 constexpr int kPoolPer = kPool / 32;
 static_assert(kPoolPer == 4, "pool warp layout: four slots per lane");
 constexpr int kArows = 128;   // pool rows per MMA (M = 128: the TMEM lanes)
@@ -56,171 +58,115 @@ struct DivScratch {
   int digit, above;
   int t, npool, tmin, nphase;
   unsigned long long tau;
-  __align__(16) int pick[kPick];        // pool slots of this iteration's candidates, ascending
+  __align__(16) unsigned long long skey[kPool];  // pool rounds: (m, slot) keys of the certain entries
+  int sorted[kPool];                    // pool rounds: slots of the certain entries in key order
+  int L;                                // pool rounds: length of the confirmed prefix
   int ptok[kPool];                      // pool slot -> token (ascending)
   float pm[kPool];                      // m of the pool tokens (bound, then exact)
   unsigned int pmx[kPool];              // order key of the largest cosine to the pick columns
   int psum[kPool], pnorm[kPool];        // pool rows: sum of u, squared code norm
+  float prs[kPool];                     // pool rows: rsqrtf of the squared code norm (0 for a zero row)
   int csum[kBrows], cnorm[kBrows];      // extra columns of the current chunk
+  float crs[kBrows];                    // their rsqrtf norms (candidate path)
   unsigned int keptbits[P4Q_MAX_TOKENS / 32];
-  int list[P4Q_MAX_TOKENS];             // the greedy picks, in order
+  int16_t list[P4Q_MAX_TOKENS];         // the greedy picks, in order
   signed char slotof[P4Q_MAX_TOKENS];   // token -> pool slot, -1 outside the pool
+  int16_t candof[P4Q_MAX_TOKENS];       // token -> candidate index, -1 for the others
+  int pci[kPool];                       // pool slot -> candidate index (-1: not a candidate)
   uint64_t bar_full[kStages];           // producer warps -> the stage is in shared memory
   uint64_t bar_empty[kStages];          // MMA commit -> the stage may be overwritten
   uint64_t bar_acc;                     // MMA commit -> the chunk's accumulator is complete
   uint64_t bar_done;                    // MMA commit at teardown -> nothing in flight
   uint32_t tmem_slot;
   volatile int abort_flag;
-  __align__(16) float cp[kPool][kPool]; // cos(ptok[i], ptok[j])
+  __align__(16) float cp[kPool][kPool]; // cos(ptok[i], ptok[j]) (Eq. 4, exact)
 };
 
 __device__ __forceinline__ float order_key_float(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
 }
 
-// Sorts four 64-bit values ascending (five compare-exchanges).
-__device__ __forceinline__ void sort4(unsigned long long (&h)[kPoolPer]) {
-  auto cx = [](unsigned long long& x, unsigned long long& y) {
-    const unsigned long long lo = x < y ? x : y, hi = x < y ? y : x;
-    x = lo;
-    y = hi;
-  };
-  cx(h[0], h[1]);
-  cx(h[2], h[3]);
-  cx(h[0], h[2]);
-  cx(h[1], h[3]);
-  cx(h[1], h[2]);
-}
-
-// Greedy rounds on the pool by warp 0 (lane l holds slots 4l .. 4l + 3, in
-// token order), with exact m of the pool entries in s.pm. The next pick is the
+// Greedy rounds on the pool, by the whole block (thread i < 128 owns pool
+// slot i), with exact m of the pool entries in s.pm. The next pick is the
 // smallest free (m, token) pair. A pool entry is certain to be in order while
 // its pair is at most tau (every token outside the pool is above tau and m
-// only grows). Per iteration the r smallest certain entries c_0 < c_1 < ...
-// are taken by r rounds of a warp minimum; c_0 is the next pick, and c_a the
-// pick after c_0 .. c_{a-1} whenever none of their cosines exceeds m(c_a)
-// (nothing else can pass it). The longest such prefix is picked, the pool's m
-// absorbs the picks' cosines, and the picks are appended to s.list. Ends when
-// Kd picks are made or no entry is certain; s.t and s.pm hold the results.
-__device__ void pool_rounds(int npool, int Kd, unsigned long long tau, DivScratch& s) {
-  const int lane = threadIdx.x & 31;
-  const unsigned int lanes_below = (1u << lane) - 1u;
+// only grows). Per iteration the certain entries are ranked by their pairs
+// (each owner counts the smaller keys), giving c_0 < c_1 < ...; c_0 is the
+// next pick, and c_a the pick after c_0 .. c_{a-1} whenever none of their
+// cosines exceeds m(c_a) (nothing else can pass it: every other pair only
+// grows). The pairs (b < a) are checked in parallel; the longest such
+// prefix (at most kPickMax) is picked at once, the pool's m absorbs the
+// picks' cosines, and the picks are appended to s.list. Ends when Kd picks
+// are made or no entry is certain; s.t and s.pm hold the results.
+template <int kThreads>
+__device__ void pool_rounds(int npool, int Kd, DivScratch& s) {
   constexpr unsigned long long kNone = ~0ull;
-  float pm[kPoolPer];
-  unsigned int alive = 0;
-#pragma unroll
-  for (int k = 0; k < kPoolPer; ++k) {
-    const int slot = kPoolPer * lane + k;
-    pm[k] = slot < npool ? s.pm[slot] : 0.0f;
-    if (slot < npool) alive |= 1u << k;
-  }
-  int t = s.t;
-  while (t < Kd) {
-    unsigned long long h[kPoolPer];
-    int nv = 0;
-#pragma unroll
-    for (int k = 0; k < kPoolPer; ++k) {
-      const unsigned long long pr =
-          (static_cast<unsigned long long>(float_order_key(pm[k])) << 32) | (kPoolPer * lane + k);
-      h[k] = ((alive >> k) & 1u) && pr <= tau ? pr : kNone;
-      nv += h[k] != kNone;
+  const int tid = threadIdx.x;
+  const unsigned long long tau = s.tau;
+  bool alive = tid < npool;
+  while (true) {
+    const int t = s.t;  // every thread has passed the barrier that published it
+    if (t >= Kd) break;
+    unsigned long long key = kNone;
+    if (alive) {
+      const unsigned long long pr = (static_cast<unsigned long long>(float_order_key(s.pm[tid])) << 32) | tid;
+      if (pr <= tau) key = pr;
     }
-    nv = __reduce_add_sync(0xFFFFFFFFu, nv);
-    const int r = min(min(kPick, Kd - t), nv);
+    if (tid < kPool) s.skey[tid] = key;
+    if (tid == 0) s.L = kPickMax;
+    const int nc = __syncthreads_count(key != kNone);
+    const int r = min(min(nc, Kd - t), kPickMax);
     if (r == 0) break;
-    sort4(h);
-    // The lane's sorted entries as 32-bit keys (the pair order is the key
-    // order, ties between lanes resolving to the lower lane) and their slots
-    // as a queue of 2-bit indices into the lane's four slots.
-    uint32_t hk[kPoolPer];
-    uint32_t perm = 0;
-#pragma unroll
-    for (int k = 0; k < kPoolPer; ++k) {
-      hk[k] = static_cast<uint32_t>(h[k] >> 32);
-      perm |= (static_cast<uint32_t>(h[k]) & 3u) << (2 * k);
-    }
-    uint32_t rks = 0, pks = 0;
-    int np = 0;
-#pragma unroll
-    for (int a = 0; a < kPick; ++a) {
-      const uint32_t wk = __reduce_min_sync(0xFFFFFFFFu, hk[0]);
-      const unsigned int tied = __ballot_sync(0xFFFFFFFFu, hk[0] == wk);
-      const bool mine = a < r && hk[0] == wk && (tied & lanes_below) == 0u;
-      if (mine) {
-        s.pick[a] = kPoolPer * lane + static_cast<int>(perm & 3u);
-        rks |= static_cast<uint32_t>(a) << (4 * np);
-        pks |= (perm & 3u) << (2 * np);
-        ++np;
-        perm >>= 2;
-#pragma unroll
-        for (int k = 0; k + 1 < kPoolPer; ++k) hk[k] = hk[k + 1];
-        hk[kPoolPer - 1] = 0xFFFFFFFFu;
+    // rank of each certain entry among them (keys are unique: the slot is in the low bits)
+    int rank = kPool;
+    if (key != kNone) {
+      rank = 0;
+#pragma unroll 8
+      for (int f = 0; f < kPool; f += 2) {
+        const ulonglong2 kk = *reinterpret_cast<const ulonglong2*>(&s.skey[f]);
+        rank += (kk.x < key ? 1 : 0) + (kk.y < key ? 1 : 0);
       }
+      if (rank < r) s.sorted[rank] = tid;
     }
-    int rk[kPoolPer];  // position among the candidates of each of this lane's slots, or -1
-#pragma unroll
-    for (int k = 0; k < kPoolPer; ++k) rk[k] = -1;
-#pragma unroll
-    for (int j = 0; j < kPoolPer; ++j) {
-      const int kj = static_cast<int>((pks >> (2 * j)) & 3u), aj = static_cast<int>((rks >> (4 * j)) & 15u);
-#pragma unroll
-      for (int k = 0; k < kPoolPer; ++k) rk[k] = (j < np && kj == k) ? aj : rk[k];
+    __syncthreads();
+    // pairs b < a < r: a violation (an earlier candidate raises c_a) ends the prefix at a
+    const int npairs = r * (r - 1) / 2;
+    for (int q = tid; q < npairs; q += kThreads) {
+      int a2 = static_cast<int>((1.0f + sqrtf(1.0f + 8.0f * static_cast<float>(q))) * 0.5f);
+      while (a2 * (a2 - 1) / 2 > q) --a2;
+      while ((a2 + 1) * a2 / 2 <= q) ++a2;
+      const int b2 = q - a2 * (a2 - 1) / 2;
+      const int ca = s.sorted[a2];
+      if (s.cp[s.sorted[b2]][ca] > s.pm[ca]) atomicMin(&s.L, a2);
     }
-    __syncwarp();
-    // cos(c_a, c_b) for this lane's slots from row c_b (the block is
-    // symmetric): one 16-byte read per earlier candidate (every entry of
-    // s.pick is a valid slot, stale past r)
-    unsigned int fail = 0;
-#pragma unroll
-    for (int c0 = 0; c0 < kPick; c0 += 4) {
-      float4 c[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) c[u] = *reinterpret_cast<const float4*>(&s.cp[s.pick[c0 + u]][kPoolPer * lane]);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int b2 = c0 + u;
-        fail |= (b2 < rk[0] && c[u].x > pm[0]) ? 1u << rk[0] : 0u;
-        fail |= (b2 < rk[1] && c[u].y > pm[1]) ? 1u << rk[1] : 0u;
-        fail |= (b2 < rk[2] && c[u].z > pm[2]) ? 1u << rk[2] : 0u;
-        fail |= (b2 < rk[3] && c[u].w > pm[3]) ? 1u << rk[3] : 0u;
-      }
-    }
-    fail = __reduce_or_sync(0xFFFFFFFFu, fail);
-    const int L = fail ? __ffs(fail) - 1 : r;  // bit 0 is never set
-#pragma unroll
-    for (int c0 = 0; c0 < kPick; c0 += 4) {
-      float4 c[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) c[u] = *reinterpret_cast<const float4*>(&s.cp[s.pick[c0 + u]][kPoolPer * lane]);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const bool use = c0 + u < L;
-        pm[0] = use ? fmaxf(pm[0], c[u].x) : pm[0]; pm[1] = use ? fmaxf(pm[1], c[u].y) : pm[1];
-        pm[2] = use ? fmaxf(pm[2], c[u].z) : pm[2]; pm[3] = use ? fmaxf(pm[3], c[u].w) : pm[3];
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < kPoolPer; ++k) {
-      if (rk[k] >= 0 && rk[k] < L) {
-        alive &= ~(1u << k);
-        const int tok = s.ptok[kPoolPer * lane + k];
-        s.list[t + rk[k]] = tok;
+    __syncthreads();
+    const int L = min(s.L, r);  // >= 1: c_0 never fails
+    if (alive) {
+      if (rank < L) {
+        alive = false;
+        const int tok = s.ptok[tid];
+        s.list[t + rank] = static_cast<int16_t>(tok);
         atomicOr(&s.keptbits[tok >> 5], 1u << (tok & 31));
+      } else {
+        float m = s.pm[tid];
+#pragma unroll 8
+        for (int b2 = 0; b2 < L; ++b2) m = fmaxf(m, s.cp[s.sorted[b2]][tid]);
+        s.pm[tid] = m;
       }
     }
-    t += L;
-    __syncwarp();
+    if (tid == 0) s.t = t + L;
+    __syncthreads();
   }
-#pragma unroll
-  for (int k = 0; k < kPoolPer; ++k)
-    if (kPoolPer * lane + k < npool) s.pm[kPoolPer * lane + k] = pm[k];
-  if (lane == 0) s.t = t;
 }
 
 // Arguments of one launch.
 struct DivArgs {
   const uint32_t* kept12;  // [B, words] R0 as bits
   const float* m;          // [B, N] largest cosine to R0 (R0 > 0)
+  const int32_t* cand;     // [B, C] candidates, ascending
+  const int32_t* candnorm; // [B, C]
+  const float* cdots;      // [B, C, cpitch] their pairwise code dot products
+  int C, cpitch;
   const uint8_t* vu;       // [B*N, d] expanded codes
   const int32_t* vsum;     // [B*N]
   const int32_t* vnorm;    // [B*N]
@@ -258,8 +204,10 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
     tmem_alloc(&s.tmem_slot, kTmemCols);
     tmem_relinquish();
   }
-  for (int i = threadIdx.x; i < N; i += kThreads) s.slotof[i] = -1;
-  if (threadIdx.x < kPick) s.pick[threadIdx.x] = 0;
+  for (int i = threadIdx.x; i < N; i += kThreads) {
+    s.slotof[i] = -1;
+    s.candof[i] = -1;
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -268,6 +216,8 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
   pdl_wait();  // R0 bits and maxima come from the kernels before
   pdl_launch_dependents();
   for (int w = threadIdx.x; w < words; w += kThreads) s.keptbits[w] = a.kept12[static_cast<size_t>(b) * words + w];
+  __syncthreads();  // candof is cleared
+  for (int c = threadIdx.x; c < a.C; c += kThreads) s.candof[a.cand[static_cast<size_t>(b) * a.C + c]] = static_cast<int16_t>(c);
   __syncthreads();
 
   bool kept[kPer];
@@ -328,7 +278,9 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
           s.pmx[pos] = 0u;  // below the key of every float
           s.psum[pos] = a.vsum[row0 + i];
           s.pnorm[pos] = a.vnorm[row0 + i];
+          s.prs[pos] = s.pnorm[pos] > 0 ? rsqrtf(static_cast<float>(s.pnorm[pos])) : 0.0f;
           s.slotof[i] = static_cast<signed char>(pos);
+          s.pci[pos] = s.candof[i];
           ++pos;
         }
       }
@@ -355,12 +307,83 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
           __reduce_max_sync(0xFFFFFFFFu, static_cast<uint32_t>(mx >> 32) == thi ? static_cast<uint32_t>(mx) : 0u);
       if (lane == 0) s.tau = (q >= nfree) ? ~0ull : ((static_cast<unsigned long long>(thi) << 32) | tlo);
     }
+    // ---- 2. the pool's exact dot products with the pool and with the picks
+    // its bounds have not seen: from the candidates' dot products when every
+    // one of those tokens is a candidate, else on the tensor cores here
+    bool mine_ok = true;
+    for (int r = threadIdx.x; r < npool + ncp; r += kThreads) {
+      const int tok = r < npool ? s.ptok[r] : s.list[tmin + r - npool];
+      mine_ok = mine_ok && s.candof[tok] >= 0;
+    }
+    const bool from_cand = __syncthreads_and(mine_ok) != 0;
+    if (from_cand) {
+      const float* cd = a.cdots + static_cast<size_t>(b) * a.C * a.cpitch;
+      // the pool block, one warp per row, four columns per lane in flight
+      for (int e = warp; e < npool; e += kWarps) {
+        const float* row = cd + static_cast<size_t>(s.pci[e]) * a.cpitch;
+        float v[kPoolPer];
+#pragma unroll
+        for (int k = 0; k < kPoolPer; ++k) {
+          const int f = lane + 32 * k;
+          v[k] = f < npool ? __ldg(row + s.pci[f]) : 0.0f;
+        }
+        const int ne = s.pnorm[e];
+#pragma unroll
+        for (int k = 0; k < kPoolPer; ++k) {
+          const int f = lane + 32 * k;
+          if (f < npool) s.cp[e][f] = code_cosine(static_cast<int>(v[k]), ne, s.pnorm[f]);
+        }
+      }
+      // per pool row: the largest cosine to the unseen picks (chunks of 128
+      // picks with their candidate index and norms in shared memory),
+      // approximate first, then exact for the columns near it
+      const int32_t* cn = a.candnorm + static_cast<size_t>(b) * a.C;
+      for (int c0 = 0; c0 < ncp; c0 += kBrows) {
+        const int nc2 = min(kBrows, ncp - c0);
+        __syncthreads();  // the previous chunk's column data is no longer read
+        for (int c = threadIdx.x; c < nc2; c += kThreads) {
+          const int cj = s.candof[s.list[tmin + c0 + c]];
+          const int nj = cn[cj];
+          s.csum[c] = cj;  // candidate index of the column
+          s.cnorm[c] = nj;
+          s.crs[c] = nj > 0 ? rsqrtf(static_cast<float>(nj)) : 0.0f;
+        }
+        __syncthreads();
+        for (int e = warp; e < npool; e += kWarps) {
+          const float* row = cd + static_cast<size_t>(s.pci[e]) * a.cpitch;
+          float v[kBrows / 32];
+#pragma unroll
+          for (int k = 0; k < kBrows / 32; ++k) {
+            const int c = lane + 32 * k;
+            v[k] = c < nc2 ? __ldg(row + s.csum[c]) : 0.0f;
+          }
+          float amax = -INFINITY;
+#pragma unroll
+          for (int k = 0; k < kBrows / 32; ++k) {
+            const int c = lane + 32 * k;
+            if (c < nc2) amax = fmaxf(amax, v[k] * s.prs[e] * s.crs[c]);
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, o));
+          float emax = -INFINITY;
+#pragma unroll
+          for (int k = 0; k < kBrows / 32; ++k) {
+            const int c = lane + 32 * k;
+            if (c < nc2 && v[k] * s.prs[e] * s.crs[c] >= amax - kCosMargin)
+              emax = fmaxf(emax, code_cosine(static_cast<int>(v[k]), s.pnorm[e], s.cnorm[c]));
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) emax = fmaxf(emax, __shfl_xor_sync(0xFFFFFFFFu, emax, o));
+          if (lane == 0) s.pmx[e] = max(s.pmx[e], float_order_key(emax));
+        }
+      }
+      __syncthreads();
+    } else {
     // the rows this phase reads, toward L2 ahead of the staged loads
     for (int r = threadIdx.x; r < npool + ncp; r += kThreads) {
       const int tok = r < npool ? s.ptok[r] : s.list[tmin + r - npool];
       prefetch_l2_bulk(a.vu + (row0 + tok) * d, static_cast<uint32_t>(d));
     }
-    // ---- 2. exact cosines of the pool rows with the pool and with the unseen picks
     // chunk 0: columns = the 128 pool rows (the A stage itself) + up to 128 picks;
     // chunk c >= 1: up to 128 further picks.
     const int extra0 = min(ncp, kArows);
@@ -490,12 +513,13 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
       tc_fence_before();
       __syncthreads();
     }
+    }  // tensor-core path
     // the bounds of the pool become m
     if (threadIdx.x < npool && s.pmx[threadIdx.x] != 0u)
       s.pm[threadIdx.x] = fmaxf(s.pm[threadIdx.x], order_key_float(s.pmx[threadIdx.x]));
     __syncthreads();
     // ---- 3. greedy rounds on the pool
-    if (warp == 0 && !s.abort_flag) pool_rounds(npool, a.Kd, s.tau, s);
+    if (!s.abort_flag) pool_rounds<kThreads>(npool, a.Kd, s);
     __syncthreads();
     // ---- 4. exact m back to the pool's tokens
     const int tn = s.t;
@@ -554,6 +578,11 @@ cudaError_t launch_select_diverse(const SelectPlan& p, const SelectWorkspace& ws
   DivArgs a;
   a.kept12 = ws.kept12;
   a.m = ws.m;
+  a.cand = ws.cand;
+  a.candnorm = ws.candnorm;
+  a.cdots = ws.cdots;
+  a.C = ws.C;
+  a.cpitch = ws.cpitch;
   a.vu = ws.vu;
   a.vsum = ws.vsum;
   a.vnorm = ws.vnorm;

@@ -164,10 +164,23 @@ struct SelectWorkspace {
   int dot_pitch;     // R0 rounded up to a multiple of 4
   int r0_tile_n;     // column tile width of that GEMM
   float* m;          // [B, N] the largest cosine of each token to R0 (stage 3's initial m)
+  int C;             // candidates of stage 3 per image (0 without a diversity stage)
+  int32_t* cand;     // [B, C] the candidates, ascending
+  uint8_t* candu;    // [B, C, d] their expanded codes
+  int32_t* candsum;  // [B, C]
+  int32_t* candnorm; // [B, C]
+  float* cdots;      // [B, C, cpitch] their code dot products (exact, fp32)
+  int cpitch;        // C rounded up to a multiple of 4
 };
 
-// Workspace of one selector call with R0 = Kq + Ks tokens after stages 1-2.
-size_t select_workspace_layout(int B, int N, int d, int J, int R0, SelectWorkspace* ws, void* base);
+// Candidates of stage 3: up to kCandExtra more than the K_d picks (a pool's
+// worth), at most kCandMax.
+constexpr int kCandExtra = 128, kCandMax = 1024;
+int select_candidates(int N, int R0, int Kd);
+
+// Workspace of one selector call with R0 = Kq + Ks tokens after stages 1-2
+// and C candidates in stage 3.
+size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, SelectWorkspace* ws, void* base);
 int r0_tile_n(int R0);
 
 // Stages 1-2: kept12 bits, r0tok, and idx when p.Kd == 0.
@@ -181,7 +194,10 @@ cudaError_t launch_gather_r0(const SelectPlan& p, const SelectWorkspace& ws, cud
 // the expanded-operand CTA-pair GEMM (tokens as A rows, R0 as B rows, int32
 // tiles), then their cosines and maxima by a full-GPU row pass.
 cudaError_t launch_r0_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
-// Stage 3 (greedy max-min diversity) from kept12 and m; writes idx.
+// The candidates of stage 3 (per image), their expanded codes, and the
+// code dot products of every pair of them (a batched tensor-core GEMM).
+cudaError_t launch_candidates(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+// Stage 3 (greedy max-min diversity) from kept12, m and the candidates; writes idx.
 cudaError_t launch_select_diverse(const SelectPlan& p, const SelectWorkspace& ws, int32_t* idx, cudaStream_t stream);
 unsigned int diverse_read_and_clear_error();
 

@@ -14,9 +14,13 @@
 //                           (per-concept top quota), stage 2 (CLS-saliency top
 //                           K_s); writes the kept set R0 as bits and as an
 //                           ascending token list (and as idx when K_d = 0).
-//   gather_r0_kernel        the expanded codes, row sums and norms of R0, row
-//                           by row, as the B operand of the GEMM that gives
-//                           every token its largest cosine to R0.
+//   gather_rows_kernel      the expanded codes, row sums and norms of listed
+//                           tokens (R0, or the diversity candidates), row by
+//                           row, as an operand of the tensor-core GEMMs.
+//   r0_cosmax_kernel        each token's largest cosine to R0 from the exact
+//                           dot products of that GEMM.
+//   select_candidates_kernel  the diversity stage's candidates: the free
+//                           tokens with the smallest of those maxima.
 // Every ranking orders by (score, lower token index first).
 #include <cuda_fp16.h>
 
@@ -107,28 +111,69 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
   }
 }
 
-// r0u[b, j] = vu[b, r0tok[b, j]] (d bytes), with its row sum and squared
-// norm: one warp per row, 16-byte chunks.
-__global__ void __launch_bounds__(256) gather_r0_kernel(const uint8_t* __restrict__ vu, const int32_t* __restrict__ vsum,
-                                                        const int32_t* __restrict__ vnorm,
-                                                        const int32_t* __restrict__ r0tok, int B, int N, int d, int R0,
-                                                        uint8_t* __restrict__ r0u, int32_t* __restrict__ r0sum,
-                                                        int32_t* __restrict__ r0norm) {
+// Candidates of the diversity stage for image blockIdx.x: the C free tokens
+// (not in R0) with the smallest (m, token) pairs, m their largest cosine to
+// R0, as an ascending list cand [B, C]. Greedy picks and pool entries are
+// taken among the smallest pairs and pairs only grow, so the stage usually
+// needs the cosines of candidates only (the GEMM over them); it checks, per
+// pool phase, that it does. Same layout and radix select as stages 1-2.
+template <int kMaxThreads>
+__global__ void __launch_bounds__(kMaxThreads, 1)
+    select_candidates_kernel(const float* __restrict__ m, const uint32_t* __restrict__ kept12, int N, int R0, int C,
+                             int32_t* __restrict__ cand) {
+  pdl_wait();
+  pdl_launch_dependents();
+  __shared__ RankScratch s;
+  const int b = blockIdx.x, nt = blockDim.x;
+  const int base = kPer * threadIdx.x;
+  const int words = (N + 31) / 32;
+  bool taken[kPer];
+  uint32_t key[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) {
+    const int i = base + e;
+    taken[e] = i < N && ((kept12[static_cast<size_t>(b) * words + (i >> 5)] >> (i & 31)) & 1u);
+    // the smallest pairs as the largest keys; m = -inf (R0 empty) ranks every token equal
+    key[e] = (i < N) ? ~float_order_key(R0 > 0 ? m[static_cast<size_t>(b) * N + i] : -INFINITY) : 0u;
+  }
+  bool in_r0[kPer];
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) in_r0[e] = taken[e];
+  block_take_top(key, taken, base, N, C, nt, s);
+  int cnt = 0;
+#pragma unroll
+  for (int e = 0; e < kPer; ++e) cnt += (base + e < N && taken[e] && !in_r0[e]) ? 1 : 0;
+  int total;
+  int pos = block_exclusive_scan(cnt, &total, nt, s);
+#pragma unroll
+  for (int e = 0; e < kPer; ++e)
+    if (base + e < N && taken[e] && !in_r0[e] && pos < C) cand[static_cast<size_t>(b) * C + pos++] = base + e;
+}
+
+// ru[b, j] = vu[b, tok[b, j]] (d bytes), with its row sum and squared norm,
+// for R listed tokens per image (the kept set R0, or the candidates of the
+// diversity stage): one warp per row, 16-byte chunks.
+__global__ void __launch_bounds__(256) gather_rows_kernel(const uint8_t* __restrict__ vu,
+                                                          const int32_t* __restrict__ vsum,
+                                                          const int32_t* __restrict__ vnorm,
+                                                          const int32_t* __restrict__ tok, int B, int N, int d, int R,
+                                                          uint8_t* __restrict__ ru, int32_t* __restrict__ rsum,
+                                                          int32_t* __restrict__ rnorm) {
   pdl_wait();
   pdl_launch_dependents();
   const int lane = threadIdx.x & 31;
-  const int rows = B * R0;
+  const int rows = B * R;
   const int nwarps = gridDim.x * (blockDim.x >> 5);
   const int chunks = d >> 4;
   for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += nwarps) {
-    const int b = r / R0;
-    const size_t src = static_cast<size_t>(b) * N + r0tok[r];
+    const int b = r / R;
+    const size_t src = static_cast<size_t>(b) * N + tok[r];
     const uint4* s = reinterpret_cast<const uint4*>(vu + src * d);
-    uint4* t = reinterpret_cast<uint4*>(r0u + static_cast<size_t>(r) * d);
+    uint4* t = reinterpret_cast<uint4*>(ru + static_cast<size_t>(r) * d);
     for (int c = lane; c < chunks; c += 32) t[c] = ldg_stream16(s + c);
     if (lane == 0) {
-      r0sum[r] = vsum[src];
-      r0norm[r] = vnorm[src];
+      rsum[r] = vsum[src];
+      rnorm[r] = vnorm[src];
     }
   }
 }
@@ -163,12 +208,14 @@ __global__ void __launch_bounds__(256) r0_cosmax_kernel(const float* __restrict_
     const int na = vnorm[row];
     const float ra = na > 0 ? rsqrtf(static_cast<float>(na)) : 0.0f;
     float amax = -INFINITY;
-    for (int j = lane; j < R0; j += 32) amax = fmaxf(amax, dr[j] * ra * rr[j]);
+#pragma unroll 4
+    for (int j = lane; j < R0; j += 32) amax = fmaxf(amax, __ldg(dr + j) * ra * rr[j]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, o));
     float emax = -INFINITY;
+#pragma unroll 4
     for (int j = lane; j < R0; j += 32) {
-      const float dot = dr[j];
+      const float dot = __ldg(dr + j);
       if (dot * ra * rr[j] >= amax - kCosMargin) emax = fmaxf(emax, code_cosine(static_cast<int>(dot), na, nr[j]));
     }
 #pragma unroll
@@ -239,8 +286,16 @@ int r0_tile_n(int R0) {
   return (per + 31) / 32 * 32;
 }
 
-size_t select_workspace_layout(int B, int N, int d, int J, int R0, SelectWorkspace* ws, void* base) {
+int select_candidates(int N, int R0, int Kd) {
+  if (Kd <= 0) return 0;
+  const int want = std::min((Kd + kCandExtra + 31) / 32 * 32, kCandMax);
+  return std::min(N - R0, want);
+}
+
+size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, SelectWorkspace* ws, void* base) {
   const size_t BN = static_cast<size_t>(B) * N, BJ = static_cast<size_t>(B) * J, BR = static_cast<size_t>(B) * R0;
+  const size_t BC = static_cast<size_t>(B) * C;
+  const int cp = (C + 3) & ~3;
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -258,6 +313,8 @@ size_t select_workspace_layout(int B, int N, int d, int J, int R0, SelectWorkspa
   const size_t o_k12 = take(static_cast<size_t>(B) * ((N + 31) / 32) * 4);
   const size_t o_r0t = take(BR * 4), o_r0u = take(BR * d), o_r0s = take(BR * 4), o_r0n = take(BR * 4);
   const size_t o_dot = take(BN * dp * 4), o_m = take(BN * 4);
+  const size_t o_ct = take(BC * 4), o_cu = take(BC * d), o_cs = take(BC * 4), o_cn = take(BC * 4);
+  const size_t o_cd = take(BC * cp * 4);
   if (ws && base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     ws->vscale = reinterpret_cast<float*>(p + o_vs);
@@ -280,6 +337,13 @@ size_t select_workspace_layout(int B, int N, int d, int J, int R0, SelectWorkspa
     ws->dot_pitch = dp;
     ws->r0_tile_n = tn;
     ws->m = reinterpret_cast<float*>(p + o_m);
+    ws->C = C;
+    ws->cand = reinterpret_cast<int32_t*>(p + o_ct);
+    ws->candu = p + o_cu;
+    ws->candsum = reinterpret_cast<int32_t*>(p + o_cs);
+    ws->candnorm = reinterpret_cast<int32_t*>(p + o_cn);
+    ws->cdots = reinterpret_cast<float*>(p + o_cd);
+    ws->cpitch = cp;
   }
   return off;
 }
@@ -330,12 +394,40 @@ cudaError_t launch_r0_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cud
                     ws.vnorm, ws.r0norm, p.N, R0, ws.m);
 }
 
+cudaError_t launch_candidates(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
+  const int C = ws.C;
+  if (C <= 0) return cudaSuccess;
+  const int R0 = p.Kq + p.Ks;
+  const int nt = ((p.N + kPer - 1) / kPer + 31) / 32 * 32;
+  auto go = [&](auto kern) {
+    return launch_pdl(kern, dim3(p.B), dim3(nt), 0, stream, ws.m, ws.kept12, p.N, R0, C, ws.cand);
+  };
+  cudaError_t e = nt <= 512 ? go(select_candidates_kernel<512>)
+                            : (nt <= 768 ? go(select_candidates_kernel<768>) : go(select_candidates_kernel<kSelThreads>));
+  if (e != cudaSuccess) return e;
+  const int rows = p.B * C;
+  const int blocks = std::min((rows + 7) / 8, 4 * num_sms());
+  e = launch_pdl(gather_rows_kernel, dim3(blocks), dim3(256), 0, stream, ws.vu, ws.vsum, ws.vnorm, ws.cand, p.B, p.N,
+                 p.d, C, ws.candu, ws.candsum, ws.candnorm);
+  if (e != cudaSuccess) return e;
+  GemmArgs g;  // every candidate against every candidate of its image
+  g.M = C;
+  g.N = C;
+  g.K = p.d;
+  g.batch = p.B;
+  g.out = GemmOut::kS32;
+  g.D = ws.cdots;
+  g.d_pitch = ws.cpitch;
+  g.f32_out = true;
+  return launch_gemm8(g, ws.candu, ws.candsum, ws.candu, ws.candsum, stream);
+}
+
 cudaError_t launch_gather_r0(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
   const int R0 = p.Kq + p.Ks;
   const int rows = p.B * R0;
   if (rows == 0) return cudaSuccess;
   const int blocks = std::min((rows + 7) / 8, 4 * num_sms());
-  return launch_pdl(gather_r0_kernel, dim3(blocks), dim3(256), 0, stream, ws.vu, ws.vsum, ws.vnorm, ws.r0tok, p.B,
+  return launch_pdl(gather_rows_kernel, dim3(blocks), dim3(256), 0, stream, ws.vu, ws.vsum, ws.vnorm, ws.r0tok, p.B,
                     p.N, p.d, R0, ws.r0u, ws.r0sum, ws.r0norm);
 }
 
