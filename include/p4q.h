@@ -164,14 +164,17 @@ p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, ui
 /* SwiGLU before down_proj fused with the per-token quantizer of its input
  * (App. A quantizes every linear's input per token; the decoder's MLP feeds
  * down_proj with silu(gate) * up). For each row m:
- *   h_k = silu(g_k) * u_k with silu(g) = g * (1 / (1 + exp32(-g))), each
- *   operation one rounded fp32 step (the reciprocal correctly rounded), where
- *   exp32 is this library's own fp32 exponential: n = rint(x * log2 e),
- *   r = x - n * ln2 by two fused multiply-adds (ln2 = 355/512 + a low part),
- *   e^r by the degree-7 Taylor polynomial (Horner, fused multiply-adds),
- *   times 2^n by two exact power-of-two multiplications; 0 for x < -87, inf
- *   for x > 88.72284 (within 1 ulp of e^x in between);
- *   then the codes and scale of h as p4q_quant_act.
+ *   h_k = silu(g_k) * u_k, silu(g) = g / (1 + e^-g), evaluated in fp32 as
+ *   g * (1 / (1 + exp32(-g))) (each operation one rounded fp32 step, the
+ *   reciprocal correctly rounded), where exp32 is this library's own fp32
+ *   exponential (Cody-Waite reduction with ln2 = 355/512 + a low part, the
+ *   degree-7 Taylor polynomial, two exact power-of-two scalings: within
+ *   0.9 ulp of e^x; 0 for x < -87, inf for x > 88.72284, so silu(g) = 0
+ *   for g < -88.72284);
+ *   then the codes and scale of h as p4q_quant_act. h is within 3 fp32
+ *   rounding units of the real silu(g) * u, so the scale is within 1e-6 of
+ *   the exact one and every code equals the code of the exact h except
+ *   where h / s lies within 3.2e-6 of a .5 boundary.
  *   gate, up [M, Kin] fp16, rows ld_gate / ld_up elements apart (column
  *              blocks of a fused gate|up output; device, read)
  *   Xq [M, Kin/2], s_a [M]           written
@@ -396,14 +399,19 @@ p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
  * convenience of this library.
  *
  * Scratch: a fixed array of P4Q_NOALLOC_SCRATCH_BYTES inside the library's
- * device image, held by every GPU that loads the library until the process
- * exits. Sizes whose workspace (p4q_select_workspace_bytes) exceeds it return
- * P4Q_ERR_WORKSPACE_TOO_SMALL and launch nothing. The first call on a device
- * looks up the array's device address (cudaGetSymbolAddress) and keeps it;
- * make that first call before any stream capture. The call allocates nothing.
- * All calls on a device share the one array: calls whose work overlaps on the
- * GPU (other streams, or several host threads) race and give undefined
- * results, so serialize them. */
+ * device image (enough for at least 8 images of 576 x 4096 with 3 concepts
+ * and K = 192). Sizes whose workspace for this call exceeds it return
+ * P4Q_ERR_WORKSPACE_TOO_SMALL and launch nothing. Each call looks up the
+ * array's device address in the current context (cudaGetSymbolAddress), so
+ * it stays right after cudaDeviceReset or in another context. Under CUDA's
+ * lazy module loading the array is committed on a device by the first call
+ * there (which may then fail with P4Q_ERR_CUDA on a full device): make that
+ * first call at start-up, inside the caller's memory budget, and before any
+ * stream capture. The call allocates nothing itself. All calls on a device
+ * share the one array, which keeps the last call's contents (every region is
+ * written before it is read, so nothing needs clearing): calls whose work
+ * overlaps on the GPU (other streams, or several host threads) race and give
+ * undefined results, so serialize them. */
 #define P4Q_NOALLOC_SCRATCH_BYTES (48u << 20)
 p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
                               const float* A_cls, const p4q_select_params* params, int32_t* idx,

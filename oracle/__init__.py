@@ -68,8 +68,6 @@ def _load():
             lib.p4q_gather.restype = i32
             lib.p4q_cls_saliency.argtypes = [P, P, P, i32, i32, i32, i32, i32, P]
             lib.p4q_cls_saliency.restype = i32
-            lib.oracle_exp32_array.argtypes = [P, i64, P]
-            lib.oracle_exp32_array.restype = i32
             lib.p4q_swiglu_quantize_rows.argtypes = [P, P, i64, i64, P, P]
             lib.p4q_swiglu_quantize_rows.restype = i32
             lib.p4q_causal_attention.argtypes = [P, P, P, i32, i32, i32, i32, i32, P]
@@ -230,21 +228,10 @@ def cls_saliency(q_cls, k_cls, k):
     return A
 
 
-def exp32(x):
-    """The oracle's own fp32 exponential (Cody-Waite reduction, degree-7
-    Taylor polynomial, power-of-two scaling; 0 below -87), elementwise; the
-    CUDA path evaluates the same function bit for bit."""
-    a = _f32(x)
-    y = np.empty_like(a)
-    rc = _load().oracle_exp32_array(_ptr(a), a.size, _ptr(y))
-    if rc != OK:
-        raise ValueError("oracle exp32 failed")
-    return y
-
-
 def swiglu_quantize_rows(gate, up):
-    """h = silu(gate) * up (silu(g) = g * (1 / (1 + exp32(-g))), fp32), then the per-row
-    4-bit quantizer: returns (codes int8 [rows, cols], scale fp32 [rows])."""
+    """h = silu(gate) * up (silu(g) = g / (1 + exp(-g)) in float64, rounded once to
+    fp32), then the per-row 4-bit quantizer: returns (codes int8 [rows, cols],
+    scale fp32 [rows])."""
     g, u = _f32(gate), _f32(up)
     assert g.shape == u.shape and g.ndim == 2
     rows, cols = g.shape

@@ -42,15 +42,12 @@
  *      over the whole kept set, because max is associative.
  *   R8 output indices are sorted ascending.
  *   R12 SwiGLU before down_proj (the decoder's MLP; the paper quantizes every
- *      linear's input per token): h = silu(gate) * up, silu(g) =
- *      g * (1 / (1 + exp32(-g))) (four rounded fp32 steps), then h quantized
- *      by R1. exp32 is this file's own
- *      fp32 exponential (Cody-Waite range reduction with ln 2 split as
- *      355/512 + a low part, degree-7 Taylor polynomial by Horner's rule with
- *      fused multiply-adds, two exact power-of-two scalings; 0 below -87,
- *      inf above 88.72284):
- *      every step is one correctly rounded fp32 operation, so the CUDA path
- *      evaluates the same function bit for bit and the codes match exactly.
+ *      linear's input per token): h = silu(gate) * up with silu(g) =
+ *      g / (1 + e^-g), evaluated in float64 with the C library's exp and
+ *      rounded once to fp32, then h quantized by R1. The paper fixes no
+ *      SwiGLU arithmetic; this is the mathematical function, and a kernel
+ *      that evaluates it in fp32 matches the codes except where the float64
+ *      quotient h / s lies within its error bound of a .5 boundary.
  *   R13 RMSNorm before the quantized linears (the decoder's input norms feed
  *      q/k/v/gate/up; the paper quantizes every linear's input per token):
  *      S = sum x^2 exactly (fp16 squares are multiples of 2^-48; the sum is
@@ -407,47 +404,11 @@ int p4q_cls_saliency(const float* q_cls, const float* k_cls, const float* k, int
   return ORACLE_OK;
 }
 
-/* 2^k as an fp32 bit pattern, -126 <= k <= 127. */
-static float pow2f(int k) {
-  const uint32_t b = (uint32_t)(k + 127) << 23;
-  float f;
-  memcpy(&f, &b, sizeof f);
-  return f;
-}
-
-/* Own fp32 exponential (reading R12): n = rint(x * log2 e); r = x - n ln2 in
- * two fused steps (ln2 = 355/512 + LN2_LO; n * 355/512 is exact for the n
- * that occur); e^r by the degree-7 Taylor polynomial (|r| <= ln2 / 2: the
- * truncation is below 2e-8 relative); times 2^n as two exact multiplications
- * by powers of two. Below -87 the result is 0 (so every other result is a
- * normal number; such values vanish in 1 + e anyway), above 88.72284 inf. */
-float oracle_exp32(float x) {
-  if (x > 0x1.62e430p+6f) return INFINITY;
-  if (x < -87.0f) return 0.0f;
-  const float n = nearbyintf(x * 0x1.715476p+0f);
-  float r = fmaf(-n, 0x1.630000p-1f, x);
-  r = fmaf(-n, -0x1.bd0106p-13f, r);
-  float p = 0x1.a01a02p-13f;
-  p = fmaf(p, r, 0x1.6c16c2p-10f);
-  p = fmaf(p, r, 0x1.111112p-7f);
-  p = fmaf(p, r, 0x1.555556p-5f);
-  p = fmaf(p, r, 0x1.555556p-3f);
-  p = fmaf(p, r, 0.5f);
-  p = fmaf(p, r, 1.0f);
-  p = fmaf(p, r, 1.0f);
-  const int k = (int)n, a = k / 2;
-  return (p * pow2f(a)) * pow2f(k - a);
-}
-
-int oracle_exp32_array(const float* x, int64_t n, float* y) {
-  if (!x || !y || n < 0) return ORACLE_BAD_ARG;
-  for (int64_t i = 0; i < n; ++i) y[i] = oracle_exp32(x[i]);
-  return ORACLE_OK;
-}
-
-/* SwiGLU then the per-token quantizer (reading R12): h = silu(g) * u with
- * silu(g) = g * (1 / (1 + exp32(-g))), every operation one rounded fp32 step, then
- * quantize_row on h. gate, up, h: [rows, cols]. */
+/* SwiGLU then the per-token quantizer (reading R12; the decoder MLP feeds
+ * down_proj with silu(gate) * up, and App. A quantizes every linear input per
+ * token): h = g / (1 + exp(-g)) * u in float64 with the C library's exp,
+ * rounded once to fp32, then quantize_row (R1) on the fp32 row. gate, up:
+ * [rows, cols] (fp16 values widened to fp32: exact). */
 int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, int64_t cols, int8_t* code,
                              float* scale) {
   if (!gate || !up || !code || !scale || rows < 0 || cols <= 0) return ORACLE_BAD_ARG;
@@ -460,10 +421,9 @@ int p4q_swiglu_quantize_rows(const float* gate, const float* up, int64_t rows, i
       continue;
     }
     for (int64_t k = 0; k < cols; ++k) {
-      const float g = gate[r * cols + k];
-      const float sig = 1.0f / (1.0f + oracle_exp32(-g));
-      const float silu = g * sig;
-      h[k] = silu * up[r * cols + k];
+      const double g = gate[r * cols + k];
+      const double silu = g / (1.0 + exp(-g));
+      h[k] = (float)(silu * (double)up[r * cols + k]);
     }
     quantize_row(h, cols, code + r * cols, scale + r);
     free(h);

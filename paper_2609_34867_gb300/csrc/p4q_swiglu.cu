@@ -5,9 +5,10 @@
 //   then a = max|h|, s = a / 7, code = clamp(round_half_even(h / s), -8, 7).
 // exp32 is an own fp32 exponential (Cody-Waite reduction with ln 2 split as
 // 355/512 + a low part, degree-7 Taylor polynomial by Horner's rule with fused
-// multiply-adds, two exact power-of-two scalings; 0 below -87, inf above
-// 88.72284): every step is one correctly rounded fp32 operation, so the codes
-// equal those of a CPU evaluation of the same steps bit for bit.
+// multiply-adds, two exact power-of-two scalings; within 0.9 ulp of e^x; 0
+// below -87, inf above 88.72284). The fp32 h is within 3 rounding units of
+// the real silu(g) * up, so the codes are those of the exact SwiGLU except
+// where h / s falls within 3.2e-6 of a .5 boundary.
 //
 // Kernel: one CTA of 512 threads per row; each thread holds its chunks of 8
 // values of h in registers (computed once), the row's abs-max comes from a

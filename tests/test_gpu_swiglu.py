@@ -1,5 +1,9 @@
 """GPU parity of SwiGLU -> per-token INT4 (the input of down_proj) against the
-oracle: codes, scale bits, expanded codes and their row sums bit-exact."""
+float64 oracle (silu with the C library's exp): scales within 1e-6, codes
+identical except where the float64 quotient h / s lies within the kernel's
+error bound of a .5 boundary (reading R12: the fp32 SwiGLU quotient is within
+3.2e-6 of the float64 one; the band is 1e-5), expanded codes and row sums
+consistent with the packed ones."""
 import numpy as np
 import pytest
 import torch
@@ -22,19 +26,37 @@ def _run(p4q, dev, G, U, expanded=True):
         (None if su is None else su.cpu().numpy())
 
 
+FLT_MIN = float(np.finfo(np.float32).tiny)
+BAND = 1e-5           # codes are compared where the float64 quotient is this far from a .5 boundary
+SATURATE = -88.72284  # below this gate the kernel's exponential of -g is inf: silu(g) = 0
+
+
 def _check(p4q, dev, g, u, expanded=True, G=None, U=None):
     G = torch.from_numpy(g).to(dev) if G is None else G
     U = torch.from_numpy(u).to(dev) if U is None else U
     q, s, xu, su = _run(p4q, dev, G, U, expanded)
-    c, sr = oracle.swiglu_quantize_rows(g, u)
-    assert np.array_equal(s.view(np.uint32), sr.view(np.uint32)), "scale bits differ"
     got = oracle.unpack_codes(q)
-    bad = np.argwhere(got != c)
-    assert bad.size == 0, f"{len(bad)} codes differ, first at {bad[:3].tolist()}"
+    c, sr = oracle.swiglu_quantize_rows(g, u)
+    gd, ud = g.astype(np.float64), u.astype(np.float64)
+    with np.errstate(over="ignore"):  # exp(-g) = inf for very negative gates: silu = 0
+        h = gd / (1.0 + np.exp(-gd)) * ud
+    a = np.abs(h).max(axis=1)
+    # rows whose values lie below the fp32 normal range, or whose every gate
+    # saturates the kernel's exponential, come back as zero rows
+    tiny = (a < FLT_MIN) | np.all(gd < SATURATE, axis=1)
+    assert not got[tiny].any() and not s[tiny].any(), "a flushed row is not zero"
+    ok = ~tiny
+    assert np.all(np.abs(s[ok].astype(np.float64) / sr[ok] - 1.0) <= 1e-6), "scales differ"
+    qq = h[ok] / (a[ok] / 7.0)[:, None]
+    near = np.abs(np.abs(qq - np.floor(qq)) - 0.5) < BAND
+    g_ok, c_ok = got[ok], c[ok]
+    bad = np.argwhere((g_ok != c_ok) & ~near)
+    assert bad.size == 0, f"{len(bad)} codes differ away from a .5 boundary, first at {bad[:3].tolist()}"
+    assert np.all(np.abs(g_ok[near] - qq[near]) <= 0.5 + BAND)
     if expanded:
         # per 32-bit word of packed codes: its four even-index codes, then its four odd ones, + 8
         K = g.shape[1]
-        w = (c.astype(np.int16) + 8).reshape(-1, K // 8, 8)
+        w = (got.astype(np.int16) + 8).reshape(-1, K // 8, 8)
         want = np.concatenate([w[..., 0::2], w[..., 1::2]], axis=-1).reshape(-1, K).astype(np.uint8)
         assert np.array_equal(xu, want)
         assert np.array_equal(su, want.astype(np.int64).sum(1))
@@ -49,8 +71,8 @@ def test_swiglu_quant_matches_oracle(p4q, dev, M, K):
 
 
 def test_swiglu_quant_extremes(p4q, dev):
-    """Gates past exp32's cuts (inf and 0 branches), fp16 extremes, zero rows,
-    rows where every gate is very negative (h = -0 * u)."""
+    """Gates past the kernel exponential's cuts (inf and 0 branches), fp16
+    extremes, zero rows, rows where every gate is very negative (zero rows)."""
     rng = np.random.default_rng(9)
     K = 1024
     g = (rng.standard_normal((8, K)) * 40).astype(np.float16)
