@@ -57,10 +57,11 @@ WORKLOAD = wl.LLAVANEXT_13B
 FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed steps
 
 # Latest ncu capture of the dominant kernel (the expanded-operand GEMM): mean
-# DRAM bytes (read + write) per launch over the three GEMMs of one step of
-# this workload, valid only while the GEMM source is unchanged since the
-# capture.
-PROFILED_GEMM = {"source_sha1": "a5aabe263180372449196085094568fbaf61e0c2", "dram_bytes_per_launch": 115333547}
+# DRAM bytes (read + write) per launch over the three GEMM shapes of one step
+# of the 32 x 2880 x 5120 workload (22528 x 43008 x 5120, 22528 x 5120 x 5120,
+# 22528 x 5120 x 13824), valid only while the GEMM source is unchanged since
+# the capture.
+PROFILED_GEMM = {"source_sha1": "8e8c6e9b8d145d3228bcfca3a69b86fdbd7b9463", "dram_bytes_per_launch": 1837964714}
 
 
 def gemm_source_sha1() -> str:

@@ -34,6 +34,8 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <algorithm>
+
 #include "p4q_device.cuh"
 #include "p4q_internal.h"
 
@@ -59,6 +61,7 @@ struct Params8 {
   int M, N, K, batch;
   int num_m, num_n, per, tiles;  // per: tiles per batch entry
   int bn;                        // int32 tiles: output columns per pair tile (<= BN)
+  int gm;                        // row tiles per raster group (tile_coords)
   int f32_out;                   // int32 tiles: store the exact integers as fp32 values instead
   const float* s_a;
   const float* s_b;
@@ -83,10 +86,12 @@ struct Lay8 {
   static_assert(SMEM <= 232448, "shared memory budget");
 };
 
-// Tile t -> (batch entry, row tile, column tile). Row tiles vary fastest,
-// except for narrow int32 tiles (bn < BN: a few column tiles over a short B),
-// whose column tiles vary fastest, so that the pairs reading the same A rows
-// run side by side and those rows come from DRAM once.
+// Tile t -> (batch entry, row tile, column tile). Narrow int32 tiles (bn <
+// BN: a few column tiles over a short B) vary their column tile fastest, so
+// that the pairs reading the same A rows run side by side. Otherwise the row
+// tiles are rastered in groups of p.gm: consecutive tiles sweep a group's row
+// tiles, then the next column tile, so a group's A rows (sized to stay in L2)
+// are read from DRAM once while the group sweeps all of B.
 __device__ __forceinline__ void tile_coords(const Params8& p, int t, int* bz, int* mt, int* nb) {
   *bz = t / p.per;
   const int r = t - *bz * p.per;
@@ -94,8 +99,12 @@ __device__ __forceinline__ void tile_coords(const Params8& p, int t, int* bz, in
     *mt = r / p.num_n;
     *nb = r - *mt * p.num_n;
   } else {
-    *nb = r / p.num_m;
-    *mt = r - *nb * p.num_m;
+    const int span = p.gm * p.num_n;  // tiles of a full group
+    const int grp = r / span;
+    const int gm = min(p.gm, p.num_m - grp * p.gm);
+    const int q = r - grp * span;
+    *nb = q / gm;
+    *mt = grp * p.gm + (q - *nb * gm);
   }
 }
 
@@ -405,6 +414,8 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
   p.num_m = (g.M + 2 * BM - 1) / (2 * BM);
   p.num_n = (g.N + bn - 1) / bn;
   p.bn = bn;
+  // a raster group's A rows: about 24 MB, so they stay in the 129 MB L2 beside B and the output
+  p.gm = std::max(1, std::min(p.num_m, static_cast<int>((24u << 20) / (static_cast<size_t>(2 * BM) * g.K))));
   p.f32_out = g.f32_out ? 1 : 0;
   p.per = p.num_m * p.num_n;
   p.tiles = p.per * batch;

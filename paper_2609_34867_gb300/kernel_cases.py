@@ -12,6 +12,7 @@
   python -m paper_2609_34867_gb300.kernel_cases mse B M D [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases topk B N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases peak {f8,s8,dp4a} ITERS [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases sweep {gemm,quant,select} [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -44,6 +45,13 @@ selects the first replayed launch.
           pipe (f8: tcgen05 kind::f8f6f4 MMAs on operands in shared memory;
           s8: mma.sync m16n8k32 s8; dp4a), ITERS rounds (ops = 2 per
           multiply-add, as counted by the probe);
+  sweep   the GEMM + quantizer sweep (every M x (K, N) of the LLaVA-shaped
+          sweep: the W4A4 linear as called, p4q_w4a4_linear_ws with its
+          operand expansion, and the GEMM kernel alone on expanded operands;
+          p4q_quant_act on every M x K) or the selector sweep (576 .. 2880
+          tokens, 1 .. 64 images, budgets 5 .. 50%, inputs drawn on the GPU
+          from a seeded generator: N(0,1) with the 8 outlier channels x20, 3
+          concepts, softmax CLS saliency), one table row per point;
   saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
           heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
           fp16 keys and queries in, 4 B N out).
@@ -112,10 +120,71 @@ def peak_tops(kind: str, dev, reps: int = 5, iters: int | None = None) -> float:
     return best
 
 
+def _sweep(kind: str, reps: int, dev):
+    if kind == "gemm":
+        print("| M | K | N | linear (ws, expansion included) us | TOPS | GEMM kernel alone us | TOPS |")
+        print("|---|---|---|---|---|---|---|")
+        g = torch.Generator(device=dev).manual_seed(wl.SWEEP_SEED)
+        for K, N in wl.SWEEP_KN:
+            Wq = torch.randint(0, 256, (N, K // 2), dtype=torch.uint8, device=dev, generator=g)
+            s_w = torch.rand(N, device=dev, generator=g) * 0.01
+            Wu, sW = p4q.expand_codes(Wq)
+            for M in wl.SWEEP_M:
+                Xq = torch.randint(0, 256, (M, K // 2), dtype=torch.uint8, device=dev, generator=g)
+                s_a = torch.rand(M, device=dev, generator=g)
+                Y = torch.empty((M, N), dtype=torch.float16, device=dev)
+                ws = p4q.linear_workspace(M, N, K, dev)
+                t_lin = _timed(lambda: p4q.p4q_w4a4_linear_ws(Xq, s_a, Wq, s_w, Y, ws), reps, dev)
+                Xu, sX = p4q.expand_codes(Xq)
+                if N >= 256 and M >= 16:
+                    t_g = _timed(lambda: p4q.p4q_w4a4_linear_expanded(Xu, sX, s_a, Wu, sW, s_w, Y), reps, dev)
+                    g8 = f"{t_g * 1e3:.1f} | {2 * M * N * K / t_g / 1e9:.1f}"
+                else:
+                    g8 = "- | -"
+                print(f"| {M} | {K} | {N} | {t_lin * 1e3:.1f} | {2 * M * N * K / t_lin / 1e9:.1f} | {g8} |", flush=True)
+                del Xq, Y, ws, Xu, sX
+            del Wq, Wu, sW
+    elif kind == "quant":
+        print("| M | K | us | GB/s |")
+        print("|---|---|---|---|")
+        for K in sorted({k for k, _ in wl.SWEEP_KN}):
+            Xall = torch.from_numpy(wl.activations(max(wl.SWEEP_M), K, seed=wl.SWEEP_SEED)).to(dev)
+            for M in wl.SWEEP_M:
+                X = Xall[:M]
+                Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)
+                sc = torch.empty((M,), dtype=torch.float32, device=dev)
+                t = _timed(lambda: p4q.p4q_quant_act(X, Xq, sc), reps, dev)
+                nbytes = 2 * M * K + M * K // 2 + 4 * M
+                print(f"| {M} | {K} | {t * 1e3:.1f} | {nbytes / t / 1e6:.1f} |", flush=True)
+            del Xall
+    else:
+        print("| N | B | budget % | K | us / call | us / image |")
+        print("|---|---|---|---|---|---|")
+        g = torch.Generator(device=dev).manual_seed(wl.SWEEP_SEED)
+        d = 4096
+        out_ch = torch.from_numpy(wl.outlier_channels(d)).to(dev)
+        points = [(N, B, pct) for N in wl.SWEEP_SEL_N for B in wl.SWEEP_SEL_B for pct in (11.1,)]
+        points += [(N, 16, pct) for N in (576, 2880) for pct in wl.SWEEP_SEL_PCT if pct != 11.1]
+        for N, B, pct in points:
+            V = torch.randn((B, N, d), device=dev, generator=g)
+            V[:, :, out_ch] *= 20.0
+            V = V.to(torch.float16)
+            pick = torch.randint(0, N, (B, 3), device=dev, generator=g)
+            Q = (V.float().gather(1, pick[:, :, None].expand(B, 3, d)) +
+                 0.5 * torch.randn((B, 3, d), device=dev, generator=g)).to(torch.float16)
+            A = torch.softmax(2.0 * torch.randn((B, N), device=dev, generator=g), dim=1)
+            K = wl.sweep_budget(N, pct)
+            ws = p4q.select_workspace(B, N, d, 3, K, dev)
+            idx = torch.empty((B, K), dtype=torch.int32, device=dev)
+            t = _timed(lambda: p4q.p4q_select(V, Q, A, K, idx, ws), reps, dev)
+            print(f"| {N} | {B} | {pct:g} | {K} | {t * 1e3:.1f} | {t * 1e3 / B:.2f} |", flush=True)
+            del V, Q, A, ws, idx
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn",
-                                     "mse", "topk", "peak"])
+                                     "mse", "topk", "peak", "sweep"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -213,6 +282,8 @@ def main(argv=None):
         rho = torch.empty((B,), dtype=torch.float32, device=dev)
         ms = _timed(lambda: p4q.p4q_topk_replacement(s1, s2, K, inter, rho), a.reps, dev)
         print(f"topk {B}x{N} K={K}: {ms * 1e3:.1f} us/call, {8 * B * N / ms / 1e6:.1f} GB/s")
+    elif a.case == "sweep":
+        _sweep(a.args[0], a.reps, dev)
     elif a.case == "peak":
         kind, iters = a.args[0], int(a.args[1])
         sink = torch.zeros((8192,), dtype=torch.int32, device=dev)
