@@ -81,12 +81,13 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   if (A_cls && !aligned16(A_cls)) return P4Q_ERR_MISALIGNED;
   const Budget bud = split(*params, have_q, A_cls != nullptr);
   const int R0 = bud.Kq + bud.Ks;
+  const bool gram = select_gram_mode(N, bud.Kd);
   const int C = select_candidates(N, R0, bud.Kd);
-  const size_t need = select_workspace_layout(B, N, d, Jeff, R0, C, nullptr, nullptr);
+  const size_t need = select_workspace_layout(B, N, d, Jeff, R0, C, gram, nullptr, nullptr);
   if (!ws || ws_bytes < need) return P4Q_ERR_WORKSPACE_TOO_SMALL;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return P4Q_ERR_MISALIGNED;
   SelectWorkspace w;
-  select_workspace_layout(B, N, d, Jeff, R0, C, &w, ws);
+  select_workspace_layout(B, N, d, Jeff, R0, C, gram, &w, ws);
   SelectPlan plan{B, N, d, Jeff, params->K, bud.Kq, bud.Ks, bud.Kd};
 
   // Fake-quantized copies of the projector features (and of the concepts):
@@ -120,12 +121,18 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     if ((e = counted(launch_select_stages12(plan, w, A_cls, idx, stream))) != cudaSuccess) return from_cuda(e);
   }
   if (bud.Kd == 0) return P4Q_OK;
-  if (R0 > 0) {
-    if ((e = counted(launch_gather_r0(plan, w, stream))) != cudaSuccess) return from_cuda(e);
-    if ((e = counted(launch_r0_cosmax(plan, w, stream), 2)) != cudaSuccess) return from_cuda(e);  // GEMM + row pass
+  if (w.gram) {
+    // small images: every token pair's dot product; stage 3 takes R0's maxima from it
+    if ((e = counted(launch_gram(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+    if (R0 > 0 && (e = counted(launch_gram_cosmax(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+  } else {
+    if (R0 > 0) {
+      if ((e = counted(launch_gather_r0(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+      if ((e = counted(launch_r0_cosmax(plan, w, stream), 2)) != cudaSuccess) return from_cuda(e);  // GEMM + row pass
+    }
+    // candidates, their rows, their pairwise dot products
+    if ((e = counted(launch_candidates(plan, w, stream), 3)) != cudaSuccess) return from_cuda(e);
   }
-  // candidates, their rows, their pairwise dot products
-  if ((e = counted(launch_candidates(plan, w, stream), 3)) != cudaSuccess) return from_cuda(e);
   return from_cuda(counted(launch_select_diverse(plan, w, idx, stream)));
 }
 
@@ -461,10 +468,11 @@ size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_p
   if (!params || B < 1 || N < 1 || d < 1 || J < 0 || N > P4Q_MAX_TOKENS || J > P4Q_MAX_CONCEPTS ||
       d % 128 != 0 || d > P4Q_MAX_ROW || params->K < 1 || params->K > N)
     return 0;
-  // the largest R0 and candidate count a call with these sizes can have:
-  // concepts and CLS saliency present (R0), or absent (K_d = K)
-  const int C = select_candidates(N, 0, params->K);
-  return select_workspace_layout(B, N, d, J, select_r0(*params, J > 0, true), C, nullptr, nullptr);
+  // every region at the largest a call with these sizes can need: R0 with
+  // concepts and CLS saliency present, the candidates with both absent (K_d = K)
+  const bool gram = select_gram_mode(N, params->K);
+  return select_workspace_layout(B, N, d, J, select_r0(*params, J > 0, true), select_candidates(N, 0, params->K),
+                                 gram, nullptr, nullptr);
 }
 
 p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
@@ -558,8 +566,9 @@ extern "C" p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d,
   // Every region of the scratch is written before it is read on each call, so
   // nothing needs clearing between calls.
   const int r0 = select_r0(*params, have_q, A_cls != nullptr);
-  if (select_workspace_layout(B, N, d, Jeff, r0, select_candidates(N, r0, params->K - r0), nullptr, nullptr) >
-      kNoAllocScratchBytes)
+  const int kd = params->K - r0;
+  if (select_workspace_layout(B, N, d, Jeff, r0, select_candidates(N, r0, kd), select_gram_mode(N, kd), nullptr,
+                              nullptr) > kNoAllocScratchBytes)
     return P4Q_ERR_WORKSPACE_TOO_SMALL;
   if ((st = check_device()) != P4Q_OK) return st;
   void* ws = nullptr;

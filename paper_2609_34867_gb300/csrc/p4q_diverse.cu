@@ -163,7 +163,7 @@ __device__ void pool_rounds(int npool, int Kd, DivScratch& s) {
 struct DivArgs {
   const uint32_t* kept12;  // [B, words] R0 as bits
   const float* m;          // [B, N] largest cosine to R0 (R0 > 0)
-  const int32_t* cand;     // [B, C] candidates, ascending
+  const int32_t* cand;     // [B, C] candidates, ascending (nullptr: every token, C = N)
   const int32_t* candnorm; // [B, C]
   const float* cdots;      // [B, C, cpitch] their pairwise code dot products
   int C, cpitch;
@@ -217,7 +217,8 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
   pdl_launch_dependents();
   for (int w = threadIdx.x; w < words; w += kThreads) s.keptbits[w] = a.kept12[static_cast<size_t>(b) * words + w];
   __syncthreads();  // candof is cleared
-  for (int c = threadIdx.x; c < a.C; c += kThreads) s.candof[a.cand[static_cast<size_t>(b) * a.C + c]] = static_cast<int16_t>(c);
+  for (int c = threadIdx.x; c < a.C; c += kThreads)
+    s.candof[a.cand ? a.cand[static_cast<size_t>(b) * a.C + c] : c] = static_cast<int16_t>(c);
   __syncthreads();
 
   bool kept[kPer];
@@ -578,8 +579,8 @@ cudaError_t launch_select_diverse(const SelectPlan& p, const SelectWorkspace& ws
   DivArgs a;
   a.kept12 = ws.kept12;
   a.m = ws.m;
-  a.cand = ws.cand;
-  a.candnorm = ws.candnorm;
+  a.cand = ws.gram ? nullptr : ws.cand;
+  a.candnorm = ws.gram ? ws.vnorm : ws.candnorm;  // Gram mode: candidate c is token c
   a.cdots = ws.cdots;
   a.C = ws.C;
   a.cpitch = ws.cpitch;

@@ -171,16 +171,22 @@ struct SelectWorkspace {
   int32_t* candnorm; // [B, C]
   float* cdots;      // [B, C, cpitch] their code dot products (exact, fp32)
   int cpitch;        // C rounded up to a multiple of 4
+  bool gram;         // small images: every token is a candidate (C = N, cdots by token, no cand lists)
 };
 
 // Candidates of stage 3: up to kCandExtra more than the K_d picks (a pool's
-// worth), at most kCandMax.
-constexpr int kCandExtra = 128, kCandMax = 1024;
+// worth), at most kCandMax. Images of at most kGramMaxTokens tokens take every
+// token as a candidate: one GEMM of all their token pairs replaces R0's GEMM,
+// the candidate selection and the gather (Gram mode).
+constexpr int kCandExtra = 128, kCandMax = 1024, kGramMaxTokens = 1024;
+bool select_gram_mode(int N, int Kd);
 int select_candidates(int N, int R0, int Kd);
 
 // Workspace of one selector call with R0 = Kq + Ks tokens after stages 1-2
-// and C candidates in stage 3.
-size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, SelectWorkspace* ws, void* base);
+// and C candidates in stage 3 (Gram mode: C = N). Every region grows with R0
+// and with C, so the layout at the largest R0 and C covers any call.
+size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, bool gram, SelectWorkspace* ws,
+                               void* base);
 int r0_tile_n(int R0);
 
 // Stages 1-2: kept12 bits, r0tok, and idx when p.Kd == 0.
@@ -197,6 +203,10 @@ cudaError_t launch_r0_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cud
 // The candidates of stage 3 (per image), their expanded codes, and the
 // code dot products of every pair of them (a batched tensor-core GEMM).
 cudaError_t launch_candidates(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+// Gram mode: the code dot products of every token pair of each image into
+// cdots; then each token's largest cosine to R0 from them (m).
+cudaError_t launch_gram(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
+cudaError_t launch_gram_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream);
 // Stage 3 (greedy max-min diversity) from kept12, m and the candidates; writes idx.
 cudaError_t launch_select_diverse(const SelectPlan& p, const SelectWorkspace& ws, int32_t* idx, cudaStream_t stream);
 unsigned int diverse_read_and_clear_error();

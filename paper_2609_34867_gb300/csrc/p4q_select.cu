@@ -187,19 +187,26 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const uint8_t* __restr
 // of it, so the maximum is exactly code_cosine's.
 constexpr int kCosmaxRows = 8;  // one row per warp: many warps in flight
 
+// cols == nullptr: column j of a row is R0 token j (the R0 GEMM's output,
+// norms r0norm); else the row holds every token (the Gram mode's cdots) and
+// column j is token cols[b, j] (norms from vnorm).
 __global__ void __launch_bounds__(256) r0_cosmax_kernel(const float* __restrict__ dots, int pitch,
                                                         const int32_t* __restrict__ vnorm,
-                                                        const int32_t* __restrict__ r0norm, int N, int R0,
+                                                        const int32_t* __restrict__ r0norm,
+                                                        const int32_t* __restrict__ cols, int N, int R0,
                                                         float* __restrict__ m) {
-  extern __shared__ int32_t nr[];  // [R0] squared norms of the image's kept tokens, then [R0] rsqrtf of them
+  extern __shared__ int32_t nr[];  // [R0] squared norms of the image's kept tokens, [R0] their rsqrtf, [R0] columns
   float* rr = reinterpret_cast<float*>(nr + R0);
+  int32_t* cj = nr + 2 * R0;
   pdl_wait();
   pdl_launch_dependents();
   const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int j = threadIdx.x; j < R0; j += blockDim.x) {
-    const int v = r0norm[static_cast<size_t>(b) * R0 + j];
+    const int c = cols ? cols[static_cast<size_t>(b) * R0 + j] : j;
+    const int v = cols ? vnorm[static_cast<size_t>(b) * N + c] : r0norm[static_cast<size_t>(b) * R0 + j];
     nr[j] = v;
     rr[j] = v > 0 ? rsqrtf(static_cast<float>(v)) : 0.0f;
+    cj[j] = c;
   }
   __syncthreads();
   for (int i = blockIdx.x * kCosmaxRows + warp; i < min(N, (blockIdx.x + 1) * kCosmaxRows); i += blockDim.x / 32) {
@@ -209,13 +216,13 @@ __global__ void __launch_bounds__(256) r0_cosmax_kernel(const float* __restrict_
     const float ra = na > 0 ? rsqrtf(static_cast<float>(na)) : 0.0f;
     float amax = -INFINITY;
 #pragma unroll 4
-    for (int j = lane; j < R0; j += 32) amax = fmaxf(amax, __ldg(dr + j) * ra * rr[j]);
+    for (int j = lane; j < R0; j += 32) amax = fmaxf(amax, __ldg(dr + cj[j]) * ra * rr[j]);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, o));
     float emax = -INFINITY;
 #pragma unroll 4
     for (int j = lane; j < R0; j += 32) {
-      const float dot = __ldg(dr + j);
+      const float dot = __ldg(dr + cj[j]);
       if (dot * ra * rr[j] >= amax - kCosMargin) emax = fmaxf(emax, code_cosine(static_cast<int>(dot), na, nr[j]));
     }
 #pragma unroll
@@ -286,15 +293,21 @@ int r0_tile_n(int R0) {
   return (per + 31) / 32 * 32;
 }
 
+bool select_gram_mode(int N, int Kd) { return Kd > 0 && N <= kGramMaxTokens; }
+
 int select_candidates(int N, int R0, int Kd) {
   if (Kd <= 0) return 0;
+  if (select_gram_mode(N, Kd)) return N;
   const int want = std::min((Kd + kCandExtra + 31) / 32 * 32, kCandMax);
   return std::min(N - R0, want);
 }
 
-size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, SelectWorkspace* ws, void* base) {
-  const size_t BN = static_cast<size_t>(B) * N, BJ = static_cast<size_t>(B) * J, BR = static_cast<size_t>(B) * R0;
-  const size_t BC = static_cast<size_t>(B) * C;
+size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, bool gram, SelectWorkspace* ws,
+                               void* base) {
+  const size_t BN = static_cast<size_t>(B) * N, BJ = static_cast<size_t>(B) * J;
+  const bool r0gemm = !gram && C > 0;  // R0's own GEMM (not in Gram mode, nor without a diversity stage)
+  const size_t BR = r0gemm ? static_cast<size_t>(B) * R0 : 0;
+  const size_t BC = gram ? 0 : static_cast<size_t>(B) * C;   // gathered candidates (not in Gram mode)
   const int cp = (C + 3) & ~3;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -311,10 +324,11 @@ size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, Select
   const size_t o_sc = take(BN * qp * 4);
   const size_t o_vu = take(BN * d), o_vsum = take(BN * 4);
   const size_t o_k12 = take(static_cast<size_t>(B) * ((N + 31) / 32) * 4);
-  const size_t o_r0t = take(BR * 4), o_r0u = take(BR * d), o_r0s = take(BR * 4), o_r0n = take(BR * 4);
-  const size_t o_dot = take(BN * dp * 4), o_m = take(BN * 4);
+  const size_t o_r0t = take(static_cast<size_t>(B) * R0 * 4);
+  const size_t o_r0u = take(BR * d), o_r0s = take(BR * 4), o_r0n = take(BR * 4);
+  const size_t o_dot = take(r0gemm ? BN * dp * 4 : 0), o_m = take(BN * 4);
   const size_t o_ct = take(BC * 4), o_cu = take(BC * d), o_cs = take(BC * 4), o_cn = take(BC * 4);
-  const size_t o_cd = take(BC * cp * 4);
+  const size_t o_cd = take(static_cast<size_t>(B) * C * cp * 4);
   if (ws && base) {
     uint8_t* p = static_cast<uint8_t*>(base);
     ws->vscale = reinterpret_cast<float*>(p + o_vs);
@@ -344,6 +358,7 @@ size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, Select
     ws->candnorm = reinterpret_cast<int32_t*>(p + o_cn);
     ws->cdots = reinterpret_cast<float*>(p + o_cd);
     ws->cpitch = cp;
+    ws->gram = gram;
   }
   return off;
 }
@@ -390,8 +405,30 @@ cudaError_t launch_r0_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cud
   cudaError_t e = launch_gemm8(g, ws.vu, ws.vsum, ws.r0u, ws.r0sum, stream);
   if (e != cudaSuccess) return e;
   const dim3 grid((p.N + kCosmaxRows - 1) / kCosmaxRows, p.B);
-  return launch_pdl(r0_cosmax_kernel, grid, dim3(256), static_cast<size_t>(R0) * 8, stream, ws.dots, ws.dot_pitch,
-                    ws.vnorm, ws.r0norm, p.N, R0, ws.m);
+  return launch_pdl(r0_cosmax_kernel, grid, dim3(256), static_cast<size_t>(R0) * 12, stream, ws.dots,
+                    ws.dot_pitch, ws.vnorm, ws.r0norm, static_cast<const int32_t*>(nullptr), p.N, R0, ws.m);
+}
+
+cudaError_t launch_gram(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
+  GemmArgs g;  // every token against every token of its image
+  g.M = p.N;
+  g.N = p.N;
+  g.K = p.d;
+  g.batch = p.B;
+  g.out = GemmOut::kS32;
+  g.D = ws.cdots;
+  g.d_pitch = ws.cpitch;
+  g.f32_out = true;
+  return launch_gemm8(g, ws.vu, ws.vsum, ws.vu, ws.vsum, stream);
+}
+
+cudaError_t launch_gram_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {
+  const int R0 = p.Kq + p.Ks;
+  if (R0 == 0) return cudaSuccess;
+  const dim3 grid((p.N + kCosmaxRows - 1) / kCosmaxRows, p.B);
+  return launch_pdl(r0_cosmax_kernel, grid, dim3(256), static_cast<size_t>(R0) * 12, stream, ws.cdots, ws.cpitch,
+                    ws.vnorm, static_cast<const int32_t*>(nullptr), static_cast<const int32_t*>(ws.r0tok), p.N, R0,
+                    ws.m);
 }
 
 cudaError_t launch_candidates(const SelectPlan& p, const SelectWorkspace& ws, cudaStream_t stream) {

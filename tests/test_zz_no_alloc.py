@@ -65,11 +65,11 @@ def test_noalloc_select_at_its_capacity_and_just_beyond(p4q, dev):
     f = _fn(p4q.lib())
     stream = torch.cuda.current_stream()
     N, d, K = 576, 4096, 192
-    w = wl.Workload("t", B=12, N=N, d=d, K=K, T=0, J=3, seed=44, heavy_tail=False, linears=())
+    w = wl.Workload("t", B=40, N=N, d=d, K=K, T=0, J=3, seed=44, heavy_tail=False, linears=())
     x = wl.selector_inputs(w)
     Vall, Qall, Aall = (torch.from_numpy(a).to(dev) for a in (x.V, x.Q, x.A))
     fits, refused = None, None
-    for B in range(1, 13):  # rejected sizes launch nothing, so probing them is safe
+    for B in range(1, 41):  # rejected sizes launch nothing, so probing them is safe
         idx = torch.full((B, K), -1, dtype=torch.int32, device=dev)
         rc = _call(f, Vall[:B], Qall[:B], Aall[:B], K, idx, stream)
         torch.cuda.synchronize()
