@@ -382,12 +382,14 @@ size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_p
  * Requires 1 <= B, 1 <= K <= N <= P4Q_MAX_TOKENS, 0 <= J <= P4Q_MAX_CONCEPTS,
  * d % 128 == 0, 128 <= d <= P4Q_MAX_ROW, 0 <= alpha, beta and
  * alpha + beta <= 1000.
- * All work is ordered on `stream`. When the cosine-matrix GEMM leaves an SM
- * per image free, stages 1-2 run beside it on a second stream the library
- * owns (one per device, created on the first call that is not being captured
- * into a CUDA graph), forked from and joined back into `stream` by events
- * inside the call, so a graph captured from `stream` contains both branches;
- * a host lock keeps concurrent callers' fork/join pairs apart. */
+ * All work is ordered on `stream`. For images of at most 1024 tokens with a
+ * diversity stage (K_d > 0) the GEMM of all token pairs runs beside the
+ * concept, query and stage 1-2 launches on a second stream the library owns
+ * (one per device, created on the first call that is not being captured into
+ * a CUDA graph; until then the order is serial), forked from and joined back
+ * into `stream` by events inside the call, so a graph captured from `stream`
+ * contains both branches; a host lock keeps concurrent callers' fork/join
+ * pairs apart. */
 p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
                       const float* A_cls, const p4q_select_params* params, int32_t* idx,
                       void* ws, size_t ws_bytes, p4q_stream_t stream);
@@ -407,7 +409,8 @@ p4q_status p4q_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
  * lazy module loading the array is committed on a device by the first call
  * there (which may then fail with P4Q_ERR_CUDA on a full device): make that
  * first call at start-up, inside the caller's memory budget, and before any
- * stream capture. The call allocates nothing itself. All calls on a device
+ * stream capture. The call allocates nothing itself and creates no stream or
+ * event (its launches run in order on `stream`). All calls on a device
  * share the one array, which keeps the last call's contents (every region is
  * written before it is read, so nothing needs clearing): calls whose work
  * overlaps on the GPU (other streams, or several host threads) race and give

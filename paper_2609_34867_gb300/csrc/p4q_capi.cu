@@ -62,19 +62,54 @@ p4q_status check_select_args(const uint16_t* V, int B, int N, int d, int J, cons
   return P4Q_OK;
 }
 
+// A second stream of the library per device, with a fork and a join event,
+// on which the selector's token-pair GEMM (Gram mode) runs beside the
+// concept, query and stage-1/2 launches; created on the first call that is
+// not being captured into a graph. Its users hold g_side_mutex from the fork
+// to the join (the events are shared).
+struct SideStream {
+  cudaStream_t s = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+  bool failed = false;
+};
+std::mutex g_side_mutex;
+SideStream g_side[64];
+
+SideStream* side_stream(cudaStream_t stream) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  SideStream& r = g_side[dev];
+  if (r.s) return &r;
+  if (r.failed) return nullptr;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return nullptr;
+  if (cudaStreamCreateWithFlags(&r.s, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&r.fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&r.join, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    r.failed = true;  // the serial order is used from now on
+    r.s = nullptr;
+    return nullptr;
+  }
+  return &r;
+}
+
 // R0 = Kq + Ks of a call (the workspace layout depends on it).
 int select_r0(const p4q_select_params& p, bool have_q, bool have_a) {
   const Budget bud = split(p, have_q, have_a);
   return bud.Kq + bud.Ks;
 }
 
-// The selector: fake-quantized copies (tokens and concepts in one launch),
-// query cosines, stages 1-2, the initial diversity maxima on the tensor cores
-// (R0's expanded codes gathered, then one GEMM with a max-cosine epilogue),
-// stage 3 (writes idx). Every launch on `stream`.
+// The selector: fake-quantized copies of the tokens and of the concepts,
+// query cosines (a narrow GEMM), stages 1-2, the initial diversity maxima on
+// the tensor cores (Gram mode: one GEMM of all token pairs; otherwise R0's
+// expanded codes gathered, a GEMM against every token and a row pass, then
+// the candidates' pairwise GEMM), stage 3 (writes idx). Work is ordered on
+// `stream`; with use_side the Gram GEMM runs on the library's second stream,
+// forked from and joined back into `stream`.
 p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J, const float* A_cls,
                       const p4q_select_params* params, int32_t* idx, void* ws, size_t ws_bytes,
-                      cudaStream_t stream) {
+                      cudaStream_t stream, bool use_side = true) {
   const bool have_q = (Q != nullptr && J > 0);
   const int Jeff = have_q ? J : 0;
   if (have_q && !aligned16(Q)) return P4Q_ERR_MISALIGNED;
@@ -104,6 +139,23 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   sv.u = w.vu;
   sv.sum_u = w.vsum;
   if ((e = counted(launch_quant_rows(src, B * N, d, sv, stream))) != cudaSuccess) return from_cuda(e);
+  // Gram mode: the token-pair GEMM needs only the token codes; it runs on the
+  // library's second stream beside the concept, query and stage-1/2 launches
+  std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
+  SideStream* side = nullptr;
+  if (w.gram && use_side) {
+    side_lock.lock();
+    side = side_stream(stream);
+    if (side) {
+      cudaError_t se = cudaEventRecord(side->fork, stream);
+      if (se == cudaSuccess) se = cudaStreamWaitEvent(side->s, side->fork, 0);
+      if (se == cudaSuccess) se = counted(launch_gram(plan, w, side->s));
+      if (se == cudaSuccess) se = cudaEventRecord(side->join, side->s);
+      if (se != cudaSuccess) return from_cuda(se);
+    } else {
+      side_lock.unlock();
+    }
+  }
   if (bud.Kq > 0) {
     RowSource qsrc;
     qsrc.X = Q;
@@ -123,7 +175,11 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   if (bud.Kd == 0) return P4Q_OK;
   if (w.gram) {
     // small images: every token pair's dot product; stage 3 takes R0's maxima from it
-    if ((e = counted(launch_gram(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+    if (side) {
+      if ((e = cudaStreamWaitEvent(stream, side->join, 0)) != cudaSuccess) return from_cuda(e);
+    } else if ((e = counted(launch_gram(plan, w, stream))) != cudaSuccess) {
+      return from_cuda(e);
+    }
     if (R0 > 0 && (e = counted(launch_gram_cosmax(plan, w, stream))) != cudaSuccess) return from_cuda(e);
   } else {
     if (R0 > 0) {
@@ -573,7 +629,8 @@ extern "C" p4q_status p4q_select_noalloc(const uint16_t* V, int B, int N, int d,
   if ((st = check_device()) != P4Q_OK) return st;
   void* ws = nullptr;
   if ((st = scratch_address(&ws)) != P4Q_OK) return st;
+  // serial order on `stream`: the call creates no stream or event either
   return run_select(V, B, N, d, Q, J, A_cls, params, idx, ws, kNoAllocScratchBytes,
-                    reinterpret_cast<cudaStream_t>(stream));
+                    reinterpret_cast<cudaStream_t>(stream), false);
 }
 
