@@ -184,7 +184,9 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   } else {
     if (R0 > 0) {
       if ((e = counted(launch_gather_r0(plan, w, stream))) != cudaSuccess) return from_cuda(e);
-      if ((e = counted(launch_r0_cosmax(plan, w, stream), 2)) != cudaSuccess) return from_cuda(e);  // GEMM + row pass
+      // one GEMM with the cosine-max epilogue, or (R0 > kCosMaxCols) a GEMM and a row pass
+      if ((e = counted(launch_r0_cosmax(plan, w, stream), R0 <= kCosMaxCols ? 1 : 2)) != cudaSuccess)
+        return from_cuda(e);
     }
     // candidates, their rows, their pairwise dot products
     if ((e = counted(launch_candidates(plan, w, stream), 3)) != cudaSuccess) return from_cuda(e);

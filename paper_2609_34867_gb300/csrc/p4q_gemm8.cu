@@ -21,6 +21,11 @@
 // int32 tiles may be narrower than 256 columns (p.bn, a multiple of 32): the
 // selector's products of every token with its few kept tokens.
 //
+// Cosine-max tiles (MODE 2, the selector's initial diversity maxima of
+// Eq. 4): the epilogue turns each row's exact dot products into its largest
+// code cosine over the tile's columns and writes that one float per row and
+// column tile (p.num_n partial maxima per row, p.part apart).
+//
 // Kernel: persistent, one cluster of two CTAs per 256 x 256 output tile,
 //   warp 0    MMA issuer (leader CTA): 4 x tcgen05.mma (M 256, N 256, K 32)
 //             per 128-deep k-block into one of two TMEM accumulators;
@@ -67,9 +72,15 @@ struct Params8 {
   const float* s_b;
   const int32_t* sum_a;  // [batch, M] sum of u over each A row
   const int32_t* sum_b;  // [batch, N]
+  const int32_t* norm_a;  // cosine-max tiles: [batch, M] squared code norms of the A rows
+  const int32_t* norm_b;  // [batch, N] of the B rows
+  float* cos_max;         // [num_n][part] with part >= batch * M: each A row's largest cosine per column tile
+  size_t part;
 };
 
-template <int MODE>  // GemmOut::kHalf or kS32
+constexpr int kCosMode = static_cast<int>(GemmOut::kCos);
+
+template <int MODE>  // GemmOut::kHalf, kS32 or kCos
 struct Lay8 {
   static constexpr int ELEM = (MODE == static_cast<int>(GemmOut::kHalf)) ? 2 : 4;
   static constexpr int BOX_BYTES = 32 * 32 * ELEM;
@@ -144,7 +155,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   const int KB = p.K / BK;
-  const int bn = (MODE == static_cast<int>(GemmOut::kS32)) ? p.bn : BN;  // columns of a pair tile
+  const int bn = (MODE != static_cast<int>(GemmOut::kHalf)) ? p.bn : BN;  // columns of a pair tile
   const int hb = bn / 2;                                                  // B rows per CTA
 
   if (threadIdx.x == 0) {
@@ -232,6 +243,98 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           mbar_wait(&full[j % S], (j / S) & 1, reinterpret_cast<volatile int*>(&fresh), &g_gemm8_err,
                     100000000ull);
       }
+    }
+  } else if (MODE == kCosMode) {
+    // ------------------------------------------------------------ epilogue warps: cosine max per row
+    const int ew = warp - kFirstEpiWarp;
+    const int q = warp & 3;  // TMEM lane quarter of this warp
+    int32_t* cnr = reinterpret_cast<int32_t*>(smem + L::OFF_BOX);  // [BN] B norms
+    float* cbias = reinterpret_cast<float*>(cnr + BN);              // [BN] 0, or -inf past N
+    const uint32_t acc_empty_leader = mapa_shared(smem_u32(acc_empty), 0);
+    int it = 0;
+    bool failed = false;
+    for (int t = cluster_id_x(); t < p.tiles; t += nclusters_x(), ++it) {
+      int bz, mt, nb;
+      tile_coords(p, t, &bz, &mt, &nb);
+      const int m0 = mt * (2 * BM) + static_cast<int>(rank) * BM;
+      const int n0 = nb * bn;
+      const int ab = it & 1;
+      if (!failed && !mbar_wait_warp(&acc_full[ab], (it >> 1) & 1, abort_flag, &g_gemm8_err)) failed = true;
+      tc_fence_after();
+      epi_sync8();  // every epilogue warp is done with the previous tile's column constants
+      if (!failed) {
+        for (int i = ew * 32 + lane; i < bn; i += kEpiWarps * 32) {
+          const int n = n0 + i;
+          const size_t nn = static_cast<size_t>(bz) * p.N + n;
+          const bool in = n < p.N;
+          const int nbv = in ? p.norm_b[nn] : 0;
+          sbw[i] = in ? static_cast<float>(-8 * p.sum_b[nn]) : 0.0f;
+          cnr[i] = nbv;
+          colv[i] = nbv > 0 ? rsqrtf(static_cast<float>(nbv)) : 0.0f;
+          cbias[i] = in ? 0.0f : -INFINITY;  // zero-filled B rows past N take no part
+        }
+      }
+      epi_sync8();
+      if (failed) continue;
+      const int m = m0 + q * 32 + lane;
+      const bool row_in = m < p.M;
+      const size_t ma = static_cast<size_t>(bz) * p.M + m;
+      const float corrA = row_in ? static_cast<float>(64 * p.K - 8 * p.sum_a[ma]) : 0.0f;
+      const int na = row_in ? p.norm_a[ma] : 0;
+      const float ra = na > 0 ? rsqrtf(static_cast<float>(na)) : 0.0f;
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ab * BN;
+      // Pass 1: the largest approximate cosine (as dot * rsqrt(na) * rsqrt(nb),
+      // within cos_approx's error bound), the runner-up, and the dot product at
+      // the largest. Only columns within kCosMargin of the largest can hold the
+      // exact maximum; when the runner-up is not among them, the exact maximum
+      // is the largest column's code cosine.
+      float amax = -INFINITY, a2 = -INFINITY, xarg = 0.0f;
+      int carg = 0;
+#pragma unroll 1
+      for (int c0 = 0; c0 < bn; c0 += 32) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(taddr + c0, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int c = c0 + i;
+          const float x = __fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c]);  // exact dot
+          const float ap = __fmul_rn(__fmul_rn(x, ra), colv[c]) + cbias[c];
+          a2 = fmaxf(a2, fminf(ap, amax));
+          if (ap > amax) {
+            amax = ap;
+            xarg = x;
+            carg = c;
+          }
+        }
+      }
+      const bool slow = a2 >= amax - kCosMargin;
+      float emax = code_cosine(static_cast<int>(xarg), na, cnr[carg]);
+      if (__any_sync(0xFFFFFFFFu, slow)) {
+        // Pass 2 (near ties): the exact cosine of every column within the margin
+        float e2 = -INFINITY;
+#pragma unroll 1
+        for (int c0 = 0; c0 < bn; c0 += 32) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(taddr + c0, v);
+          tmem_ld_wait();
+          if (slow) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int c = c0 + i;
+              const float x = __fmaf_rn(__uint_as_float(v[i]), 262144.0f, corrA + sbw[c]);
+              const float ap = __fmul_rn(__fmul_rn(x, ra), colv[c]) + cbias[c];
+              if (ap >= amax - kCosMargin) e2 = fmaxf(e2, code_cosine(static_cast<int>(x), na, cnr[c]));
+            }
+          }
+        }
+        if (slow) emax = e2;
+      }
+      // the accumulator is free for the next tile
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(acc_empty_leader + 8u * ab);
+      if (row_in) p.cos_max[static_cast<size_t>(nb) * p.part + ma] = emax;
     }
   } else {
     // ------------------------------------------------------------ epilogue warps
@@ -388,8 +491,9 @@ size_t ws8_layout(int M, int N, int K, void* base, Ws8* w) {
 
 template <int MODE>
 cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
-  const int bn = (MODE == static_cast<int>(GemmOut::kS32)) ? g.tile_n : BN;
+  const int bn = (MODE != static_cast<int>(GemmOut::kHalf)) ? g.tile_n : BN;
   if (bn < 32 || bn > BN || bn % 32 != 0) return cudaErrorInvalidValue;
+  if (MODE == kCosMode && (!g.norm_a || !g.norm_b || !g.D)) return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(w4a4_gemm8_pair_kernel<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -401,11 +505,15 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
   const int batch = g.batch > 0 ? g.batch : 1;
   if (!make_expanded_map(&ma, w.a8, g.K, g.M, batch, BM)) return cudaErrorInvalidValue;
   if (!make_expanded_map(&mb, w.b8, g.K, g.N, batch, bn / 2)) return cudaErrorInvalidValue;
-  const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
-  // a row narrower than 16 bytes is stored over its whole pitch (the extra
-  // columns hold the products with zero-filled B rows)
-  const int ocols = (g.N * 4 < 16) ? pitch : g.N;
-  if (!make_output_map(&md, g.D, g.out, g.M, ocols, pitch, batch)) return cudaErrorInvalidValue;
+  if (MODE == kCosMode) {
+    md = ma;  // no tiles are stored: one float per A row and column tile
+  } else {
+    const int pitch = g.d_pitch > 0 ? g.d_pitch : g.N;
+    // a row narrower than 16 bytes is stored over its whole pitch (the extra
+    // columns hold the products with zero-filled B rows)
+    const int ocols = (g.N * 4 < 16) ? pitch : g.N;
+    if (!make_output_map(&md, g.D, g.out, g.M, ocols, pitch, batch)) return cudaErrorInvalidValue;
+  }
   Params8 p;
   p.M = g.M;
   p.N = g.N;
@@ -423,6 +531,10 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
   p.s_b = g.s_b;
   p.sum_a = w.sum_a;
   p.sum_b = w.sum_b;
+  p.norm_a = g.norm_a;
+  p.norm_b = g.norm_b;
+  p.cos_max = MODE == kCosMode ? static_cast<float*>(g.D) : nullptr;
+  p.part = static_cast<size_t>(batch) * g.M;
   const int pairs = p.tiles < num_sms() / 2 ? p.tiles : num_sms() / 2;
   return launch_pdl(w4a4_gemm8_pair_kernel<MODE>, dim3(2 * pairs), dim3(kThreads), Lay8<MODE>::SMEM, stream, ma,
                     mb, md, p);
@@ -449,7 +561,11 @@ cudaError_t launch_gemm8(const GemmArgs& g, const uint8_t* a8, const int32_t* su
   w.b8 = const_cast<uint8_t*>(b8);
   w.sum_a = const_cast<int32_t*>(sum_a);
   w.sum_b = const_cast<int32_t*>(sum_b);
-  return g.out == GemmOut::kHalf ? launch8<0>(g, w, stream) : launch8<1>(g, w, stream);
+  switch (g.out) {
+    case GemmOut::kHalf: return launch8<0>(g, w, stream);
+    case GemmOut::kS32: return launch8<1>(g, w, stream);
+    default: return launch8<kCosMode>(g, w, stream);
+  }
 }
 
 cudaError_t launch_w4a4_gemm8(const GemmArgs& g, void* ws, size_t ws_bytes, cudaStream_t stream) {

@@ -160,7 +160,10 @@ struct SelectWorkspace {
   uint8_t* r0u;      // [B, R0, d] its expanded codes
   int32_t* r0sum;    // [B, R0]
   int32_t* r0norm;   // [B, R0]
-  float* dots;       // [B, N, dot_pitch] code dot products of every token with every token of R0 (exact, fp32)
+  float* dots;       // [B, N, dot_pitch] code dot products of every token with every token of R0 (exact,
+                     // fp32), for R0 > kCosMaxCols
+  float* mpart;      // [r0_parts, B, N] each token's largest cosine per column tile of R0 (r0_parts > 1)
+  int r0_parts;      // column tiles of the R0 GEMM (cosine-max epilogue), else 0
   int dot_pitch;     // R0 rounded up to a multiple of 4
   int r0_tile_n;     // column tile width of that GEMM
   float* m;          // [B, N] the largest cosine of each token to R0 (stage 3's initial m)
@@ -179,6 +182,11 @@ struct SelectWorkspace {
 // token as a candidate: one GEMM of all their token pairs replaces R0's GEMM,
 // the candidate selection and the gather (Gram mode).
 constexpr int kCandExtra = 128, kCandMax = 1024, kGramMaxTokens = 1024;
+// Kept sets of at most kCosMaxCols tokens take their tokens' cosine maxima
+// from one GEMM with a cosine-max epilogue (a partial maximum per column tile,
+// merged by the candidate selection); larger ones from an int32-tile GEMM and
+// a row pass.
+constexpr int kCosMaxCols = 1024;
 bool select_gram_mode(int N, int Kd);
 int select_candidates(int N, int R0, int Kd);
 

@@ -18,9 +18,12 @@
 //                           tokens (R0, or the diversity candidates), row by
 //                           row, as an operand of the tensor-core GEMMs.
 //   r0_cosmax_kernel        each token's largest cosine to R0 from the exact
-//                           dot products of that GEMM.
+//                           dot products of an int32-tile GEMM (kept sets of
+//                           more than kCosMaxCols tokens; smaller ones take
+//                           the maxima from the GEMM's cosine-max epilogue).
 //   select_candidates_kernel  the diversity stage's candidates: the free
-//                           tokens with the smallest of those maxima.
+//                           tokens with the smallest of those maxima (after
+//                           merging the epilogue's per-column-tile maxima).
 // Every ranking orders by (score, lower token index first).
 #include <cuda_fp16.h>
 
@@ -119,10 +122,21 @@ __global__ void __launch_bounds__(kMaxThreads, 1)
 // pool phase, that it does. Same layout and radix select as stages 1-2.
 template <int kMaxThreads>
 __global__ void __launch_bounds__(kMaxThreads, 1)
-    select_candidates_kernel(const float* __restrict__ m, const uint32_t* __restrict__ kept12, int N, int R0, int C,
-                             int32_t* __restrict__ cand) {
+    select_candidates_kernel(float* __restrict__ m, const float* __restrict__ mpart, int parts,
+                             const uint32_t* __restrict__ kept12, int N, int R0, int C, int32_t* __restrict__ cand) {
   pdl_wait();
   pdl_launch_dependents();
+  if (mpart != nullptr) {
+    // m = the largest of the per-column-tile maxima (stage 3 reads m too)
+    const size_t part = static_cast<size_t>(gridDim.x) * N;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+      const size_t t = static_cast<size_t>(blockIdx.x) * N + i;
+      float v = mpart[t];
+      for (int k = 1; k < parts; ++k) v = fmaxf(v, mpart[k * part + t]);
+      m[t] = v;
+    }
+    __syncthreads();
+  }
   __shared__ RankScratch s;
   const int b = blockIdx.x, nt = blockDim.x;
   const int base = kPer * threadIdx.x;
@@ -326,7 +340,10 @@ size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, bool g
   const size_t o_k12 = take(static_cast<size_t>(B) * ((N + 31) / 32) * 4);
   const size_t o_r0t = take(static_cast<size_t>(B) * R0 * 4);
   const size_t o_r0u = take(BR * d), o_r0s = take(BR * 4), o_r0n = take(BR * 4);
-  const size_t o_dot = take(r0gemm ? BN * dp * 4 : 0), o_m = take(BN * 4);
+  const bool rowpass = r0gemm && R0 > kCosMaxCols;  // int32 tiles and a row pass
+  const int parts = (r0gemm && !rowpass && R0 > 0) ? (R0 + tn - 1) / tn : 0;
+  const size_t o_dot = take(rowpass ? BN * dp * 4 : 0), o_m = take(BN * 4);
+  const size_t o_mp = take(parts > 1 ? parts * BN * 4 : 0);
   const size_t o_ct = take(BC * 4), o_cu = take(BC * d), o_cs = take(BC * 4), o_cn = take(BC * 4);
   const size_t o_cd = take(static_cast<size_t>(B) * C * cp * 4);
   if (ws && base) {
@@ -348,6 +365,8 @@ size_t select_workspace_layout(int B, int N, int d, int J, int R0, int C, bool g
     ws->r0sum = reinterpret_cast<int32_t*>(p + o_r0s);
     ws->r0norm = reinterpret_cast<int32_t*>(p + o_r0n);
     ws->dots = reinterpret_cast<float*>(p + o_dot);
+    ws->mpart = reinterpret_cast<float*>(p + o_mp);
+    ws->r0_parts = parts;
     ws->dot_pitch = dp;
     ws->r0_tile_n = tn;
     ws->m = reinterpret_cast<float*>(p + o_m);
@@ -397,11 +416,19 @@ cudaError_t launch_r0_cosmax(const SelectPlan& p, const SelectWorkspace& ws, cud
   g.N = R0;   // B rows: its kept set
   g.K = p.d;
   g.batch = p.B;
+  g.tile_n = ws.r0_tile_n;
+  if (R0 <= kCosMaxCols) {
+    // each token's largest cosine per column tile straight from the accumulators
+    g.out = GemmOut::kCos;
+    g.D = ws.r0_parts > 1 ? ws.mpart : ws.m;
+    g.norm_a = ws.vnorm;
+    g.norm_b = ws.r0norm;
+    return launch_gemm8(g, ws.vu, ws.vsum, ws.r0u, ws.r0sum, stream);
+  }
   g.out = GemmOut::kS32;
   g.D = ws.dots;
   g.d_pitch = ws.dot_pitch;
   g.f32_out = true;
-  g.tile_n = ws.r0_tile_n;
   cudaError_t e = launch_gemm8(g, ws.vu, ws.vsum, ws.r0u, ws.r0sum, stream);
   if (e != cudaSuccess) return e;
   const dim3 grid((p.N + kCosmaxRows - 1) / kCosmaxRows, p.B);
@@ -437,7 +464,8 @@ cudaError_t launch_candidates(const SelectPlan& p, const SelectWorkspace& ws, cu
   const int R0 = p.Kq + p.Ks;
   const int nt = ((p.N + kPer - 1) / kPer + 31) / 32 * 32;
   auto go = [&](auto kern) {
-    return launch_pdl(kern, dim3(p.B), dim3(nt), 0, stream, ws.m, ws.kept12, p.N, R0, C, ws.cand);
+    return launch_pdl(kern, dim3(p.B), dim3(nt), 0, stream, ws.m, ws.r0_parts > 1 ? ws.mpart : nullptr,
+                      ws.r0_parts, ws.kept12, p.N, R0, C, ws.cand);
   };
   cudaError_t e = nt <= 512 ? go(select_candidates_kernel<512>)
                             : (nt <= 768 ? go(select_candidates_kernel<768>) : go(select_candidates_kernel<kSelThreads>));
