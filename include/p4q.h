@@ -384,7 +384,7 @@ size_t p4q_select_workspace_bytes(int B, int N, int d, int J, const p4q_select_p
  * alpha + beta <= 1000.
  * All work is ordered on `stream`. For images of at most 1024 tokens with a
  * diversity stage (K_d > 0) the GEMM of all token pairs runs beside the
- * concept, query and stage 1-2 launches on a second stream the library owns
+ * stage 1-2 launch on a second stream the library owns
  * (one per device, created on the first call that is not being captured into
  * a CUDA graph; until then the order is serial), forked from and joined back
  * into `stream` by events inside the call, so a graph captured from `stream`

@@ -100,8 +100,8 @@ int select_r0(const p4q_select_params& p, bool have_q, bool have_a) {
   return bud.Kq + bud.Ks;
 }
 
-// The selector: fake-quantized copies of the tokens and of the concepts,
-// query cosines (a narrow GEMM), stages 1-2, the initial diversity maxima on
+// The selector: fake-quantized copies of the concepts and of the tokens with
+// the query dot products (in the token pass, or a narrow GEMM), stages 1-2, the initial diversity maxima on
 // the tensor cores (Gram mode: one GEMM of all token pairs; otherwise R0's
 // expanded codes gathered, a GEMM against every token and a row pass, then
 // the candidates' pairwise GEMM), stage 3 (writes idx). Work is ordered on
@@ -125,22 +125,42 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
   select_workspace_layout(B, N, d, Jeff, R0, C, gram, &w, ws);
   SelectPlan plan{B, N, d, Jeff, params->K, bud.Kq, bud.Ks, bud.Kd};
 
-  // Fake-quantized copies of the projector features (and of the concepts):
+  // Fake-quantized copies of the concepts, then of the projector features:
   // the codes expanded to one byte each (what the tensor-core stages read),
-  // their row sums and squared norms; then the code dot products of every
-  // token with its image's concepts on the tensor cores (the query cosines
-  // are taken from them in stages 1-2).
+  // their row sums and squared norms, and the code dot products of every
+  // token with its image's concepts (the query cosines are taken from them
+  // in stages 1-2): in the token pass itself where it applies, else on the
+  // tensor cores after it.
   cudaError_t e;
-  RowSource src;
-  src.X = V;
+  const int Jq = bud.Kq > 0 ? Jeff : 0;  // concepts whose dot products stage 1 reads
+  if (Jq > 0) {
+    RowSource qsrc;
+    qsrc.X = Q;
+    RowSinks oq;
+    oq.codes = w.qcodes;
+    oq.scale = w.qscale;
+    oq.norm2 = w.qnorm;
+    oq.u = w.qu;
+    oq.sum_u = w.qsum;
+    if ((e = counted(launch_quant_rows(qsrc, B * Jeff, d, oq, stream))) != cudaSuccess) return from_cuda(e);
+  }
   RowSinks sv;
   sv.scale = w.vscale;
   sv.norm2 = w.vnorm;
   sv.u = w.vu;
   sv.sum_u = w.vsum;
-  if ((e = counted(launch_quant_rows(src, B * N, d, sv, stream))) != cudaSuccess) return from_cuda(e);
+  if (select_token_quant_applies(d, Jq)) {
+    if ((e = counted(launch_select_token_quant(V, B, N, d, Jq, w.qu, w.qsum, sv, w.qdots, w.q_pitch, stream))) !=
+        cudaSuccess)
+      return from_cuda(e);
+  } else {
+    RowSource src;
+    src.X = V;
+    if ((e = counted(launch_quant_rows(src, B * N, d, sv, stream))) != cudaSuccess) return from_cuda(e);
+    if (Jq > 0 && (e = counted(launch_query_dots(plan, w, stream))) != cudaSuccess) return from_cuda(e);
+  }
   // Gram mode: the token-pair GEMM needs only the token codes; it runs on the
-  // library's second stream beside the concept, query and stage-1/2 launches
+  // library's second stream beside the stage-1/2 launch
   std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
   SideStream* side = nullptr;
   if (w.gram && use_side) {
@@ -155,18 +175,6 @@ p4q_status run_select(const uint16_t* V, int B, int N, int d, const uint16_t* Q,
     } else {
       side_lock.unlock();
     }
-  }
-  if (bud.Kq > 0) {
-    RowSource qsrc;
-    qsrc.X = Q;
-    RowSinks oq;
-    oq.codes = w.qcodes;
-    oq.scale = w.qscale;
-    oq.norm2 = w.qnorm;
-    oq.u = w.qu;
-    oq.sum_u = w.qsum;
-    if ((e = counted(launch_quant_rows(qsrc, B * Jeff, d, oq, stream))) != cudaSuccess) return from_cuda(e);
-    if ((e = counted(launch_query_dots(plan, w, stream))) != cudaSuccess) return from_cuda(e);
   }
   if (R0 > 0 || bud.Kd > 0) {
     // stages 1-2 (also the bits of an empty R0, and idx when Kd = 0)

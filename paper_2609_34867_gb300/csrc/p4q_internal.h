@@ -58,6 +58,17 @@ struct RowSinks {
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
                               cudaStream_t stream, const RowSinks* out2 = nullptr);
 
+// The selector's token pass: V [B, N, d] fake-quantized per row into out's
+// scale, norm2, u and sum_u (all required), and, for J > 0, the exact code
+// dot products with the image's J concepts (expanded codes qu [B, J, d], row
+// sums qsum [B, J]) as floats qdots [B * N, qp]. For d % 256 == 0, d <=
+// kTokenQuantMaxRow and J * d <= 96 KB (select_token_quant_applies).
+constexpr int kTokenQuantMaxRow = 5120;
+bool select_token_quant_applies(int d, int J);
+cudaError_t launch_select_token_quant(const uint16_t* V, int B, int N, int d, int J, const uint8_t* qu,
+                                      const int32_t* qsum, const RowSinks& out, float* qdots, int qp,
+                                      cudaStream_t stream);
+
 // ------------------------------------------------------------ GEMM
 enum class GemmOut { kHalf = 0, kS32 = 1, kCos = 2 };
 

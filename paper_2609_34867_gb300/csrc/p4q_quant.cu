@@ -19,6 +19,7 @@
 #include <cuda_fp16.h>
 
 #include <algorithm>
+#include <type_traits>
 
 #include "p4q_device.cuh"
 #include "p4q_internal.h"
@@ -310,7 +311,140 @@ cudaError_t launch_norm(const RowSource& src, int rows, int L, const RowSinks& o
   }
 }
 
+// ---------------------------------------------------------------- selector token pass
+// The selector's fake-quantized tokens (the quantizer above with the squared
+// code norm and the expanded codes) with the Eq. 4 query dot products fused:
+// one warp per token row, the row held in registers (CH 16-byte chunks per
+// lane, all loads of a row in flight at once), the abs-max a warp reduction,
+// no shared-memory pass and no block barrier. CTA (x, b) takes rows of image
+// b only, so the image's J concept rows (expanded codes, written by the
+// concept pass before this launch) sit in shared memory and each chunk's
+// bytes u are multiplied into them by dp4a as they are produced: the exact
+// code dot product with concept j is sum u u_j - 8 sum u - 8 sum u_j + 64 L.
+template <int CH, int JMAX>
+__global__ void __launch_bounds__(256, 2)
+    select_token_quant_kernel(const uint16_t* __restrict__ V, int N, int L, int J, const uint8_t* __restrict__ qu,
+                              const int32_t* __restrict__ qsum, RowSinks out, float* __restrict__ qdots, int qp) {
+  extern __shared__ __align__(16) uint8_t cq[];  // [J, L] the image's concept codes, expanded
+  const int b = blockIdx.y, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  pdl_wait();  // the concept codes come from the previous launch
+  pdl_launch_dependents();
+  if (JMAX > 0) {
+    const uint4* src = reinterpret_cast<const uint4*>(qu + static_cast<size_t>(b) * J * L);
+    for (int i = threadIdx.x; i < J * L / 16; i += blockDim.x) reinterpret_cast<uint4*>(cq)[i] = src[i];
+    __syncthreads();
+  }
+  const int nch = L >> 3;
+  const int wpi = gridDim.x * (blockDim.x >> 5);  // warps per image
+  for (int r = blockIdx.x * (blockDim.x >> 5) + warp; r < N; r += wpi) {
+    const size_t row = static_cast<size_t>(b) * N + r;
+    const uint4* x = reinterpret_cast<const uint4*>(V + row * L);
+    uint4 v[CH];
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      const int c = lane + 32 * i;
+      v[i] = (c < nch) ? ldg_stream16(x + c) : make_uint4(0u, 0u, 0u, 0u);
+    }
+    uint32_t m = 0;  // per-halfword max of |x| bit patterns
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      m = __vmaxu2(m, v[i].x & 0x7FFF7FFFu);
+      m = __vmaxu2(m, v[i].y & 0x7FFF7FFFu);
+      m = __vmaxu2(m, v[i].z & 0x7FFF7FFFu);
+      m = __vmaxu2(m, v[i].w & 0x7FFF7FFFu);
+    }
+    const uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+    const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
+    const float s = __fdiv_rn(a, 7.0f);
+    const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
+    float2 n2 = make_float2(0.0f, 0.0f);
+    uint32_t su = 0;
+    uint32_t dq[JMAX > 0 ? JMAX : 1];
+#pragma unroll
+    for (int j = 0; j < (JMAX > 0 ? JMAX : 1); ++j) dq[j] = 0;
+    uint2* up = reinterpret_cast<uint2*>(out.u + row * L);
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      const int c = lane + 32 * i;
+      if (c < nch) {
+        const uint32_t pw = (a != 0.0f) ? quant_chunk<true>(v[i], s, inv, n2) : 0u;
+        // one byte per code, u = v + 8: the word's four low-nibble codes, then its four high-nibble codes
+        const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+        up[c] = make_uint2(eu, ou);
+        su = __dp4a(eu + ou, 0x01010101u, su);
+#pragma unroll
+        for (int j = 0; j < JMAX; ++j) {
+          if (j < J) {
+            const uint2 w = *reinterpret_cast<const uint2*>(cq + static_cast<size_t>(j) * L + 8 * c);
+            dq[j] = __dp4a(eu, w.x, __dp4a(ou, w.y, dq[j]));
+          }
+        }
+      }
+    }
+    const int wn = __reduce_add_sync(0xFFFFFFFFu, static_cast<int>(n2.x + n2.y));
+    const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
+#pragma unroll
+    for (int j = 0; j < JMAX; ++j) {
+      if (j < J) {
+        const int p = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, dq[j]));
+        if (lane == j) {
+          // exact (|dot| <= 49 L < 2^24), so the float holds it exactly
+          const int dot = p - 8 * wu - 8 * qsum[b * J + j] + 64 * L;
+          qdots[row * qp + j] = static_cast<float>(dot);
+        }
+      }
+    }
+    if (lane == 0) {
+      out.scale[row] = (a != 0.0f) ? s : 0.0f;
+      out.norm2[row] = wn;
+      out.sum_u[row] = wu;
+    }
+  }
+}
+
+template <int CH, int JMAX>
+cudaError_t launch_token_quant(const uint16_t* V, int B, int N, int L, int J, const uint8_t* qu, const int32_t* qsum,
+                               const RowSinks& out, float* qdots, int qp, cudaStream_t stream) {
+  const size_t smem = static_cast<size_t>(J) * L;
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(select_token_quant_kernel<CH, JMAX>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  // at most two CTAs of 8 warps per SM over the whole batch (one wave: rows are dealt out per CTA in
+  // advance, so a second wave would double the time), never more warps than an image has rows
+  const int per_image = std::max(1, std::min((N + 7) / 8, 2 * sm_count() / B));
+  return launch_pdl(select_token_quant_kernel<CH, JMAX>, dim3(per_image, B), dim3(256), smem, stream, V, N, L, J, qu,
+                    qsum, out, qdots, qp);
+}
+
 }  // namespace
+
+bool select_token_quant_applies(int d, int J) {
+  return d % 256 == 0 && d <= kTokenQuantMaxRow && static_cast<size_t>(J) * d <= 96u * 1024u;
+}
+
+cudaError_t launch_select_token_quant(const uint16_t* V, int B, int N, int d, int J, const uint8_t* qu,
+                                      const int32_t* qsum, const RowSinks& out, float* qdots, int qp,
+                                      cudaStream_t stream) {
+  if (!select_token_quant_applies(d, J) || !out.u || !out.sum_u || !out.norm2 || !out.scale) return cudaErrorInvalidValue;
+  if (J > 0 && (!qu || !qsum || !qdots)) return cudaErrorInvalidValue;
+  const int ch = d / 256;
+  auto go = [&](auto ch_tag) -> cudaError_t {
+    constexpr int C = decltype(ch_tag)::value;
+    if (J == 0) return launch_token_quant<C, 0>(V, B, N, d, J, qu, qsum, out, qdots, qp, stream);
+    if (J <= 4) return launch_token_quant<C, 4>(V, B, N, d, J, qu, qsum, out, qdots, qp, stream);
+    return launch_token_quant<C, 16>(V, B, N, d, J, qu, qsum, out, qdots, qp, stream);
+  };
+  if (ch <= 4) return go(std::integral_constant<int, 4>());
+  if (ch <= 8) return go(std::integral_constant<int, 8>());
+  if (ch <= 12) return go(std::integral_constant<int, 12>());
+  if (ch <= 16) return go(std::integral_constant<int, 16>());
+  return go(std::integral_constant<int, 20>());
+}
+
 
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
                               cudaStream_t stream, const RowSinks* out2) {

@@ -96,10 +96,13 @@ def test_select_duplicate_tokens(p4q, dev):
         assert np.array_equal(idx.cpu().numpy(), oracle.select_batch(V, K))
 
 
-@pytest.mark.parametrize("N,K,d", [(2880, 640, 256), (4096, 1024, 128), (2049, 2000, 128)])
+@pytest.mark.parametrize("N,K,d", [(2880, 640, 256), (4096, 1024, 128), (2049, 2000, 128), (4096, 2048, 128),
+                                   (4096, 2400, 128)])
 def test_select_large_token_sets(p4q, dev, N, K, d):
     """Block sizes of 768 and 1024 ranking threads, several column chunks per
-    pool phase (up to K_d picks unseen by a pool), K close to N."""
+    pool phase (up to K_d picks unseen by a pool), K close to N; kept sets R0
+    of 320, 512, 1000 and 1024 tokens (two to four column tiles of the
+    cosine-max epilogue) and 1200 (int32 tiles and the row pass)."""
     w = wl.Workload("t", B=2, N=N, d=d, K=K, T=0, J=3, seed=31, heavy_tail=True, linears=())
     got, ref = _select(p4q, dev, wl.selector_inputs(w), K)
     assert np.array_equal(got, ref)
