@@ -321,6 +321,9 @@ cudaError_t launch_norm(const RowSource& src, int rows, int L, const RowSinks& o
 // concept pass before this launch) sit in shared memory and each chunk's
 // bytes u are multiplied into them by dp4a as they are produced: the exact
 // code dot product with concept j is sum u u_j - 8 sum u - 8 sum u_j + 64 L.
+// Rolling prefetch: as soon as a chunk is quantized its registers take the
+// same chunk of the warp's next row, so the next row's loads are in flight
+// during the rest of this row's work without more registers.
 template <int CH, int JMAX>
 __global__ void __launch_bounds__(256, 2)
     select_token_quant_kernel(const uint16_t* __restrict__ V, int N, int L, int J, const uint8_t* __restrict__ qu,
@@ -336,15 +339,20 @@ __global__ void __launch_bounds__(256, 2)
   }
   const int nch = L >> 3;
   const int wpi = gridDim.x * (blockDim.x >> 5);  // warps per image
-  for (int r = blockIdx.x * (blockDim.x >> 5) + warp; r < N; r += wpi) {
-    const size_t row = static_cast<size_t>(b) * N + r;
-    const uint4* x = reinterpret_cast<const uint4*>(V + row * L);
-    uint4 v[CH];
+  const int r_first = blockIdx.x * (blockDim.x >> 5) + warp;
+  uint4 v[CH];
+  if (r_first < N) {
+    const uint4* x = reinterpret_cast<const uint4*>(V + (static_cast<size_t>(b) * N + r_first) * L);
 #pragma unroll
     for (int i = 0; i < CH; ++i) {
       const int c = lane + 32 * i;
       v[i] = (c < nch) ? ldg_stream16(x + c) : make_uint4(0u, 0u, 0u, 0u);
     }
+  }
+  for (int r = r_first; r < N; r += wpi) {
+    const size_t row = static_cast<size_t>(b) * N + r;
+    const bool more = r + wpi < N;
+    const uint4* xn = reinterpret_cast<const uint4*>(V + (row + (more ? wpi : 0)) * L);  // the warp's next row
     uint32_t m = 0;  // per-halfword max of |x| bit patterns
 #pragma unroll
     for (int i = 0; i < CH; ++i) {
@@ -368,6 +376,7 @@ __global__ void __launch_bounds__(256, 2)
       const int c = lane + 32 * i;
       if (c < nch) {
         const uint32_t pw = (a != 0.0f) ? quant_chunk<true>(v[i], s, inv, n2) : 0u;
+        if (more) v[i] = ldg_stream16(xn + c);
         // one byte per code, u = v + 8: the word's four low-nibble codes, then its four high-nibble codes
         const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
         up[c] = make_uint2(eu, ou);
