@@ -61,7 +61,7 @@ FLUSH_BYTES = 512 << 20  # > 129 MB L2, written and then read between timed step
 # of the 32 x 2880 x 5120 workload (22528 x 43008 x 5120, 22528 x 5120 x 5120,
 # 22528 x 5120 x 13824), valid only while the GEMM source is unchanged since
 # the capture.
-PROFILED_GEMM = {"source_sha1": "8e8c6e9b8d145d3228bcfca3a69b86fdbd7b9463", "dram_bytes_per_launch": 1837964714}
+PROFILED_GEMM = {"source_sha1": "fab1d1384c4ec3b311a94787f2d0bf845cdafd5f", "dram_bytes_per_launch": 1839311360}
 
 
 def gemm_source_sha1() -> str:
@@ -775,6 +775,23 @@ class OracleSampler:
             est += float(np.mean(self.times[i])) * (w.B if kind == "select" else w.layers * w.M / self.rows)
         return est
 
+    def breakdown(self) -> dict:
+        """The selector piece's mean time per image and the sampled linears'
+        integer-op throughput (their ops over their mean times)."""
+        sel, ops, sec = None, 0.0, 0.0
+        lin = {l.name: l for l in self.w.linears}
+        for i, (kind, name) in enumerate(self.pieces):
+            if not self.times[i]:
+                continue
+            t = float(np.mean(self.times[i]))
+            if kind == "select":
+                sel = t
+            else:
+                ops += 2.0 * self.rows * lin[name].k_in * lin[name].n_out
+                sec += t
+        return {"select_ms_per_image": round(sel * 1e3, 3) if sel is not None else None,
+                "linear_gops": round(ops / sec / 1e9, 3) if sec > 0 else None}
+
     def describe(self) -> str:
         w = self.w
         lay = f" x {w.layers} layers" if w.layers > 1 else ""
@@ -792,7 +809,7 @@ def cpu_baseline(w: wl.Workload, threads: int, reps: int = 2):
     est = s.estimate()
     return {"value": round(linear_ops(w) / est / 1e12, 6), "unit": "TOPS", "cores": s.cores, "kind": "oracle",
             "sample": s.describe(), "pieces_timed": len(timed),
-            "ms_per_piece": round(float(np.mean(timed)) * 1e3, 3), "est_step_s": round(est, 3)}
+            "ms_per_piece": round(float(np.mean(timed)) * 1e3, 3), "est_step_s": round(est, 3), **s.breakdown()}
 
 
 def run_reference(args, rank):
@@ -829,7 +846,8 @@ def run_reference(args, rank):
         "step_note": "each of the K steps is one piece of the workload (steps and ms_per_step describe the pieces "
                      "that ran); value = the full step's integer ops / est_step_s",
         "cpu_baseline": {"value": round(value, 6), "unit": "TOPS", "cores": s.cores, "kind": "oracle",
-                         "sample": "each step one piece: " + s.describe(), "est_step_s": round(est, 3)},
+                         "sample": "each step one piece: " + s.describe(), "est_step_s": round(est, 3),
+                         **s.breakdown()},
         "e2e": {"value": round(value, 6), "unit": "TOPS", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
 
