@@ -171,10 +171,11 @@ p4q_status p4q_quant_act_expanded(const uint16_t* X, int ldx, int M, int Kin, ui
  *   degree-7 Taylor polynomial, two exact power-of-two scalings: within
  *   0.9 ulp of e^x; 0 for x < -87, inf for x > 88.72284, so silu(g) = 0
  *   for g < -88.72284);
- *   then the codes and scale of h as p4q_quant_act. h is within 3 fp32
- *   rounding units of the real silu(g) * u, so the scale is within 1e-6 of
- *   the exact one and every code equals the code of the exact h except
- *   where h / s lies within 3.2e-6 of a .5 boundary.
+ *   then the codes and scale of h as p4q_quant_act. h is within 2.9 ulp
+ *   (3.5e-7 relative) of the real silu(g) * u, so the scale is within 1e-6
+ *   of the exact one, the quotient h / s within 5.7e-6 of the exact
+ *   quotient, and every code equals the code of the exact h except where
+ *   that quotient lies within 5.7e-6 of a .5 boundary.
  *   gate, up [M, Kin] fp16, rows ld_gate / ld_up elements apart (column
  *              blocks of a fused gate|up output; device, read)
  *   Xq [M, Kin/2], s_a [M]           written

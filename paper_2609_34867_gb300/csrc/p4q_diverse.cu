@@ -5,8 +5,9 @@
 // m (lower index on ties) and m absorbs its cosines.
 //
 // One CTA per image. The largest cosine of every token to R0 comes from the
-// tensor-core GEMM and row pass before this kernel (m). After that no cosine row of
-// the whole image is ever formed. The kernel holds, for every free token, a
+// tensor-core GEMM before this kernel (its cosine-max epilogue, or a row pass
+// over its int32 tiles; in Gram mode a row pass over the token-pair GEMM)
+// as m. After that no cosine row of the whole image is ever formed. The kernel holds, for every free token, a
 // lower bound of m (exact up to the first ex picks) and runs in phases:
 //   1. pool: the 128 smallest free (bound, token) pairs (block radix select);
 //      tau = the largest of them. Every token outside the pool has a pair

@@ -2,12 +2,12 @@
 // query relevance and saliency stages, and the operand preparation of the
 // diversity stage (p4q_diverse.cu runs the greedy rounds).
 //
-// Inputs are the fake-quantized copies produced by the per-row quantizer (the
-// codes of every visual token and concept expanded to one byte each, u = v +
-// 8, with their row sums, and the squared code norms) and the exact code dot
-// products of every token with its image's concepts (a tensor-core GEMM). The cosine of two
-// fake-quantized rows is evaluated on their codes (code_cosine: the positive
-// per-row scales cancel).
+// Inputs are the fake-quantized copies produced by the quantizers (the codes
+// of every visual token and concept expanded to one byte each, u = v + 8,
+// with their row sums, and the squared code norms) and the exact code dot
+// products of every token with its image's concepts (from the token pass, or
+// a narrow tensor-core GEMM). The cosine of two fake-quantized rows is
+// evaluated on their codes (code_cosine: the positive per-row scales cancel).
 //
 // Kernels:
 //   select_stages12_kernel  one CTA per image, one thread per 4 tokens: stage 1
@@ -17,10 +17,12 @@
 //   gather_rows_kernel      the expanded codes, row sums and norms of listed
 //                           tokens (R0, or the diversity candidates), row by
 //                           row, as an operand of the tensor-core GEMMs.
-//   r0_cosmax_kernel        each token's largest cosine to R0 from the exact
-//                           dot products of an int32-tile GEMM (kept sets of
-//                           more than kCosMaxCols tokens; smaller ones take
-//                           the maxima from the GEMM's cosine-max epilogue).
+//   r0_cosmax_kernel        each token's largest cosine to R0 from exact dot
+//                           products in fp32 rows: the token-pair GEMM of
+//                           Gram mode (columns through R0's token list), or
+//                           an int32-tile GEMM against R0 (kept sets of more
+//                           than kCosMaxCols tokens; smaller ones take the
+//                           maxima from the GEMM's cosine-max epilogue).
 //   select_candidates_kernel  the diversity stage's candidates: the free
 //                           tokens with the smallest of those maxima (after
 //                           merging the epilogue's per-column-tile maxima).

@@ -6,9 +6,13 @@
 // exp32 is an own fp32 exponential (Cody-Waite reduction with ln 2 split as
 // 355/512 + a low part, degree-7 Taylor polynomial by Horner's rule with fused
 // multiply-adds, two exact power-of-two scalings; within 0.9 ulp of e^x; 0
-// below -87, inf above 88.72284). The fp32 h is within 3 rounding units of
-// the real silu(g) * up, so the codes are those of the exact SwiGLU except
-// where h / s falls within 3.2e-6 of a .5 boundary.
+// below -87, inf above 88.72284). The fp32 h is within 2.9 ulp (3.5e-7
+// relative: 0.9 ulp from exp32 and four roundings of 2^-24) of the real
+// silu(g) * up, the row's abs-max likewise, the scale a / 7 adds one
+// rounding and the quotient h / s one more, so h / s is within 8.1e-7
+// relative, 5.7e-6 absolute (|h / s| <= 7), of the exact quotient: the codes
+// are those of the exact SwiGLU except where that quotient falls within
+// 5.7e-6 of a .5 boundary.
 //
 // Kernel: one CTA of 512 threads per row; each thread holds its chunks of 8
 // values of h in registers (computed once), the row's abs-max comes from a

@@ -106,13 +106,18 @@ def test_llava15_7b_batch_8x576_to_192(run_step):
     check_step(run_step(w), w, images=list(range(w.B)), rows=sample_rows(w.M, 62, 1))
 
 
+def spread(B, n=4):
+    """n image indices spread across a batch of B, first and last included."""
+    return sorted({round(i * (B - 1) / (n - 1)) for i in range(n)})
+
+
 def test_llavanext_7b_batch_16x2880_to_320(run_step):
     # two of the 32 layers: every layer launches the same kernels on the same
     # shapes, and the second checks that the layer chain reads its own weights
     w = dataclasses.replace(wl.LLAVANEXT_7B, layers=2)
-    check_step(run_step(w), w, images=[0, w.B - 1], rows=sample_rows(w.M, 46, 2))
+    check_step(run_step(w), w, images=spread(w.B), rows=sample_rows(w.M, 46, 2))
 
 
 def test_llavanext_13b_batch_32x2880_to_640_heavy_tails(run_step):
     w = wl.LLAVANEXT_13B
-    check_step(run_step(w), w, images=[0, w.B - 1], rows=sample_rows(w.M, 30, 3))
+    check_step(run_step(w), w, images=spread(w.B), rows=sample_rows(w.M, 30, 3))
