@@ -291,6 +291,18 @@ class Step:
         for name in self.Xq_re:
             self.Xu_re[name] = torch.empty((M, dims[name].k_in), dtype=torch.uint8, device=dev)
             self.sXu_re[name] = torch.empty((M,), dtype=torch.int32, device=dev)
+        # When every re-quantized block is a column block of one GEMM's output,
+        # that GEMM records each row's abs-max per block (its row-max epilogue)
+        # and each block is quantized in one streaming pass
+        # (p4q_quant_act_expanded_rowmax) instead of two.
+        srcs = {self.col[self.REQUANT[n]][0] for n in self.Xq_re}
+        self.rm_gemm = None
+        if len(srcs) == 1 and 1 <= len(self.Xq_re) <= 2:
+            names = sorted(self.Xq_re, key=lambda n: self.col[self.REQUANT[n]][1])
+            blocks = [tuple(self.col[self.REQUANT[n]][1:]) for n in names]
+            if all(off % 32 == 0 and n % 256 == 0 for off, n in blocks):
+                self.rm_gemm, self.rm_names, self.rm_blocks = srcs.pop(), names, blocks
+                self.rowmax = torch.empty((len(names), M), dtype=torch.int32, device=dev)
         # one weight scratch per GEMM of a layer: the weights expand on a side
         # stream, ahead of the GEMMs that read them (see body)
         self.slot = {g: i for i, (g, _) in enumerate(self.gemms)}
@@ -308,8 +320,7 @@ class Step:
             for gname, members in self.gemms:
                 if members[0] in self.REQUANT:
                     name = members[0]
-                    self.segments.append(("quant", "quant_" + name, (lambda n=name: p4q.p4q_quant_act_expanded(
-                        self.output(self.REQUANT[n]), self.Xq_re[n], self.s_re[n], self.Xu_re[n], self.sXu_re[n]))))
+                    self.segments.append(("quant", "quant_" + name, (lambda n=name: self._requant(n))))
                     xin = (lambda n=name: (self.Xu_re[n], self.sXu_re[n], self.s_re[n]))
                 else:
                     xin = (lambda: (self.Xu, self.sXu, self.s_a))
@@ -340,9 +351,27 @@ class Step:
         k = self.slot[gname]
         self.p4q.p4q_expand_codes(self.Wq[layer, gname], self.Wu[k], self.sWu[k], stream)
 
-    def _gemm(self, layer, gname, Xu, sXu, s):
+    def _gemm(self, layer, gname, Xu, sXu, s, stream=None):
         k = self.slot[gname]
-        self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, self.Wu[k], self.sWu[k], self.s_w[layer, gname], self.Y[gname])
+        if gname == self.rm_gemm:
+            self.p4q.p4q_w4a4_linear_expanded_rowmax(Xu, sXu, s, self.Wu[k], self.sWu[k], self.s_w[layer, gname],
+                                                     self.Y[gname], self.rm_blocks, self.rowmax, stream)
+        else:
+            self.p4q.p4q_w4a4_linear_expanded(Xu, sXu, s, self.Wu[k], self.sWu[k], self.s_w[layer, gname],
+                                              self.Y[gname], stream)
+
+    def _requant(self, name, stream=None):
+        """The per-token codes of the block of the source GEMM's output that
+        linear `name` reads (R10): one pass with the row maxima the GEMM
+        recorded, else the two-pass quantizer."""
+        if self.rm_gemm is None:
+            self.p4q.p4q_quant_act_expanded(self.output(self.REQUANT[name]), self.Xq_re[name], self.s_re[name],
+                                            self.Xu_re[name], self.sXu_re[name], stream)
+            return
+        b = self.rm_names.index(name)
+        self.p4q.p4q_quant_act_expanded_rowmax(self.Y[self.rm_gemm], [self.rm_blocks[b]], self.rowmax[b:b + 1],
+                                               [self.Xq_re[name]], [self.s_re[name]], [self.Xu_re[name]],
+                                               [self.sXu_re[name]], stream)
 
     def body_serial(self):
         """The step's segments one after another on the current stream."""
@@ -383,19 +412,15 @@ class Step:
                 with torch.cuda.stream(self.aux):
                     if src_done is not None:
                         self.aux.wait_event(src_done)
-                    self.p4q.p4q_quant_act_expanded(self.output("q"), self.Xq_re["o"], self.s_re["o"],
-                                                    self.Xu_re["o"], self.sXu_re["o"], self.aux)
+                    self._requant("o", self.aux)
                     o_read = torch.cuda.Event()
                     o_read.record(self.aux)
                     self.aux.wait_event(ready[i])
-                    self.p4q.p4q_w4a4_linear_expanded(*xin(), self.Wu[self.slot[gname]], self.sWu[self.slot[gname]],
-                                                      self.s_w[layer, gname], self.Y[gname], self.aux)
+                    self._gemm(layer, gname, *xin(), self.aux)
                     freed[i].record(self.aux)
                 continue
             if first in self.REQUANT:
-                src = self.REQUANT[first]
-                self.p4q.p4q_quant_act_expanded(self.output(src), self.Xq_re[first], self.s_re[first],
-                                                self.Xu_re[first], self.sXu_re[first])
+                self._requant(first)
             if gname == o_src and o_read is not None:
                 main.wait_event(o_read)  # the previous layer's o chain has read this GEMM's output
             if out_free is not None and self.out_name in members[gname]:

@@ -328,6 +328,43 @@ p4q_status p4q_w4a4_linear_expanded(const uint8_t* Xu, const int32_t* sum_xu, co
                                     const uint8_t* Wu, const int32_t* sum_wu, const float* s_w, int N, uint16_t* Y,
                                     p4q_stream_t stream);
 
+/* p4q_w4a4_linear_expanded that also records, for nblk <= 2 column blocks
+ * of Y, each row's abs-max over the block as the fp16 bit pattern the
+ * per-token quantizer of the next linear reads first (App. A: per-token
+ * activations; the block is that linear's input, e.g. the q or up part of a
+ * fused q|k|v|gate|up output):
+ *   rowmax[b * M + m] = max over c in [col0[b], col0[b] + ncols[b]) of
+ *                       (bits(Y[m, c]) & 0x7FFF)
+ * (non-negative fp16 values order as their bit patterns). The call clears
+ * rowmax on `stream`, then the GEMM's epilogue takes the maxima with one
+ * atomic per row and tile. Y and every other output as
+ * p4q_w4a4_linear_expanded. The paper has no counterpart.
+ *   col0, ncols  host arrays of nblk entries, multiples of 32,
+ *                col0[b] + ncols[b] <= N
+ *   rowmax       [nblk, M] uint32 (device, written), 16-byte aligned */
+p4q_status p4q_w4a4_linear_expanded_rowmax(const uint8_t* Xu, const int32_t* sum_xu, const float* s_a, int M,
+                                           int Kin, const uint8_t* Wu, const int32_t* sum_wu, const float* s_w, int N,
+                                           uint16_t* Y, int nblk, const int* col0, const int* ncols,
+                                           uint32_t* rowmax, p4q_stream_t stream);
+
+/* p4q_quant_act_expanded of nblk <= 2 column blocks of Y [M, ldy] fp16
+ * (block b: columns col0[b] .. col0[b] + ncols[b] - 1) whose row abs-max is
+ * given (rowmax as p4q_w4a4_linear_expanded_rowmax writes it): the same
+ * codes, scales, expanded codes and row sums bit for bit, in one streaming
+ * pass over both blocks (no abs-max pass). The paper has no counterpart.
+ *   Xq[b]   [M, ncols[b]/2] packed INT4, or Xq == NULL / Xq[b] == NULL to
+ *           skip the packed form (device, written)
+ *   s_a[b]  [M] fp32; Xu[b] [M, ncols[b]] bytes; sum_xu[b] [M] int32
+ *           (device, written)
+ *   col0, ncols and the pointer arrays are host arrays of nblk entries.
+ * Requires ncols[b] % 256 == 0, ncols[b] <= P4Q_MAX_ROW, col0[b] % 8 == 0,
+ * col0[b] + ncols[b] <= ldy, ldy % 8 == 0, 16-byte aligned pointers. M == 0
+ * is a no-op. */
+p4q_status p4q_quant_act_expanded_rowmax(const uint16_t* Y, int ldy, int M, int nblk, const int* col0,
+                                         const int* ncols, const uint32_t* rowmax, uint8_t* const* Xq,
+                                         float* const* s_a, uint8_t* const* Xu, int32_t* const* sum_xu,
+                                         p4q_stream_t stream);
+
 /* Test view of the same path: the exact int32 accumulators (as
  * p4q_w4a4_gemm_s32). */
 p4q_status p4q_w4a4_gemm_s32_ws(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,

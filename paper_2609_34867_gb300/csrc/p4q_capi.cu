@@ -514,6 +514,71 @@ p4q_status p4q_w4a4_linear_expanded(const uint8_t* Xu, const int32_t* sum_xu, co
   return from_cuda(counted(launch_gemm8(g, Xu, sum_xu, Wu, sum_wu, reinterpret_cast<cudaStream_t>(stream))));
 }
 
+p4q_status p4q_w4a4_linear_expanded_rowmax(const uint8_t* Xu, const int32_t* sum_xu, const float* s_a, int M,
+                                           int Kin, const uint8_t* Wu, const int32_t* sum_wu, const float* s_w, int N,
+                                           uint16_t* Y, int nblk, const int* col0, const int* ncols,
+                                           uint32_t* rowmax, p4q_stream_t stream) {
+  if (M < 0 || N < 1 || Kin < 1 || !Wu || !sum_wu || !s_w || (M > 0 && (!Xu || !sum_xu || !s_a || !Y)))
+    return P4Q_ERR_INVALID_ARG;
+  if (nblk < 1 || nblk > 2 || !col0 || !ncols || (M > 0 && !rowmax)) return P4Q_ERR_INVALID_ARG;
+  for (int b = 0; b < nblk; ++b) {
+    if (col0[b] < 0 || ncols[b] < 1 || col0[b] > N - ncols[b]) return P4Q_ERR_INVALID_ARG;
+    if (col0[b] % 32 != 0 || ncols[b] % 32 != 0) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  }
+  if (Kin % 128 != 0 || Kin > P4Q_MAX_ROW || N % 8 != 0 || N < 256) return P4Q_ERR_UNSUPPORTED_SHAPE;
+  if (!aligned16(Wu) || (M > 0 && (!aligned16(Xu) || !aligned16(Y) || !aligned16(rowmax)))) return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemsetAsync(rowmax, 0, sizeof(uint32_t) * static_cast<size_t>(nblk) * M, cs);
+  if (e != cudaSuccess) return from_cuda(e);
+  GemmArgs g;
+  g.M = M;
+  g.N = N;
+  g.K = Kin;
+  g.out = GemmOut::kHalf;
+  g.D = Y;
+  g.s_a = s_a;
+  g.s_b = s_w;
+  g.rowmax = rowmax;
+  g.rm_n = nblk;
+  for (int b = 0; b < nblk; ++b) {
+    g.rm_c0[b] = col0[b];
+    g.rm_c1[b] = col0[b] + ncols[b];
+  }
+  return from_cuda(counted(launch_gemm8(g, Xu, sum_xu, Wu, sum_wu, cs)));
+}
+
+p4q_status p4q_quant_act_expanded_rowmax(const uint16_t* Y, int ldy, int M, int nblk, const int* col0,
+                                         const int* ncols, const uint32_t* rowmax, uint8_t* const* Xq,
+                                         float* const* s_a, uint8_t* const* Xu, int32_t* const* sum_xu,
+                                         p4q_stream_t stream) {
+  if (M < 0 || nblk < 1 || nblk > 2 || !col0 || !ncols || !s_a || !Xu || !sum_xu) return P4Q_ERR_INVALID_ARG;
+  if (M > 0 && (!Y || !rowmax)) return P4Q_ERR_INVALID_ARG;
+  RowmaxBlock blk[2];
+  for (int b = 0; b < nblk; ++b) {
+    if (col0[b] < 0 || ncols[b] < 1 || ldy < ncols[b] || col0[b] > ldy - ncols[b]) return P4Q_ERR_INVALID_ARG;
+    if (ncols[b] % 256 != 0 || ncols[b] > P4Q_MAX_ROW) return P4Q_ERR_UNSUPPORTED_SHAPE;
+    if (col0[b] % 8 != 0) return P4Q_ERR_MISALIGNED;
+    if (M > 0 && (!s_a[b] || !Xu[b] || !sum_xu[b])) return P4Q_ERR_INVALID_ARG;
+    if (M > 0 && (!aligned16(s_a[b]) || !aligned16(Xu[b]) || !aligned16(sum_xu[b]) ||
+                  (Xq && Xq[b] && !aligned16(Xq[b]))))
+      return P4Q_ERR_MISALIGNED;
+    blk[b].col0 = col0[b];
+    blk[b].L = ncols[b];
+    blk[b].codes = Xq ? Xq[b] : nullptr;
+    blk[b].scale = M > 0 ? s_a[b] : nullptr;
+    blk[b].u = M > 0 ? Xu[b] : nullptr;
+    blk[b].sum_u = M > 0 ? sum_xu[b] : nullptr;
+  }
+  if (ldy % 8 != 0 || (M > 0 && (!aligned16(Y) || !aligned16(rowmax)))) return P4Q_ERR_MISALIGNED;
+  if (M == 0) return P4Q_OK;
+  p4q_status st = check_device();
+  if (st != P4Q_OK) return st;
+  return from_cuda(counted(launch_quant_rowmax(Y, ldy, M, nblk, blk, rowmax, reinterpret_cast<cudaStream_t>(stream))));
+}
+
 p4q_status p4q_w4a4_gemm_s32(const uint8_t* Xq, int M, int Kin, const uint8_t* Wq, int N, int32_t* acc,
                              p4q_stream_t stream) {
   p4q_status st = check_gemm(Xq, M, Kin, Wq, N, acc);

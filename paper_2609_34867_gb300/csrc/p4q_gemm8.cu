@@ -76,6 +76,9 @@ struct Params8 {
   const int32_t* norm_b;  // [batch, N] of the B rows
   float* cos_max;         // [num_n][part] with part >= batch * M: each A row's largest cosine per column tile
   size_t part;
+  uint32_t* rowmax;       // fp16 tiles: [rm_n, M] each row's largest |Y| bit pattern per column range
+  int rm_n;
+  int rm_c0[2], rm_c1[2];
 };
 
 constexpr int kCosMode = static_cast<int>(GemmOut::kCos);
@@ -368,9 +371,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       // result is an integer of magnitude < 2^24, so the fused multiply-add is exact.
       const float corrA = (m < p.M) ? static_cast<float>(64 * p.K - 8 * p.sum_a[static_cast<size_t>(bz) * p.M + m]) : 0.0f;
       const float sa = (MODE == static_cast<int>(GemmOut::kHalf) && m < p.M) ? p.s_a[m] : 0.0f;
+      uint32_t rmx0 = 0, rmx1 = 0;  // fp16 tiles: |Y| bit-pattern maxima (two halfwords) per column range
 #pragma unroll 1
       for (int cc = 0; cc < bn / 32; ++cc) {
         uint8_t* box = boxes + (nbox & 1) * BOX_BYTES;
+        uint32_t cmx = 0;
         if (lane == 0) bulk_wait_group_read<1>();
         __syncwarp();
         uint8_t* rowp = box + lane * (32 * L::ELEM);
@@ -398,6 +403,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
                 const float y1 = __fmul_rn(__fmul_rn(a1, sa), colv[c0 + i0 + 1]);
                 const __half2 hh = __floats2half2_rn(y0, y1);
                 w[e] = *reinterpret_cast<const uint32_t*>(&hh);
+                cmx = __vmaxu2(cmx, w[e] & 0x7FFF7FFFu);
               }
               // 64-byte rows, 64-byte swizzle: 16-byte chunk (2h + g2) of row `lane`
               const int ch = 2 * h + g2;
@@ -426,6 +432,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           bulk_commit_group();
         }
         ++nbox;
+        if (MODE == static_cast<int>(GemmOut::kHalf) && p.rm_n > 0) {
+          // this 32-column chunk lies wholly inside or outside each range (multiples of 32)
+          const int c = n0 + cc * 32;
+          if (c >= p.rm_c0[0] && c < p.rm_c1[0]) rmx0 = __vmaxu2(rmx0, cmx);
+          if (p.rm_n > 1 && c >= p.rm_c0[1] && c < p.rm_c1[1]) rmx1 = __vmaxu2(rmx1, cmx);
+        }
+      }
+      if (MODE == static_cast<int>(GemmOut::kHalf) && p.rm_n > 0 && m < p.M) {
+        // one atomic per row and range the tile meets
+        if (n0 < p.rm_c1[0] && n0 + bn > p.rm_c0[0])
+          atomicMax(p.rowmax + m, max(rmx0 & 0xFFFFu, rmx0 >> 16));
+        if (p.rm_n > 1 && n0 < p.rm_c1[1] && n0 + bn > p.rm_c0[1])
+          atomicMax(p.rowmax + static_cast<size_t>(p.M) + m, max(rmx1 & 0xFFFFu, rmx1 >> 16));
       }
     }
     if (lane == 0) bulk_wait_group_all();
@@ -535,6 +554,12 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
   p.norm_b = g.norm_b;
   p.cos_max = MODE == kCosMode ? static_cast<float*>(g.D) : nullptr;
   p.part = static_cast<size_t>(batch) * g.M;
+  p.rowmax = g.rowmax;
+  p.rm_n = (MODE == static_cast<int>(GemmOut::kHalf) && g.rowmax && batch == 1) ? g.rm_n : 0;
+  for (int r = 0; r < 2; ++r) {
+    p.rm_c0[r] = g.rm_c0[r];
+    p.rm_c1[r] = g.rm_c1[r];
+  }
   const int pairs = p.tiles < num_sms() / 2 ? p.tiles : num_sms() / 2;
   return launch_pdl(w4a4_gemm8_pair_kernel<MODE>, dim3(2 * pairs), dim3(kThreads), Lay8<MODE>::SMEM, stream, ma,
                     mb, md, p);

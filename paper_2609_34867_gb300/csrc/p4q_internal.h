@@ -58,6 +58,20 @@ struct RowSinks {
 cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSinks& out,
                               cudaStream_t stream, const RowSinks* out2 = nullptr);
 
+// Per-token quantizer of up to two column blocks of Y [M, ldy] fp16 whose
+// rows' abs-max is known (fp16 bit patterns rowmax [nblk, M], as the GEMM's
+// row-max epilogue writes them): the codes, scales and expanded codes of
+// launch_quant_rows, one streaming pass (one warp per block row).
+struct RowmaxBlock {
+  int col0 = 0, L = 0;        // columns col0 .. col0 + L of Y (L % 256 == 0)
+  uint8_t* codes = nullptr;   // [M, L/2] or null
+  float* scale = nullptr;     // [M]
+  uint8_t* u = nullptr;       // [M, L]
+  int32_t* sum_u = nullptr;   // [M]
+};
+cudaError_t launch_quant_rowmax(const uint16_t* Y, int ldy, int M, int nblk, const RowmaxBlock* blk,
+                                const uint32_t* rowmax, cudaStream_t stream);
+
 // The selector's token pass: V [B, N, d] fake-quantized per row into out's
 // scale, norm2, u and sum_u (all required), and, for J > 0, the exact code
 // dot products with the image's J concepts (expanded codes qu [B, J, d], row
@@ -87,6 +101,12 @@ struct GemmArgs {
   const int32_t* norm_b = nullptr;  // kCos: [batch, N]
   int tile_n = 256;                 // expanded-operand int32 tiles: columns per tile (multiple of 32, <= 256)
   bool f32_out = false;             // expanded-operand int32 tiles: the exact integers as fp32 values
+  // expanded-operand fp16 output: per row, the largest |Y| bit pattern over
+  // each of rm_n <= 2 column ranges [rm_c0, rm_c1) (multiples of 32), into
+  // rowmax [rm_n, M] by atomicMax (cleared by the caller first)
+  uint32_t* rowmax = nullptr;
+  int rm_n = 0;
+  int rm_c0[2] = {0, 0}, rm_c1[2] = {0, 0};
 };
 
 // Returns cudaSuccess or the launch error; sets *unsupported when the shape

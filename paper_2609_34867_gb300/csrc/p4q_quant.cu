@@ -429,7 +429,93 @@ cudaError_t launch_token_quant(const uint16_t* V, int B, int N, int L, int J, co
                     qsum, out, qdots, qp);
 }
 
+// ---------------------------------------------------------------- known row abs-max
+// Up to two column blocks of Y quantized per row with the abs-max already
+// known (the GEMM's row-max epilogue): no abs-max pass, no reduction before
+// the codes, so one warp streams a block row in 256-element steps (one
+// 16-byte chunk per lane, kRmUnroll steps in flight) and only the row sum of
+// the expanded codes is reduced at the end. Same arithmetic as
+// quant_rows_kernel (s = a / 7, quant_chunk), so the same codes and scales.
+struct RowmaxArgs {
+  const uint16_t* Y;
+  int ldy, M, nblk;
+  RowmaxBlock b[2];
+  const uint32_t* rowmax;
+};
+
+constexpr int kRmUnroll = 4;  // 256-element steps in flight per warp
+
+__global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
+  pdl_wait();  // Y and its row maxima come from the previous kernel
+  pdl_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  const int tasks = a.nblk * a.M;
+  for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < tasks; t += warps) {
+    const int bi = t / a.M, m = t - bi * a.M;
+    const bool b1 = bi != 0;  // field by field: no dynamic index into the parameter array
+    RowmaxBlock B;
+    B.col0 = b1 ? a.b[1].col0 : a.b[0].col0;
+    B.L = b1 ? a.b[1].L : a.b[0].L;
+    B.codes = b1 ? a.b[1].codes : a.b[0].codes;
+    B.scale = b1 ? a.b[1].scale : a.b[0].scale;
+    B.u = b1 ? a.b[1].u : a.b[0].u;
+    B.sum_u = b1 ? a.b[1].sum_u : a.b[0].sum_u;
+    const float amax = __half2float(__ushort_as_half(static_cast<unsigned short>(a.rowmax[t])));
+    const float s = __fdiv_rn(amax, 7.0f);
+    const float inv = (amax != 0.0f) ? __frcp_rn(s) : 0.0f;
+    const uint4* x = reinterpret_cast<const uint4*>(a.Y + static_cast<size_t>(m) * a.ldy + B.col0);
+    uint32_t* q4 = B.codes ? reinterpret_cast<uint32_t*>(B.codes + static_cast<size_t>(m) * (B.L >> 1)) : nullptr;
+    uint2* up = reinterpret_cast<uint2*>(B.u + static_cast<size_t>(m) * B.L);
+    const int steps = B.L >> 8;  // 256 elements per warp step
+    float2 n2 = make_float2(0.0f, 0.0f);
+    uint32_t su = 0;
+    for (int j0 = 0; j0 < steps; j0 += kRmUnroll) {
+      uint4 v[kRmUnroll];
+#pragma unroll
+      for (int k = 0; k < kRmUnroll; ++k)
+        v[k] = (j0 + k < steps) ? ldg_stream16(x + (j0 + k) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+      for (int k = 0; k < kRmUnroll; ++k) {
+        if (j0 + k < steps) {
+          const int c = (j0 + k) * 32 + lane;
+          const uint32_t pw = (amax != 0.0f) ? quant_chunk<false>(v[k], s, inv, n2) : 0u;
+          if (q4) q4[c] = pw;
+          const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+          up[c] = make_uint2(eu, ou);
+          su = __dp4a(eu + ou, 0x01010101u, su);
+        }
+      }
+    }
+    const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
+    if (lane == 0) {
+      B.scale[m] = (amax != 0.0f) ? s : 0.0f;
+      B.sum_u[m] = wu;
+    }
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_quant_rowmax(const uint16_t* Y, int ldy, int M, int nblk, const RowmaxBlock* blk,
+                                const uint32_t* rowmax, cudaStream_t stream) {
+  if (M <= 0) return cudaSuccess;
+  if (nblk < 1 || nblk > 2 || !Y || !rowmax) return cudaErrorInvalidValue;
+  RowmaxArgs a;
+  a.Y = Y;
+  a.ldy = ldy;
+  a.M = M;
+  a.nblk = nblk;
+  a.rowmax = rowmax;
+  for (int i = 0; i < nblk; ++i) {
+    if (blk[i].L <= 0 || blk[i].L % 256 != 0 || !blk[i].scale || !blk[i].u || !blk[i].sum_u)
+      return cudaErrorInvalidValue;
+    a.b[i] = blk[i];
+  }
+  const int tasks = nblk * M;
+  const int blocks = std::max(1, std::min((tasks + 7) / 8, 8 * sm_count()));
+  return launch_pdl(quant_rowmax_kernel, dim3(blocks), dim3(256), 0, stream, a);
+}
 
 bool select_token_quant_applies(int d, int J) {
   return d % 256 == 0 && d <= kTokenQuantMaxRow && static_cast<size_t>(J) * d <= 96u * 1024u;

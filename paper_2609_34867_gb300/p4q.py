@@ -92,6 +92,10 @@ def lib() -> ctypes.CDLL:
         L.p4q_expand_codes.restype = st
         L.p4q_w4a4_linear_expanded.argtypes = [P, P, P, I, I, P, P, P, I, P, P]
         L.p4q_w4a4_linear_expanded.restype = st
+        L.p4q_w4a4_linear_expanded_rowmax.argtypes = [P, P, P, I, I, P, P, P, I, P, I, P, P, P, P]
+        L.p4q_w4a4_linear_expanded_rowmax.restype = st
+        L.p4q_quant_act_expanded_rowmax.argtypes = [P, I, I, I, P, P, P, P, P, P, P, P]
+        L.p4q_quant_act_expanded_rowmax.restype = st
         L.p4q_select_workspace_bytes.argtypes = [I, I, I, I, ctypes.POINTER(SelectParams)]
         L.p4q_select_workspace_bytes.restype = S
         L.p4q_select.argtypes = [P, I, I, I, P, I, P, ctypes.POINTER(SelectParams), P, P, S, P]
@@ -433,6 +437,46 @@ def p4q_w4a4_linear_expanded(Xu, sum_xu, s_a, Wu, sum_wu, s_w, Y, stream=None):
     N = Wu.shape[0]
     _check(lib().p4q_w4a4_linear_expanded(_ptr(Xu), _ptr(sum_xu), _ptr(s_a), M, K, _ptr(Wu), _ptr(sum_wu), _ptr(s_w),
                                           N, _ptr(Y), _stream(stream)), "p4q_w4a4_linear_expanded")
+
+
+def _host_ints(vals):
+    return (ctypes.c_int * len(vals))(*vals)
+
+
+def _host_ptrs(ts):
+    return (ctypes.c_void_p * len(ts))(*[(_ptr(t) if t is not None else None) for t in ts])
+
+
+def p4q_w4a4_linear_expanded_rowmax(Xu, sum_xu, s_a, Wu, sum_wu, s_w, Y, blocks, rowmax, stream=None):
+    """p4q_w4a4_linear_expanded plus each row's |Y| abs-max (fp16 bits) over
+    the column blocks [(col0, ncols), ...] (at most two) into rowmax [nblk, M]."""
+    _need(Xu, torch.uint8, 2, "Xu"); _need(Wu, torch.uint8, 2, "Wu"); _need(Y, torch.float16, 2, "Y")
+    _need(rowmax, torch.int32, 2, "rowmax")
+    M, K = Xu.shape
+    N = Wu.shape[0]
+    c0, nc = _host_ints([b[0] for b in blocks]), _host_ints([b[1] for b in blocks])
+    _check(lib().p4q_w4a4_linear_expanded_rowmax(_ptr(Xu), _ptr(sum_xu), _ptr(s_a), M, K, _ptr(Wu), _ptr(sum_wu),
+                                                 _ptr(s_w), N, _ptr(Y), len(blocks), c0, nc, _ptr(rowmax),
+                                                 _stream(stream)), "p4q_w4a4_linear_expanded_rowmax")
+
+
+def p4q_quant_act_expanded_rowmax(Y, blocks, rowmax, Xq, s_a, Xu, sum_xu, stream=None):
+    """p4q_quant_act_expanded of the column blocks [(col0, ncols), ...] of Y with
+    the row abs-max given; Xq, s_a, Xu, sum_xu: one tensor per block (Xq
+    entries may be None)."""
+    if not isinstance(Y, torch.Tensor) or Y.dtype != torch.float16 or Y.dim() != 2 or Y.stride(1) != 1 or not Y.is_cuda:
+        raise TypeError("Y: expected a CUDA fp16 2-D tensor with unit column stride")
+    _need(rowmax, torch.int32, 2, "rowmax")
+    for b in range(len(blocks)):
+        if Xq is not None and Xq[b] is not None:
+            _need(Xq[b], torch.uint8, 2, "Xq")
+        _need(s_a[b], torch.float32, 1, "s_a"); _need(Xu[b], torch.uint8, 2, "Xu")
+        _need(sum_xu[b], torch.int32, 1, "sum_xu")
+    c0, nc = _host_ints([b[0] for b in blocks]), _host_ints([b[1] for b in blocks])
+    _check(lib().p4q_quant_act_expanded_rowmax(_ptr(Y), Y.stride(0), Y.shape[0], len(blocks), c0, nc, _ptr(rowmax),
+                                               _host_ptrs(Xq) if Xq is not None else None, _host_ptrs(s_a),
+                                               _host_ptrs(Xu), _host_ptrs(sum_xu),
+                                               _stream(stream)), "p4q_quant_act_expanded_rowmax")
 
 
 def w4a4_gemm_s32(Xq, Wq, stream=None):

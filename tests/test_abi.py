@@ -198,3 +198,28 @@ def test_strided_quantizer_validates_its_row_pitch(lib):
     assert lib.p4q_quant_act_ld(P(16), 64, 4, 128, P(16), P(16), None) == 1   # pitch below the row length
     assert lib.p4q_quant_act_ld(P(16), 132, 4, 128, P(16), P(16), None) == 3  # rows not 16-byte aligned
     assert lib.p4q_quant_act_ld(None, 128, 0, 128, None, None, None) == 0     # empty is a no-op
+
+
+def test_rowmax_entries_validate_their_blocks(lib):
+    P, I = ctypes.c_void_p, ctypes.c_int
+    ints = lambda *v: (ctypes.c_int * len(v))(*v)
+    ptrs = lambda *v: (ctypes.c_void_p * len(v))(*v)
+    g = lib.p4q_w4a4_linear_expanded_rowmax
+    g.argtypes = [P, P, P, I, I, P, P, P, I, P, I, P, P, P, P]
+    a = (P(16), P(16), P(16), 4, 128, P(16), P(16), P(16), 512, P(16))
+    assert g(*a, 3, ints(0, 0, 0), ints(32, 32, 32), P(16), None) == 1          # at most two blocks
+    assert g(*a, 1, ints(480), ints(64), P(16), None) == 1                      # past N
+    assert g(*a, 1, ints(16), ints(64), P(16), None) == 2                       # not a multiple of 32
+    assert g(*a, 1, ints(0), ints(64), None, None) == 1                         # no rowmax
+    assert g(P(16), P(16), P(16), 0, 128, P(16), P(16), P(16), 512, P(16), 1, ints(0), ints(64), None,
+             None) == 0                                                          # M == 0 is a no-op
+    q = lib.p4q_quant_act_expanded_rowmax
+    q.argtypes = [P, I, I, I, P, P, P, P, P, P, P, P]
+    sinks = (ptrs(16, 16), ptrs(16, 16), ptrs(16, 16), ptrs(16, 16))
+    assert q(P(16), 1024, 4, 2, ints(0, 512), ints(256, 384), P(16), *sinks, None) == 2   # 384 % 256
+    assert q(P(16), 1024, 4, 2, ints(0, 896), ints(256, 256), P(16), *sinks, None) == 1   # past ldy
+    assert q(P(16), 1024, 4, 1, ints(4), ints(256), P(16), *sinks, None) == 3             # col0 % 8
+    assert q(P(16), 1024, 4, 1, ints(0), ints(256), P(16), ptrs(16), ptrs(8), ptrs(16), ptrs(16),
+             None) == 3                                                                  # misaligned s_a
+    assert q(P(16), 1024, 0, 1, ints(0), ints(256), None, None, ptrs(16), ptrs(16), ptrs(16),
+             None) == 0                                                                  # M == 0
