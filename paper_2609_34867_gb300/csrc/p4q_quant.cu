@@ -39,53 +39,81 @@ constexpr uint32_t kStageBudget = 100u * 1024u;    // shared memory for row buff
 constexpr uint32_t kInflightTarget = 48u * 1024u;  // bytes on their way per CTA (HBM latency x bandwidth share)
 constexpr int kSmemMax = 110 * 1024;
 
-// Codes of eight fp16 values (one 16-byte chunk), packed two per byte.
+// Codes of eight fp16 values (one 16-byte chunk).
 //
-// code = round_half_even(fl(x / s)) is computed as round(x * inv) with
-// inv = fl(1 / s): the two quotients differ by less than 2^-19 for |x / s| <= 7
-// (three roundings of relative size 2^-24), so they round to the same integer
-// unless x * inv lies within 2^-17 of a .5 boundary; a chunk with such a value
-// is recomputed with exact quotients fl(x / s). Rounding uses the magic
-// constant 1.5 * 2^23: q + 1.5 * 2^23 rounds q to the nearest integer (ties
-// to even) and leaves its two's complement in the low mantissa bits, which
-// are the packed nibble. |x| <= max|x| bounds the codes to [-7, 7], so the
-// clamp to [-8, 7] cannot bind. With NORM, squares of the codes are added to n2.
+// code = round_half_even(fl(x / s)). With inv = fl(1 / s) correctly rounded,
+// fl(x / s) lies within 2^-23 (relative) of x * inv, so ip = fl(inv (1 +
+// 2^-21)) and im = fl(inv (1 - 2^-21)) give products x * ip and x * im that
+// enclose fl(x / s) (each is at least 2^-21 - 2^-23 away from x * inv). One
+// fused multiply-add with the magic constant 1.5 * 2^23 rounds each exact
+// product to the nearest integer (ties to even: the constant is even) and
+// leaves its two's complement in the low mantissa bits. Rounding is
+// monotone, so where the two agree their integer is the code of fl(x / s);
+// a chunk where they differ for some value (a quotient within about 2^-21 of
+// a .5 boundary) is recomputed with exact quotients fl(x / s). |x| <= max|x|
+// bounds the codes to [-7, 7], so the clamp to [-8, 7] cannot bind. With
+// NORM, squares of the codes are added to n2 (exact: sums below 2^24).
+struct QRow {
+  float s, ip, im;  // scale a / 7 and the two bracketing reciprocals (0 when a == 0)
+};
+
+__device__ __forceinline__ QRow quant_row(float a) {
+  QRow r;
+  r.s = __fdiv_rn(a, 7.0f);
+  const float inv = (a != 0.0f) ? __frcp_rn(r.s) : 0.0f;
+  r.ip = __fmul_rn(inv, 1.0f + 0x1p-21f);
+  r.im = __fmul_rn(inv, 1.0f - 0x1p-21f);
+  return r;
+}
+
+// Byte k of e holds the code of element 2k, byte k of o the code of element
+// 2k + 1 (two's complement; the low nibble is the 4-bit code).
+struct Codes8 {
+  uint32_t e, o;
+};
+
+// packed: even-index codes in the low nibbles, odd-index codes in the high nibbles
+__device__ __forceinline__ uint32_t packed4(Codes8 c) { return (c.e & 0x0F0F0F0Fu) | ((c.o << 4) & 0xF0F0F0F0u); }
+// expanded, one byte per code u = v + 8: the four even-index codes, then the four odd-index codes
+__device__ __forceinline__ uint32_t expanded_even(Codes8 c) { return (c.e & 0x0F0F0F0Fu) ^ 0x08080808u; }
+__device__ __forceinline__ uint32_t expanded_odd(Codes8 c) { return (c.o & 0x0F0F0F0Fu) ^ 0x08080808u; }
+
 template <bool NORM>
-__device__ __forceinline__ uint32_t quant_chunk(const uint4 v, float s, float inv, float2& n2) {
-  const float2 inv2 = make_float2(inv, inv);
+__device__ __forceinline__ Codes8 quant_chunk(const uint4 v, const QRow& q, float2& n2) {
+  const float2 ip2 = make_float2(q.ip, q.ip), im2 = make_float2(q.im, q.im);
   const float2 mg = make_float2(12582912.0f, 12582912.0f);
-  const float2 nmg = make_float2(-12582912.0f, -12582912.0f);
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  float2 f[4], c[4];
+  float2 f[4];
   uint32_t tb[8];
-  float dmax = 0.0f;
+  uint32_t diff = 0;
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
     f[k] = __half22float2(*reinterpret_cast<const __half2*>(&w[k]));
-    const float2 q = __fmul2_rn(f[k], inv2);
-    const float2 t = __fadd2_rn(q, mg);
-    tb[2 * k] = __float_as_uint(t.x);
-    tb[2 * k + 1] = __float_as_uint(t.y);
-    c[k] = __fadd2_rn(t, nmg);
-    const float2 d = __fadd2_rn(q, make_float2(-c[k].x, -c[k].y));
-    dmax = fmaxf(dmax, fmaxf(fabsf(d.x), fabsf(d.y)));
+    const float2 tp = __ffma2_rn(f[k], ip2, mg);
+    const float2 tm = __ffma2_rn(f[k], im2, mg);
+    tb[2 * k] = __float_as_uint(tp.x);
+    tb[2 * k + 1] = __float_as_uint(tp.y);
+    diff |= (tb[2 * k] ^ __float_as_uint(tm.x)) | (tb[2 * k + 1] ^ __float_as_uint(tm.y));
   }
-  if (dmax > 0.5f - 0x1p-17f) {
+  if (diff != 0) {
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-      c[k] = make_float2(rintf(__fdiv_rn(f[k].x, s)), rintf(__fdiv_rn(f[k].y, s)));
-      tb[2 * k] = __float_as_uint(c[k].x + 12582912.0f);
-      tb[2 * k + 1] = __float_as_uint(c[k].y + 12582912.0f);
+      tb[2 * k] = __float_as_uint(rintf(__fdiv_rn(f[k].x, q.s)) + 12582912.0f);
+      tb[2 * k + 1] = __float_as_uint(rintf(__fdiv_rn(f[k].y, q.s)) + 12582912.0f);
     }
   }
   if (NORM) {
+    const float2 nmg = make_float2(-12582912.0f, -12582912.0f);
 #pragma unroll
-    for (int k = 0; k < 4; ++k) n2 = __ffma2_rn(c[k], c[k], n2);
+    for (int k = 0; k < 4; ++k) {
+      const float2 c = __fadd2_rn(make_float2(__uint_as_float(tb[2 * k]), __uint_as_float(tb[2 * k + 1])), nmg);
+      n2 = __ffma2_rn(c, c, n2);
+    }
   }
-  // even-index codes in the low nibbles, odd-index codes in the high nibbles
-  const uint32_t e = __byte_perm(__byte_perm(tb[0], tb[2], 0x0040), __byte_perm(tb[4], tb[6], 0x0040), 0x5410);
-  const uint32_t o = __byte_perm(__byte_perm(tb[1], tb[3], 0x0040), __byte_perm(tb[5], tb[7], 0x0040), 0x5410);
-  return (e & 0x0F0F0F0Fu) | ((o << 4) & 0xF0F0F0F0u);
+  Codes8 r;
+  r.e = __byte_perm(__byte_perm(tb[0], tb[2], 0x0040), __byte_perm(tb[4], tb[6], 0x0040), 0x5410);
+  r.o = __byte_perm(__byte_perm(tb[1], tb[3], 0x0040), __byte_perm(tb[5], tb[7], 0x0040), 0x5410);
+  return r;
 }
 
 __device__ __forceinline__ const uint16_t* row_ptr(const RowSource& src, int row, int L) {
@@ -175,8 +203,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       for (int w = 0; w < G; ++w) mm = max(mm, red[grp * G + w]);
     }
     const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
-    const float s = __fdiv_rn(a, 7.0f);
-    const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
+    const QRow qr = quant_row(a);
 
     float2 n2 = make_float2(0.0f, 0.0f);  // exact: sums of squared codes <= 49 * 16384 < 2^24
     uint32_t su = 0;                      // sum of the expanded codes u = v + 8 (expanded output)
@@ -187,12 +214,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 #pragma unroll 4
       for (int c = gt; c < nch; c += kGroupThreads) {
         const uint4 v = v4[c];
-        const uint32_t pw = (a != 0.0f) ? quant_chunk<NORM>(v, s, inv, n2) : 0u;
-        if (q4) q4[c] = pw;
+        const Codes8 cd = (a != 0.0f) ? quant_chunk<NORM>(v, qr, n2) : Codes8{0u, 0u};
+        if (q4) q4[c] = packed4(cd);
         if (cp) cp[c] = v;
         if (up) {
-          // one byte per code, u = v + 8: the word's four low-nibble codes, then its four high-nibble codes
-          const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+          const uint32_t eu = expanded_even(cd), ou = expanded_odd(cd);
           up[c] = make_uint2(eu, ou);
           su = __dp4a(eu + ou, 0x01010101u, su);
         }
@@ -224,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     }
     if (leader) {
       if (!failed) {
-        out.scale[row] = (a != 0.0f) ? s : 0.0f;
+        out.scale[row] = (a != 0.0f) ? qr.s : 0.0f;
         if (NORM) out.norm2[row] = wn;
         if (out.sum_u) out.sum_u[row] = wu;
         if (issued < mine) {
@@ -363,10 +389,9 @@ __global__ void __launch_bounds__(256, 2)
     }
     const uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
     const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
-    const float s = __fdiv_rn(a, 7.0f);
-    const float inv = (a != 0.0f) ? __frcp_rn(s) : 0.0f;
-    float2 n2 = make_float2(0.0f, 0.0f);
-    uint32_t su = 0;
+    const QRow qr = quant_row(a);
+    float2 n2 = make_float2(0.0f, 0.0f);  // unused: the norm comes from the expanded codes
+    uint32_t su = 0, uu = 0;              // sums of u and of u^2
     uint32_t dq[JMAX > 0 ? JMAX : 1];
 #pragma unroll
     for (int j = 0; j < (JMAX > 0 ? JMAX : 1); ++j) dq[j] = 0;
@@ -375,12 +400,12 @@ __global__ void __launch_bounds__(256, 2)
     for (int i = 0; i < CH; ++i) {
       const int c = lane + 32 * i;
       if (c < nch) {
-        const uint32_t pw = (a != 0.0f) ? quant_chunk<true>(v[i], s, inv, n2) : 0u;
+        const Codes8 cd = (a != 0.0f) ? quant_chunk<false>(v[i], qr, n2) : Codes8{0u, 0u};
         if (more) v[i] = ldg_stream16(xn + c);
-        // one byte per code, u = v + 8: the word's four low-nibble codes, then its four high-nibble codes
-        const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+        const uint32_t eu = expanded_even(cd), ou = expanded_odd(cd);
         up[c] = make_uint2(eu, ou);
         su = __dp4a(eu + ou, 0x01010101u, su);
+        uu = __dp4a(eu, eu, __dp4a(ou, ou, uu));
 #pragma unroll
         for (int j = 0; j < JMAX; ++j) {
           if (j < J) {
@@ -390,8 +415,9 @@ __global__ void __launch_bounds__(256, 2)
         }
       }
     }
-    const int wn = __reduce_add_sync(0xFFFFFFFFu, static_cast<int>(n2.x + n2.y));
     const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
+    // sum of squared codes (u - 8)^2 over the row's L codes, exactly
+    const int wn = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, uu)) - 16 * wu + 64 * L;
 #pragma unroll
     for (int j = 0; j < JMAX; ++j) {
       if (j < J) {
@@ -404,7 +430,7 @@ __global__ void __launch_bounds__(256, 2)
       }
     }
     if (lane == 0) {
-      out.scale[row] = (a != 0.0f) ? s : 0.0f;
+      out.scale[row] = (a != 0.0f) ? qr.s : 0.0f;
       out.norm2[row] = wn;
       out.sum_u[row] = wu;
     }
@@ -462,8 +488,7 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
     B.u = b1 ? a.b[1].u : a.b[0].u;
     B.sum_u = b1 ? a.b[1].sum_u : a.b[0].sum_u;
     const float amax = __half2float(__ushort_as_half(static_cast<unsigned short>(a.rowmax[t])));
-    const float s = __fdiv_rn(amax, 7.0f);
-    const float inv = (amax != 0.0f) ? __frcp_rn(s) : 0.0f;
+    const QRow qr = quant_row(amax);
     const uint4* x = reinterpret_cast<const uint4*>(a.Y + static_cast<size_t>(m) * a.ldy + B.col0);
     uint32_t* q4 = B.codes ? reinterpret_cast<uint32_t*>(B.codes + static_cast<size_t>(m) * (B.L >> 1)) : nullptr;
     uint2* up = reinterpret_cast<uint2*>(B.u + static_cast<size_t>(m) * B.L);
@@ -479,9 +504,9 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
       for (int k = 0; k < kRmUnroll; ++k) {
         if (j0 + k < steps) {
           const int c = (j0 + k) * 32 + lane;
-          const uint32_t pw = (amax != 0.0f) ? quant_chunk<false>(v[k], s, inv, n2) : 0u;
-          if (q4) q4[c] = pw;
-          const uint32_t eu = (pw & 0x0F0F0F0Fu) ^ 0x08080808u, ou = ((pw >> 4) & 0x0F0F0F0Fu) ^ 0x08080808u;
+          const Codes8 cd = (amax != 0.0f) ? quant_chunk<false>(v[k], qr, n2) : Codes8{0u, 0u};
+          if (q4) q4[c] = packed4(cd);
+          const uint32_t eu = expanded_even(cd), ou = expanded_odd(cd);
           up[c] = make_uint2(eu, ou);
           su = __dp4a(eu + ou, 0x01010101u, su);
         }
@@ -489,7 +514,7 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
     }
     const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
     if (lane == 0) {
-      B.scale[m] = (amax != 0.0f) ? s : 0.0f;
+      B.scale[m] = (amax != 0.0f) ? qr.s : 0.0f;
       B.sum_u[m] = wu;
     }
   }
