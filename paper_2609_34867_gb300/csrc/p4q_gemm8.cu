@@ -105,7 +105,8 @@ struct Lay8 {
 // that the pairs reading the same A rows run side by side. Otherwise the row
 // tiles are rastered in groups of p.gm: consecutive tiles sweep a group's row
 // tiles, then the next column tile, so a group's A rows (sized to stay in L2)
-// are read from DRAM once while the group sweeps all of B.
+// are read from DRAM once while the group sweeps all of B; p.gm = 1 (a B
+// that fits L2) is plain row-major order.
 __device__ __forceinline__ void tile_coords(const Params8& p, int t, int* bz, int* mt, int* nb) {
   *bz = t / p.per;
   const int r = t - *bz * p.per;
@@ -541,8 +542,13 @@ cudaError_t launch8(const GemmArgs& g, const Ws8& w, cudaStream_t stream) {
   p.num_m = (g.M + 2 * BM - 1) / (2 * BM);
   p.num_n = (g.N + bn - 1) / bn;
   p.bn = bn;
-  // a raster group's A rows: about 24 MB, so they stay in the 129 MB L2 beside B and the output
-  p.gm = std::max(1, std::min(p.num_m, static_cast<int>((24u << 20) / (static_cast<size_t>(2 * BM) * g.K))));
+  // Raster: a B of at most 32 MB stays in L2 while the row tiles stream past
+  // it (row-major order, every A row read once; measured: a 71 MB B did not
+  // stay, as the L2 is split between the two dies); a larger B is swept by
+  // groups of row tiles whose A rows (about 24 MB) stay in L2.
+  const bool b_fits = static_cast<size_t>(g.N) * g.K <= (32u << 20);
+  p.gm = b_fits ? 1
+                : std::max(1, std::min(p.num_m, static_cast<int>((24u << 20) / (static_cast<size_t>(2 * BM) * g.K))));
   p.f32_out = g.f32_out ? 1 : 0;
   p.per = p.num_m * p.num_n;
   p.tiles = p.per * batch;
