@@ -598,14 +598,16 @@ def run_gpu(args, rank, world, local_rank):
             if i >= 2:
                 times.append(a.elapsed_time(b))
         e2e_serial_ms = float(np.mean(times))
-        # a stream of batches: while step i computes, a copy stream brings in the
-        # inputs of step i + 1 (two device input sets, alternating) and copies
-        # out the result of step i - 1; every step still copies its own inputs
-        # in from pinned host memory and its result out. No L2 flush between
+        # a stream of batches: while step i computes, one copy stream brings in
+        # the inputs of step i + 1 (two device input sets, alternating) and
+        # another copies out the result of step i - 1 (the host link carries
+        # both directions at once); every step still copies its own inputs in
+        # from pinned host memory and its result out. No L2 flush between
         # steps: each step moves more than the L2 holds (V, the packed weights
         # and their expanded copies).
         main = torch.cuda.current_stream()
-        copy = torch.cuda.Stream(device=dev)
+        copy = torch.cuda.Stream(device=dev)      # host -> device
+        copy_out = torch.cuda.Stream(device=dev)  # device -> host
         sets = [(step.V, step.Q, step.A, step.text, step.idx),
                 tuple(torch.empty_like(t) for t in (step.V, step.Q, step.A, step.text, step.idx))]
         outYs = [outY, torch.empty_like(outY).pin_memory()]
@@ -633,6 +635,7 @@ def run_gpu(args, rank, world, local_rank):
             t_host = time.perf_counter()
             a.record(main)
             copy.wait_event(a)
+            copy_out.wait_event(a)
             h2d(0)
             for i in range(E):
                 if i + 1 < E:
@@ -643,12 +646,13 @@ def run_gpu(args, rank, world, local_rank):
                 step.V, step.Q, step.A, step.text, step.idx = sets[i % 2]
                 step.body(out_free=copied[i - 1] if i >= 1 else None)
                 done[i].record(main)
-                with torch.cuda.stream(copy):
-                    copy.wait_event(done[i])
+                with torch.cuda.stream(copy_out):
+                    copy_out.wait_event(done[i])
                     outYs[i % 2].copy_(step.output(step.out_name), non_blocking=True)
                     outIs[i % 2].copy_(step.idx, non_blocking=True)
-                    copied[i].record(copy)
+                    copied[i].record(copy_out)
             main.wait_stream(copy)
+            main.wait_stream(copy_out)
             b.record(main)
             host_ms = (time.perf_counter() - t_host) * 1e3 / E  # enqueueing only: nothing waited on yet
             torch.cuda.synchronize()
@@ -736,9 +740,9 @@ def run_gpu(args, rank, world, local_rank):
                       "h2d_bytes_per_step": int(h2d_bytes), "d2h_bytes_per_step": int(d2h_bytes),
                       "ms_per_step": round(e2e_max, 4), "steps": args.e2e_steps,
                       "timing": "a stream of steps through the C-ABI calls (no graph): each step's inputs copied in "
-                                "from pinned host memory and its result copied out on a copy stream, overlapping the "
-                                "neighbouring steps' compute; total time / steps, no L2 flush (each step moves more "
-                                "than the L2 holds)",
+                                "from pinned host memory on one copy stream and its result copied out on another, "
+                                "overlapping the neighbouring steps' compute; total time / steps, no L2 flush (each "
+                                "step moves more than the L2 holds)",
                       "serial_ms_per_step": round(e2e_serial_ms, 4),
                       "host_enqueue_ms_per_step": round(e2e_host_ms, 4),
                       "serial_value": round(whole_job_tops(ops, world, e2e_serial_ms), 3)}
