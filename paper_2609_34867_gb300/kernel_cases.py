@@ -13,6 +13,7 @@
   python -m paper_2609_34867_gb300.kernel_cases topk B N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases peak {f8,s8,dp4a} ITERS [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases sweep {gemm,quant,select} [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases hostlink MIB [--reps R]
 
 Each case builds seeded synthetic inputs (workloads.py), makes one untimed
 warm-up call of the C-ABI entry point on cuda:0, captures the call in a CUDA
@@ -54,7 +55,11 @@ selects the first replayed launch.
           concepts, softmax CLS saliency), one table row per point;
   saliency p4q_cls_saliency on B images of N tokens (576-token crops, 16
           heads x 64, the CLIP ViT-L vision tower's final layer; bytes: the
-          fp16 keys and queries in, 4 B N out).
+          fp16 keys and queries in, 4 B N out);
+  hostlink the copies the end-to-end path makes: MIB MiB from pinned host
+          memory to the device, back, and both directions at once on two
+          streams (the best of the replays; no graph, no kernel of the
+          library).
 """
 from __future__ import annotations
 
@@ -184,7 +189,7 @@ def _sweep(kind: str, reps: int, dev):
 def main(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn",
-                                     "mse", "topk", "peak", "sweep"])
+                                     "mse", "topk", "peak", "sweep", "hostlink"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
     a = ap.parse_args(argv)
@@ -284,6 +289,36 @@ def main(argv=None):
         print(f"topk {B}x{N} K={K}: {ms * 1e3:.1f} us/call, {8 * B * N / ms / 1e6:.1f} GB/s")
     elif a.case == "sweep":
         _sweep(a.args[0], a.reps, dev)
+    elif a.case == "hostlink":
+        # the host link the end-to-end path copies over: pinned host <-> device, each direction alone and both at once
+        nbytes = int(a.args[0]) << 20
+        h_in = torch.empty((nbytes,), dtype=torch.uint8).pin_memory()
+        h_out = torch.empty((nbytes,), dtype=torch.uint8).pin_memory()
+        d_in = torch.empty((nbytes,), dtype=torch.uint8, device=dev)
+        d_out = torch.empty((nbytes,), dtype=torch.uint8, device=dev)
+        s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+
+        def run(h2d, d2h):
+            torch.cuda.synchronize()
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record()
+            s_in.wait_event(a0)
+            s_out.wait_event(a0)
+            if h2d:
+                with torch.cuda.stream(s_in):
+                    d_in.copy_(h_in, non_blocking=True)
+            if d2h:
+                with torch.cuda.stream(s_out):
+                    h_out.copy_(d_out, non_blocking=True)
+            torch.cuda.current_stream().wait_stream(s_in)
+            torch.cuda.current_stream().wait_stream(s_out)
+            a1.record()
+            torch.cuda.synchronize()
+            return a0.elapsed_time(a1)
+
+        for name, h2d, d2h in (("host->device", True, False), ("device->host", False, True), ("both at once", True, True)):
+            ms = min(run(h2d, d2h) for _ in range(max(a.reps, 2)))
+            print(f"hostlink {name} {nbytes >> 20} MiB each: {ms * 1e3:.1f} us, {nbytes / ms / 1e6:.1f} GB/s per direction")
     elif a.case == "peak":
         kind, iters = a.args[0], int(a.args[1])
         sink = torch.zeros((8192,), dtype=torch.int32, device=dev)
