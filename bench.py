@@ -303,6 +303,9 @@ class Step:
             if all(off % 32 == 0 and n % 256 == 0 for off, n in blocks):
                 self.rm_gemm, self.rm_names, self.rm_blocks = srcs.pop(), names, blocks
                 self.rowmax = torch.empty((len(names), M), dtype=torch.int32, device=dev)
+        # the one-pass re-quantization writes only the expanded codes the next
+        # GEMM reads (no packed copy: nothing in the step reads it)
+        self.packed_requant = self.rm_gemm is None
         # one weight scratch per GEMM of a layer: the weights expand on a side
         # stream, ahead of the GEMMs that read them (see body)
         self.slot = {g: i for i, (g, _) in enumerate(self.gemms)}
@@ -370,8 +373,8 @@ class Step:
             return
         b = self.rm_names.index(name)
         self.p4q.p4q_quant_act_expanded_rowmax(self.Y[self.rm_gemm], [self.rm_blocks[b]], self.rowmax[b:b + 1],
-                                               [self.Xq_re[name]], [self.s_re[name]], [self.Xu_re[name]],
-                                               [self.sXu_re[name]], stream)
+                                               None, [self.s_re[name]], [self.Xu_re[name]], [self.sXu_re[name]],
+                                               stream)
 
     def body_serial(self):
         """The step's segments one after another on the current stream."""

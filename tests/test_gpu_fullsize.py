@@ -32,7 +32,7 @@ import torch
 import bench
 import oracle
 from paper_2609_34867_gb300 import workloads as wl
-from parity import assert_close, assert_codes_equal, sample_rows, take
+from parity import assert_close, assert_codes_equal, assert_expanded_codes_equal, sample_rows, take
 
 pytestmark = pytest.mark.gpu
 
@@ -46,7 +46,7 @@ def run_step(p4q, dev):
         torch.cuda.synchronize()
         step.capture()
         for t in [step.X, step.Xq, step.s_a] + list(step.Y.values()) + list(step.Xq_re.values()) + \
-                list(step.s_re.values()):
+                list(step.s_re.values()) + list(step.Xu_re.values()) + list(step.sXu_re.values()):
             t.zero_()
         step.idx.fill_(-1)
         step()
@@ -89,7 +89,11 @@ def check_step(step, w, images, rows):
             every = Yin.numel() <= (64 << 20)
             r = np.arange(w.M) if every else rows
             cq, sq = oracle.quantize_rows(take(Yin, r))
-            assert_codes_equal(take(step.Xq_re[lin.name], r), take(step.s_re[lin.name], r), cq, sq)
+            if step.packed_requant:
+                assert_codes_equal(take(step.Xq_re[lin.name], r), take(step.s_re[lin.name], r), cq, sq)
+            else:  # the step writes only the expanded codes its GEMM reads
+                assert_expanded_codes_equal(take(step.Xu_re[lin.name], r), take(step.sXu_re[lin.name], r),
+                                            take(step.s_re[lin.name], r), cq, sq)
             a, s = (cq[rows], sq[rows]) if every else (cq, sq)
         else:
             a, s = ca[rows], sa[rows]
