@@ -347,8 +347,9 @@ class Step:
         return self.Wq[layer, g][off:off + n], self.s_w[layer, g][off:off + n]
 
     def _select(self):
+        # the pruned sequence's expanded codes only: the GEMMs read them, nothing reads a packed copy
         self.p4q.p4q_select_gather_quant_expanded(self.V, self.Q, self.A, self.text, self.w.K, self.idx, self.X,
-                                                  self.Xq, self.s_a, self.Xu, self.sXu, self.ws)
+                                                  None, self.s_a, self.Xu, self.sXu, self.ws)
 
     def _expand_w(self, layer, gname, stream=None):
         k = self.slot[gname]

@@ -478,7 +478,8 @@ p4q_status p4q_select_gather_quant(const uint16_t* V, int B, int N, int d, const
 /* p4q_select_gather_quant that also writes the pruned sequence's codes in
  * the expanded form of p4q_expand_codes (Xu [B*(K+T), d] bytes, sum_xu
  * [B*(K+T)] int32; both NULL or both set), for p4q_w4a4_linear_expanded,
- * without a second pass over the codes. The paper has no counterpart. */
+ * without a second pass over the codes. With Xu set, Xq may be NULL (only
+ * the expanded form is written). The paper has no counterpart. */
 p4q_status p4q_select_gather_quant_expanded(const uint16_t* V, int B, int N, int d, const uint16_t* Q, int J,
                                             const float* A_cls, const uint16_t* text, int T,
                                             const p4q_select_params* params, int32_t* idx, uint16_t* X,

@@ -630,8 +630,10 @@ p4q_status p4q_select_gather_quant_expanded(const uint16_t* V, int B, int N, int
                                             size_t ws_bytes, p4q_stream_t stream) {
   p4q_status st = check_select_args(V, B, N, d, J, params, idx);
   if (st != P4Q_OK) return st;
-  if (T < 0 || (T > 0 && !text) || !X || !Xq || !s_a || (!Xu != !sum_xu)) return P4Q_ERR_INVALID_ARG;
-  if ((T > 0 && !aligned16(text)) || !aligned16(X) || !aligned16(Xq) || !aligned16(s_a)) return P4Q_ERR_MISALIGNED;
+  // the packed codes may be left out when the expanded ones are written
+  if (T < 0 || (T > 0 && !text) || !X || (!Xq && !Xu) || !s_a || (!Xu != !sum_xu)) return P4Q_ERR_INVALID_ARG;
+  if ((T > 0 && !aligned16(text)) || !aligned16(X) || (Xq && !aligned16(Xq)) || !aligned16(s_a))
+    return P4Q_ERR_MISALIGNED;
   if (Xu && (!aligned16(Xu) || !aligned16(sum_xu))) return P4Q_ERR_MISALIGNED;
   if ((st = check_device()) != P4Q_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

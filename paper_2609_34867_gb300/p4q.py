@@ -330,9 +330,12 @@ def p4q_select_gather_quant(V, Q, A_cls, text, K, idx, X, Xq, s_a, ws, alpha_per
 
 def p4q_select_gather_quant_expanded(V, Q, A_cls, text, K, idx, X, Xq, s_a, Xu, sum_xu, ws, alpha_permille=300,
                                      beta_permille=200, stream=None):
-    """p4q_select_gather_quant plus the pruned sequence's expanded codes (see p4q_expand_codes)."""
+    """p4q_select_gather_quant plus the pruned sequence's expanded codes (see p4q_expand_codes);
+    Xq may be None (only the expanded codes are written)."""
     _need(V, torch.float16, 3, "V"); _need(idx, torch.int32, 2, "idx"); _need(ws, torch.uint8, 1, "ws")
-    _need(X, torch.float16, 3, "X"); _need(Xq, torch.uint8, 2, "Xq"); _need(s_a, torch.float32, 1, "s_a")
+    _need(X, torch.float16, 3, "X"); _need(s_a, torch.float32, 1, "s_a")
+    if Xq is not None:
+        _need(Xq, torch.uint8, 2, "Xq")
     _need(Xu, torch.uint8, 2, "Xu"); _need(sum_xu, torch.int32, 1, "sum_xu")
     B, N, d = V.shape
     J = 0 if Q is None else Q.shape[1]

@@ -45,7 +45,7 @@ def run_step(p4q, dev):
         step.body()
         torch.cuda.synchronize()
         step.capture()
-        for t in [step.X, step.Xq, step.s_a] + list(step.Y.values()) + list(step.Xq_re.values()) + \
+        for t in [step.X, step.Xq, step.s_a, step.Xu, step.sXu] + list(step.Y.values()) + list(step.Xq_re.values()) + \
                 list(step.s_re.values()) + list(step.Xu_re.values()) + list(step.sXu_re.values()):
             t.zero_()
         step.idx.fill_(-1)
@@ -76,7 +76,8 @@ def check_step(step, w, images, rows):
     assert torch.equal(step.X[:, K:].view(torch.int16), step.text.view(torch.int16))
 
     ca, sa = oracle.quantize_rows(step.X.reshape(-1, d).cpu().numpy())
-    assert_codes_equal(step.Xq.cpu().numpy(), step.s_a.cpu().numpy(), ca, sa)
+    # the step writes the pruned sequence's expanded codes (what its GEMMs read)
+    assert_expanded_codes_equal(step.Xu.cpu().numpy(), step.sXu.cpu().numpy(), step.s_a.cpu().numpy(), ca, sa)
 
     layer = w.layers - 1  # Y holds the last layer's outputs
     for lid, lin in enumerate(w.linears):
