@@ -520,6 +520,91 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
   }
 }
 
+// ---------------------------------------------------------------- dense rows in registers
+// Dense rows of L <= kRegRowMax elements (L % 256 == 0): one warp per row,
+// the row in registers (CH 16-byte chunks per lane, all loads of a row in
+// flight), abs-max by a warp reduction, and the rolling prefetch of the
+// warp's next row (as in the selector's token pass). Same arithmetic as
+// quant_rows_kernel; NORM takes the squared code norm from the expanded
+// codes by dp4a.
+constexpr int kRegRowMax = 5120;
+
+template <int CH, bool NORM>
+__global__ void __launch_bounds__(256, 2)
+    quant_rows_reg_kernel(const uint16_t* __restrict__ X, long long ldx, int rows, int L, RowSinks out) {
+  pdl_wait();  // rows come from the previous kernel
+  pdl_launch_dependents();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nch = L >> 3;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  const int r_first = blockIdx.x * (blockDim.x >> 5) + warp;
+  uint4 v[CH];
+  if (r_first < rows) {
+    const uint4* x = reinterpret_cast<const uint4*>(X + static_cast<size_t>(r_first) * ldx);
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      const int c = lane + 32 * i;
+      v[i] = (c < nch) ? ldg_stream16(x + c) : make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+  for (int r = r_first; r < rows; r += warps) {
+    const bool more = r + warps < rows;
+    const uint4* xn = reinterpret_cast<const uint4*>(X + static_cast<size_t>(more ? r + warps : r) * ldx);
+    uint32_t m = 0;
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      m = __vmaxu2(m, v[i].x & 0x7FFF7FFFu);
+      m = __vmaxu2(m, v[i].y & 0x7FFF7FFFu);
+      m = __vmaxu2(m, v[i].z & 0x7FFF7FFFu);
+      m = __vmaxu2(m, v[i].w & 0x7FFF7FFFu);
+    }
+    const uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+    const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
+    const QRow qr = quant_row(a);
+    float2 n2 = make_float2(0.0f, 0.0f);  // unused: NORM comes from the expanded codes
+    uint32_t su = 0, uu = 0;
+    uint32_t* q4 = out.codes ? reinterpret_cast<uint32_t*>(out.codes + static_cast<size_t>(r) * (L >> 1)) : nullptr;
+    uint2* up = out.u ? reinterpret_cast<uint2*>(out.u + static_cast<size_t>(r) * L) : nullptr;
+#pragma unroll
+    for (int i = 0; i < CH; ++i) {
+      const int c = lane + 32 * i;
+      if (c < nch) {
+        const Codes8 cd = (a != 0.0f) ? quant_chunk<false>(v[i], qr, n2) : Codes8{0u, 0u};
+        if (more) v[i] = ldg_stream16(xn + c);
+        if (q4) q4[c] = packed4(cd);
+        const uint32_t eu = expanded_even(cd), ou = expanded_odd(cd);
+        if (up) up[c] = make_uint2(eu, ou);
+        su = __dp4a(eu + ou, 0x01010101u, su);
+        if (NORM) uu = __dp4a(eu, eu, __dp4a(ou, ou, uu));
+      }
+    }
+    const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
+    const int wn = NORM ? static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, uu)) - 16 * wu + 64 * L : 0;
+    if (lane == 0) {
+      out.scale[r] = (a != 0.0f) ? qr.s : 0.0f;
+      if (NORM) out.norm2[r] = wn;
+      if (out.sum_u) out.sum_u[r] = wu;
+    }
+  }
+}
+
+template <int CH, bool NORM>
+cudaError_t launch_reg(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
+  const long long ldx = src.ldx > 0 ? src.ldx : L;
+  const int blocks = std::max(1, std::min((rows + 7) / 8, 2 * sm_count()));  // one wave
+  return launch_pdl(quant_rows_reg_kernel<CH, NORM>, dim3(blocks), dim3(256), 0, stream, src.X, ldx, rows, L, out);
+}
+
+template <bool NORM>
+cudaError_t launch_reg_norm(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
+  const int ch = L / 256;
+  if (ch <= 4) return launch_reg<4, NORM>(src, rows, L, out, stream);
+  if (ch <= 8) return launch_reg<8, NORM>(src, rows, L, out, stream);
+  if (ch <= 12) return launch_reg<12, NORM>(src, rows, L, out, stream);
+  if (ch <= 16) return launch_reg<16, NORM>(src, rows, L, out, stream);
+  return launch_reg<20, NORM>(src, rows, L, out, stream);
+}
+
 }  // namespace
 
 cudaError_t launch_quant_rowmax(const uint16_t* Y, int ldy, int M, int nblk, const RowmaxBlock* blk,
@@ -575,6 +660,10 @@ cudaError_t launch_quant_rows(const RowSource& src, int rows, int L, const RowSi
   // packed codes may be left out when the expanded ones are written
   if (out.scale == nullptr || (out.codes == nullptr && out.u == nullptr)) return cudaErrorInvalidValue;
   const RowSinks& o2 = out2 ? *out2 : out;
+  // dense rows of at most kRegRowMax elements: the register-resident kernel
+  if (src.X2 == nullptr && src.idx == nullptr && out.copy == nullptr && L % 256 == 0 && L <= kRegRowMax &&
+      (out.u == nullptr) == (out.sum_u == nullptr))
+    return out.norm2 ? launch_reg_norm<true>(src, rows, L, out, stream) : launch_reg_norm<false>(src, rows, L, out, stream);
   return out.norm2 ? launch_norm<true>(src, rows, L, out, o2, stream)
                    : launch_norm<false>(src, rows, L, out, o2, stream);
 }
