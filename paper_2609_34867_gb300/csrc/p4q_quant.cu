@@ -521,35 +521,38 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
 }
 
 // ---------------------------------------------------------------- dense rows in registers
-// Dense rows of L <= kRegRowMax elements (L % 256 == 0): one warp per row,
-// the row in registers (CH 16-byte chunks per lane, all loads of a row in
-// flight), abs-max by a warp reduction, and the rolling prefetch of the
-// warp's next row (as in the selector's token pass). Same arithmetic as
-// quant_rows_kernel; NORM takes the squared code norm from the expanded
-// codes by dp4a.
-constexpr int kRegRowMax = 5120;
+// Dense rows of L <= kRegRowMax elements (L % 256 == 0): a group of G warps
+// per row, the row in registers (CH 16-byte chunks per thread, all loads of
+// a row in flight), abs-max by warp reductions (and, for G > 1, a named
+// barrier of the group), and the rolling prefetch of the group's next row
+// (as in the selector's token pass). Same arithmetic as quant_rows_kernel;
+// NORM takes the squared code norm from the expanded codes by dp4a.
+constexpr int kRegRowMax = 16384;
 
-template <int CH, bool NORM>
+template <int CH, int G, bool NORM>
 __global__ void __launch_bounds__(256, 2)
     quant_rows_reg_kernel(const uint16_t* __restrict__ X, long long ldx, int rows, int L, RowSinks out) {
+  __shared__ uint32_t red[8][3];  // per warp: abs-max, sum of u, sum of u^2 (G > 1)
   pdl_wait();  // rows come from the previous kernel
   pdl_launch_dependents();
+  constexpr int kGroups = 8 / G;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int grp = warp / G, gt = (warp % G) * 32 + lane;  // thread index inside the group
   const int nch = L >> 3;
-  const int warps = gridDim.x * (blockDim.x >> 5);
-  const int r_first = blockIdx.x * (blockDim.x >> 5) + warp;
+  const int groups = gridDim.x * kGroups;
+  const int r_first = blockIdx.x * kGroups + grp;
   uint4 v[CH];
   if (r_first < rows) {
     const uint4* x = reinterpret_cast<const uint4*>(X + static_cast<size_t>(r_first) * ldx);
 #pragma unroll
     for (int i = 0; i < CH; ++i) {
-      const int c = lane + 32 * i;
+      const int c = gt + 32 * G * i;
       v[i] = (c < nch) ? ldg_stream16(x + c) : make_uint4(0u, 0u, 0u, 0u);
     }
   }
-  for (int r = r_first; r < rows; r += warps) {
-    const bool more = r + warps < rows;
-    const uint4* xn = reinterpret_cast<const uint4*>(X + static_cast<size_t>(more ? r + warps : r) * ldx);
+  for (int r = r_first; r < rows; r += groups) {  // uniform across the group
+    const bool more = r + groups < rows;
+    const uint4* xn = reinterpret_cast<const uint4*>(X + static_cast<size_t>(more ? r + groups : r) * ldx);
     uint32_t m = 0;
 #pragma unroll
     for (int i = 0; i < CH; ++i) {
@@ -558,7 +561,13 @@ __global__ void __launch_bounds__(256, 2)
       m = __vmaxu2(m, v[i].z & 0x7FFF7FFFu);
       m = __vmaxu2(m, v[i].w & 0x7FFF7FFFu);
     }
-    const uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+    uint32_t mm = __reduce_max_sync(0xFFFFFFFFu, max(m & 0xFFFFu, m >> 16));
+    if (G > 1) {
+      if (lane == 0) red[warp][0] = mm;
+      named_bar_sync(1 + grp, 32 * G);
+#pragma unroll
+      for (int w = 0; w < G; ++w) mm = max(mm, red[grp * G + w][0]);
+    }
     const float a = __half2float(__ushort_as_half(static_cast<unsigned short>(mm)));
     const QRow qr = quant_row(a);
     float2 n2 = make_float2(0.0f, 0.0f);  // unused: NORM comes from the expanded codes
@@ -567,7 +576,7 @@ __global__ void __launch_bounds__(256, 2)
     uint2* up = out.u ? reinterpret_cast<uint2*>(out.u + static_cast<size_t>(r) * L) : nullptr;
 #pragma unroll
     for (int i = 0; i < CH; ++i) {
-      const int c = lane + 32 * i;
+      const int c = gt + 32 * G * i;
       if (c < nch) {
         const Codes8 cd = (a != 0.0f) ? quant_chunk<false>(v[i], qr, n2) : Codes8{0u, 0u};
         if (more) v[i] = ldg_stream16(xn + c);
@@ -578,31 +587,52 @@ __global__ void __launch_bounds__(256, 2)
         if (NORM) uu = __dp4a(eu, eu, __dp4a(ou, ou, uu));
       }
     }
-    const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
-    const int wn = NORM ? static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, uu)) - 16 * wu + 64 * L : 0;
-    if (lane == 0) {
+    int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
+    int wuu = NORM ? static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, uu)) : 0;
+    if (G > 1) {
+      if (lane == 0) {
+        red[warp][1] = static_cast<uint32_t>(wu);
+        red[warp][2] = static_cast<uint32_t>(wuu);
+      }
+      named_bar_sync(1 + grp, 32 * G);
+      wu = wuu = 0;
+#pragma unroll
+      for (int w = 0; w < G; ++w) {
+        wu += static_cast<int>(red[grp * G + w][1]);
+        wuu += static_cast<int>(red[grp * G + w][2]);
+      }
+    }
+    if (gt == 0) {
       out.scale[r] = (a != 0.0f) ? qr.s : 0.0f;
-      if (NORM) out.norm2[r] = wn;
+      if (NORM) out.norm2[r] = wuu - 16 * wu + 64 * L;
       if (out.sum_u) out.sum_u[r] = wu;
     }
+    if (G > 1) named_bar_sync(1 + grp, 32 * G);  // the group's reductions are read before the next row writes them
   }
 }
 
-template <int CH, bool NORM>
+template <int CH, int G, bool NORM>
 cudaError_t launch_reg(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
   const long long ldx = src.ldx > 0 ? src.ldx : L;
-  const int blocks = std::max(1, std::min((rows + 7) / 8, 2 * sm_count()));  // one wave
-  return launch_pdl(quant_rows_reg_kernel<CH, NORM>, dim3(blocks), dim3(256), 0, stream, src.X, ldx, rows, L, out);
+  const int groups = 8 / G;
+  const int blocks = std::max(1, std::min((rows + groups - 1) / groups, 2 * sm_count()));  // one wave
+  return launch_pdl(quant_rows_reg_kernel<CH, G, NORM>, dim3(blocks), dim3(256), 0, stream, src.X, ldx, rows, L,
+                    out);
 }
 
+// One warp per row up to 5120 elements (at most 20 chunks per lane), else a
+// group of 4 warps (at most 16 chunks per thread: 16384 elements).
 template <bool NORM>
 cudaError_t launch_reg_norm(const RowSource& src, int rows, int L, const RowSinks& out, cudaStream_t stream) {
   const int ch = L / 256;
-  if (ch <= 4) return launch_reg<4, NORM>(src, rows, L, out, stream);
-  if (ch <= 8) return launch_reg<8, NORM>(src, rows, L, out, stream);
-  if (ch <= 12) return launch_reg<12, NORM>(src, rows, L, out, stream);
-  if (ch <= 16) return launch_reg<16, NORM>(src, rows, L, out, stream);
-  return launch_reg<20, NORM>(src, rows, L, out, stream);
+  if (ch <= 4) return launch_reg<4, 1, NORM>(src, rows, L, out, stream);
+  if (ch <= 8) return launch_reg<8, 1, NORM>(src, rows, L, out, stream);
+  if (ch <= 12) return launch_reg<12, 1, NORM>(src, rows, L, out, stream);
+  if (ch <= 16) return launch_reg<16, 1, NORM>(src, rows, L, out, stream);
+  if (ch <= 20) return launch_reg<20, 1, NORM>(src, rows, L, out, stream);
+  const int ch4 = (ch + 3) / 4;
+  if (ch4 <= 12) return launch_reg<12, 4, NORM>(src, rows, L, out, stream);
+  return launch_reg<16, 4, NORM>(src, rows, L, out, stream);
 }
 
 }  // namespace
