@@ -4,11 +4,11 @@
 //   o_i = sum_{j <= i} p_ij v_j,  p_i. = softmax_j(q_i . k_j / sqrt(d_h)),
 // key/value head h / (H / H_kv).
 //
-// One CTA per (128-query block, head, sample), 16 warps: warp w reads TMEM
-// lanes 32 (w % 4) .. + 31 (query rows) and takes every fourth 32-column
-// chunk from chunk w / 4 on (keys for S, head dimensions for O). The keys the
-// block can see (rounded up to 64) are taken 256 at a time, with an online
-// softmax (running row maxima and sums):
+// One CTA per (128-query block, head, sample), 8 warps, two CTAs per SM:
+// warp w reads TMEM lanes 32 (w % 4) .. + 31 (query rows) and takes every
+// second 32-column chunk from chunk w / 4 on (keys for S, head dimensions
+// for O). The keys the block can see (rounded up to 64) are taken 128 at a
+// time, with an online softmax (running row maxima and sums):
 //   1. thread 0 loads the query block once, and per key chunk the keys and
 //      values by TMA into 128-byte swizzled tiles (after the previous chunk's
 //      P V has released them), and issues S = Q K^T on the tensor cores
@@ -26,8 +26,9 @@
 //      when a row's maximum moved);
 //   4. thread 0 issues O += P V^T. After the last chunk each warp scales its
 //      32 columns of O by 1 / sum and stores fp16.
-// One chunk (m <= 256) is a plain two-pass softmax. Every wait is bounded; a
-// time-out sets the kernel's device error word.
+// One chunk (a block that sees at most 128 keys) is a plain two-pass
+// softmax. Every wait is bounded; a time-out sets the kernel's device error
+// word.
 #include <cuda_fp16.h>
 
 #include "p4q.h"
