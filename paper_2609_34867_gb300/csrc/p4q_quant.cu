@@ -6,16 +6,30 @@
 // and zero codes. Codes are written packed, two per byte, the even index in
 // the low nibble (two's complement).
 //
-// Rows stream through shared memory. A group of G warps owns a ring of S row
-// buffers that its leader thread fills with bulk asynchronous copies
-// (cp.async.bulk, completion counted on one mbarrier per buffer), so that
-// while the group quantizes one row the next S - 1 rows are already on their
-// way from HBM; the group reads each row from shared memory twice, once for
-// the abs-max and once to quantize. Two persistent CTAs of 8 warps per SM. The
-// same kernel serves the activation quantizer, the weight quantizer, the
-// selector's fake-quantized copies (with the squared code norm as an extra
-// output) and the fused gather of the pruned sequence (rows addressed through
-// the kept indices, fp16 copy written beside the codes).
+// Kernels:
+//   quant_rows_reg_kernel     dense rows of up to 16384 elements (a multiple
+//                             of 256): each row held in the registers of one
+//                             warp (up to 5120 elements) or of four, every
+//                             load of a row in flight, the group's next row
+//                             prefetched chunk by chunk as the current one is
+//                             quantized. Activations, weights, the selector's
+//                             concepts.
+//   quant_rows_kernel         every other case (the fused gather of the
+//                             pruned sequence through the kept indices with
+//                             its fp16 copy, two row sets in one launch, other
+//                             row lengths): rows stream through shared memory,
+//                             a group of G warps owning a ring of S row
+//                             buffers that its leader fills with bulk
+//                             asynchronous copies (cp.async.bulk, one mbarrier
+//                             per buffer); each row is read from shared memory
+//                             twice (abs-max, then codes). Two persistent CTAs
+//                             of 8 warps per SM.
+//   select_token_quant_kernel the selector's tokens with the query dot
+//                             products fused (register-resident, per image).
+//   quant_rowmax_kernel       column blocks of a GEMM output whose row
+//                             abs-max is known: one streaming pass.
+// Optional outputs: the codes expanded one byte each (u = code + 8, the
+// GEMM's operand form) with their row sums, and the squared code norm.
 #include <cuda_fp16.h>
 
 #include <algorithm>
