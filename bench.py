@@ -386,7 +386,12 @@ class Step:
         """The step as plain C-ABI calls (no graph), on three streams:
         - side: every GEMM's weight expansion, into that GEMM's scratch, in
           step order (a later layer's waits until the previous layer's GEMM
-          has read the scratch), overlapping the selector and the GEMMs;
+          has read the scratch). The first GEMM of a layer has its weights
+          expanded ahead (beside the selector, or beside the previous
+          layer's GEMMs); the layer's other GEMMs have theirs expanded once
+          that first GEMM is about to start, so the expansion streams beside
+          a tensor-bound GEMM instead of competing with the memory-bound
+          selector for HBM;
         - aux: the o chain (re-quantization of the q block, o GEMM), beside
           the down chain (re-quantization of the up block, down GEMM);
         - the current stream: everything else.
@@ -400,18 +405,31 @@ class Step:
         ngemm = len(self.gemms)
         ready = [torch.cuda.Event() for _ in range(n)]
         freed = [torch.cuda.Event() for _ in range(n)]
-        with torch.cuda.stream(self.side):
-            for i, (layer, gname, _) in enumerate(self.gemm_calls):
+
+        def expand(i, after=None):
+            """Call i's weights into its GEMM's scratch, on the side stream."""
+            layer, gname, _ = self.gemm_calls[i]
+            with torch.cuda.stream(self.side):
                 if i >= ngemm:
                     self.side.wait_event(freed[i - ngemm])
+                if after is not None:
+                    self.side.wait_event(after)
                 self._expand_w(layer, gname, self.side)
                 ready[i].record(self.side)
+
+        expand(0)
         self._select()
         members = dict(self.gemms)
         o_src = self.col[self.REQUANT["o"]][0] if "o" in self.Xq_re else None
         src_done, o_read = None, None
         for i, (layer, gname, xin) in enumerate(self.gemm_calls):
             first = members[gname][0]
+            if i % ngemm == 0:
+                # the layer's first GEMM is next: its other GEMMs' weights now
+                go = torch.cuda.Event()
+                go.record(main)
+                for j in range(i + 1, i + ngemm):
+                    expand(j, go)
             if first == "o":
                 with torch.cuda.stream(self.aux):
                     if src_done is not None:
@@ -432,6 +450,8 @@ class Step:
             main.wait_event(ready[i])
             self._gemm(layer, gname, *xin())
             freed[i].record(main)
+            if i % ngemm == 0 and i + ngemm < n:
+                expand(i + ngemm)  # the next layer's first GEMM, once this one has read the scratch
             if gname == o_src:
                 src_done = torch.cuda.Event()
                 src_done.record(main)
