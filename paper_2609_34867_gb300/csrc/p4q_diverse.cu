@@ -80,7 +80,7 @@ struct DivScratch {
   uint64_t bar_done;                    // MMA commit at teardown -> nothing in flight
   uint32_t tmem_slot;
   volatile int abort_flag;
-  __align__(16) float cp[kPool][kPool]; // cos(ptok[i], ptok[j]) (Eq. 4, exact)
+  __align__(16) float cp[kPool][kPool + 1]; // cos(ptok[i], ptok[j]) (Eq. 4, exact; padded: column writes)
 };
 
 __device__ __forceinline__ float order_key_float(uint32_t k) {
@@ -330,10 +330,15 @@ __global__ void __launch_bounds__(kThreads, 1) select_diverse_kernel(const DivAr
           v[k] = f < npool ? __ldg(row + s.pci[f]) : 0.0f;
         }
         const int ne = s.pnorm[e];
+        // the block is symmetric: each pair once (f >= e), written both ways
 #pragma unroll
         for (int k = 0; k < kPoolPer; ++k) {
           const int f = lane + 32 * k;
-          if (f < npool) s.cp[e][f] = code_cosine(static_cast<int>(v[k]), ne, s.pnorm[f]);
+          if (f < npool && f >= e) {
+            const float c = code_cosine(static_cast<int>(v[k]), ne, s.pnorm[f]);
+            s.cp[e][f] = c;
+            s.cp[f][e] = c;
+          }
         }
       }
       // per pool row: the largest cosine to the unseen picks (chunks of 128
