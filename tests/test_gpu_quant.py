@@ -28,7 +28,8 @@ def _check(p4q, dev, x):
 
 
 @pytest.mark.parametrize("M,K", [(1, 16), (7, 128), (33, 4096), (96, 4096), (300, 11008), (17, 13824),
-                                 (5, 16384), (257, 5120)])
+                                 (5, 16384), (257, 5120),
+                                 (2100, 5120), (2049, 11008)])  # from 2048 rows: the register-resident kernel
 def test_quant_act_matches_oracle(p4q, dev, M, K):
     _check(p4q, dev, wl.activations(M, K, seed=M + K))
 
@@ -97,7 +98,7 @@ def test_quant_act_on_a_column_block_matches_dense(p4q, dev):
 def test_quant_act_expanded_matches_quant_then_expand(p4q, dev):
     """The quantizer's expanded output equals p4q_expand_codes of its packed
     codes (bytes and row sums), for one-warp and multi-warp row lengths."""
-    for M, K, seed in [(300, 1024, 31), (77, 11008, 32), (129, 5120, 33)]:
+    for M, K, seed in [(300, 1024, 31), (77, 11008, 32), (129, 5120, 33), (2048, 5120, 34), (2053, 13824, 35)]:
         X = torch.from_numpy(wl.activations(M, K, seed=seed)).to(dev)
         X[3].zero_()
         Xq = torch.empty((M, K // 2), dtype=torch.uint8, device=dev)

@@ -27,7 +27,8 @@ def _select(p4q, dev, x, K, use_q=True, use_a=True, alpha=300, beta=200):
 
 @pytest.mark.parametrize("B,N,d,K,J,seed", [(2, 100, 128, 20, 3, 0), (3, 576, 256, 64, 3, 1),
                                             (1, 30, 128, 10, 2, 2), (2, 301, 384, 77, 5, 3),
-                                            (1, 1152, 128, 200, 3, 4)])
+                                            (1, 1152, 128, 200, 3, 4),
+                                            (1, 2048, 5376, 160, 2, 5)])  # rows wider than the token pass
 def test_select_matches_oracle(p4q, dev, B, N, d, K, J, seed):
     w = wl.Workload("t", B=B, N=N, d=d, K=K, T=0, J=J, seed=seed, heavy_tail=False, linears=())
     got, ref = _select(p4q, dev, wl.selector_inputs(w), K)
