@@ -472,9 +472,12 @@ cudaError_t launch_token_quant(const uint16_t* V, int B, int N, int L, int J, co
 // ---------------------------------------------------------------- known row abs-max
 // Up to two column blocks of Y quantized per row with the abs-max already
 // known (the GEMM's row-max epilogue): no abs-max pass, no reduction before
-// the codes, so one warp streams a block row in 256-element steps (one
-// 16-byte chunk per lane, kRmUnroll steps in flight) and only the row sum of
-// the expanded codes is reduced at the end. Same arithmetic as
+// the codes, so G warps stream a block row in 256-element steps (one 16-byte
+// chunk per lane, steps interleaved over the G warps, kRmUnroll in flight per
+// warp) and only the row sum of the expanded codes is reduced at the end. The
+// pass is issue-bound (about 14 instructions per code at a quarter of the
+// warp slots), so a few thousand rows (the short sequences) take G = 2 or 4
+// warps per row to fill the GPU; G = 1 otherwise. Same arithmetic as
 // quant_rows_kernel (s = a / 7, quant_chunk), so the same codes and scales.
 struct RowmaxArgs {
   const uint16_t* Y;
@@ -485,13 +488,17 @@ struct RowmaxArgs {
 
 constexpr int kRmUnroll = 4;  // 256-element steps in flight per warp
 
-__global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
+template <int G>
+__global__ void __launch_bounds__(256, 4) quant_rowmax_kernel(RowmaxArgs a) {
+  __shared__ uint32_t red[2][8];  // per warp: its part of the row sum (two buffers: one barrier per row)
   pdl_wait();  // Y and its row maxima come from the previous kernel
   pdl_launch_dependents();
-  const int lane = threadIdx.x & 31;
-  const int warps = gridDim.x * (blockDim.x >> 5);
+  constexpr int kRows = 8 / G;  // rows in flight per CTA
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int grp = warp / G, seg = warp % G;
   const int tasks = a.nblk * a.M;
-  for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < tasks; t += warps) {
+  int par = 0;
+  for (int t = blockIdx.x * kRows + grp; t < tasks; t += gridDim.x * kRows, par ^= 1) {  // uniform across the group
     const int bi = t / a.M, m = t - bi * a.M;
     const bool b1 = bi != 0;  // field by field: no dynamic index into the parameter array
     RowmaxBlock B;
@@ -509,15 +516,18 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
     const int steps = B.L >> 8;  // 256 elements per warp step
     float2 n2 = make_float2(0.0f, 0.0f);
     uint32_t su = 0;
-    for (int j0 = 0; j0 < steps; j0 += kRmUnroll) {
+    for (int j0 = seg; j0 < steps; j0 += kRmUnroll * G) {
       uint4 v[kRmUnroll];
 #pragma unroll
-      for (int k = 0; k < kRmUnroll; ++k)
-        v[k] = (j0 + k < steps) ? ldg_stream16(x + (j0 + k) * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+      for (int k = 0; k < kRmUnroll; ++k) {
+        const int j = j0 + k * G;
+        v[k] = (j < steps) ? ldg_stream16(x + j * 32 + lane) : make_uint4(0u, 0u, 0u, 0u);
+      }
 #pragma unroll
       for (int k = 0; k < kRmUnroll; ++k) {
-        if (j0 + k < steps) {
-          const int c = (j0 + k) * 32 + lane;
+        const int j = j0 + k * G;
+        if (j < steps) {
+          const int c = j * 32 + lane;
           const Codes8 cd = (amax != 0.0f) ? quant_chunk<false>(v[k], qr, n2) : Codes8{0u, 0u};
           if (q4) q4[c] = packed4(cd);
           const uint32_t eu = expanded_even(cd), ou = expanded_odd(cd);
@@ -526,10 +536,17 @@ __global__ void __launch_bounds__(256) quant_rowmax_kernel(RowmaxArgs a) {
         }
       }
     }
-    const int wu = static_cast<int>(__reduce_add_sync(0xFFFFFFFFu, su));
-    if (lane == 0) {
+    uint32_t wu = __reduce_add_sync(0xFFFFFFFFu, su);
+    if (G > 1) {
+      if (lane == 0) red[par][warp] = wu;
+      named_bar_sync(1 + grp, 32 * G);
+      wu = 0;
+#pragma unroll
+      for (int i = 0; i < G; ++i) wu += red[par][grp * G + i];
+    }
+    if (seg == 0 && lane == 0) {
       B.scale[m] = (amax != 0.0f) ? qr.s : 0.0f;
-      B.sum_u[m] = wu;
+      B.sum_u[m] = static_cast<int>(wu);
     }
   }
 }
@@ -667,9 +684,17 @@ cudaError_t launch_quant_rowmax(const uint16_t* Y, int ldy, int M, int nblk, con
       return cudaErrorInvalidValue;
     a.b[i] = blk[i];
   }
+  // warps per row: as many as fill the resident warp slots (32 per SM at the
+  // kernel's registers), at most one per 256-element step of the shorter block
   const int tasks = nblk * M;
-  const int blocks = std::max(1, std::min((tasks + 7) / 8, 8 * sm_count()));
-  return launch_pdl(quant_rowmax_kernel, dim3(blocks), dim3(256), 0, stream, a);
+  const int steps = std::min(a.b[0].L, a.b[nblk - 1].L) >> 8;
+  const long long slots = 32LL * sm_count();
+  const int G = (4LL * tasks <= slots && steps >= 4) ? 4 : (2LL * tasks <= slots && steps >= 2) ? 2 : 1;
+  const int rows_per_cta = 8 / G;
+  const int blocks = std::max(1, std::min((tasks + rows_per_cta - 1) / rows_per_cta, 8 * sm_count()));
+  if (G == 4) return launch_pdl(quant_rowmax_kernel<4>, dim3(blocks), dim3(256), 0, stream, a);
+  if (G == 2) return launch_pdl(quant_rowmax_kernel<2>, dim3(blocks), dim3(256), 0, stream, a);
+  return launch_pdl(quant_rowmax_kernel<1>, dim3(blocks), dim3(256), 0, stream, a);
 }
 
 bool select_token_quant_applies(int d, int J) {

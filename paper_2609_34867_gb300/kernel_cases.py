@@ -3,7 +3,7 @@
   python -m paper_2609_34867_gb300.kernel_cases gemm M N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases gemm8 M N K [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases quant M K [--reps R]
-  python -m paper_2609_34867_gb300.kernel_cases requant M L LD [--reps R]
+  python -m paper_2609_34867_gb300.kernel_cases {requant,requant1} M L LD [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases select WORKLOAD [B] [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases saliency B N [--reps R]
   python -m paper_2609_34867_gb300.kernel_cases swiglu M K LD [--reps R]
@@ -31,6 +31,9 @@ selects the first replayed launch.
   requant p4q_quant_act_expanded on the last L columns of an M x LD fp16
           matrix (a linear's output block inside a fused GEMM's output), with
           the expanded codes (bytes: 2 M L in, 3 M L / 2 + 8 M out);
+  requant1 p4q_quant_act_expanded_rowmax on the same block with its row
+          abs-max given (as a GEMM's row-max epilogue records it), expanded
+          codes only (bytes: 2 M L in, M L + 8 M out);
   select  p4q_select_gather_quant on one of the LLaVA-shaped workloads (B:
           its first B images instead of all);
   swiglu  p4q_swiglu_quant_expanded on gate / up, the last 2 K columns of an
@@ -188,7 +191,7 @@ def _sweep(kind: str, reps: int, dev):
 
 def main(argv=None):
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "select", "saliency", "swiglu", "rmsnorm", "attn",
+    ap.add_argument("case", choices=["gemm", "gemm8", "quant", "requant", "requant1", "select", "saliency", "swiglu", "rmsnorm", "attn",
                                      "mse", "topk", "peak", "sweep", "hostlink"])
     ap.add_argument("args", nargs="+")
     ap.add_argument("--reps", type=int, default=3)
@@ -231,6 +234,18 @@ def main(argv=None):
         ms = _timed(lambda: p4q.p4q_quant_act_expanded(X, Xq, s, Xu, su), a.reps, dev)
         nbytes = 2 * M * L + 3 * M * L // 2 + 8 * M
         print(f"requant {M}x{L} of {LD}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
+    elif a.case == "requant1":
+        M, L, LD = (int(x) for x in a.args)
+        g = torch.Generator(device=dev).manual_seed(0)
+        Y = (torch.randn((M, LD), generator=g, device=dev) * 4.0).to(torch.float16)
+        rowmax = (Y[:, LD - L:].contiguous().view(torch.int16).to(torch.int32) & 0x7FFF).amax(dim=1)[None]
+        s = torch.empty((M,), dtype=torch.float32, device=dev)
+        Xu = torch.empty((M, L), dtype=torch.uint8, device=dev)
+        su = torch.empty((M,), dtype=torch.int32, device=dev)
+        ms = _timed(lambda: p4q.p4q_quant_act_expanded_rowmax(Y, [(LD - L, L)], rowmax, None, [s], [Xu], [su]),
+                    a.reps, dev)
+        nbytes = 2 * M * L + M * L + 8 * M
+        print(f"requant1 {M}x{L} of {LD}: {ms * 1e3:.1f} us/call, {nbytes / ms / 1e6:.1f} GB/s")
     elif a.case == "swiglu":
         M, K, LD = (int(x) for x in a.args)
         g = torch.Generator(device=dev).manual_seed(0)

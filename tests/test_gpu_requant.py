@@ -62,7 +62,10 @@ def _quant_ref(p4q, Yb):
 @pytest.mark.parametrize("M,ldy,blocks,packed", [(33, 2048, [(0, 512), (768, 1280)], True),
                                                  (2048, 4096 * 3 + 11008 * 2, [(0, 4096), (23296, 11008)], True),
                                                  (300, 1024, [(256, 768)], False),
-                                                 (5, 5120, [(0, 5120), (0, 5120)], True)])
+                                                 (5, 5120, [(0, 5120), (0, 5120)], True),
+                                                 (5000, 1536, [(0, 512), (1024, 512)], True),  # one warp per row
+                                                 (2048, 6144, [(2048, 4096)], True),           # two warps per row
+                                                 (1000, 12032, [(1024, 11008)], False)])       # four, 43 steps
 def test_known_max_quantizer_matches_two_pass(p4q, dev, M, ldy, blocks, packed):
     g = torch.Generator(device=dev).manual_seed(M)
     Y = (torch.randn((M, ldy), generator=g, device=dev) * 3.0).to(torch.float16)
