@@ -213,7 +213,7 @@ p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t
  *   o_i = sum_{j <= i} p_ij v_j, p_i. = softmax_j(q_i . k_j / sqrt(dh)),
  * with key/value head h / (H / Hkv). Position encodings are applied by the
  * caller. fp16 inputs, products accumulated in fp32, p rounded to fp16 before
- * the product with v (keys taken 256 at a time with running row maxima: p is
+ * the product with v (keys taken 128 at a time with running row maxima: p is
  * relative to the maximum so far, the earlier partial sums and products
  * rescaled when it moves), fp32 row sums, fp16 output.
  *   q [B*m, ldq] fp16: row b*m + i holds position i of sample b, head h in

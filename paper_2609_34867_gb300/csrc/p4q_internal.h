@@ -138,7 +138,7 @@ cudaError_t launch_rmsnorm_quant(const uint16_t* X, long long ldx, const uint16_
                                  uint8_t* Xq, float* s_a, uint8_t* Xu, int32_t* sum_xu, cudaStream_t stream);
 
 // ------------------------------------------------------------ causal attention (FP16 K/V)
-// Longest sample the kernel takes (the keys stream through in chunks of 256).
+// Longest sample the kernel takes (the keys stream through in chunks of 128).
 constexpr int kAttnMaxLen = 8192;
 // Dynamic shared memory of one CTA for samples of m positions.
 size_t causal_attention_smem_bytes(int m);
