@@ -214,8 +214,9 @@ p4q_status p4q_rmsnorm_quant_expanded(const uint16_t* X, int ldx, const uint16_t
  * with key/value head h / (H / Hkv). Position encodings are applied by the
  * caller. fp16 inputs, products accumulated in fp32, p rounded to fp16 before
  * the product with v (keys taken 128 at a time with running row maxima: p is
- * relative to the maximum so far, the earlier partial sums and products
- * rescaled when it moves), fp32 row sums, fp16 output.
+ * relative to a reference maximum of the keys so far, which moves when a
+ * chunk's maximum exceeds it by 2^8 in p, the earlier partial sums and
+ * products rescaled then), fp32 row sums, fp16 output.
  *   q [B*m, ldq] fp16: row b*m + i holds position i of sample b, head h in
  *                      columns h*dh .. h*dh + dh - 1   (device, read)
  *   k, v [B*m, ldk / ldv] fp16, Hkv heads likewise   (device, read; rows may
