@@ -68,9 +68,11 @@ struct AttnParams {
 // Shared memory: two query buffers, two key stages, two value stages (two
 // tiles each: head dims 0-63, 64-127), the row maxima / sums of the two
 // halves of each row, barriers.
+constexpr int kQBufs = 2;    // query buffers (units in flight)
+constexpr int kKStages = 2;  // key stages
 constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + 4 * kTileBytes;
-constexpr int kOffV = kOffK + 4 * kTileBytes;
+constexpr int kOffK = kOffQ + 2 * kQBufs * kTileBytes;
+constexpr int kOffV = kOffK + 2 * kKStages * kTileBytes;
 constexpr int kOffRed = kOffV + 4 * kTileBytes;  // float [3 (chunk parity; row sums)][2 (half)][128]
 constexpr int kOffBar = kOffRed + 6 * kBQ * 4;
 constexpr int kNumBars = 18;
@@ -194,7 +196,8 @@ struct ChunkIt {
 };
 
 struct Bars {
-  uint64_t q_full[2], q_empty[2], k_full[2], k_empty[2], v_full[2], v_empty[2], s_full[2];
+  uint64_t q_full[kQBufs], q_empty[kQBufs], k_full[kKStages], k_empty[kKStages];
+  uint64_t v_full[2], v_empty[2], s_full[2];
   uint64_t o_free[2];  // per O buffer: a unit's output has been read out
   uint64_t p_ready, pv_done, mma_done;
   uint32_t tmem_slot;
@@ -212,11 +215,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   volatile int* abort_flag = &br.abort_flag;
 
   if (t == 0) {
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < kQBufs; ++i) {
       mbar_init(&br.q_full[i], 1);
       mbar_init(&br.q_empty[i], 1);
+    }
+    for (int i = 0; i < kKStages; ++i) {
       mbar_init(&br.k_full[i], 1);
       mbar_init(&br.k_empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
       mbar_init(&br.v_full[i], 1);
       mbar_init(&br.v_empty[i], 1);
       mbar_init(&br.s_full[i], 1);
@@ -255,8 +262,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto load_k = [&](const ChunkIt& it) {
         const int hk = it.h / p.group;
         if (it.c == 0) {
-          const int qbuf = it.uq & 1;
-          if (it.uq >= 2) ok = ok && mbar_wait_spin(&br.q_empty[qbuf], ((it.uq >> 1) - 1) & 1, abort_flag, &g_attn_err);
+          const int qbuf = it.uq % kQBufs;
+          if (it.uq >= kQBufs)
+            ok = ok && mbar_wait_spin(&br.q_empty[qbuf], ((it.uq / kQBufs) - 1) & 1, abort_flag, &g_attn_err);
           if (!ok) return;
           mbar_arrive_expect_tx(&br.q_full[qbuf], 2 * kTileBytes);
           for (int kb = 0; kb < 2; ++kb)
@@ -264,8 +272,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                         it.qb * kBQ, it.b);
           ++q_issued;
         }
-        const int st = static_cast<int>(it.j & 1);
-        if (it.j >= 2) ok = ok && mbar_wait_spin(&br.k_empty[st], ((it.j >> 1) - 1) & 1, abort_flag, &g_attn_err);
+        const int st = static_cast<int>(it.j % kKStages);
+        if (it.j >= kKStages)
+          ok = ok && mbar_wait_spin(&br.k_empty[st], ((it.j / kKStages) - 1) & 1, abort_flag, &g_attn_err);
         if (!ok) return;
         mbar_arrive_expect_tx(&br.k_full[st], 2 * kTileBytes);
         for (int kb = 0; kb < 2; ++kb)
@@ -297,12 +306,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // nothing of this CTA's loads may still be in flight when it exits
       volatile int never = 0;
-      for (long long jj = k_issued - 1; jj >= 0 && jj >= k_issued - 2; --jj)
-        mbar_wait(&br.k_full[jj & 1], (jj >> 1) & 1, &never, &g_attn_err);
+      for (long long jj = k_issued - 1; jj >= 0 && jj >= k_issued - kKStages; --jj)
+        mbar_wait(&br.k_full[jj % kKStages], (jj / kKStages) & 1, &never, &g_attn_err);
       for (long long jj = v_issued - 1; jj >= 0 && jj >= v_issued - 2; --jj)
         mbar_wait(&br.v_full[jj & 1], (jj >> 1) & 1, &never, &g_attn_err);
-      for (int qq = q_issued - 1; qq >= 0 && qq >= q_issued - 2; --qq)
-        mbar_wait(&br.q_full[qq & 1], (qq >> 1) & 1, &never, &g_attn_err);
+      for (int qq = q_issued - 1; qq >= 0 && qq >= q_issued - kQBufs; --qq)
+        mbar_wait(&br.q_full[qq % kQBufs], (qq / kQBufs) & 1, &never, &g_attn_err);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMAs
@@ -315,22 +324,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       pit.start(p);
       // S = Q K^T of a chunk into S buffer j & 1
       auto issue_s = [&](const ChunkIt& it) {
-        const int qbuf = it.uq & 1, st = static_cast<int>(it.j & 1);
-        if (it.c == 0) ok = ok && mbar_wait_spin(&br.q_full[qbuf], (it.uq >> 1) & 1, abort_flag, &g_attn_err);
-        ok = ok && mbar_wait_spin(&br.k_full[st], (it.j >> 1) & 1, abort_flag, &g_attn_err);
+        const int qbuf = it.uq % kQBufs, st = static_cast<int>(it.j & 1), ks = static_cast<int>(it.j % kKStages);
+        if (it.c == 0) ok = ok && mbar_wait_spin(&br.q_full[qbuf], (it.uq / kQBufs) & 1, abort_flag, &g_attn_err);
+        ok = ok && mbar_wait_spin(&br.k_full[ks], (it.j / kKStages) & 1, abort_flag, &g_attn_err);
         if (!ok) return;
         tc_fence_after();
         const uint32_t d = tmem + kColS + 128u * static_cast<uint32_t>(st);
 #pragma unroll
         for (int kb = 0; kb < 2; ++kb) {
           const uint32_t a0 = smem_u32(smem + kOffQ + (2 * qbuf + kb) * kTileBytes);
-          const uint32_t b0 = smem_u32(smem + kOffK + (2 * st + kb) * kTileBytes);
+          const uint32_t b0 = smem_u32(smem + kOffK + (2 * ks + kb) * kTileBytes);
 #pragma unroll
           for (int k = 0; k < 4; ++k)
             mma_f16(d, sw128_kmajor_desc(a0 + 32 * k), sw128_kmajor_desc(b0 + 32 * k), idS, (kb | k) != 0 ? 1u : 0u);
         }
         mma_commit(&br.s_full[st]);
-        mma_commit(&br.k_empty[st]);
+        mma_commit(&br.k_empty[ks]);
         if (it.c == it.qb) mma_commit(&br.q_empty[qbuf]);
       };
       if (sit.valid) {

@@ -91,3 +91,14 @@ def test_attention_fullsize_sampled(p4q, dev, B, m, H):
         cols = slice(h * DH, (h + 1) * DH)
         want = oracle.causal_attention(q[rows, cols], k[rows, cols], v[rows, cols], 1, m, 1, 1, DH)
         _check(got[rows, cols], want, v[rows, cols], 1, m, 1, 1)
+
+
+def test_attention_many_units_per_cta(p4q, dev):
+    """Enough (sample, head) pairs that every persistent CTA works through
+    several units of mixed length (three query blocks per sample, the last
+    one ragged) and the last group of pairs is partly empty: the O buffers
+    and their read-out barriers cycle many times."""
+    B, m, H, Hkv = 8, 300, 40, 8  # 960 units on 150 CTAs; 320 pairs in groups of 50
+    q, k, v = _inputs(B, m, H, Hkv, seed=31)
+    got = _run(p4q, dev, q, k, v, B, m, H, Hkv)
+    _check(got, oracle.causal_attention(q, k, v, B, m, H, Hkv, DH), v, B, m, H, Hkv)
