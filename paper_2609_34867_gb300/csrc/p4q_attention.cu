@@ -23,7 +23,7 @@
 //              place as an MN-major operand (no transposed copy);
 //   warps 2-9  two threads per query row (its TMEM lane), one per half of
 //              the chunk's keys and of O's columns: the chunk's row maximum
-//              (the halves meet in shared memory), p = 2^((s - m_new)
+//              (the halves meet in shared memory), p = 2^((s - m)
 //              log2(e) / sqrt(d_h)) (0 past the causal limit on the diagonal
 //              chunk) rounded to fp16 into TMEM over the chunk's S, and the
 //              row sum. The reference maximum m of a row moves only when the
@@ -34,8 +34,8 @@
 //              a unit's O / sum -> fp16 runs after the next unit's first
 //              chunk.
 // Keys and rows past m read as zeros (3-D tensor maps over [B][m][cols]).
-// Every wait polls (a suspended thread wakes up too late for this pipeline)
-// and is bounded; a time-out sets the kernel's device error word.
+// Every wait of the pipeline polls the barrier and is bounded; a time-out
+// sets the kernel's device error word.
 #include <cuda_fp16.h>
 
 #include <algorithm>
