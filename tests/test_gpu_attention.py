@@ -102,3 +102,12 @@ def test_attention_many_units_per_cta(p4q, dev):
     q, k, v = _inputs(B, m, H, Hkv, seed=31)
     got = _run(p4q, dev, q, k, v, B, m, H, Hkv)
     _check(got, oracle.causal_attention(q, k, v, B, m, H, Hkv, DH), v, B, m, H, Hkv)
+
+
+def test_attention_longest_sample(p4q, dev):
+    """The documented maximum, m = 8192 positions (64 query blocks, up to 64
+    key chunks per block): the row sums and P V accumulate over 8192 keys."""
+    B, m, H, Hkv = 1, 8192, 1, 1
+    q, k, v = _inputs(B, m, H, Hkv, seed=41)
+    got = _run(p4q, dev, q, k, v, B, m, H, Hkv)
+    _check(got, oracle.causal_attention(q, k, v, B, m, H, Hkv, DH), v, B, m, H, Hkv)
