@@ -160,6 +160,37 @@ def test_select_gather_quant_expanded_matches(p4q, dev):
     assert torch.equal(Xq, ref_q) and torch.equal(Xu, ref_u) and torch.equal(su, ref_su)
 
 
+def test_select_gather_quant_expanded_nine_images_matches_oracle(p4q, dev):
+    """Nine images of more than 1024 tokens (no Gram mode: the kept set's
+    cosine-max GEMM and the candidates' pair GEMM), twice on the same
+    workspace: every image's indices, gathered rows, codes, scales and
+    expanded codes against the oracle."""
+    w = wl.Workload("t", B=9, N=1100, d=256, K=150, T=12, J=3, seed=23, heavy_tail=False, linears=())
+    x = wl.selector_inputs(w)
+    V, Q, A, T = (_t(a, dev) for a in (x.V, x.Q, x.A, x.text))
+    ws = p4q.select_workspace(w.B, w.N, w.d, w.J, w.K, dev)
+    M = w.B * (w.K + w.T)
+    idx = torch.full((w.B, w.K), -1, dtype=torch.int32, device=dev)
+    X = torch.empty((w.B, w.K + w.T, w.d), dtype=torch.float16, device=dev)
+    Xq = torch.empty((M, w.d // 2), dtype=torch.uint8, device=dev)
+    s = torch.empty((M,), dtype=torch.float32, device=dev)
+    Xu = torch.empty((M, w.d), dtype=torch.uint8, device=dev)
+    su = torch.empty((M,), dtype=torch.int32, device=dev)
+    for _ in range(2):
+        p4q.p4q_select_gather_quant_expanded(V, Q, A, T, w.K, idx, X, Xq, s, Xu, su, ws)
+    ref_u, ref_su = p4q.expand_codes(Xq)
+    torch.cuda.synchronize()
+    assert p4q.p4q_device_status() == 0
+    ref_idx = oracle.select_batch(x.V, w.K, x.Q, x.A)
+    assert np.array_equal(idx.cpu().numpy(), ref_idx)
+    Xr = oracle.gather(x.V, ref_idx, x.text)
+    assert np.array_equal(X.cpu().numpy().astype(np.float32), Xr)
+    c, sr = oracle.quantize_rows(Xr.reshape(-1, w.d))
+    assert np.array_equal(oracle.unpack_codes(Xq.cpu().numpy()), c)
+    assert np.array_equal(s.cpu().numpy().view(np.uint32), sr.view(np.uint32))
+    assert torch.equal(Xu, ref_u) and torch.equal(su, ref_su)
+
+
 def test_select_from_two_host_threads_on_two_streams(p4q, dev):
     """Concurrent calls from two host threads on two streams, each with its own
     workspace: the library keeps no state between the launches of a call, so
