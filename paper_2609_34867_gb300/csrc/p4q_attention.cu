@@ -322,7 +322,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       ChunkIt sit, pit;
       sit.start(p);
       pit.start(p);
-      // S = Q K^T of a chunk into S buffer j & 1
+      // S = Q K^T of a chunk into S buffer j & 1. The buffer held the S, then
+      // the P, of chunk j - 2, whose P V this thread issued earlier: the
+      // tcgen05.mma operations of one thread run in issue order, so that P V
+      // has read its P before this S overwrites it.
       auto issue_s = [&](const ChunkIt& it) {
         const int qbuf = it.uq % kQBufs, st = static_cast<int>(it.j & 1), ks = static_cast<int>(it.j % kKStages);
         if (it.c == 0) ok = ok && mbar_wait_spin(&br.q_full[qbuf], (it.uq / kQBufs) & 1, abort_flag, &g_attn_err);
